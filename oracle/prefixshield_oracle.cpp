@@ -63,9 +63,11 @@ enum Stat {
   S_DEBT_RAW, S_DEBT_NORM
 };
 
-// Recency stamp: (step, request, reversed position).  A request releases its
-// blocks tail first, so within a request the deeper block is older.
-constexpr uint64_t POS_BITS = 20, REQ_BITS = 20, STEP_BITS = 24;
+// Recency stamp: (step, request, reversed position), 62 bits in all.  A
+// request releases its blocks tail first, so within a request the deeper block
+// is older.  Limits: 2^18-1 requests per step and full blocks per request,
+// 2^26-1 steps.
+constexpr uint64_t POS_BITS = 18, REQ_BITS = 18, STEP_BITS = 26;
 constexpr uint64_t MAX_POS = (1ull << POS_BITS) - 1;
 uint64_t make_stamp(uint64_t step, uint64_t req, uint64_t pos) {
   return (step << (REQ_BITS + POS_BITS)) | (req << POS_BITS) | (MAX_POS - pos);
@@ -403,7 +405,9 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
       int32_t j = owner[{g[i], keys[i][m]}];
       if (granted_rank(j, m) < avail) ++e[i]; else break;
     }
-    if (e[i] < s[i] - h[i]) a[i] = 0;  // cannot materialize past an ungranted block
+    // When e_i < s_i - h_i some earlier rank r >= avail is not granted, and
+    // base_i > r, so a_i is already 0: no block is materialized past an
+    // ungranted one.
     hit[i] = h[i] + e[i];
   }
 

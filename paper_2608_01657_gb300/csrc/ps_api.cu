@@ -1,0 +1,450 @@
+// C ABI of the prefix-cache step library (declared in include/prefixshield.h).
+//
+// Host side only: argument checks, the workspace layout, the handle, and the
+// copies of the test hooks.  Every stage of a step runs in the kernels of
+// ps_kernels.cu.
+#include <cstdlib>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "ps_internal.cuh"
+
+using namespace ps;
+
+struct ps_handle {
+  DevState base;        // constants and carved pointers; per-step fields unused
+  void* workspace;
+  size_t workspace_bytes;
+  int device;
+  // staging area for ps_step_host()
+  int32_t* st_group;
+  int64_t* st_offsets;
+  int32_t* st_tokens;
+  int32_t* st_contract;
+  uint64_t* st_prefix;
+  ps_step_out_t st_out;
+};
+
+namespace {
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+inline uint32_t log2_pow2_at_least(uint64_t v) {
+  uint32_t l = 0;
+  while ((1ull << l) < v) ++l;
+  return l;
+}
+
+// SplitMix64 stream (Steele, Lea, Flood 2014) for the NH key schedule.
+uint64_t splitmix_next(uint64_t* st) {
+  *st += 0x9E3779B97F4A7C15ull;
+  return mix64(*st);
+}
+
+int32_t check_params(int64_t N, int32_t bs, int32_t G, int32_t policy, const ps_params_t* P) {
+  if (!P || N <= 0 || N > (1ll << 30)) return PS_ERR_INVALID_ARG;
+  if (bs != 2 && bs != 4 && bs != 8 && bs != 16 && bs != 32 && bs != 64) return PS_ERR_INVALID_ARG;
+  if (G <= 0 || G > PS_MAX_GROUPS || policy < 0 || policy > 2) return PS_ERR_INVALID_ARG;
+  if (P->num_contracts < 1 || P->num_contracts > PS_MAX_CONTRACTS) return PS_ERR_INVALID_ARG;
+  if (P->fp_shift < 0 || P->fp_shift > 30 || P->epsilon_fp < 0) return PS_ERR_INVALID_ARG;
+  int64_t rmin = P->rho_fp[0], rmax = P->rho_fp[0];
+  for (int c = 0; c < P->num_contracts; ++c) {
+    if (P->rho_fp[c] <= 0 || P->beta_fp[c] < 0) return PS_ERR_INVALID_ARG;
+    if (P->beta_fp[c] > (1ll << 52) || P->rho_fp[c] > (1ll << 52)) return PS_ERR_INVALID_ARG;
+    if (P->rho_fp[c] < rmin) rmin = P->rho_fp[c];
+    if (P->rho_fp[c] > rmax) rmax = P->rho_fp[c];
+  }
+  // Eq. 8's decrement rho_min/rho_max in fixed point must be at least 1.
+  if ((int64_t)(((__int128)1 << P->fp_shift) * rmin / rmax) < 1) return PS_ERR_INVALID_ARG;
+  for (int g = 0; g < G; ++g)
+    if (P->contract_of_group[g] < 0 || P->contract_of_group[g] >= P->num_contracts) return PS_ERR_INVALID_ARG;
+  if (P->s3_small_pct < 1 || P->s3_small_pct > 100 || P->s3_freq_cap < 1 || P->s3_freq_cap > 255)
+    return PS_ERR_INVALID_ARG;
+  if (P->s3_move_min_freq < 1 || P->history_capacity < 1 || P->history_capacity > (1ll << 28))
+    return PS_ERR_INVALID_ARG;
+  return PS_OK;
+}
+
+// Workspace carving.  One pass computes offsets (base == nullptr) or
+// assigns pointers; every region starts on a 256-byte boundary.
+struct Carver {
+  char* base;
+  size_t off = 0;
+  template <typename T>
+  T* take(size_t count) {
+    off = align_up(off, 256);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += sizeof(T) * (count ? count : 1);
+    return p;
+  }
+};
+
+struct Dims {
+  int64_t N, max_tokens, max_blocks, nwords, hist_cap;
+  int32_t bs, G, C, max_requests;
+  uint32_t tb_log2, cl_log2, hist_log2;
+};
+
+Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t max_requests, int64_t max_tokens) {
+  Dims d{};
+  d.N = N; d.bs = bs; d.G = G; d.C = P->num_contracts; d.max_requests = max_requests;
+  d.max_tokens = max_tokens;
+  d.max_blocks = max_tokens / bs;
+  d.nwords = (N + 31) / 32;
+  // native table: 8-way buckets at load <= 1/2
+  d.tb_log2 = log2_pow2_at_least((uint64_t)((N + 3) / 4 > 1 ? (N + 3) / 4 : 1));
+  if (d.tb_log2 < 1) d.tb_log2 = 1;
+  // claim map: 4-way buckets, capacity >= 2 x blocks of a step
+  d.cl_log2 = log2_pow2_at_least((uint64_t)(d.max_blocks / 2 > 1 ? d.max_blocks / 2 : 1));
+  if (d.cl_log2 < 1) d.cl_log2 = 1;
+  d.hist_log2 = log2_pow2_at_least((uint64_t)(2 * (P->history_capacity + max_requests)));
+  if (d.hist_log2 < 1) d.hist_log2 = 1;
+  d.hist_cap = P->history_capacity;
+  return d;
+}
+
+// Returns the total size; fills s / h pointers when base != nullptr.
+size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
+  Carver cv{base};
+  const size_t N = (size_t)d.N, R = (size_t)d.max_requests, B = (size_t)d.max_blocks, G = (size_t)d.G;
+  DevState t{};
+  t.ctl = cv.take<Ctl>(1);
+  t.blk_key = cv.take<uint64_t>(N);
+  t.blk_stamp = cv.take<uint64_t>(N);
+  t.blk_prefix = cv.take<uint64_t>(N);
+  t.blk_promo = cv.take<uint64_t>(N);
+  t.blk_s3seq = cv.take<uint64_t>(N);
+  t.blk_group = cv.take<uint16_t>(N);
+  t.blk_contract = cv.take<uint8_t>(N);
+  t.blk_klass = cv.take<uint8_t>(N);
+  t.blk_flags = cv.take<uint8_t>(N);
+  t.blk_freq = cv.take<uint32_t>(N);
+  t.blk_acc = cv.take<uint32_t>(N);
+  t.blk_slot = cv.take<uint32_t>(N);
+  t.blk_pin = cv.take<uint32_t>(N);
+  t.blk_inval = cv.take<uint32_t>(N);
+  const size_t zero_end = cv.off;  // everything above starts zeroed
+  t.res_bits = cv.take<uint32_t>((size_t)d.nwords);
+  t.table = cv.take<TableEntry>((size_t)kTableWays << d.tb_log2);
+  t.table_ovf = cv.take<uint32_t>((size_t)1 << d.tb_log2);
+  t.ledger = cv.take<int64_t>(G * d.C);
+  t.contract_of_group = cv.take<int32_t>(G);
+  t.key_words = cv.take<uint32_t>((size_t)d.bs + 2);
+  t.stats = cv.take<int64_t>(G * PS_NUM_STATS);
+  t.hist = cv.take<HistEntry>((size_t)1 << d.hist_log2);
+  t.rq_n = cv.take<int32_t>(R);
+  t.rq_pbase = cv.take<int32_t>(R);
+  t.rq_h = cv.take<int32_t>(R);
+  t.rq_s = cv.take<int32_t>(R);
+  t.rq_cbase = cv.take<int32_t>(R);
+  t.rq_a = cv.take<int32_t>(R);
+  t.rq_e = cv.take<int32_t>(R);
+  t.rq_cid = cv.take<int32_t>(R);
+  t.rq_hs = cv.take<uint32_t>(R);
+  t.rq_p = cv.take<uint64_t>(R);
+  t.rq_flags = cv.take<uint8_t>(R);
+  t.rq_knew = cv.take<uint8_t>(R);
+  t.pos_key = cv.take<uint64_t>(B);
+  t.pos_blk = cv.take<uint32_t>(B);
+  t.pos_claim = cv.take<uint32_t>(B);
+  t.pos_elig = cv.take<uint8_t>(B);
+  t.claims = cv.take<ClaimEntry>((size_t)kClaimWays << d.cl_log2);
+  t.bm_victim = cv.take<uint32_t>((size_t)d.nwords);
+  t.bm_alloc = cv.take<uint32_t>((size_t)d.nwords);
+  t.bm_inval = cv.take<uint32_t>((size_t)d.nwords);
+  t.csk = cv.take<uint64_t>(N);
+  t.grp_qsize = cv.take<int64_t>(G);
+  t.grp_P = cv.take<int64_t>(G);
+  t.grp_delta = cv.take<int64_t>(G);
+  t.grp_x = cv.take<int64_t>(G);
+  t.sel = cv.take<SelSeg>(G);
+  t.hist_bins = cv.take<uint32_t>(G * kRadixBins);
+  t.bm_chunk_cnt = cv.take<int32_t>(3 * (((size_t)d.nwords + 1023) / 1024));
+  // staging for ps_step_host
+  int32_t* st_group = cv.take<int32_t>(R);
+  int64_t* st_offsets = cv.take<int64_t>(R + 1);
+  int32_t* st_tokens = cv.take<int32_t>((size_t)d.max_tokens);
+  int32_t* st_contract = cv.take<int32_t>(R);
+  uint64_t* st_prefix = cv.take<uint64_t>(R);
+  ps_step_out_t so{};
+  so.hit_blocks = cv.take<int32_t>(R);
+  so.admitted_blocks = cv.take<int32_t>(R);
+  so.admitted_offsets = cv.take<int32_t>(R + 1);
+  so.admitted_ids = cv.take<int32_t>(B);
+  so.evicted_ids = cv.take<int32_t>(B);
+  so.invalidated_ids = cv.take<int32_t>(B);
+  so.counts = cv.take<int32_t>(4);
+  so.debt_raw = cv.take<int64_t>(G);
+  so.debt_norm = cv.take<int64_t>(G);
+  const size_t total = align_up(cv.off, 256);
+  if (base) {
+    *s = t;
+    h->st_group = st_group; h->st_offsets = st_offsets; h->st_tokens = st_tokens;
+    h->st_contract = st_contract; h->st_prefix = st_prefix; h->st_out = so;
+  }
+  (void)zero_end;
+  return total;
+}
+
+int32_t init_state(ps_handle* h, cudaStream_t st) {
+  const DevState& s = h->base;
+  // everything zero, then the non-zero patterns
+  if (cudaMemsetAsync(h->workspace, 0, h->workspace_bytes, st) != cudaSuccess) return PS_ERR_CUDA;
+  if (cudaMemsetAsync(s.table, 0xFF, sizeof(TableEntry) * ((size_t)kTableWays << s.tb_nbuckets_log2), st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  launch_init(s, st);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+inline cudaStream_t as_stream(void* p) { return reinterpret_cast<cudaStream_t>(p); }
+
+}  // namespace
+
+extern "C" {
+
+size_t ps_workspace_bytes(int64_t capacity_blocks, int32_t block_size, int32_t num_groups, const ps_params_t* params,
+                          int32_t max_requests, int64_t max_tokens) {
+  if (check_params(capacity_blocks, block_size, num_groups, 0, params) != PS_OK) return 0;
+  if (max_requests < 0 || max_requests > PS_MAX_REQUESTS_PER_STEP || max_tokens < 0 || max_tokens > (1ll << 31))
+    return 0;
+  const Dims d = make_dims(capacity_blocks, block_size, num_groups, params, max_requests, max_tokens);
+  return carve(d, nullptr, nullptr, nullptr);
+}
+
+int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size, int32_t num_groups, int32_t policy,
+                  const ps_params_t* params, void* d_workspace, size_t workspace_bytes, int32_t max_requests,
+                  int64_t max_tokens, void* stream) {
+  if (!out) return PS_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (check_params(capacity_blocks, block_size, num_groups, policy, params) != PS_OK) return PS_ERR_INVALID_ARG;
+  if (policy == PS_S3FIFO) return PS_ERR_INVALID_ARG;  // not built yet
+  const size_t need = ps_workspace_bytes(capacity_blocks, block_size, num_groups, params, max_requests, max_tokens);
+  if (need == 0 || !d_workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(d_workspace) & 255))
+    return PS_ERR_INVALID_ARG;
+  ps_handle* h = new (std::nothrow) ps_handle();
+  if (!h) return PS_ERR_INVALID_ARG;
+  const Dims d = make_dims(capacity_blocks, block_size, num_groups, params, max_requests, max_tokens);
+  h->workspace = d_workspace;
+  h->workspace_bytes = need;
+  cudaGetDevice(&h->device);
+  DevState s{};
+  carve(d, static_cast<char*>(d_workspace), &s, h);
+  s.N = capacity_blocks; s.bs = block_size; s.G = num_groups; s.C = params->num_contracts; s.policy = policy;
+  s.flags = params->flags; s.fp_shift = params->fp_shift; s.eps = params->epsilon_fp; s.hash_seed = params->hash_seed;
+  s.rho_min = params->rho_fp[0];
+  for (int c = 0; c < PS_MAX_CONTRACTS; ++c) {
+    s.rho[c] = c < s.C ? params->rho_fp[c] : 1;
+    s.beta[c] = c < s.C ? params->beta_fp[c] : 0;
+    if (c < s.C && params->rho_fp[c] < s.rho_min) s.rho_min = params->rho_fp[c];
+  }
+  s.s3_small_pct = params->s3_small_pct; s.s3_freq_cap = params->s3_freq_cap; s.s3_move_min = params->s3_move_min_freq;
+  s.max_requests = max_requests; s.max_tokens = max_tokens; s.max_blocks = d.max_blocks;
+  s.history_capacity = params->history_capacity;
+  s.tb_nbuckets_log2 = d.tb_log2; s.cl_nbuckets_log2 = d.cl_log2; s.hist_cap_log2 = d.hist_log2;
+  s.nwords = d.nwords;
+  h->base = s;
+  cudaStream_t st = as_stream(stream);
+  int32_t rc = init_state(h, st);
+  if (rc == PS_OK) {
+    std::vector<uint32_t> kw((size_t)block_size + 2);
+    uint64_t seed = params->hash_seed;
+    for (auto& w : kw) w = (uint32_t)splitmix_next(&seed);
+    std::vector<int32_t> cog(params->contract_of_group, params->contract_of_group + num_groups);
+    if (cudaMemcpyAsync(s.key_words, kw.data(), kw.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+        cudaMemcpyAsync(s.contract_of_group, cog.data(), cog.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+      rc = PS_ERR_CUDA;
+  }
+  if (rc != PS_OK) {
+    delete h;
+    return rc;
+  }
+  *out = h;
+  return PS_OK;
+}
+
+int32_t ps_step(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t num_requests, const int32_t* d_group_ids,
+                const int64_t* d_token_offsets, const int32_t* d_tokens, const int32_t* d_contract_ids,
+                const uint64_t* d_prefix_ids, const ps_step_out_t* out) {
+  if (!h || !out || num_requests < 0 || num_requests > h->base.max_requests || !d_token_offsets) return PS_ERR_INVALID_ARG;
+  if (num_requests > 0 && (!d_group_ids || !d_tokens)) return PS_ERR_INVALID_ARG;
+  if (!out->hit_blocks || !out->admitted_blocks || !out->admitted_offsets || !out->admitted_ids || !out->evicted_ids ||
+      !out->invalidated_ids || !out->counts || !out->debt_raw || !out->debt_norm)
+    return PS_ERR_INVALID_ARG;
+  DevState s = h->base;
+  s.now = now_ticks;
+  s.R = num_requests;
+  s.in_group = d_group_ids;
+  s.in_offsets = d_token_offsets;
+  s.in_tokens = d_tokens;
+  s.in_contract = d_contract_ids;
+  s.in_prefix = d_prefix_ids;
+  s.tokens_aligned16 = (reinterpret_cast<uintptr_t>(d_tokens) & 15) == 0;
+  s.out = *out;
+  return launch_step(s, as_stream(stream));
+}
+
+int32_t ps_step_host(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t num_requests, const int32_t* h_group_ids,
+                     const int64_t* h_token_offsets, const int32_t* h_tokens, const int32_t* h_contract_ids,
+                     const uint64_t* h_prefix_ids, const ps_host_out_t* h_out) {
+  if (!h || !h_out || num_requests < 0 || num_requests > h->base.max_requests || !h_token_offsets)
+    return PS_ERR_INVALID_ARG;
+  const int64_t T = num_requests > 0 ? h_token_offsets[num_requests] : 0;
+  if (T < 0 || T > h->base.max_tokens || (num_requests > 0 && (!h_group_ids || (T > 0 && !h_tokens))))
+    return PS_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  const size_t R = (size_t)num_requests;
+  auto h2d = [&](void* d, const void* src, size_t bytes) {
+    return bytes == 0 || cudaMemcpyAsync(d, src, bytes, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  };
+  if (!h2d(h->st_offsets, h_token_offsets, (R + 1) * 8) || !h2d(h->st_group, h_group_ids, R * 4) ||
+      !h2d(h->st_tokens, h_tokens, (size_t)T * 4) ||
+      (h_contract_ids && !h2d(h->st_contract, h_contract_ids, R * 4)) ||
+      (h_prefix_ids && !h2d(h->st_prefix, h_prefix_ids, R * 8)))
+    return PS_ERR_CUDA;
+  int32_t rc = ps_step(h, stream, now_ticks, num_requests, h->st_group, h->st_offsets, h->st_tokens,
+                       h_contract_ids ? h->st_contract : nullptr, h_prefix_ids ? h->st_prefix : nullptr, &h->st_out);
+  if (rc != PS_OK) return rc;
+  const ps_step_out_t& o = h->st_out;
+  auto d2h = [&](void* dst, const void* d, size_t bytes) {
+    return bytes == 0 || !dst || cudaMemcpyAsync(dst, d, bytes, cudaMemcpyDeviceToHost, st) == cudaSuccess;
+  };
+  const size_t G = (size_t)h->base.G;
+  if (!d2h(h_out->counts, o.counts, 16) || !d2h(h_out->hit_blocks, o.hit_blocks, R * 4) ||
+      !d2h(h_out->admitted_blocks, o.admitted_blocks, R * 4) ||
+      !d2h(h_out->admitted_offsets, o.admitted_offsets, (R + 1) * 4) || !d2h(h_out->debt_raw, o.debt_raw, G * 8) ||
+      !d2h(h_out->debt_norm, o.debt_norm, G * 8) || cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  if (!h_out->counts || h_out->counts[3] != PS_OK) return h_out->counts ? h_out->counts[3] : PS_OK;
+  if (!d2h(h_out->admitted_ids, o.admitted_ids, (size_t)h_out->counts[0] * 4) ||
+      !d2h(h_out->evicted_ids, o.evicted_ids, (size_t)h_out->counts[1] * 4) ||
+      !d2h(h_out->invalidated_ids, o.invalidated_ids, (size_t)h_out->counts[2] * 4) ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  return PS_OK;
+}
+
+int32_t ps_stats(ps_handle_t* h, void* stream, int64_t* h_stats) {
+  if (!h || !h_stats) return PS_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  int32_t sticky = PS_OK;
+  if (cudaMemcpyAsync(h_stats, h->base.stats, sizeof(int64_t) * h->base.G * PS_NUM_STATS, cudaMemcpyDeviceToHost, st) !=
+          cudaSuccess ||
+      cudaMemcpyAsync(&sticky, &h->base.ctl->sticky, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  return sticky;
+}
+
+int32_t ps_clear_status(ps_handle_t* h, void* stream) {
+  if (!h) return PS_ERR_INVALID_ARG;
+  return cudaMemsetAsync(&h->base.ctl->sticky, 0, 4, as_stream(stream)) == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+int32_t ps_reset(ps_handle_t* h, void* stream) {
+  if (!h) return PS_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  // key words and contract map survive in host copies: rebuild them
+  std::vector<uint32_t> kw((size_t)h->base.bs + 2);
+  std::vector<int32_t> cog((size_t)h->base.G);
+  if (cudaMemcpyAsync(kw.data(), h->base.key_words, kw.size() * 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaMemcpyAsync(cog.data(), h->base.contract_of_group, cog.size() * 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  int32_t rc = init_state(h, st);
+  if (rc != PS_OK) return rc;
+  if (cudaMemcpyAsync(h->base.key_words, kw.data(), kw.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+      cudaMemcpyAsync(h->base.contract_of_group, cog.data(), cog.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  return PS_OK;
+}
+
+void ps_destroy(ps_handle_t* h) { delete h; }
+
+const char* ps_status_string(int32_t status) {
+  switch (status) {
+    case PS_OK: return "ok";
+    case PS_ERR_INVALID_ARG: return "invalid argument";
+    case PS_ERR_CAPACITY: return "capacity exceeded";
+    case PS_ERR_CLOCK: return "accounting clock went backwards";
+    case PS_ERR_CUDA: return "CUDA error";
+    case PS_ERR_TIMEOUT: return "device wait timed out";
+    case PS_ERR_DEVICE_STATUS: return "device reported an error";
+    default: return "unknown status";
+  }
+}
+
+int32_t ps_export_state(ps_handle_t* h, void* stream, ps_state_view_t* v) {
+  if (!h || !v) return PS_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  const DevState& s = h->base;
+  const size_t N = (size_t)s.N;
+  std::vector<uint8_t> flags(N), contract(N), klass(N);
+  std::vector<uint16_t> group(N);
+  std::vector<uint32_t> freq(N);
+  Ctl ctl{};
+  bool ok = true;
+  auto d2h = [&](void* dst, const void* src, size_t bytes) {
+    ok = ok && cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, st) == cudaSuccess;
+  };
+  d2h(flags.data(), s.blk_flags, N);
+  d2h(contract.data(), s.blk_contract, N);
+  d2h(klass.data(), s.blk_klass, N);
+  d2h(group.data(), s.blk_group, N * 2);
+  d2h(freq.data(), s.blk_freq, N * 4);
+  d2h(&ctl, s.ctl, sizeof(Ctl));
+  if (v->key) d2h(v->key, s.blk_key, N * 8);
+  if (v->prefix) d2h(v->prefix, s.blk_prefix, N * 8);
+  if (v->stamp) d2h(v->stamp, s.blk_stamp, N * 8);
+  if (v->acc) d2h(v->acc, s.blk_acc, N * 4);
+  if (v->s3seq) d2h(v->s3seq, s.blk_s3seq, N * 8);
+  if (v->balances) d2h(v->balances, s.ledger, sizeof(int64_t) * s.G * s.C);
+  if (!ok || cudaStreamSynchronize(st) != cudaSuccess) return PS_ERR_CUDA;
+  for (size_t b = 0; b < N; ++b) {
+    if (v->resident) v->resident[b] = flags[b] & 1;
+    if (v->group) v->group[b] = group[b];
+    if (v->contract) v->contract[b] = contract[b];
+    if (v->klass) v->klass[b] = klass[b];
+    if (v->freq) v->freq[b] = (int32_t)(freq[b] < (uint32_t)s.s3_freq_cap ? freq[b] : (uint32_t)s.s3_freq_cap);
+    if (v->s3q) v->s3q[b] = (flags[b] >> 1) & 1;
+  }
+  v->t_prev = ctl.t_prev;
+  v->step = ctl.step;
+  v->s3_ctr = ctl.s3_ctr;
+  v->ghost_ctr = ctl.ghost_ctr;
+  return PS_OK;
+}
+
+int64_t ps_export_history(ps_handle_t* h, void* stream, int32_t* h_group, uint64_t* h_prefix, uint64_t* h_refcount,
+                          uint8_t* h_admitted, int64_t cap) {
+  if (!h) return PS_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  const size_t n = (size_t)1 << h->base.hist_cap_log2;
+  std::vector<HistEntry> e(n);
+  if (cudaMemcpyAsync(e.data(), h->base.hist, n * sizeof(HistEntry), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  int64_t k = 0;
+  for (const HistEntry& x : e) {
+    if (x.g1 == 0) continue;
+    const uint32_t rc = x.refadm & 0x7FFFFFFFu;
+    const bool adm = x.refadm >> 31;
+    if (rc == 0 && !adm) continue;
+    if (h_group && k < cap) {
+      h_group[k] = (int32_t)x.g1 - 1;
+      h_prefix[k] = x.p;
+      h_refcount[k] = rc;
+      h_admitted[k] = adm;
+    }
+    ++k;
+  }
+  return k;
+}
+
+int64_t ps_export_ghost(ps_handle_t* h, void* stream, int32_t* h_group, uint64_t* h_key, uint64_t* h_seq, int64_t cap) {
+  (void)h; (void)stream; (void)h_group; (void)h_key; (void)h_seq; (void)cap;
+  return 0;
+}
+
+}  // extern "C"

@@ -1,0 +1,204 @@
+// Internal declarations of the GB300 prefix-cache step library.
+//
+// Device state lives in one caller-provided workspace, carved into the
+// structure-of-arrays layout below.  Every kernel receives a DevState by
+// value: the carved pointers, the handle's constants and the current step's
+// input/output pointers.
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+
+#include <cuda_runtime.h>
+
+#include "prefixshield.h"
+
+namespace ps {
+
+// ---- constants -------------------------------------------------------------
+constexpr uint32_t kNone = 0xFFFFFFFFu;           // empty slot / no block
+constexpr int kProb = 0, kNormal = 1, kReuse = 2;  // retention classes (Eq. 9 order)
+constexpr int kStampPosBits = 18, kStampReqBits = 18, kStampStepBits = 26;
+constexpr uint64_t kMaxPos = (1ull << kStampPosBits) - 1;
+constexpr uint64_t kMaxStep = (1ull << kStampStepBits) - 1;
+constexpr int kTableWays = 8;    // native prefix table: 8 x 16 B entries per 128 B bucket
+constexpr int kClaimWays = 4;    // per-step claim map: 4 x 32 B entries per bucket
+constexpr int kRadixBits = 8;
+constexpr int kRadixBins = 1 << kRadixBits;
+
+// Recency stamp (native free-queue order): larger = more recently released.
+__host__ __device__ __forceinline__ uint64_t make_stamp(uint64_t step, uint64_t req, uint64_t pos) {
+  return (step << (kStampReqBits + kStampPosBits)) | (req << kStampPosBits) | (kMaxPos - pos);
+}
+
+// ---- table entries ---------------------------------------------------------
+struct __align__(16) TableEntry {   // native prefix table (group, key) -> block
+  uint64_t key;
+  uint32_t blk;   // kNone when the slot is empty
+  uint32_t grp;
+};
+
+struct __align__(32) ClaimEntry {   // per-step: first request that needs a new key
+  uint64_t key;     // 0 when empty
+  uint32_t minreq;  // lowest request index containing the key (atomicMin)
+  uint32_t last;    // 1 + highest request index that hit it in-step (atomicMax)
+  uint32_t tcnt;    // in-step touches
+  uint32_t promo;   // lowest request index whose touch promotes it
+  uint32_t pad0, pad1;
+};
+
+struct __align__(32) HistEntry {    // (group, prefix id) -> reference history
+  uint64_t p;       // 0 when empty
+  uint32_t g1;      // group + 1
+  uint32_t refadm;  // reference count (bits 0..30) | admitted (bit 31)
+  uint64_t ftag;    // (step << 32) | ~first request of the step with this entry
+  uint64_t atag;    // (step << 32) | ~first request of the step that admitted
+};
+
+// Device-resident control block: persistent scalars and per-step scalars.
+struct Ctl {
+  // persistent
+  int32_t sticky;          // PS_OK or PS_ERR_CAPACITY
+  int32_t pad0;
+  uint64_t step;           // index of the step being / next to be processed (from 1)
+  int64_t t_prev;          // last refill time
+  int64_t n_resident;
+  int64_t hist_live;
+  uint64_t s3_ctr, ghost_ctr;
+  int64_t s3_nS, s3_nM;
+  uint64_t ringS_head, ringS_tail, ringM_head, ringM_tail;
+  uint64_t ghost_head, ghost_tail;
+  int64_t ghost_live;
+  // per step
+  int32_t status;          // this step's status
+  int32_t pad1;
+  int64_t T, nblocks;
+  int64_t pinned, n_inval, total_claims, avail, need, nfree, ftake, mvict;
+  int64_t hist_new;
+  int64_t n_evicted, n_alloc, n_victims_marked;
+  int64_t m_fb;            // prefixshield: victims left to the global fallback
+  int32_t sel_ntie, sel_k; // prefixshield tie bookkeeping
+  uint32_t ticket;         // last-block-done counter for the radix passes
+  int32_t internal_error;  // an invariant of the step failed (reported, never expected)
+};
+
+// Per-segment state of the segmented radix select.
+struct __align__(16) SelSeg {
+  uint64_t prefix;   // key bits fixed so far
+  uint64_t mask;     // which bits are fixed
+  int64_t rank;      // 1-based rank still to locate inside the prefix class
+  int32_t active;    // 1 while this segment selects
+  int32_t incl;      // 1: victims are keys <= prefix; 0: keys < prefix
+};
+
+struct DevState {
+  // constants
+  int64_t N;
+  int32_t bs, G, C, policy;
+  uint32_t flags;
+  int32_t fp_shift;
+  int64_t eps;
+  uint64_t hash_seed;
+  int64_t rho[PS_MAX_CONTRACTS], beta[PS_MAX_CONTRACTS];
+  int64_t rho_min;
+  int32_t s3_small_pct, s3_freq_cap, s3_move_min;
+  int32_t max_requests;
+  int64_t max_tokens, max_blocks;
+  int64_t history_capacity;
+  uint32_t tb_nbuckets_log2, cl_nbuckets_log2, hist_cap_log2;
+  int64_t nwords;          // resident bitmap words
+  // persistent state
+  Ctl* ctl;
+  uint64_t* blk_key;
+  uint64_t* blk_stamp;
+  uint64_t* blk_prefix;
+  uint64_t* blk_promo;     // (step << 32) | ~promoting request (atomicMax)
+  uint64_t* blk_s3seq;
+  uint16_t* blk_group;
+  uint8_t* blk_contract;
+  uint8_t* blk_klass;
+  uint8_t* blk_flags;      // bit0 resident, bit1 S3-FIFO main queue
+  uint32_t* blk_freq;      // S3-FIFO counter, unclamped (read as min(cap, f))
+  uint32_t* blk_acc;
+  uint32_t* blk_slot;      // table slot of a resident block
+  uint32_t* blk_pin;       // step tag: hit in this step
+  uint32_t* blk_inval;     // step tag: invalidated in this step
+  uint32_t* res_bits;      // resident bitmap
+  TableEntry* table;
+  uint32_t* table_ovf;     // per bucket: live keys probing past it
+  int64_t* ledger;         // B_{g,c}, fixed point
+  int32_t* contract_of_group;
+  uint32_t* key_words;     // NH key schedule, bs + 2 words
+  int64_t* stats;          // [G][PS_NUM_STATS]
+  HistEntry* hist;
+  // per-step scratch
+  int32_t* rq_n;           // full blocks
+  int32_t* rq_pbase;       // first position index of the request
+  int32_t* rq_h;           // cached prefix length
+  int32_t* rq_s;           // first own claim
+  int32_t* rq_cbase;       // exclusive scan of claims
+  int32_t* rq_a;           // granted (admitted) blocks
+  int32_t* rq_e;           // in-step hits
+  int32_t* rq_cid;         // contract
+  uint32_t* rq_hs;         // history slot
+  uint64_t* rq_p;          // prefix id
+  uint8_t* rq_flags;       // bit0 proven, bit1 gate open
+  uint8_t* rq_knew;        // class of newly admitted blocks
+  uint64_t* pos_key;
+  uint32_t* pos_blk;       // resident block hit by lookup (or kNone)
+  uint32_t* pos_claim;     // claim-map slot (or kNone)
+  uint8_t* pos_elig;       // touch was promotion-eligible
+  ClaimEntry* claims;
+  uint32_t* bm_victim;     // per-step bitmaps over block ids
+  uint32_t* bm_alloc;
+  uint32_t* bm_inval;
+  uint64_t* csk;           // candidate sort keys (~0 = not a candidate)
+  int64_t* grp_qsize;      // candidates per group
+  int64_t* grp_P;          // projected score P^(0)_g = normalized debt
+  int64_t* grp_delta;      // Eq. 8 decrement
+  int64_t* grp_x;          // victims taken from the group in the debt phase
+  SelSeg* sel;             // [G] segments
+  uint32_t* hist_bins;     // [G][256] radix histogram
+  int32_t* bm_chunk_cnt;   // [3][chunks] bitmap compaction counts
+  // current step inputs / outputs
+  int64_t now;
+  int32_t R;
+  const int32_t* in_group;
+  const int64_t* in_offsets;
+  const int32_t* in_tokens;
+  const int32_t* in_contract;
+  const uint64_t* in_prefix;
+  int32_t tokens_aligned16;
+  ps_step_out_t out;
+};
+
+// ---- hashing (published definitions, implemented here independently) -----
+// SplitMix64 output function (Steele, Lea, Flood 2014), used as a mixer.
+__host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+__host__ __device__ __forceinline__ uint64_t fix_reserved(uint64_t h) {
+  return (h == 0 || h == ~0ull) ? 1ull : h;
+}
+__host__ __device__ __forceinline__ uint64_t chain_seed(uint64_t seed, int32_t g) {
+  return mix64(seed ^ ((uint64_t)(g + 1) * 0x9E3779B97F4A7C15ull));
+}
+__device__ __forceinline__ uint32_t table_home(uint64_t key, uint32_t g, uint32_t log2nb) {
+  uint64_t x = (key ^ ((uint64_t)(g + 1) * 0x9E3779B97F4A7C15ull)) * 0xD6E8FEB86659FD93ull;
+  return (uint32_t)(x >> (64 - log2nb));
+}
+__device__ __forceinline__ uint32_t claim_home(uint64_t key, uint32_t log2nb) {
+  return (uint32_t)((key * 0xC2B2AE3D27D4EB4Full) >> (64 - log2nb));
+}
+__device__ __forceinline__ uint32_t hist_home(uint64_t p, uint32_t g, uint32_t log2cap) {
+  uint64_t x = (p ^ ((uint64_t)(g + 1) * 0xFF51AFD7ED558CCDull)) * 0x9E3779B97F4A7C15ull;
+  return (uint32_t)(x >> (64 - log2cap));
+}
+
+// ---- host launchers (ps_kernels.cu) ----------------------------------------
+void launch_init(const DevState& s, cudaStream_t st);
+int32_t launch_step(const DevState& s, cudaStream_t st);
+
+}  // namespace ps

@@ -173,3 +173,40 @@ def check_step(oc, before, after, step_inputs, res, policy):
             want = sorted(queues[g][j] for g, j in sel)
         assert E.tolist() == want
     return hres
+
+
+# ---------------------------------------------------------------------------
+# GPU-vs-oracle comparison helpers.
+OUT_KEYS = ("hit_blocks", "admitted_blocks", "admitted_offsets", "admitted_ids", "evicted_ids",
+            "invalidated_ids", "debt_raw", "debt_norm")
+BLOCK_KEYS = ("key", "group", "contract", "prefix", "klass", "stamp", "acc", "freq")
+
+
+def compare_outputs(got, want, where=""):
+    assert got["status"] == want["status"], f"{where}: status {got['status']} != {want['status']}"
+    if want["status"] != 0:
+        return
+    for k in OUT_KEYS:
+        a, b = np.asarray(got[k]), np.asarray(want[k])
+        assert a.shape == b.shape and np.array_equal(a, b), (
+            f"{where}: {k} differs" + (f" first at {int(np.nonzero(a != b)[0][0])}" if a.shape == b.shape else
+                                       f" (len {a.shape} vs {b.shape})"))
+
+
+def compare_state(got, want, where="", s3=False):
+    assert np.array_equal(got["resident"], want["resident"]), f"{where}: residency differs"
+    r = want["resident"].astype(bool)
+    keys = BLOCK_KEYS + (("s3q", "s3seq") if s3 else ())
+    for k in keys:
+        a, b = got[k][r], want[k][r]
+        if not np.array_equal(a, b):
+            bad = np.nonzero(a != b)[0][0]
+            raise AssertionError(f"{where}: block field {k} differs at resident #{bad}: {a[bad]} != {b[bad]}")
+    assert np.array_equal(got["B"], want["B"]), f"{where}: balances differ"
+    assert got["t_prev"] == want["t_prev"] and got["step"] == want["step"], f"{where}: clock/step differ"
+    for a, b in zip(got["history"], want["history"]):
+        assert np.array_equal(a, b), f"{where}: history differs"
+    if s3:
+        assert got["s3_ctr"] == want["s3_ctr"] and got["ghost_ctr"] == want["ghost_ctr"]
+        for a, b in zip(got["ghost"], want["ghost"]):
+            assert np.array_equal(a, b), f"{where}: ghost differs"

@@ -1,0 +1,161 @@
+"""GPU-vs-oracle parity of the prefix-cache step, through the C ABI.
+
+The CUDA library and the CPU oracle run the same seeded steps; every output
+(hit and admitted counts, CSR offsets, admitted / evicted / invalidated ids,
+raw and normalized debt) must match bit for bit after every step, and so must
+the exported policy state (per-block key, owner, contract, prefix id, class,
+recency stamp, access count, frequency; balances; clock; history) and the
+per-group statistics.  Everything here is integer or fixed-point arithmetic,
+so the tolerance is zero.
+"""
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2608_01657_gb300 import workloads as W
+from _util import compare_outputs, compare_state
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+def _pair(N, bs, G, policy, params_kw, max_requests, max_tokens):
+    from paper_2608_01657_gb300 import binding as B
+    gpu = B.Cache(N, bs, G, policy, B.Params(**params_kw), max_requests=max_requests, max_tokens=max_tokens)
+    orc = O.OracleCache(N, bs, G, policy, O.Params(**params_kw))
+    return gpu, orc
+
+
+def _run(gpu, orc, steps, state_every=1, s3=False, label=""):
+    dev = torch.device("cuda")
+    for k, st in enumerate(steps):
+        g = torch.from_numpy(st.groups).to(dev)
+        o = torch.from_numpy(st.offsets).to(dev)
+        t = torch.from_numpy(st.tokens if st.num_tokens else np.zeros(4, np.int32)).to(dev)
+        c = None if st.contracts is None else torch.from_numpy(st.contracts).to(dev)
+        p = None if st.prefixes is None else torch.from_numpy(st.prefixes.view(np.int64)).to(dev)
+        rc = gpu.step(st.now, g, o, t, c, p)
+        assert rc == 0, f"{label} step {k}: launch rc {rc}"
+        got = gpu.fetch(st.num_requests)
+        want = orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts, st.prefixes)
+        compare_outputs(got, want, f"{label} step {k}")
+        if state_every and (k % state_every == 0 or k == len(steps) - 1):
+            compare_state(gpu.export(), orc.export(), f"{label} step {k}", s3=s3)
+    assert np.array_equal(gpu.stats(), orc.stats()), f"{label}: stats differ"
+
+
+GPU_POLICIES = ["lru", "prefixshield"]
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+@pytest.mark.parametrize("seed,N,G,R,contracts,prefixes,flags", [
+    (1, 24, 2, 3, 0, False, 0),
+    (2, 40, 3, 6, 0, False, 0),
+    (3, 64, 4, 8, 3, True, 0),
+    (4, 12, 1, 2, 0, False, 0),
+    (5, 30, 3, 5, 3, True, 1),
+    (6, 30, 3, 5, 3, True, 2),
+    (11, 20, 2, 4, 2, False, 0),
+])
+def test_parity_fuzz(policy, seed, N, G, R, contracts, prefixes, flags):
+    steps = W.fuzz_steps(seed, G, R, 60, docs_per_group=3, doc_blocks=7, fresh_max_blocks=2,
+                         with_contracts=contracts, with_prefixes=prefixes, now_stride=2, empty_every=9)
+    kw = dict(rho=(2.0, 1.5, 1.0), beta=(6.0, 5.0, 4.0), flags=flags, contract_of_group=[g % 3 for g in range(G)])
+    gpu, orc = _pair(N, 16, G, policy, kw, max_requests=R, max_tokens=4096)
+    _run(gpu, orc, steps, label=f"fuzz{seed}/{policy}")
+
+
+@pytest.mark.parametrize("bs", [2, 4, 8, 32, 64])
+def test_parity_block_sizes(bs):
+    steps = W.fuzz_steps(21, 2, 4, 25, block_size=bs, docs_per_group=3, doc_blocks=40, fresh_max_blocks=40)
+    gpu, orc = _pair(200, bs, 2, "prefixshield", dict(rho=(8.0,), beta=(40.0,)), max_requests=4,
+                     max_tokens=4 * 90 * bs)
+    _run(gpu, orc, steps, label=f"bs{bs}")
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+def test_parity_tiny_one_touch(policy):
+    wl = W.make_workload(0, seed=1)
+    sp = wl.spec
+    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, dict(rho=sp.rho, beta=sp.beta),
+                     max_requests=sp.requests_per_step, max_tokens=sp.requests_per_step * 1100)
+    _run(gpu, orc, list(wl.steps()), state_every=5, label=f"cfg0/{policy}")
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+@pytest.mark.parametrize("cfg,nsteps,rps", [(1, 40, None), (1, 60, 8), (2, 40, 8), (3, 30, None)])
+def test_parity_configs(policy, cfg, nsteps, rps):
+    wl = W.make_workload(cfg, seed=2, requests_per_step=rps)
+    sp = wl.spec
+    steps = list(wl.steps(nsteps))
+    maxT = max(s.num_tokens for s in steps)
+    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, dict(rho=sp.rho, beta=sp.beta),
+                     max_requests=sp.requests_per_step, max_tokens=maxT)
+    _run(gpu, orc, steps, state_every=10, label=f"cfg{cfg}/{policy}")
+
+
+def test_parity_alg2_ties():
+    """Groups with equal debt and equal decrements force Eq. 7's tie rule."""
+    G = 6
+    steps = W.fuzz_steps(31, G, 6, 50, docs_per_group=2, doc_blocks=6, fresh_max_blocks=3)
+    kw = dict(rho=(1.0,), beta=(2.0,))
+    gpu, orc = _pair(36, 16, G, "prefixshield", kw, max_requests=6, max_tokens=4096)
+    _run(gpu, orc, steps, label="ties")
+
+
+def test_invalid_inputs_leave_state_unchanged():
+    gpu, orc = _pair(32, 16, 2, "prefixshield", dict(rho=(1.0,), beta=(2.0,), history_capacity=3),
+                     max_requests=4, max_tokens=512)
+    dev = torch.device("cuda")
+    from _util import make_step, obj_tokens
+
+    def both(now, prompts, groups, contracts=None, prefixes=None, offsets=None):
+        g, o, t, _ = make_step(prompts, groups)
+        if offsets is not None:
+            o = np.asarray(offsets, np.int64)
+        rc = gpu.step(now, torch.from_numpy(g).to(dev), torch.from_numpy(o).to(dev),
+                      torch.from_numpy(t if len(t) else np.zeros(4, np.int32)).to(dev),
+                      None if contracts is None else torch.from_numpy(np.asarray(contracts, np.int32)).to(dev),
+                      None if prefixes is None else torch.from_numpy(np.asarray(prefixes, np.int64)).to(dev))
+        assert rc == 0
+        got = gpu.fetch(len(g))
+        want = orc.step(now, g, o, t, None if contracts is None else np.asarray(contracts, np.int32),
+                        None if prefixes is None else np.asarray(prefixes, np.uint64))
+        compare_outputs(got, want, f"now={now}")
+        return got["status"]
+
+    A = obj_tokens("a", blocks=2)
+    assert both(5, [A], [0]) == 0
+    snap = gpu.export()
+    assert both(4, [A], [0]) == O.ERR_CLOCK
+    assert both(5, [A], [2]) == O.ERR_INVALID_ARG
+    assert both(5, [A], [0], offsets=[1, 32]) == O.ERR_INVALID_ARG
+    assert both(5, [A], [0], contracts=[1]) == O.ERR_INVALID_ARG
+    assert both(5, [A], [0], prefixes=[0]) == O.ERR_INVALID_ARG
+    compare_state(gpu.export(), snap, "after invalid steps")
+    compare_state(gpu.export(), orc.export(), "after invalid steps vs oracle")
+    P = [obj_tokens(x) for x in "pqr"]
+    assert both(6, P[:2], [0, 1]) == 0
+    assert both(6, P[2:], [1]) == O.ERR_CAPACITY
+    assert both(7, [], []) == O.ERR_CAPACITY
+    gpu.clear_status(); orc.clear_status()
+    assert both(7, [], []) == 0
+
+
+def test_step_host_matches_step():
+    from paper_2608_01657_gb300 import binding as B
+    steps = W.fuzz_steps(41, 3, 5, 30, docs_per_group=3, doc_blocks=6)
+    kw = dict(rho=(2.0,), beta=(6.0,))
+    a = B.Cache(40, 16, 3, "prefixshield", B.Params(**kw), max_requests=5, max_tokens=2048)
+    orc = O.OracleCache(40, 16, 3, "prefixshield", O.Params(**kw))
+    for st in steps:
+        out = a.step_host(st.now, st.groups, st.offsets, st.tokens)
+        assert out["rc"] == 0
+        cnt = out["counts"]
+        got = {"status": int(cnt[3]), "hit_blocks": out["hit_blocks"][:st.num_requests],
+               "admitted_blocks": out["admitted_blocks"][:st.num_requests],
+               "admitted_offsets": out["admitted_offsets"][:st.num_requests + 1],
+               "admitted_ids": out["admitted_ids"][:cnt[0]], "evicted_ids": out["evicted_ids"][:cnt[1]],
+               "invalidated_ids": out["invalidated_ids"][:cnt[2]], "debt_raw": out["debt_raw"],
+               "debt_norm": out["debt_norm"]}
+        compare_outputs(got, orc.step(st.now, st.groups, st.offsets, st.tokens), f"step {st.index}")
