@@ -1,0 +1,394 @@
+#!/usr/bin/env python3
+"""Benchmark of the batched prefix-cache step (PrefixShield, arXiv 2608.01657).
+
+Workload: the scale trace (64 accounting groups: 8 victim, 8 attacker and 48
+benign chat groups; a pool of 1,048,576 KV blocks of 16 tokens; 4096 requests
+per step), policy prefixshield, synthetic seeded inputs.  A step is one pass
+of the whole hot path over one batch: hashing, lookup, metering, gating,
+reclamation and insertion.
+
+The pool starts empty, so ``--prefill`` untimed steps fill it before the
+``--warmup`` steps; then ``--steps`` steps are timed one by one with CUDA
+events on the launching stream, with an L2 flush (a 256 MiB write) between
+steps outside the events.  Step inputs are resident in HBM before timing.
+
+``--impl reference`` times the CPU oracle (the plain sequential statement of
+the same step) on the host cores instead.
+
+Prints one JSON line (rank 0).  Multi-GPU runs are independent replicas, one
+pool per GPU with its own trace seed (weak scaling, no collective on the data
+path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "prefix-cache step requests/s and KV blocks/s on 1 GB300; % of HBM roofline"
+WORKLOAD = ("scale: 64 groups (8 victim, 8 attacker, 48 benign chat), pool 1,048,576 blocks, "
+            "block_size 16, 4096 requests/step")
+CONFIG_INDEX = 4
+STAGES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
+          "freetake_evict", "id_lists", "insert", "commit")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--prefill", type=int, default=6, help="untimed steps that fill the empty pool")
+    ap.add_argument("--impl", choices=("own", "reference"), default="own")
+    ap.add_argument("--policy", choices=("prefixshield", "lru"), default="prefixshield")
+    ap.add_argument("--seed", type=int, default=1)
+    ap.add_argument("--cpu-steps", type=int, default=3, help="timed oracle steps for cpu_baseline")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def algorithmic_bytes(T, R, H, A, E, Ag, V):
+    """Bytes a step must touch (tokens, descriptors, table probes, claims,
+    metadata touches, insertions, victims, outputs)."""
+    return (4 * T + 12 * R + 16 * (H + R) + 32 * A + 16 * (H + E) + 48 * Ag + 32 * V + 4 * (Ag + V) + 8 * R)
+
+
+def hash_lookup_bytes(T, R, H, A):
+    """Algorithmic bytes of the hash + lookup kernel: tokens, request
+    descriptors, one table probe per cached block and per request, claims."""
+    return 4 * T + 12 * R + 16 * (H + R) + 32 * A
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for l in getattr(self, "lines", []):
+            f = [x.strip() for x in l.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unavailable"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def make_steps(seed, n):
+    from paper_2608_01657_gb300 import workloads as W
+    wl = W.make_workload(CONFIG_INDEX, seed=seed)
+    return wl.spec, list(wl.steps(n))
+
+
+def run_oracle_steps(spec, steps, timed_from):
+    """Oracle over steps; returns (seconds over steps[timed_from:], requests timed)."""
+    import oracle as O
+    oc = O.OracleCache(spec.capacity_blocks, spec.block_size, spec.num_groups, "prefixshield",
+                       O.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20))
+    t_sum, reqs = 0.0, 0
+    for k, st in enumerate(steps):
+        t0 = time.perf_counter()
+        r = oc.step(st.now, st.groups, st.offsets, st.tokens)
+        dt = time.perf_counter() - t0
+        if r["status"] != 0:
+            raise RuntimeError(f"oracle step {k} failed: {r['status']}")
+        if k >= timed_from:
+            t_sum += dt
+            reqs += st.num_requests
+    return t_sum, reqs
+
+
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return ws, rank, local
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(ws, v):
+    if ws == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda") if torch.cuda.is_available() else torch.device("cpu")
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(ws, v):
+    if ws == 1:
+        return v
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda") if torch.cuda.is_available() else torch.device("cpu")
+    t = torch.tensor([v], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+def run_reference(args, ws, rank):
+    """The oracle arm: the CPU oracle on the host cores, same workload."""
+    if rank != 0:
+        return
+    n = args.prefill + args.warmup + args.steps
+    spec, steps = make_steps(args.seed, n)
+    t, reqs = run_oracle_steps(spec, steps, args.prefill + args.warmup)
+    value = reqs / t
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / max(1, args.steps),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "policy": "prefixshield", "prefill_steps": args.prefill},
+        "cpu_baseline": {"value": value, "unit": "requests/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{args.steps} steps of the scale trace after {args.prefill + args.warmup} "
+                                   f"untimed ones ({reqs} requests)"},
+        "e2e": {"value": value, "unit": "requests/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_own(args, ws, rank, local):
+    import numpy as np
+    import torch
+
+    from paper_2608_01657_gb300 import binding as B
+    from paper_2608_01657_gb300 import build as BLD
+
+    if not BLD.up_to_date():
+        BLD.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    n_total = args.prefill + args.warmup + args.steps
+    spec, steps = make_steps(args.seed + rank, n_total)
+    maxT = max(s.num_tokens for s in steps)
+    R = spec.requests_per_step
+    dsteps = []
+    for st in steps:
+        dsteps.append((st.now, torch.from_numpy(st.groups).to(dev), torch.from_numpy(st.offsets).to(dev),
+                       torch.from_numpy(st.tokens).to(dev)))
+    params = B.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20)
+    cache = B.Cache(spec.capacity_blocks, spec.block_size, spec.num_groups, args.policy, params,
+                    max_requests=R, max_tokens=maxT)
+    cache.set_stage_timing(True)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def run(k):
+        now, g, o, t = dsteps[k]
+        rc = cache.step(now, g, o, t)
+        if rc != 0:
+            raise RuntimeError(f"ps_step rc={rc}")
+
+    for k in range(args.prefill + args.warmup):
+        run(k)
+    torch.cuda.synchronize()
+    if int(cache.out["counts"][3].item()) != 0:
+        raise RuntimeError("step status error during warmup")
+    s0 = cache.stats()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    stage_ms = np.zeros(len(STAGES))
+    launches = 0
+    barrier(ws)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for j in range(args.steps):
+            flush.zero_()
+            e0, e1 = evs[j]
+            e0.record(stream)
+            run(args.prefill + args.warmup + j)
+            e1.record(stream)
+            ms, nl = cache.stage_times()
+            stage_ms[: len(ms)] += ms
+            launches += nl
+        torch.cuda.synchronize()
+    barrier(ws)
+    step_ms = [e0.elapsed_time(e1) for e0, e1 in evs]
+    total_s = sum(step_ms) / 1e3
+    status = int(cache.out["counts"][3].item())
+    if status != 0:
+        raise RuntimeError(f"step status {status}")
+    s1 = cache.stats()
+    d = s1 - s0
+    col = {n: i for i, n in enumerate(B.STAT_NAMES)}
+    timed = steps[args.prefill + args.warmup:]
+    T = sum(s.num_tokens for s in timed)
+    nreq = sum(s.num_requests for s in timed)
+    nblocks = int(d[:, col["full_blocks"]].sum())
+    hit = int(d[:, col["hit_blocks"]].sum())
+    inst = int(d[:, col["instep_hit_blocks"]].sum())
+    adm = int(d[:, col["admitted_blocks"]].sum())
+    ungr = int(d[:, col["ungranted_blocks"]].sum())
+    ev = int(d[:, col["evicted_blocks"]].sum())
+    H = hit - inst
+    A = adm + ungr
+    alg = algorithmic_bytes(T, nreq, H, A, inst, adm, ev)
+    peak, peak_kind = peaks()
+    total_max = max_over_ranks(ws, total_s)
+    req_all = sum_over_ranks(ws, nreq)
+    blk_all = sum_over_ranks(ws, nblocks)
+    value = req_all / total_max
+    # dominant single kernel: hash + lookup (one launch per step)
+    hl_ms = stage_ms[STAGES.index("hash_lookup")] / args.steps
+    hl_bytes = hash_lookup_bytes(T, nreq, H, A) / args.steps
+    hl_gbs = hl_bytes / (hl_ms / 1e3) / 1e9
+    step_gbs = alg / total_s / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, cache, steps, dsteps, flush, R)
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        n_cpu = args.prefill + args.cpu_steps
+        t_cpu, r_cpu = run_oracle_steps(spec, steps[:n_cpu], args.prefill)
+        cpu = {"value": r_cpu / t_cpu, "unit": "requests/s", "cores": 1, "kind": "oracle",
+               "sample": f"{args.cpu_steps} steps of the scale trace ({r_cpu} requests) after {args.prefill} "
+                         f"untimed fill steps, single-threaded C++ oracle"}
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": 1e3 * total_max / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "policy": args.policy, "prefill_steps": args.prefill,
+                   "requests_per_step": R, "block_size": spec.block_size, "capacity_blocks": spec.capacity_blocks,
+                   "groups": spec.num_groups, "l2": "flushed (256 MiB write) between timed steps",
+                   "parallelism": f"replicas x{ws}"},
+        "kv_blocks_per_s": blk_all / total_max,
+        "step_roofline": {"bound": "hbm", "achieved": step_gbs, "peak": peak, "unit": "GB/s",
+                          "frac": step_gbs / peak, "algorithmic_bytes_per_step": alg / args.steps,
+                          "peak_kind": peak_kind},
+        "roofline": {"bound": "hbm", "kernel": "k_hash_lookup", "achieved": hl_gbs, "peak": peak, "unit": "GB/s",
+                     "frac": hl_gbs / peak, "traffic": None, "bytes_per_launch": hl_bytes,
+                     "ms_per_launch": hl_ms, "peak_kind": peak_kind},
+        "stages_ms_per_step": {n: round(float(v) / args.steps, 4) for n, v in zip(STAGES, stage_ms)},
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "step_ms": {"min": min(step_ms), "median": statistics.median(step_ms), "max": max(step_ms)},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_e2e(args, cache, steps, dsteps, flush, R):
+    """Same steps through ps_step_host: pinned host inputs copied in, outputs
+    copied back, inside the timed region."""
+    import numpy as np
+    import torch
+
+    from paper_2608_01657_gb300 import binding as B
+    cache.reset()
+    for k in range(args.prefill + args.warmup):
+        now, g, o, t = dsteps[k]
+        cache.step(now, g, o, t)
+    torch.cuda.synchronize()
+
+    def pin(a):
+        t = torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+        return t.numpy()
+
+    timed = steps[args.prefill + args.warmup:]
+    host = [(st.now, pin(st.groups), pin(st.offsets), pin(st.tokens)) for st in timed]
+    out = B.host_outputs(R, cache.max_blocks, cache.G, pinned=True)
+    h2d = d2h = 0
+    t_sum = 0.0
+    for (now, g, o, t) in host:
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        r = cache.step_host(now, g, o, t, out=out)
+        t_sum += time.perf_counter() - t0
+        if r["rc"] != 0:
+            raise RuntimeError(f"ps_step_host rc={r['rc']}")
+        cnt = out["counts"]
+        h2d += g.nbytes + o.nbytes + t.nbytes
+        d2h += 16 + 4 * (2 * len(g) + len(g) + 1) + 16 * cache.G + 4 * int(cnt[0] + cnt[1] + cnt[2])
+    n = len(host)
+    return {"value": sum(len(h[1]) for h in host) / t_sum, "unit": "requests/s",
+            "h2d_bytes_per_step": h2d // n, "d2h_bytes_per_step": d2h // n,
+            "ms_per_step": 1e3 * t_sum / n}
+
+
+def main():
+    args = parse_args()
+    ws, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, ws, rank)
+    else:
+        run_own(args, ws, rank, local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

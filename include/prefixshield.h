@@ -201,6 +201,21 @@ int64_t ps_export_history(ps_handle_t* h, void* stream, int32_t* h_group, uint64
 int64_t ps_export_ghost(ps_handle_t* h, void* stream, int32_t* h_group, uint64_t* h_key, uint64_t* h_seq,
                         int64_t cap);
 
+/* Profiling hook.  When enabled, ps_step() records a CUDA event on its
+ * stream before each of its PS_NUM_STAGES stages and after the last one:
+ *   0 validate, 1 hash + lookup, 2 claims + orphans, 3 grant + in-step hits,
+ *   4 metering, 5 touch + gate, 6 victim selection, 7 free-take + eviction,
+ *   8 id lists, 9 insertion, 10 commit.
+ * Creating the events is the only work; no device memory is allocated. */
+#define PS_NUM_STAGES 11
+int32_t ps_set_stage_timing(ps_handle_t* h, int32_t enable);
+
+/* Per-stage durations in milliseconds of the last timed step (synchronizes on
+ * its last event).  Writes min(max_stages, PS_NUM_STAGES) values and, if
+ * h_launches is not NULL, the number of kernels that step launched.  Returns
+ * the number of stages written, or an error. */
+int32_t ps_get_stage_times(ps_handle_t* h, float* h_ms, int32_t max_stages, int32_t* h_launches);
+
 #ifdef __cplusplus
 }
 #endif

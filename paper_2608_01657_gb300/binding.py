@@ -31,7 +31,10 @@ PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE = 1, 2
 
 EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_stats", "ps_clear_status",
             "ps_reset", "ps_destroy", "ps_status_string", "ps_export_state", "ps_export_history",
-            "ps_export_ghost")
+            "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times")
+PS_NUM_STAGES = 11
+STAGE_NAMES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
+               "freetake_evict", "id_lists", "insert", "commit")
 
 
 class PsParams(C.Structure):
@@ -102,6 +105,10 @@ def load():
     L.ps_export_history.argtypes = [vp, vp, vp, vp, vp, vp, i64]
     L.ps_export_ghost.restype = i64
     L.ps_export_ghost.argtypes = [vp, vp, vp, vp, vp, i64]
+    L.ps_set_stage_timing.restype = i32
+    L.ps_set_stage_timing.argtypes = [vp, i32]
+    L.ps_get_stage_times.restype = i32
+    L.ps_get_stage_times.argtypes = [vp, vp, i32, vp]
     _lib = L
     return L
 
@@ -253,6 +260,20 @@ class Cache:
         if rc not in (PS_OK, PS_ERR_CAPACITY):
             raise RuntimeError(f"ps_stats failed ({rc})")
         return s
+
+    def set_stage_timing(self, enable: bool = True):
+        rc = load().ps_set_stage_timing(self._h, int(enable))
+        if rc != PS_OK:
+            raise RuntimeError(f"ps_set_stage_timing failed ({rc})")
+
+    def stage_times(self):
+        """(per-stage ms of the last timed step, kernel launches of that step)."""
+        ms = np.zeros(PS_NUM_STAGES, np.float32)
+        nl = np.zeros(1, np.int32)
+        n = load().ps_get_stage_times(self._h, _ptr(ms), PS_NUM_STAGES, _ptr(nl))
+        if n < 0:
+            raise RuntimeError(f"ps_get_stage_times failed ({n})")
+        return ms[:n].copy(), int(nl[0])
 
     def clear_status(self, stream=None):
         return load().ps_clear_status(self._h, _stream_ptr(stream))

@@ -24,6 +24,7 @@ struct ps_handle {
   int32_t* st_contract;
   uint64_t* st_prefix;
   ps_step_out_t st_out;
+  StepTrace trace;
 };
 
 namespace {
@@ -281,7 +282,7 @@ int32_t ps_step(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t num_req
   s.in_prefix = d_prefix_ids;
   s.tokens_aligned16 = (reinterpret_cast<uintptr_t>(d_tokens) & 15) == 0;
   s.out = *out;
-  return launch_step(s, as_stream(stream));
+  return launch_step(s, as_stream(stream), &h->trace);
 }
 
 int32_t ps_step_host(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t num_requests, const int32_t* h_group_ids,
@@ -360,7 +361,36 @@ int32_t ps_reset(ps_handle_t* h, void* stream) {
   return PS_OK;
 }
 
-void ps_destroy(ps_handle_t* h) { delete h; }
+void ps_destroy(ps_handle_t* h) {
+  if (!h) return;
+  if (h->trace.timing)
+    for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
+  delete h;
+}
+
+int32_t ps_set_stage_timing(ps_handle_t* h, int32_t enable) {
+  if (!h) return PS_ERR_INVALID_ARG;
+  if (enable && !h->trace.timing) {
+    for (cudaEvent_t& e : h->trace.ev)
+      if (cudaEventCreate(&e) != cudaSuccess) return PS_ERR_CUDA;
+    h->trace.timing = true;
+  } else if (!enable && h->trace.timing) {
+    for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
+    h->trace.timing = false;
+  }
+  return PS_OK;
+}
+
+int32_t ps_get_stage_times(ps_handle_t* h, float* h_ms, int32_t max_stages, int32_t* h_launches) {
+  if (!h || (!h_ms && max_stages > 0)) return PS_ERR_INVALID_ARG;
+  if (h_launches) *h_launches = h->trace.launches;
+  if (!h->trace.timing) return 0;
+  if (cudaEventSynchronize(h->trace.ev[PS_NUM_STAGES]) != cudaSuccess) return PS_ERR_CUDA;
+  const int n = max_stages < PS_NUM_STAGES ? max_stages : PS_NUM_STAGES;
+  for (int k = 0; k < n; ++k)
+    if (cudaEventElapsedTime(h_ms + k, h->trace.ev[k], h->trace.ev[k + 1]) != cudaSuccess) return PS_ERR_CUDA;
+  return n;
+}
 
 const char* ps_status_string(int32_t status) {
   switch (status) {

@@ -198,7 +198,13 @@ __device__ __forceinline__ uint32_t hist_home(uint64_t p, uint32_t g, uint32_t l
 }
 
 // ---- host launchers (ps_kernels.cu) ----------------------------------------
+// Optional stage events (profiling hook) and the launch count of a step.
+struct StepTrace {
+  cudaEvent_t ev[PS_NUM_STAGES + 1];
+  bool timing = false;
+  int launches = 0;
+};
 void launch_init(const DevState& s, cudaStream_t st);
-int32_t launch_step(const DevState& s, cudaStream_t st);
+int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr);
 
 }  // namespace ps

@@ -1195,55 +1195,73 @@ static void launch_hash(const DevState& s, cudaStream_t st) {
   k_hash_lookup<PPB><<<(s.R + kWarpsPerCta - 1) / kWarpsPerCta, kWarpsPerCta * 32, smem, st>>>(s);
 }
 
-int32_t launch_step(const DevState& s, cudaStream_t st) {
+int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   const int R = s.R;
   const int wgrid = R > 0 ? (R + kWarpsPerCta - 1) / kWarpsPerCta : 1;
   const int wthreads = kWarpsPerCta * 32;
   const int ngrid = grid_for(s.N, 256, 152 * 8);
-  k_validate<<<1, 1024, 0, st>>>(s);
+  int launches = 0;
+  auto mark = [&](int stage) {
+    if (tr && tr->timing) cudaEventRecord(tr->ev[stage], st);
+  };
+#define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
+  mark(0);
+  PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s));
+  mark(1);
   if (R > 0) {
     switch (s.bs / 2) {
-      case 1: launch_hash<1>(s, st); break;
-      case 2: launch_hash<2>(s, st); break;
-      case 4: launch_hash<4>(s, st); break;
-      case 8: launch_hash<8>(s, st); break;
-      case 16: launch_hash<16>(s, st); break;
-      case 32: launch_hash<32>(s, st); break;
+      case 1: PS_LAUNCH(launch_hash<1>(s, st)); break;
+      case 2: PS_LAUNCH(launch_hash<2>(s, st)); break;
+      case 4: PS_LAUNCH(launch_hash<4>(s, st)); break;
+      case 8: PS_LAUNCH(launch_hash<8>(s, st)); break;
+      case 16: PS_LAUNCH(launch_hash<16>(s, st)); break;
+      case 32: PS_LAUNCH(launch_hash<32>(s, st)); break;
       default: return PS_ERR_INVALID_ARG;
     }
   }
-  k_claims<<<wgrid, wthreads, 0, st>>>(s);
-  k_grant<<<1, 1024, 0, st>>>(s);
-  k_instep<<<wgrid, wthreads, 0, st>>>(s);
-  k_meter<<<s.G, 1024, 0, st>>>(s);
-  k_touch<<<wgrid, wthreads, 0, st>>>(s);
-  k_touch2<<<wgrid, wthreads, 0, st>>>(s);
-  // reclamation
-  k_cand<<<ngrid, 256, 0, st>>>(s);
+  mark(2);
+  PS_LAUNCH(k_claims<<<wgrid, wthreads, 0, st>>>(s));
+  mark(3);
+  PS_LAUNCH(k_grant<<<1, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_instep<<<wgrid, wthreads, 0, st>>>(s));
+  mark(4);
+  PS_LAUNCH(k_meter<<<s.G, 1024, 0, st>>>(s));
+  mark(5);
+  PS_LAUNCH(k_touch<<<wgrid, wthreads, 0, st>>>(s));
+  PS_LAUNCH(k_touch2<<<wgrid, wthreads, 0, st>>>(s));
+  mark(6);
+  PS_LAUNCH(k_cand<<<ngrid, 256, 0, st>>>(s));
   if (s.policy == PS_PREFIXSHIELD) {
-    k_waterfill<<<1, 1024, 0, st>>>(s);
-    for (int pass = 0; pass < 8; ++pass) k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 0, 0);
-    k_tie<<<1, 1024, 0, st>>>(s);
-    k_mark<<<ngrid, 256, 0, st>>>(s, 0, 0);
-    k_sel_single<<<1, 32, 0, st>>>(s, 1);
-    for (int pass = 0; pass < 8; ++pass) k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 1, 1);
-    k_mark<<<ngrid, 256, 0, st>>>(s, 1, 1);
+    PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));
+    for (int pass = 0; pass < 8; ++pass) PS_LAUNCH(k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 0, 0));
+    PS_LAUNCH(k_tie<<<1, 1024, 0, st>>>(s));
+    PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 0, 0));
+    PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 1));
+    for (int pass = 0; pass < 8; ++pass) PS_LAUNCH(k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 1, 1));
+    PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 1));
   } else if (s.policy == PS_LRU) {
-    k_sel_single<<<1, 32, 0, st>>>(s, 0);
-    for (int pass = 0; pass < 8; ++pass) k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 1, 0);
-    k_mark<<<ngrid, 256, 0, st>>>(s, 1, 0);
+    PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
+    for (int pass = 0; pass < 8; ++pass) PS_LAUNCH(k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 1, 0));
+    PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 0));
   } else {
     return PS_ERR_INVALID_ARG;  // S3-FIFO: not yet
   }
-  k_freetake<<<1, 1024, 0, st>>>(s);
-  k_evict<<<grid_for(s.nwords, 256, 152 * 4), 256, 0, st>>>(s);
+  mark(7);
+  PS_LAUNCH(k_freetake<<<1, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_evict<<<grid_for(s.nwords, 256, 152 * 4), 256, 0, st>>>(s));
+  mark(8);
   const int nchunks = (int)((s.nwords + kBmChunk - 1) / kBmChunk);
-  k_bm_count<<<nchunks, 1024, 0, st>>>(s);
-  k_bm_write<<<nchunks, 1024, 0, st>>>(s);
-  k_insert<<<wgrid, wthreads, 0, st>>>(s);
-  k_hist_commit<<<grid_for(R, 256, 1 << 20), 256, 0, st>>>(s);
-  k_claim_clear<<<wgrid, wthreads, 0, st>>>(s);
-  k_finalize<<<1, 32, 0, st>>>(s);
+  PS_LAUNCH(k_bm_count<<<nchunks, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_bm_write<<<nchunks, 1024, 0, st>>>(s));
+  mark(9);
+  PS_LAUNCH(k_insert<<<wgrid, wthreads, 0, st>>>(s));
+  mark(10);
+  PS_LAUNCH(k_hist_commit<<<grid_for(R, 256, 1 << 20), 256, 0, st>>>(s));
+  PS_LAUNCH(k_claim_clear<<<wgrid, wthreads, 0, st>>>(s));
+  PS_LAUNCH(k_finalize<<<1, 32, 0, st>>>(s));
+  mark(11);
+#undef PS_LAUNCH
+  if (tr) tr->launches = launches;
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 

@@ -159,3 +159,28 @@ def test_step_host_matches_step():
                "invalidated_ids": out["invalidated_ids"][:cnt[2]], "debt_raw": out["debt_raw"],
                "debt_norm": out["debt_norm"]}
         compare_outputs(got, orc.step(st.now, st.groups, st.offsets, st.tokens), f"step {st.index}")
+
+
+_SCALE = {}
+
+
+def _scale_steps(n):
+    if n not in _SCALE:
+        wl = W.make_workload(4, seed=1)
+        _SCALE[n] = (wl.spec, list(wl.steps(n)))
+    return _SCALE[n]
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+def test_parity_scale_full_size(policy):
+    """The benchmarked configuration itself (64 groups, 1,048,576 blocks,
+    4096 requests per step), from the empty pool through the fill and into
+    steady-state reclamation: every output of every step and the complete
+    final state equal the oracle's."""
+    spec, steps = _scale_steps(9)
+    maxT = max(s.num_tokens for s in steps)
+    gpu, orc = _pair(spec.capacity_blocks, spec.block_size, spec.num_groups, policy,
+                     dict(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20),
+                     max_requests=spec.requests_per_step, max_tokens=maxT)
+    _run(gpu, orc, steps, state_every=4, label=f"scale/{policy}")
+    assert orc.stats()[:, O.STAT_NAMES.index("evicted_blocks")].sum() > 0  # reclamation was exercised
