@@ -230,7 +230,7 @@ class Cache:
         R = int(len(groups))
         if out is None:
             out = host_outputs(R, self.max_blocks, self.G)
-        o = PsStepOut(**{k: _ptr(v) for k, v in out.items()})
+        o = PsStepOut(**{k: _ptr(out[k]) for k, _ in PsStepOut._fields_})
         rc = load().ps_step_host(self._h, _stream_ptr(stream), int(now), R, _ptr(groups), _ptr(offsets),
                                  _ptr(tokens), _ptr(contracts), _ptr(prefixes), C.byref(o))
         out["rc"] = rc
