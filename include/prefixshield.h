@@ -131,8 +131,8 @@ size_t ps_workspace_bytes(int64_t capacity_blocks, int32_t block_size, int32_t n
 
 /* Create a pool of capacity_blocks blocks (all free, every balance full:
  * B = beta at t = 0, Sec. III-B) inside the caller's workspace, and
- * initialize it on 'stream'.  block_size: tokens per KV block, even, 2..256
- * (16 in the paper).  max_requests / max_tokens bound every later step.
+ * initialize it on 'stream'.  block_size: tokens per KV block, one of 2, 4, 8,
+ * 16, 32, 64 (16 in the paper).  max_requests / max_tokens bound every later step.
  * The workspace must stay allocated and untouched until ps_destroy().
  * Returns PS_ERR_INVALID_ARG for bad arguments or a workspace that is too
  * small or misaligned. */
@@ -200,6 +200,18 @@ int64_t ps_export_history(ps_handle_t* h, void* stream, int32_t* h_group, uint64
  * same convention as ps_export_history. */
 int64_t ps_export_ghost(ps_handle_t* h, void* stream, int32_t* h_group, uint64_t* h_key, uint64_t* h_seq,
                         int64_t cap);
+
+/* Read-only probe of the cache: for each request, the number of leading full
+ * blocks of its prompt resident in the pool now (n_cached of Alg. 1 as
+ * ps_step() would find it before any request of the batch materializes a
+ * block).  Nothing in the pool changes.  Arguments as for ps_step();
+ * d_cached_blocks [R] receives the counts and d_status (device int32) the
+ * outcome: PS_OK, or PS_ERR_INVALID_ARG for bad offsets or group ids or more
+ * than max_tokens tokens.  Uses the handle's workspace as scratch: do not run
+ * it concurrently with a ps_step() of the same handle.  Enqueued on 'stream'. */
+int32_t ps_cached_prefix(ps_handle_t* h, void* stream, int32_t num_requests, const int32_t* d_group_ids,
+                         const int64_t* d_token_offsets, const int32_t* d_tokens, int32_t* d_cached_blocks,
+                         int32_t* d_status);
 
 /* Profiling hook.  When enabled, ps_step() records a CUDA event on its
  * stream before each of its PS_NUM_STAGES stages and after the last one:

@@ -82,6 +82,7 @@ def lib():
         L.orc_step.restype = i32
         L.orc_step.argtypes = [vp, i64, i32, vp, vp, vp, vp, vp, C.POINTER(OrcOut)]
         L.orc_clear_status.argtypes = [vp]
+        L.orc_cached_prefix.argtypes = [vp, i32, vp, vp, vp, vp]
         L.orc_stats.argtypes = [vp, vp]
         L.orc_export_blocks.argtypes = [vp] + [vp] * 11
         L.orc_export_ledger.argtypes = [vp, vp, vp, vp, vp, vp]
@@ -197,6 +198,14 @@ class OracleCache:
         res["evicted_ids"] = res["evicted_ids"][: out.n_evicted].copy()
         res["invalidated_ids"] = res["invalidated_ids"][: out.n_invalidated].copy()
         return res
+
+    def cached_prefix(self, groups, offsets, tokens) -> np.ndarray:
+        g = np.ascontiguousarray(groups, dtype=np.int32)
+        o = np.ascontiguousarray(offsets, dtype=np.int64)
+        t = np.ascontiguousarray(tokens, dtype=np.int32)
+        out = np.zeros(max(1, len(g)), np.int32)
+        lib().orc_cached_prefix(self._h, len(g), _ptr(g), _ptr(o), _ptr(t), _ptr(out))
+        return out[: len(g)]
 
     def clear_status(self):
         lib().orc_clear_status(self._h)

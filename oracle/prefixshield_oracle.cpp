@@ -145,21 +145,35 @@ uint64_t nh_digest(const uint32_t* K, int off, const int32_t* M, int bs) {
   return sum;
 }
 
+// Arithmetic modulo the Mersenne prime p = 2^61 - 1.
+constexpr uint64_t P61 = (1ull << 61) - 1;
+uint64_t mod61(uint64_t x) { return x % P61; }
+uint64_t mulmod61(uint64_t a, uint64_t b) { return (uint64_t)(((unsigned __int128)a * b) % P61); }
+
 // Chained content key of every full block of one token sequence (Sec. III,
 // "native content-hash lookup key"; only full blocks are cached, Sec. III-B).
-// h_{-1} = mix(seed ^ (g+1)*phi); h_m = mix(mix(h_{m-1} ^ NH0) ^ NH2 ^ m);
-// 0 and all-ones are reserved and map to 1.
+// Key schedule from SplitMix64(seed): bs+2 NH words, then the chain
+// multiplier Kc and the digest multiplier Kd (both in [1, p)).
+//   D_m = (NH0_m + Kd * NH2_m) mod p           (the block's 128-bit NH digest)
+//   C_{-1} = mix(seed ^ (g+1)*phi) mod p       (namespace of group g)
+//   C_m = (Kc * C_{m-1} + D_m) mod p           (chain over the prefix)
+//   key_m = mix(C_m ^ (m+1)*c), with 0 and all-ones mapped to 1.
 std::vector<uint64_t> chain_keys(uint64_t seed, int32_t group, int bs, const int32_t* tok, int64_t len) {
   std::vector<uint32_t> K(bs + 2);
   uint64_t st = seed;
   for (int j = 0; j < bs + 2; ++j) K[j] = (uint32_t)splitmix64_next(&st);
+  uint64_t Kc = mod61(splitmix64_next(&st));
+  uint64_t Kd = mod61(splitmix64_next(&st));
+  if (Kc == 0) Kc = 1;
+  if (Kd == 0) Kd = 1;
   int64_t n = len / bs;
   std::vector<uint64_t> keys(n);
-  uint64_t h = mix64(seed ^ ((uint64_t)(group + 1) * 0x9E3779B97F4A7C15ull));
+  uint64_t C = mod61(mix64(seed ^ ((uint64_t)(group + 1) * 0x9E3779B97F4A7C15ull)));
   for (int64_t m = 0; m < n; ++m) {
     const int32_t* blk = tok + m * bs;
-    uint64_t x = mix64(h ^ nh_digest(K.data(), 0, blk, bs)) ^ nh_digest(K.data(), 2, blk, bs) ^ (uint64_t)m;
-    h = mix64(x);
+    uint64_t D = (mod61(nh_digest(K.data(), 0, blk, bs)) + mulmod61(Kd, mod61(nh_digest(K.data(), 2, blk, bs)))) % P61;
+    C = (mulmod61(Kc, C) + D) % P61;
+    uint64_t h = mix64(C ^ ((uint64_t)(m + 1) * 0xD1B54A32D192ED03ull));
     if (h == 0 || h == ~0ull) h = 1;
     keys[m] = h;
   }
@@ -699,6 +713,19 @@ int32_t orc_step(void* h, int64_t now, int32_t R, const int32_t* group, const in
 }
 
 void orc_clear_status(void* h) { static_cast<Oracle*>(h)->sticky = OK; }
+
+// Read-only: leading full blocks of each prompt resident now (n_cached of
+// Alg. 1 against the current pool, no state change).
+void orc_cached_prefix(void* h, int32_t R, const int32_t* group, const int64_t* offsets, const int32_t* tokens,
+                       int32_t* out) {
+  Oracle* o = static_cast<Oracle*>(h);
+  for (int32_t i = 0; i < R; ++i) {
+    std::vector<uint64_t> k = chain_keys(o->P.hash_seed, group[i], o->bs, tokens + offsets[i], offsets[i + 1] - offsets[i]);
+    int32_t n = 0;
+    while (n < (int32_t)k.size() && o->table.count({group[i], k[n]})) ++n;
+    out[i] = n;
+  }
+}
 
 void orc_stats(void* h, int64_t* out) {
   Oracle* o = static_cast<Oracle*>(h);

@@ -31,7 +31,7 @@ PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE = 1, 2
 
 EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_stats", "ps_clear_status",
             "ps_reset", "ps_destroy", "ps_status_string", "ps_export_state", "ps_export_history",
-            "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times")
+            "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times", "ps_cached_prefix")
 PS_NUM_STAGES = 11
 STAGE_NAMES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
                "freetake_evict", "id_lists", "insert", "commit")
@@ -105,6 +105,8 @@ def load():
     L.ps_export_history.argtypes = [vp, vp, vp, vp, vp, vp, i64]
     L.ps_export_ghost.restype = i64
     L.ps_export_ghost.argtypes = [vp, vp, vp, vp, vp, i64]
+    L.ps_cached_prefix.restype = i32
+    L.ps_cached_prefix.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
     L.ps_set_stage_timing.restype = i32
     L.ps_set_stage_timing.argtypes = [vp, i32]
     L.ps_get_stage_times.restype = i32
@@ -223,6 +225,21 @@ class Cache:
         R = int(groups.shape[0])
         return load().ps_step(self._h, _stream_ptr(stream), int(now), R, _ptr(groups), _ptr(offsets), _ptr(tokens),
                               _ptr(contracts), _ptr(prefixes), C.byref(self._out))
+
+    def cached_prefix(self, groups, offsets, tokens, out=None, status=None, stream=None):
+        """Read-only probe: leading resident full blocks of each prompt (device
+        tensors in, device int32 counts out).  Returns (counts, status tensor)."""
+        import torch
+        R = int(groups.shape[0])
+        if out is None:
+            out = torch.empty(max(1, R), dtype=torch.int32, device=groups.device)
+        if status is None:
+            status = torch.zeros(1, dtype=torch.int32, device=groups.device)
+        rc = load().ps_cached_prefix(self._h, _stream_ptr(stream), R, _ptr(groups), _ptr(offsets), _ptr(tokens),
+                                     _ptr(out), _ptr(status))
+        if rc != PS_OK:
+            raise RuntimeError(f"ps_cached_prefix failed ({rc})")
+        return out, status
 
     def step_host(self, now: int, groups, offsets, tokens, contracts=None, prefixes=None, stream=None,
                   out: Optional[dict] = None) -> dict:

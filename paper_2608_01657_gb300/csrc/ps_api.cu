@@ -25,6 +25,7 @@ struct ps_handle {
   uint64_t* st_prefix;
   ps_step_out_t st_out;
   StepTrace trace;
+  std::vector<int32_t> contract_of_group;
 };
 
 namespace {
@@ -36,10 +37,45 @@ inline uint32_t log2_pow2_at_least(uint64_t v) {
   return l;
 }
 
-// SplitMix64 stream (Steele, Lea, Flood 2014) for the NH key schedule.
+// SplitMix64 stream (Steele, Lea, Flood 2014) for the key schedule.
 uint64_t splitmix_next(uint64_t* st) {
   *st += 0x9E3779B97F4A7C15ull;
   return mix64(*st);
+}
+uint64_t host_mul61(uint64_t a, uint64_t b) { return (uint64_t)(((unsigned __int128)a * b) % kP61); }
+
+// Key schedule: bs + 2 NH words, then the chain and digest multipliers.
+struct KeySchedule {
+  std::vector<uint32_t> words;
+  uint64_t kc, kd;
+  std::vector<uint64_t> kc_pow;
+};
+KeySchedule key_schedule(uint64_t seed, int32_t bs) {
+  KeySchedule k;
+  uint64_t st = seed;
+  k.words.resize((size_t)bs + 2);
+  for (auto& w : k.words) w = (uint32_t)splitmix_next(&st);
+  k.kc = splitmix_next(&st) % kP61;
+  k.kd = splitmix_next(&st) % kP61;
+  if (k.kc == 0) k.kc = 1;
+  if (k.kd == 0) k.kd = 1;
+  k.kc_pow.resize(kSegBlocks + 1);
+  k.kc_pow[0] = 1;
+  for (int j = 1; j <= kSegBlocks; ++j) k.kc_pow[j] = host_mul61(k.kc_pow[j - 1], k.kc);
+  return k;
+}
+
+int32_t upload_constants(ps_handle* h, cudaStream_t st) {
+  const KeySchedule ks = key_schedule(h->base.hash_seed, h->base.bs);
+  if (cudaMemcpyAsync(h->base.key_words, ks.words.data(), ks.words.size() * 4, cudaMemcpyHostToDevice, st) !=
+          cudaSuccess ||
+      cudaMemcpyAsync(h->base.kc_pow, ks.kc_pow.data(), ks.kc_pow.size() * 8, cudaMemcpyHostToDevice, st) !=
+          cudaSuccess ||
+      cudaMemcpyAsync(h->base.contract_of_group, h->contract_of_group.data(), h->contract_of_group.size() * 4,
+                      cudaMemcpyHostToDevice, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  return PS_OK;
 }
 
 int32_t check_params(int64_t N, int32_t bs, int32_t G, int32_t policy, const ps_params_t* P) {
@@ -81,7 +117,7 @@ struct Carver {
 };
 
 struct Dims {
-  int64_t N, max_tokens, max_blocks, nwords, hist_cap;
+  int64_t N, max_tokens, max_blocks, nwords, hist_cap, max_segments;
   int32_t bs, G, C, max_requests;
   uint32_t tb_log2, cl_log2, hist_log2;
 };
@@ -91,6 +127,7 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   d.N = N; d.bs = bs; d.G = G; d.C = P->num_contracts; d.max_requests = max_requests;
   d.max_tokens = max_tokens;
   d.max_blocks = max_tokens / bs;
+  d.max_segments = d.max_blocks / kSegBlocks + max_requests + 1;
   d.nwords = (N + 31) / 32;
   // native table: 8-way buckets at load <= 1/2
   d.tb_log2 = log2_pow2_at_least((uint64_t)((N + 3) / 4 > 1 ? (N + 3) / 4 : 1));
@@ -131,6 +168,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.ledger = cv.take<int64_t>(G * d.C);
   t.contract_of_group = cv.take<int32_t>(G);
   t.key_words = cv.take<uint32_t>((size_t)d.bs + 2);
+  t.kc_pow = cv.take<uint64_t>((size_t)kSegBlocks + 1);
   t.stats = cv.take<int64_t>(G * PS_NUM_STATS);
   t.hist = cv.take<HistEntry>((size_t)1 << d.hist_log2);
   t.rq_n = cv.take<int32_t>(R);
@@ -140,12 +178,18 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.rq_cbase = cv.take<int32_t>(R);
   t.rq_a = cv.take<int32_t>(R);
   t.rq_e = cv.take<int32_t>(R);
+  t.rq_sbase = cv.take<int32_t>(R);
+  t.rq_fu = cv.take<uint32_t>(R);
   t.rq_cid = cv.take<int32_t>(R);
   t.rq_hs = cv.take<uint32_t>(R);
   t.rq_p = cv.take<uint64_t>(R);
   t.rq_flags = cv.take<uint8_t>(R);
   t.rq_knew = cv.take<uint8_t>(R);
   t.pos_key = cv.take<uint64_t>(B);
+  t.pos_req = cv.take<uint32_t>(B);
+  t.seg_req = cv.take<uint32_t>((size_t)d.max_segments);
+  t.seg_cin = cv.take<uint64_t>((size_t)d.max_segments);
+  t.seg_tot = cv.take<uint64_t>((size_t)d.max_segments);
   t.pos_blk = cv.take<uint32_t>(B);
   t.pos_claim = cv.take<uint32_t>(B);
   t.pos_elig = cv.take<uint8_t>(B);
@@ -243,19 +287,15 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   s.history_capacity = params->history_capacity;
   s.tb_nbuckets_log2 = d.tb_log2; s.cl_nbuckets_log2 = d.cl_log2; s.hist_cap_log2 = d.hist_log2;
   s.nwords = d.nwords;
+  s.max_segments = d.max_segments;
+  const KeySchedule ks = key_schedule(params->hash_seed, block_size);
+  s.chain_mul = ks.kc;
+  s.digest_mul = ks.kd;
   h->base = s;
+  h->contract_of_group.assign(params->contract_of_group, params->contract_of_group + num_groups);
   cudaStream_t st = as_stream(stream);
   int32_t rc = init_state(h, st);
-  if (rc == PS_OK) {
-    std::vector<uint32_t> kw((size_t)block_size + 2);
-    uint64_t seed = params->hash_seed;
-    for (auto& w : kw) w = (uint32_t)splitmix_next(&seed);
-    std::vector<int32_t> cog(params->contract_of_group, params->contract_of_group + num_groups);
-    if (cudaMemcpyAsync(s.key_words, kw.data(), kw.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-        cudaMemcpyAsync(s.contract_of_group, cog.data(), cog.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-        cudaStreamSynchronize(st) != cudaSuccess)
-      rc = PS_ERR_CUDA;
-  }
+  if (rc == PS_OK) rc = upload_constants(h, st);
   if (rc != PS_OK) {
     delete h;
     return rc;
@@ -345,20 +385,25 @@ int32_t ps_clear_status(ps_handle_t* h, void* stream) {
 int32_t ps_reset(ps_handle_t* h, void* stream) {
   if (!h) return PS_ERR_INVALID_ARG;
   cudaStream_t st = as_stream(stream);
-  // key words and contract map survive in host copies: rebuild them
-  std::vector<uint32_t> kw((size_t)h->base.bs + 2);
-  std::vector<int32_t> cog((size_t)h->base.G);
-  if (cudaMemcpyAsync(kw.data(), h->base.key_words, kw.size() * 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
-      cudaMemcpyAsync(cog.data(), h->base.contract_of_group, cog.size() * 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
-      cudaStreamSynchronize(st) != cudaSuccess)
-    return PS_ERR_CUDA;
-  int32_t rc = init_state(h, st);
-  if (rc != PS_OK) return rc;
-  if (cudaMemcpyAsync(h->base.key_words, kw.data(), kw.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-      cudaMemcpyAsync(h->base.contract_of_group, cog.data(), cog.size() * 4, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-      cudaStreamSynchronize(st) != cudaSuccess)
-    return PS_ERR_CUDA;
-  return PS_OK;
+  const int32_t rc = init_state(h, st);
+  return rc != PS_OK ? rc : upload_constants(h, st);
+}
+
+int32_t ps_cached_prefix(ps_handle_t* h, void* stream, int32_t num_requests, const int32_t* d_group_ids,
+                         const int64_t* d_token_offsets, const int32_t* d_tokens, int32_t* d_cached_blocks,
+                         int32_t* d_status) {
+  if (!h || num_requests < 0 || num_requests > h->base.max_requests || !d_token_offsets || !d_status)
+    return PS_ERR_INVALID_ARG;
+  if (num_requests > 0 && (!d_group_ids || !d_tokens || !d_cached_blocks)) return PS_ERR_INVALID_ARG;
+  DevState s = h->base;
+  s.R = num_requests;
+  s.in_group = d_group_ids;
+  s.in_offsets = d_token_offsets;
+  s.in_tokens = d_tokens;
+  s.in_contract = nullptr;
+  s.in_prefix = nullptr;
+  s.tokens_aligned16 = (reinterpret_cast<uintptr_t>(d_tokens) & 15) == 0;
+  return launch_probe(s, as_stream(stream), d_cached_blocks, d_status);
 }
 
 void ps_destroy(ps_handle_t* h) {

@@ -25,6 +25,8 @@ constexpr int kTableWays = 8;    // native prefix table: 8 x 16 B entries per 12
 constexpr int kClaimWays = 4;    // per-step claim map: 4 x 32 B entries per bucket
 constexpr int kRadixBits = 8;
 constexpr int kRadixBins = 1 << kRadixBits;
+constexpr int kSegBlocks = 256;  // blocks of one prompt hashed by one warp
+constexpr uint64_t kP61 = (1ull << 61) - 1;  // chain modulus, a Mersenne prime
 
 // Recency stamp (native free-queue order): larger = more recently released.
 __host__ __device__ __forceinline__ uint64_t make_stamp(uint64_t step, uint64_t req, uint64_t pos) {
@@ -72,7 +74,7 @@ struct Ctl {
   // per step
   int32_t status;          // this step's status
   int32_t pad1;
-  int64_t T, nblocks;
+  int64_t T, nblocks, nsegs;
   int64_t pinned, n_inval, total_claims, avail, need, nfree, ftake, mvict;
   int64_t hist_new;
   int64_t n_evicted, n_alloc, n_victims_marked;
@@ -89,6 +91,7 @@ struct __align__(16) SelSeg {
   int64_t rank;      // 1-based rank still to locate inside the prefix class
   int32_t active;    // 1 while this segment selects
   int32_t incl;      // 1: victims are keys <= prefix; 0: keys < prefix
+  uint64_t kmin, kmax;  // smallest / largest candidate key of the segment
 };
 
 struct DevState {
@@ -99,6 +102,8 @@ struct DevState {
   int32_t fp_shift;
   int64_t eps;
   uint64_t hash_seed;
+  uint64_t chain_mul, digest_mul;  // Kc, Kd of the key chain (mod 2^61-1)
+  int64_t max_segments;
   int64_t rho[PS_MAX_CONTRACTS], beta[PS_MAX_CONTRACTS];
   int64_t rho_min;
   int32_t s3_small_pct, s3_freq_cap, s3_move_min;
@@ -129,6 +134,7 @@ struct DevState {
   int64_t* ledger;         // B_{g,c}, fixed point
   int32_t* contract_of_group;
   uint32_t* key_words;     // NH key schedule, bs + 2 words
+  uint64_t* kc_pow;        // Kc^k mod p, k = 0..kSegBlocks
   int64_t* stats;          // [G][PS_NUM_STATS]
   HistEntry* hist;
   // per-step scratch
@@ -139,12 +145,18 @@ struct DevState {
   int32_t* rq_cbase;       // exclusive scan of claims
   int32_t* rq_a;           // granted (admitted) blocks
   int32_t* rq_e;           // in-step hits
+  int32_t* rq_sbase;       // first hashing segment of the request
+  uint32_t* rq_fu;         // first ungranted in-step position
   int32_t* rq_cid;         // contract
   uint32_t* rq_hs;         // history slot
   uint64_t* rq_p;          // prefix id
   uint8_t* rq_flags;       // bit0 proven, bit1 gate open
   uint8_t* rq_knew;        // class of newly admitted blocks
-  uint64_t* pos_key;
+  uint64_t* pos_key;       // chain partial, then the block key
+  uint32_t* pos_req;       // request of the position
+  uint32_t* seg_req;       // request of each hashing segment
+  uint64_t* seg_cin;       // chain value entering the segment
+  uint64_t* seg_tot;       // local chain value at the segment's end
   uint32_t* pos_blk;       // resident block hit by lookup (or kNone)
   uint32_t* pos_claim;     // claim-map slot (or kNone)
   uint8_t* pos_elig;       // touch was promotion-eligible
@@ -206,5 +218,7 @@ struct StepTrace {
 };
 void launch_init(const DevState& s, cudaStream_t st);
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr);
+// Read-only cached-prefix probe; 'out' receives h_i per request, 'status' the outcome.
+int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* status);
 
 }  // namespace ps

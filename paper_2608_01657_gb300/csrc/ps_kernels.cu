@@ -2,8 +2,11 @@
 //
 // One step is a fixed sequence of launches on the caller's stream.  Nothing on
 // the path goes back to the host: every size (tokens, blocks, claims, victims)
-// lives in device memory, and a kernel whose work is empty exits at once.
-// Each kernel's comment names the stage and the passage it implements.
+// lives in device memory, grids are sized from the handle's bounds, and a
+// thread whose item does not exist exits at once.  Apart from the one-CTA
+// scans, every stage runs a thread per block position, per request or per
+// victim, so a long prompt is spread over many warps instead of serializing
+// one.  Each kernel's comment names the stage and the passage it implements.
 #include <climits>
 #include <cstdio>
 
@@ -12,7 +15,8 @@
 namespace ps {
 
 constexpr unsigned kFull = 0xFFFFFFFFu;
-constexpr int kWarpsPerCta = 8;  // warp-per-request kernels
+constexpr int kWarpsPerCta = 8;   // warp-per-segment hashing kernel
+constexpr int kThreads = 256;     // position-parallel kernels
 
 // ---------------------------------------------------------------------------
 // small device helpers
@@ -70,14 +74,24 @@ __device__ T block_sum(T v) {
 __device__ __forceinline__ void atomic_add_i64(int64_t* p, int64_t v) {
   atomicAdd(reinterpret_cast<unsigned long long*>(p), static_cast<unsigned long long>(v));
 }
-__device__ __forceinline__ int64_t& stat_ref(const DevState& s, int g, int k) {
-  return s.stats[(int64_t)g * PS_NUM_STATS + k];
+__device__ __forceinline__ int64_t* stat_ptr(const DevState& s, int g, int k) {
+  return s.stats + (int64_t)g * PS_NUM_STATS + k;
+}
+// Add v to stat k of group g, combining lanes of the warp with equal g.
+__device__ __forceinline__ void agg_stat(const DevState& s, uint32_t g, int k, int64_t v, bool active) {
+  const bool on = active && v != 0;
+  const unsigned act = __ballot_sync(kFull, on);
+  if (!on) return;
+  const unsigned peers = __match_any_sync(act, g);
+  int64_t sum = 0;
+  for (unsigned m = peers; m; m &= m - 1) sum += __shfl_sync(peers, v, __ffs(m) - 1);
+  if (lane_id() == __ffs(peers) - 1) atomic_add_i64(stat_ptr(s, (int)g, k), sum);
 }
 // Warp-aggregated increment of bins[idx] for the lanes with 'active'.
 __device__ __forceinline__ void agg_inc(uint32_t* bins, uint32_t idx, bool active) {
-  unsigned act = __ballot_sync(kFull, active);
+  const unsigned act = __ballot_sync(kFull, active);
   if (!active) return;
-  unsigned peers = __match_any_sync(act, idx);
+  const unsigned peers = __match_any_sync(act, idx);
   if (lane_id() == __ffs(peers) - 1) atomicAdd(bins + idx, (uint32_t)__popc(peers));
 }
 __device__ __forceinline__ uint64_t ldcg_u64(const uint64_t* p) { return __ldcg(reinterpret_cast<const unsigned long long*>(p)); }
@@ -111,7 +125,7 @@ __device__ __forceinline__ uint32_t tag_req(uint64_t tag, uint64_t step) {
 }
 __device__ __forceinline__ int64_t refill(int64_t b, int64_t beta, int64_t rho, int64_t dt) {
   // Eq. 1, min{beta, b + rho*dt}, without overflow (dt >= ceil(need/rho) saturates).
-  int64_t need = beta - b;
+  const int64_t need = beta - b;
   if (need <= 0 || dt >= (need + rho - 1) / rho) return beta;
   return b + rho * dt;
 }
@@ -119,42 +133,39 @@ __device__ __forceinline__ int64_t muldiv(int64_t a, int64_t b, int64_t c) {
   return (int64_t)(((__int128)a * (__int128)b) / (__int128)c);
 }
 
+// ---- arithmetic modulo p = 2^61 - 1 (Mersenne reduction: 2^61 == 1) ------
+__device__ __forceinline__ uint64_t red61(uint64_t x) {  // any 64-bit x -> [0, p)
+  const uint64_t r = (x & kP61) + (x >> 61);
+  return r >= kP61 ? r - kP61 : r;
+}
+__device__ __forceinline__ uint64_t add61(uint64_t a, uint64_t b) {  // a, b < p
+  const uint64_t r = a + b;
+  return r >= kP61 ? r - kP61 : r;
+}
+__device__ __forceinline__ uint64_t mul61(uint64_t a, uint64_t b) {  // a, b < p
+  const uint64_t lo = a * b, hi = __umul64hi(a, b);
+  uint64_t r = (lo & kP61) + ((lo >> 61) | (hi << 3));
+  r = (r & kP61) + (r >> 61);
+  return r >= kP61 ? r - kP61 : r;
+}
+
 // ---- native prefix table ---------------------------------------------------
-// Lookup of 4 keys per warp, 8 lanes per key: each lane loads one 16-byte
-// entry of the key's 128-byte bucket.  A bucket whose overflow count is zero
-// ends the probe.  Returns (for lane m in [kk, kk+4)) the block of key kk+...
-__device__ uint32_t table_lookup4(const DevState& s, uint64_t key_of_group, uint32_t g, bool act_in) {
-  const int lane = lane_id();
+// Lookup by one thread: the 128-byte home bucket (8 entries), then following
+// buckets while the overflow count says some key probed past.
+__device__ uint32_t table_find(const DevState& s, uint64_t key, uint32_t g) {
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
-  bool act = act_in;
-  uint32_t b = table_home(key_of_group, g, s.tb_nbuckets_log2);
-  uint32_t found = kNone;
+  uint32_t b = table_home(key, g, s.tb_nbuckets_log2);
   for (uint32_t it = 0; it <= mask; ++it) {
-    bool hit = false;
-    uint32_t eblk = kNone;
-    if (act) {
-      const uint4 raw = __ldcg(reinterpret_cast<const uint4*>(s.table + (size_t)b * kTableWays + (lane & 7)));
-      const uint64_t ek = ((uint64_t)raw.y << 32) | raw.x;
-      eblk = raw.z;
-      hit = eblk != kNone && ek == key_of_group && raw.w == g;
+    const uint4* e = reinterpret_cast<const uint4*>(s.table + (size_t)b * kTableWays);
+#pragma unroll
+    for (int w = 0; w < kTableWays; ++w) {
+      const uint4 raw = __ldg(e + w);
+      if (raw.z != kNone && raw.x == (uint32_t)key && raw.y == (uint32_t)(key >> 32) && raw.w == g) return raw.z;
     }
-    const unsigned mh = __ballot_sync(kFull, hit);
-    const unsigned gm = (mh >> (lane & ~7)) & 0xFFu;
-    const int src = gm ? (lane & ~7) + __ffs(gm) - 1 : lane;
-    const uint32_t v = __shfl_sync(kFull, eblk, src);
-    if (act) {
-      if (gm) {
-        found = v;
-        act = false;
-      } else if (ldcg_u32(s.table_ovf + b) == 0) {
-        act = false;
-      } else {
-        b = (b + 1) & mask;
-      }
-    }
-    if (!__any_sync(kFull, act)) break;
+    if (__ldg(s.table_ovf + b) == 0) return kNone;
+    b = (b + 1) & mask;
   }
-  return found;
+  return kNone;
 }
 
 __device__ uint32_t table_insert(const DevState& s, uint64_t key, uint32_t g, uint32_t blk) {
@@ -215,21 +226,26 @@ __device__ void drop_block(const DevState& s, uint32_t b, int stat_kind) {
   const uint8_t fl = s.blk_flags[b];
   s.blk_flags[b] = 0;
   atomicAnd(s.res_bits + (b >> 5), ~(1u << (b & 31)));
-  atomic_add_i64(&s.ctl->n_resident, -1);
-  atomic_add_i64(&stat_ref(s, g, stat_kind), 1);
-  atomic_add_i64(&stat_ref(s, g, PS_STAT_RESIDENT_BLOCKS), -1);
+  atomic_add_i64(stat_ptr(s, g, stat_kind), 1);
+  atomic_add_i64(stat_ptr(s, g, PS_STAT_RESIDENT_BLOCKS), -1);
   if (s.policy == PS_S3FIFO) atomic_add_i64((fl & 2) ? &s.ctl->s3_nM : &s.ctl->s3_nS, -1);
+}
+
+// Position -> (request, position within the request).
+struct PosRef {
+  uint32_t i;
+  int m;
+};
+__device__ __forceinline__ bool pos_ref(const DevState& s, int64_t pos, PosRef* r) {
+  if (pos >= s.ctl->nblocks) return false;
+  r->i = s.pos_req[pos];
+  r->m = (int)(pos - s.rq_pbase[r->i]);
+  return true;
 }
 
 // ===========================================================================
 // Init: an empty pool, every balance at beta (Sec. III-B, B = beta at t = 0).
 __global__ void k_init_blocks(DevState s) {
-  for (int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; b < s.N; b += (int64_t)gridDim.x * blockDim.x) {
-    s.blk_flags[b] = 0;
-    s.blk_pin[b] = 0;
-    s.blk_inval[b] = 0;
-    s.blk_promo[b] = 0;
-  }
   const int64_t nclaims = (int64_t)kClaimWays << s.cl_nbuckets_log2;
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < nclaims; c += (int64_t)gridDim.x * blockDim.x) {
     ClaimEntry e{};
@@ -247,8 +263,9 @@ __global__ void k_init_ctl(DevState s) {
 }
 
 // ===========================================================================
-// Stage 0: validation of the step's inputs; n_i and block positions.
-__global__ void __launch_bounds__(1024) k_validate(DevState s) {
+// Stage 0: validation of the step's inputs; n_i, block positions, hashing
+// segments.  One CTA.  'probe' skips the clock and step checks.
+__global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
   Ctl* c = s.ctl;
   __shared__ int s_bad;
   if (threadIdx.x == 0) s_bad = 0;
@@ -265,76 +282,94 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s) {
   __syncthreads();
   int32_t st = PS_OK;
   const int64_t T = R > 0 ? s.in_offsets[R] : 0;
-  if (c->sticky != PS_OK) st = c->sticky;
-  else if (s.now < c->t_prev) st = PS_ERR_CLOCK;
-  else if (c->step > kMaxStep) st = PS_ERR_CAPACITY;
+  if (!probe && c->sticky != PS_OK) st = c->sticky;
+  else if (!probe && s.now < c->t_prev) st = PS_ERR_CLOCK;
+  else if (!probe && c->step > kMaxStep) st = PS_ERR_CAPACITY;
   else if (s_bad || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens) st = PS_ERR_INVALID_ARG;
   if (st != PS_OK) {
-    if (threadIdx.x == 0) c->status = st;
+    __syncthreads();
+    if (threadIdx.x == 0) { c->status = st; c->nblocks = 0; c->nsegs = 0; }
     return;
   }
-  int32_t carry = 0;
+  int32_t carry = 0, scarry = 0;
   for (int t0 = 0; t0 < R; t0 += blockDim.x) {
     const int i = t0 + threadIdx.x;
-    int32_t n = 0;
+    int32_t n = 0, nseg = 0;
     if (i < R) {
       n = (int32_t)((s.in_offsets[i + 1] - s.in_offsets[i]) / s.bs);
+      nseg = (n + kSegBlocks - 1) / kSegBlocks;
       s.rq_n[i] = n;
-      s.rq_cid[i] = s.in_contract ? s.in_contract[i] : s.contract_of_group[s.in_group[i]];
+      s.rq_h[i] = n;
+      s.rq_s[i] = n;
+      s.rq_fu[i] = kNone;
+      if (!probe) s.rq_cid[i] = s.in_contract ? s.in_contract[i] : s.contract_of_group[s.in_group[i]];
     }
-    int32_t tot;
+    int32_t tot, stot;
     const int32_t ex = block_excl_scan(n, &tot);
-    if (i < R) s.rq_pbase[i] = carry + ex;
+    const int32_t sex = block_excl_scan(nseg, &stot);
+    if (i < R) {
+      s.rq_pbase[i] = carry + ex;
+      s.rq_sbase[i] = scarry + sex;
+      for (int j = 0; j < nseg; ++j) s.seg_req[scarry + sex + j] = (uint32_t)i;
+    }
     carry += tot;
+    scarry += stot;
   }
   if (threadIdx.x == 0) {
     c->status = PS_OK;
     c->T = T;
     c->nblocks = carry;
-    c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
-    c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
-    c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
-    c->internal_error = 0;
+    c->nsegs = scarry;
+    if (!probe) {
+      c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
+      c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
+      c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
+      c->internal_error = 0;
+    }
   }
 }
 
 // ===========================================================================
-// Stages 1-2: chained block hashing and longest cached prefix, one warp per
-// request (Sec. III-B native content key; n_cached of Alg. 1).
+// Stage 1: chained block hashing (Sec. III-B native content key), one warp
+// per segment of up to kSegBlocks blocks of one prompt.
 //
 // Tokens of 32 blocks at a time are staged in shared memory with coalesced
 // 16-byte loads.  NH products are spread over the warp: lane l takes pair
 // (l % PPB) of block (l / PPB + (32 / PPB) r) in round r, PPB = bs / 2; the
 // pair sums are reduced with xor shuffles and routed to lane = block.  The
-// chain h_m = mix(mix(h_{m-1} ^ NH0) ^ NH2 ^ m) is then serial over the lanes.
-// Every key is looked up in the table; the first miss ends the cached prefix
-// h_i; blocks before it are pinned; every position at or past it is claimed in
-// the step's claim map (lowest request index wins, invariant I1).
+// chain C_m = Kc C_{m-1} + D_m (mod 2^61-1) is a composition of affine maps,
+// so a warp scan gives every block its chain value relative to the segment
+// start (B_m, with the value before the segment taken as 0); k_seg_carry then
+// supplies the true value entering each segment.
 template <int PPB>
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash_lookup(DevState s) {
+__global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash(DevState s) {
   extern __shared__ int32_t smem_tokens[];
-  if (s.ctl->status != PS_OK) return;
+  const Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
   constexpr int BS = 2 * PPB;
   constexpr int G32 = 32 / PPB;
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int i = blockIdx.x * kWarpsPerCta + warp;
-  if (i >= s.R) return;
+  const int64_t seg = (int64_t)blockIdx.x * kWarpsPerCta + warp;
+  if (seg >= c->nsegs) return;
   int32_t* buf = smem_tokens + warp * (32 * BS + 4);
-  const uint32_t g = (uint32_t)s.in_group[i];
-  const int64_t o0 = s.in_offsets[i];
+  const uint32_t i = s.seg_req[seg];
   const int n = s.rq_n[i];
+  const int m0 = (int)(seg - s.rq_sbase[i]) * kSegBlocks;
+  const int m1 = tmin(n, m0 + kSegBlocks);
+  const int64_t o0 = s.in_offsets[i];
   const int pbase = s.rq_pbase[i];
-  const int64_t T = s.ctl->T;
-  const uint32_t step32 = (uint32_t)s.ctl->step;
+  const int64_t T = c->T;
   const int k = lane % PPB;
   const uint32_t K0 = s.key_words[2 * k], K1 = s.key_words[2 * k + 1];
   const uint32_t K2 = s.key_words[2 * k + 2], K3 = s.key_words[2 * k + 3];
-  uint64_t h = chain_seed(s.hash_seed, (int32_t)g);
-  uint64_t key0 = 0;
-  int hfirst = -1;
-  int pinned_new = 0;
-  for (int c0 = 0; c0 < n; c0 += 32) {
-    const int nb = min(32, n - c0);
+  const uint64_t Kd = s.digest_mul;
+  uint64_t kp[5];
+#pragma unroll
+  for (int j = 0; j < 5; ++j) kp[j] = s.kc_pow[1 << j];
+  const uint64_t kpl = s.kc_pow[lane + 1];
+  uint64_t carry = 0;  // local chain value at the block before the chunk
+  for (int c0 = m0; c0 < m1; c0 += 32) {
+    const int nb = tmin(32, m1 - c0);
     const int64_t cs = o0 + (int64_t)c0 * BS, ce = cs + (int64_t)nb * BS;
     if (s.tokens_aligned16) {
       const int64_t q1 = (ce + 3) >> 2;
@@ -376,56 +411,94 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash_lookup(DevState s) {
       if (lane / G32 == r) { d1 = q1; d2 = q2; }
     }
     __syncwarp();
-    uint64_t key = 0;
-    for (int j = 0; j < nb; ++j) {
-      const uint64_t x = __shfl_sync(kFull, d1, j), y = __shfl_sync(kFull, d2, j);
-      h = fix_reserved(mix64(mix64(h ^ x) ^ y ^ (uint64_t)(c0 + j)));
-      if (lane == j) key = h;
+    // D_m, then the inclusive scan of the affine maps x -> Kc x + D
+    uint64_t b = lane < nb ? add61(red61(d1), mul61(Kd, red61(d2))) : 0;
+#pragma unroll
+    for (int j = 0; j < 5; ++j) {
+      const uint64_t t = __shfl_up_sync(kFull, b, 1 << j);
+      if (lane >= (1 << j)) b = add61(b, mul61(kp[j], t));
     }
-    if (c0 == 0) key0 = __shfl_sync(kFull, key, 0);
-    const bool valid = lane < nb;
-    const int pos = pbase + c0 + lane;
-    if (valid) s.pos_key[pos] = key;
-    // lookup, 4 keys per pass
-    uint32_t blk = kNone;
-    for (int kk = 0; kk < nb; kk += 4) {
-      const int my = kk + (lane >> 3);
-      const uint64_t kkey = __shfl_sync(kFull, key, my & 31);
-      const uint32_t f = table_lookup4(s, kkey, g, my < nb);
-      const uint32_t r = __shfl_sync(kFull, f, ((lane - kk) & 3) * 8);
-      if (lane >= kk && lane < kk + 4) blk = r;
+    const uint64_t B = add61(mul61(kpl, carry), b);
+    if (lane < nb) {
+      s.pos_key[pbase + c0 + lane] = B;
+      s.pos_req[pbase + c0 + lane] = i;
     }
-    if (valid) s.pos_blk[pos] = blk;
-    const unsigned miss = __ballot_sync(kFull, valid && blk == kNone);
-    if (hfirst < 0 && miss) hfirst = c0 + __ffs(miss) - 1;
-    const int hcur = hfirst < 0 ? INT_MAX : hfirst;
-    const int m = c0 + lane;
-    bool newpin = false;
-    if (valid) {
-      if (m < hcur) {
-        newpin = atomicExch(s.blk_pin + blk, step32) != step32;
-        s.pos_claim[pos] = kNone;
-      } else {
-        s.pos_claim[pos] = claim_insert(s, key, (uint32_t)i);
-      }
-    }
-    pinned_new += __popc(__ballot_sync(kFull, newpin));
+    carry = __shfl_sync(kFull, B, nb - 1);
   }
-  const int h_i = hfirst < 0 ? n : hfirst;
-  if (lane == 0) {
-    s.rq_h[i] = h_i;
-    if (pinned_new) atomic_add_i64(&s.ctl->pinned, pinned_new);
+  if (lane == 0) s.seg_tot[seg] = carry;
+}
+
+// Chain value entering each segment, serially over a request's segments
+// (thread per request): C = Kc^len C + B_end.
+__global__ void k_seg_carry(DevState s) {
+  const Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= s.R) return;
+  const int n = s.rq_n[i];
+  const int64_t sb = s.rq_sbase[i];
+  uint64_t C = red61(chain_seed(s.hash_seed, s.in_group[i]));
+  for (int j = 0; j * kSegBlocks < n; ++j) {
+    s.seg_cin[sb + j] = C;
+    const int len = tmin(kSegBlocks, n - j * kSegBlocks);
+    C = add61(mul61(s.kc_pow[len], C), s.seg_tot[sb + j]);
+  }
+}
+
+// Stage 2: block keys and the longest cached prefix (n_cached of Alg. 1),
+// thread per position: key_m = mix(C_m ^ (m+1) c), C_m = Kc^(k+1) C_in + B_m,
+// then a table probe; a miss lowers the request's h_i to its position.
+__global__ void __launch_bounds__(kThreads) k_keys_lookup(DevState s) {
+  const Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  PosRef r;
+  if (!pos_ref(s, pos, &r)) return;
+  const int64_t seg = s.rq_sbase[r.i] + r.m / kSegBlocks;
+  const uint64_t C = add61(mul61(s.kc_pow[r.m % kSegBlocks + 1], s.seg_cin[seg]), s.pos_key[pos]);
+  const uint64_t key = fix_reserved(mix64(C ^ ((uint64_t)(r.m + 1) * 0xD1B54A32D192ED03ull)));
+  s.pos_key[pos] = key;
+  const uint32_t blk = table_find(s, key, (uint32_t)s.in_group[r.i]);
+  s.pos_blk[pos] = blk;
+  if (blk == kNone) atomicMin(reinterpret_cast<uint32_t*>(s.rq_h) + r.i, (uint32_t)r.m);
+}
+
+// Stage 2 (cont.): blocks of the cached prefix are pinned for the step;
+// every position at or past the first miss is claimed in the step's claim
+// map (lowest request index wins: one materialization, one charge, I1).
+// Threads past the positions record each request's history entry
+// (OnRequest of Alg. 1) under its prefix id.
+__global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t nb = c->nblocks;
+  const uint32_t step32 = (uint32_t)c->step;
+  bool newpin = false;
+  if (t < nb) {
+    PosRef r;
+    pos_ref(s, t, &r);
+    if (r.m < s.rq_h[r.i]) {
+      newpin = atomicExch(s.blk_pin + s.pos_blk[t], step32) != step32;
+      s.pos_claim[t] = kNone;
+    } else {
+      s.pos_claim[t] = claim_insert(s, s.pos_key[t], r.i);
+    }
+  } else if (t < nb + s.R) {
+    const int i = (int)(t - nb);
+    const int n = s.rq_n[i];
+    const uint32_t g = (uint32_t)s.in_group[i];
     uint32_t hs = kNone;
     uint64_t p = 0;
     if (n > 0) {
-      p = s.in_prefix ? s.in_prefix[i] : key0;
+      p = s.in_prefix ? s.in_prefix[i] : s.pos_key[s.rq_pbase[i]];
       const uint32_t hmask = (1u << s.hist_cap_log2) - 1;
       uint32_t x = hist_home(p, g, s.hist_cap_log2);
       for (uint32_t it = 0; it <= hmask; ++it, x = (x + 1) & hmask) {
         uint64_t olo, ohi;
         cas128(s.hist + x, 0ull, 0ull, p, (uint64_t)(g + 1), &olo, &ohi);
         if (olo == 0 && ohi == 0) {
-          atomic_add_i64(&s.ctl->hist_new, 1);
+          atomic_add_i64(&c->hist_new, 1);
           hs = x;
           break;
         }
@@ -436,53 +509,47 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash_lookup(DevState s) {
       }
       if (hs != kNone)
         atomicMax(reinterpret_cast<unsigned long long*>(&s.hist[hs].ftag),
-                  (unsigned long long)step_tag(s.ctl->step, (uint32_t)i));
+                  (unsigned long long)step_tag(c->step, (uint32_t)i));
     }
     s.rq_hs[i] = hs;
     s.rq_p[i] = p;
   }
+  const int np = __popc(__ballot_sync(kFull, newpin));
+  if (lane_id() == 0 && np) atomic_add_i64(&c->pinned, np);
 }
 
-// ===========================================================================
-// Stage 2 (cont.): first own claim s_i of each request, and orphans.  A
+// Stage 2 (cont.): the first own claim s_i of each request, and orphans.  A
 // resident block past a request's first miss cannot be reached by lookup; it
 // is dropped (invalidated) unless some request pinned it.
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_claims(DevState s) {
+__global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   if (c->hist_live + c->hist_new > s.history_capacity) {  // history capacity is sticky
     if (blockIdx.x == 0 && threadIdx.x == 0) { c->status = PS_ERR_CAPACITY; c->sticky = PS_ERR_CAPACITY; }
     return;
   }
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int i = blockIdx.x * kWarpsPerCta + warp;
-  if (i >= s.R) return;
-  const int n = s.rq_n[i], h = s.rq_h[i], pbase = s.rq_pbase[i];
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const uint32_t step32 = (uint32_t)c->step;
-  int s_i = n;
-  for (int c0 = h; c0 < n; c0 += 32) {
-    const int m = c0 + lane;
-    bool own = false;
-    if (m < n) own = ldcg_u32(&s.claims[s.pos_claim[pbase + m]].minreq) == (uint32_t)i;
-    const unsigned b = __ballot_sync(kFull, own);
-    if (b) { s_i = c0 + __ffs(b) - 1; break; }
-  }
-  if (lane == 0) s.rq_s[i] = s_i;
-  int ninv = 0;
-  for (int c0 = h + 1; c0 < n; c0 += 32) {
-    const int m = c0 + lane;
-    bool inv = false;
-    if (m < n) {
-      const uint32_t b = s.pos_blk[pbase + m];
+  bool inv = false;
+  PosRef r;
+  if (pos_ref(s, pos, &r)) {
+    const int h = s.rq_h[r.i];
+    if (r.m >= h && ldcg_u32(&s.claims[s.pos_claim[pos]].minreq) == r.i)
+      atomicMin(reinterpret_cast<uint32_t*>(s.rq_s) + r.i, (uint32_t)r.m);
+    if (r.m > h) {
+      const uint32_t b = s.pos_blk[pos];
       if (b != kNone && ldcg_u32(s.blk_pin + b) != step32 && atomicExch(s.blk_inval + b, step32) != step32) {
         drop_block(s, b, PS_STAT_INVALIDATED_BLOCKS);
         atomicOr(s.bm_inval + (b >> 5), 1u << (b & 31));
         inv = true;
       }
     }
-    ninv += __popc(__ballot_sync(kFull, inv));
   }
-  if (lane == 0 && ninv) atomic_add_i64(&c->n_inval, ninv);
+  const int ni = __popc(__ballot_sync(kFull, inv));
+  if (lane_id() == 0 && ni) {
+    atomic_add_i64(&c->n_inval, ni);
+    atomic_add_i64(&c->n_resident, -ni);
+  }
 }
 
 // ===========================================================================
@@ -511,7 +578,8 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
     carry += tot;
   }
   const int64_t need = tmin<int64_t>(avail, carry);
-  for (int i = threadIdx.x; i < R; i += blockDim.x) s.out.admitted_offsets[i] = (int32_t)tmin<int64_t>(s.rq_cbase[i], need);
+  for (int i = threadIdx.x; i < R; i += blockDim.x)
+    s.out.admitted_offsets[i] = (int32_t)tmin<int64_t>(s.rq_cbase[i], need);
   if (threadIdx.x == 0) {
     s.out.admitted_offsets[R] = (int32_t)need;
     const int64_t nfree = s.N - c->n_resident;
@@ -519,41 +587,41 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
     c->total_claims = carry;
     c->need = need;
     c->nfree = nfree;
-    c->ftake = min(need, nfree);
-    c->mvict = need - min(need, nfree);
+    c->ftake = tmin(need, nfree);
+    c->mvict = need - tmin(need, nfree);
   }
 }
 
-// In-step hits: leading positions of [h_i, s_i) whose owner's claim was
-// granted; hit_i = h_i + e_i.  Also records the first admitting request of
-// each (group, prefix) entry.
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_instep(DevState s) {
-  Ctl* c = s.ctl;
+// In-step hits: positions of [h_i, s_i) belong to earlier requests' claims;
+// the leading granted ones are hits.  A position whose owner's rank is past
+// avail lowers the request's first-ungranted mark.
+__global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
+  const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int i = blockIdx.x * kWarpsPerCta + warp;
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  PosRef r;
+  if (!pos_ref(s, pos, &r)) return;
+  if (r.m < s.rq_h[r.i] || r.m >= s.rq_s[r.i]) return;
+  const uint32_t j = s.claims[s.pos_claim[pos]].minreq;
+  const int64_t rank = (int64_t)s.rq_cbase[j] + (r.m - s.rq_s[j]);
+  if (rank >= c->avail) atomicMin(s.rq_fu + r.i, (uint32_t)r.m);
+}
+
+// hit_i = h_i + e_i per request; records the first admitting request of each
+// (group, prefix) history entry of the step.
+__global__ void k_instep_fin(DevState s) {
+  const Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= s.R) return;
-  const int h = s.rq_h[i], si = s.rq_s[i], pbase = s.rq_pbase[i];
-  const int64_t avail = c->avail;
-  int e = si - h;
-  for (int c0 = h; c0 < si; c0 += 32) {
-    const int m = c0 + lane;
-    bool ungranted = false;
-    if (m < si) {
-      const uint32_t j = s.claims[s.pos_claim[pbase + m]].minreq;
-      const int64_t rank = (int64_t)s.rq_cbase[j] + (m - s.rq_s[j]);
-      ungranted = rank >= avail;
-    }
-    const unsigned b = __ballot_sync(kFull, ungranted);
-    if (b) { e = c0 + __ffs(b) - 1 - h; break; }
-  }
-  if (lane == 0) {
-    s.rq_e[i] = e;
-    s.out.hit_blocks[i] = h + e;
-    const uint32_t hs = s.rq_hs[i];
-    if (s.rq_a[i] > 0 && hs != kNone)
-      atomicMax(reinterpret_cast<unsigned long long*>(&s.hist[hs].atag), (unsigned long long)step_tag(c->step, (uint32_t)i));
-  }
+  const int h = s.rq_h[i], si = s.rq_s[i];
+  const uint32_t fu = s.rq_fu[i];
+  const int e = (int)tmin<uint32_t>(fu, (uint32_t)si) - h;
+  s.rq_e[i] = e;
+  s.out.hit_blocks[i] = h + e;
+  const uint32_t hs = s.rq_hs[i];
+  if (s.rq_a[i] > 0 && hs != kNone)
+    atomicMax(reinterpret_cast<unsigned long long*>(&s.hist[hs].atag), (unsigned long long)step_tag(c->step, (uint32_t)i));
 }
 
 // ===========================================================================
@@ -639,7 +707,7 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s) {
       const int64_t def = tmax<int64_t>(0, -b);
       raw += def;                                    // Eq. 3
       norm += muldiv(def, s.rho_min, s.rho[cc]);     // Eq. 5
-      if (b < 0) rmax = max(rmax, s.rho[cc]);
+      if (b < 0) rmax = tmax(rmax, s.rho[cc]);
     }
     row[PS_STAT_DEBT_RAW] = raw;
     row[PS_STAT_DEBT_NORM] = norm;
@@ -648,119 +716,123 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s) {
     s.grp_P[g] = norm;
     s.grp_delta[g] = rmax ? muldiv(unit, s.rho_min, rmax) : 0;  // 1/W_g of Eq. 8
     s.grp_qsize[g] = 0;
+    SelSeg z{};
+    z.kmin = ~0ull;
+    z.kmax = 0;
+    s.sel[g] = z;
   }
 }
 
 // ===========================================================================
-// Stage 4: OnTouch (Alg. 1, Eq. 4) for every hit block, resident or in-step.
-// Pass 1 applies the access updates (stamp = max, access count, S3-FIFO
-// frequency) and records, per block, the lowest request whose touch promotes
-// it.  Pass 2 counts the gated touches that precede the promotion (or all of
-// them when none promotes) and applies the promotion of resident blocks.
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_touch(DevState s) {
-  Ctl* c = s.ctl;
+// Stage 4: OnTouch (Alg. 1, Eq. 4) for every hit block, resident or in-step,
+// thread per position.  Pass 1 applies the access updates (stamp = max,
+// access count, S3-FIFO frequency) and records, per block, the lowest request
+// whose touch promotes it.  Pass 2 counts the gated touches that precede the
+// promotion (or all of them when none promotes) and applies the promotion of
+// resident blocks.
+__global__ void __launch_bounds__(kThreads) k_touch(DevState s) {
+  const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int i = blockIdx.x * kWarpsPerCta + warp;
-  if (i >= s.R) return;
-  const int n = s.rq_n[i];
-  if (n == 0) return;
-  const int h = s.rq_h[i], hit = h + s.rq_e[i], pbase = s.rq_pbase[i];
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  PosRef r;
+  if (!pos_ref(s, pos, &r)) return;
+  const uint32_t i = r.i;
+  const int m = r.m;
+  const int h = s.rq_h[i];
+  if (m >= h + s.rq_e[i]) return;
   const uint8_t fl = s.rq_flags[i];
   const bool proven = fl & 1, gate = fl & 2;
   const int cid = s.rq_cid[i];
   const uint64_t p = s.rq_p[i];
   const uint64_t step = c->step;
-  for (int m = lane; m < hit; m += 32) {
-    const int pos = pbase + m;
-    bool elig;
-    if (m < h) {
-      const uint32_t b = s.pos_blk[pos];
-      atomicMax(reinterpret_cast<unsigned long long*>(s.blk_stamp + b), (unsigned long long)make_stamp(step, i, m));
-      atomicAdd(s.blk_acc + b, 1u);
-      atomicAdd(s.blk_freq + b, 1u);
-      elig = proven && s.blk_contract[b] == cid && s.blk_prefix[b] == p && s.blk_klass[b] != kReuse;
-      if (elig && gate)
-        atomicMax(reinterpret_cast<unsigned long long*>(s.blk_promo + b), (unsigned long long)step_tag(step, (uint32_t)i));
-    } else {
-      ClaimEntry* e = s.claims + s.pos_claim[pos];
-      const uint32_t j = e->minreq;
-      atomicMax(&e->last, (uint32_t)i + 1);
-      atomicAdd(&e->tcnt, 1u);
-      elig = proven && s.rq_cid[j] == cid && s.rq_p[j] == p;  // new blocks are never Reuse yet
-      if (elig && gate) atomicMin(&e->promo, (uint32_t)i);
-    }
-    s.pos_elig[pos] = elig;
+  bool elig;
+  if (m < h) {
+    const uint32_t b = s.pos_blk[pos];
+    atomicMax(reinterpret_cast<unsigned long long*>(s.blk_stamp + b), (unsigned long long)make_stamp(step, i, m));
+    atomicAdd(s.blk_acc + b, 1u);
+    atomicAdd(s.blk_freq + b, 1u);
+    elig = proven && s.blk_contract[b] == cid && s.blk_prefix[b] == p && s.blk_klass[b] != kReuse;
+    if (elig && gate)
+      atomicMax(reinterpret_cast<unsigned long long*>(s.blk_promo + b), (unsigned long long)step_tag(step, i));
+  } else {
+    ClaimEntry* e = s.claims + s.pos_claim[pos];
+    const uint32_t j = e->minreq;
+    atomicMax(&e->last, i + 1);
+    atomicAdd(&e->tcnt, 1u);
+    elig = proven && s.rq_cid[j] == cid && s.rq_p[j] == p;  // new blocks are never Reuse yet
+    if (elig && gate) atomicMin(&e->promo, i);
   }
+  s.pos_elig[pos] = elig;
 }
 
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_touch2(DevState s) {
-  Ctl* c = s.ctl;
+__global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
+  const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int i = blockIdx.x * kWarpsPerCta + warp;
-  if (i >= s.R) return;
-  const int n = s.rq_n[i];
-  if (n == 0) return;
-  const int h = s.rq_h[i], hit = h + s.rq_e[i], pbase = s.rq_pbase[i];
-  const bool gate = s.rq_flags[i] & 2;
-  const uint64_t step = c->step;
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  PosRef r;
   int gated = 0, promoted = 0;
-  for (int m = lane; m < hit; m += 32) {
-    const int pos = pbase + m;
-    if (!s.pos_elig[pos]) continue;
-    uint32_t promoter;
-    uint32_t b = kNone;
-    if (m < h) {
+  uint32_t g = 0;
+  if (pos_ref(s, pos, &r) && r.m < s.rq_h[r.i] + s.rq_e[r.i] && s.pos_elig[pos]) {
+    const uint32_t i = r.i;
+    g = (uint32_t)s.in_group[i];
+    const bool gate = s.rq_flags[i] & 2;
+    uint32_t promoter, b = kNone;
+    if (r.m < s.rq_h[i]) {
       b = s.pos_blk[pos];
-      promoter = tag_req(ldcg_u64(s.blk_promo + b), step);
+      promoter = tag_req(ldcg_u64(s.blk_promo + b), c->step);
     } else {
       promoter = ldcg_u32(&s.claims[s.pos_claim[pos]].promo);
     }
     if (!gate) {
-      if ((uint32_t)i < promoter) ++gated;
-    } else if ((uint32_t)i == promoter) {
-      ++promoted;
+      gated = i < promoter;
+    } else if (i == promoter) {
+      promoted = 1;
       if (b != kNone) s.blk_klass[b] = kReuse;
     }
   }
-  gated = warp_sum(gated);
-  promoted = warp_sum(promoted);
-  if (lane == 0) {
-    const int g = s.in_group[i];
-    if (gated) atomic_add_i64(&stat_ref(s, g, PS_STAT_GATED_REUSES), gated);
-    if (promoted) atomic_add_i64(&stat_ref(s, g, PS_STAT_PROMOTIONS), promoted);
-  }
+  agg_stat(s, g, PS_STAT_GATED_REUSES, gated, gated != 0);
+  agg_stat(s, g, PS_STAT_PROMOTIONS, promoted, promoted != 0);
 }
 
 // ===========================================================================
 // Stage 5: reclamation.  Candidates are resident blocks not hit in this step.
 // The order key is (class, stamp) for prefixshield (Eq. 9; stamp only with
-// the no-segmentation ablation) and the stamp for lru.
+// the no-segmentation ablation) and the stamp for lru.  Also the smallest
+// and largest key of every segment, so the radix select can skip the bytes
+// its candidates share.
 __global__ void k_cand(DevState s) {
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const uint32_t step32 = (uint32_t)c->step;
-  const bool seg = s.policy == PS_PREFIXSHIELD && !(s.flags & PS_FLAG_NO_SEGMENTATION);
+  const bool ps = s.policy == PS_PREFIXSHIELD;
+  const bool seg = ps && !(s.flags & PS_FLAG_NO_SEGMENTATION);
   for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
     const int64_t b = b0 + threadIdx.x;
     bool cand = false;
     uint32_t g = 0;
+    uint64_t key = ~0ull;
     if (b < s.N) {
       cand = (s.blk_flags[b] & 1) && s.blk_pin[b] != step32;
-      uint64_t key = ~0ull;
       if (cand) {
         key = s.blk_stamp[b];
         if (seg) key |= (uint64_t)s.blk_klass[b] << 62;
-        g = s.blk_group[b];
+        g = ps ? s.blk_group[b] : 0;
       }
       s.csk[b] = key;
     }
-    if (s.policy == PS_PREFIXSHIELD) {
-      const unsigned act = __ballot_sync(kFull, cand);
-      if (cand) {
-        const unsigned peers = __match_any_sync(act, g);
-        if (lane_id() == __ffs(peers) - 1) atomic_add_i64(s.grp_qsize + g, __popc(peers));
+    const unsigned act = __ballot_sync(kFull, cand);
+    if (cand) {
+      const unsigned peers = __match_any_sync(act, g);
+      uint64_t mn = key, mx = key;
+      for (unsigned m = peers; m; m &= m - 1) {
+        const uint64_t v = __shfl_sync(peers, key, __ffs(m) - 1);
+        mn = tmin(mn, v);
+        mx = tmax(mx, v);
+      }
+      if (lane_id() == __ffs(peers) - 1) {
+        if (ps) atomic_add_i64(s.grp_qsize + g, __popc(peers));
+        atomicMin(reinterpret_cast<unsigned long long*>(&s.sel[g].kmin), (unsigned long long)mn);
+        atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[g].kmax), (unsigned long long)mx);
       }
     }
   }
@@ -771,10 +843,15 @@ __global__ void k_sel_single(DevState s, int fallback) {
   if (threadIdx.x != 0) return;
   int64_t m = 0;
   if (c->status == PS_OK) m = fallback ? c->m_fb : c->mvict;
+  const SelSeg old = s.sel[0];
   SelSeg z{};
   z.rank = m;
   z.active = m > 0;
   z.incl = 1;
+  // the fallback selects among the candidates the debt phase left over all
+  // groups: its key range is not known, so it starts from the top byte
+  z.kmin = fallback ? 0 : old.kmin;
+  z.kmax = fallback ? ~0ull : old.kmax;
   s.sel[0] = z;
 }
 
@@ -789,7 +866,7 @@ __global__ void k_sel_single(DevState s, int fallback) {
 // to the global fallback in (class, stamp) order.
 __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
   Ctl* c = s.ctl;
-  __shared__ int64_t s_tau;
+  __shared__ int64_t s_pmax;
   const int G = s.G;
   const int64_t eps = s.eps;
   const int64_t m = (c->status == PS_OK) ? c->mvict : 0;
@@ -798,8 +875,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     if (threadIdx.x == 0) c->m_fb = 0;
     return;
   }
-  // count of items with value > t, summed over groups
-  auto count_gt = [&](int64_t t) -> int64_t {
+  auto count_gt = [&](int64_t t) -> int64_t {  // items with value > t over all groups
     int64_t tot = 0;
     for (int g = threadIdx.x; g < G; g += blockDim.x) {
       const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
@@ -813,32 +889,30 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
       const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
       const int64_t x = (P > eps && d > 0) ? tmin<int64_t>(q, (P - eps - 1) / d + 1) : 0;
       s.grp_x[g] = x;
-      SelSeg z{};
-      z.rank = x; z.active = x > 0; z.incl = 1;
-      s.sel[g] = z;
+      s.sel[g].rank = x;
+      s.sel[g].active = x > 0;
+      s.sel[g].incl = 1;
     }
     if (threadIdx.x == 0) { c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; }
     return;
   }
-  // tau = max{t > eps : count_gt(t - 1) >= m}; binary search on [eps + 1, max P]
   int64_t pmax = 0;
-  for (int g = threadIdx.x; g < G; g += blockDim.x) pmax = max(pmax, s.grp_P[g]);
+  for (int g = threadIdx.x; g < G; g += blockDim.x) pmax = tmax(pmax, s.grp_P[g]);
   {
     __shared__ int64_t red[32];
     int64_t v = pmax;
-    for (int o = 16; o > 0; o >>= 1) v = max(v, __shfl_xor_sync(kFull, v, o));
+    for (int o = 16; o > 0; o >>= 1) v = tmax(v, (int64_t)__shfl_xor_sync(kFull, v, o));
     if (lane_id() == 0) red[threadIdx.x >> 5] = v;
     __syncthreads();
     if (threadIdx.x == 0) {
-      int64_t r = 0;
-      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) r = max(r, red[w]);
-      s_tau = r;
+      int64_t rr = 0;
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) rr = tmax(rr, red[w]);
+      s_pmax = rr;
     }
     __syncthreads();
-    pmax = s_tau;
-    __syncthreads();
+    pmax = s_pmax;
   }
-  int64_t lo = eps + 1, hi = pmax;  // invariant: count_gt(lo - 1) >= m
+  int64_t lo = eps + 1, hi = pmax;  // tau = max{t > eps : count_gt(t - 1) >= m}
   while (lo < hi) {
     const int64_t mid = lo + (hi - lo + 1) / 2;
     if (count_gt(mid - 1) >= m) lo = mid; else hi = mid - 1;
@@ -853,11 +927,9 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     if (d > 0 && P >= tau && (P - tau) % d == 0 && (P - tau) / d < q) tied = true;
     above += xa;
     ntie += tied;
-    SelSeg z{};
-    z.rank = xa + (tied ? 1 : 0);
-    z.active = z.rank > 0;
-    z.incl = tied ? 2 : 1;  // 2: the tie item is taken only if k_tie chooses it
-    s.sel[g] = z;
+    s.sel[g].rank = xa + (tied ? 1 : 0);
+    s.sel[g].active = xa + (tied ? 1 : 0) > 0;
+    s.sel[g].incl = tied ? 2 : 1;  // 2: the tie item is taken only if k_tie chooses it
     s.grp_x[g] = xa + (tied ? 1 : 0);
   }
   above = block_sum(above);
@@ -871,30 +943,56 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
 
 // One MSB-first radix digit of the segmented select.  Every candidate of an
 // active segment whose key matches the segment's prefix adds to that
-// segment's histogram of the next 8-bit digit; the last CTA to finish picks,
-// for every segment, the digit whose cumulative count reaches the rank.
+// segment's histogram of the next 8-bit digit (a shared-memory histogram per
+// CTA, flushed as non-zero bins); the last CTA to finish picks, for every
+// segment, the digit whose cumulative count reaches the rank.  Bytes that all
+// of a segment's candidates share (from its smallest and largest key) are
+// taken without counting.
+__device__ __forceinline__ bool digit_known(const SelSeg& ss, int shift) {
+  return ((ss.kmin ^ ss.kmax) & (~0ull << shift)) == 0;
+}
+
 __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int single, int fallback) {
+  extern __shared__ uint32_t shist[];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const int nseg = single ? 1 : s.G;
   if (single && !s.sel[0].active) return;
   const int shift = 64 - kRadixBits * (pass + 1);
-  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t b = b0 + threadIdx.x;
-    bool act = false;
-    uint32_t idx = 0;
-    if (b < s.N) {
-      const uint64_t key = s.csk[b];
-      if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
-        const int seg = single ? 0 : s.blk_group[b];
-        const SelSeg ss = s.sel[seg];
-        if (ss.active && (key & ss.mask) == ss.prefix) {
-          act = true;
-          idx = (uint32_t)seg * kRadixBins + (uint32_t)((key >> shift) & (kRadixBins - 1));
+  const bool use_smem = nseg <= 64;
+  __shared__ int s_work;
+  if (threadIdx.x == 0) s_work = 0;
+  __syncthreads();
+  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+    const SelSeg ss = s.sel[g];
+    if (ss.active && !digit_known(ss, shift)) s_work = 1;
+  }
+  __syncthreads();
+  if (s_work) {
+    if (use_smem)
+      for (int k = threadIdx.x; k < nseg * kRadixBins; k += blockDim.x) shist[k] = 0;
+    __syncthreads();
+    for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
+      const int64_t b = b0 + threadIdx.x;
+      bool act = false;
+      uint32_t idx = 0;
+      if (b < s.N) {
+        const uint64_t key = s.csk[b];
+        if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
+          const int seg = single ? 0 : s.blk_group[b];
+          const SelSeg ss = s.sel[seg];
+          if (ss.active && (key & ss.mask) == ss.prefix && !digit_known(ss, shift)) {
+            act = true;
+            idx = (uint32_t)seg * kRadixBins + (uint32_t)((key >> shift) & (kRadixBins - 1));
+          }
         }
       }
+      agg_inc(use_smem ? shist : s.hist_bins, idx, act);
     }
-    agg_inc(s.hist_bins, idx, act);
+    __syncthreads();
+    if (use_smem)
+      for (int k = threadIdx.x; k < nseg * kRadixBins; k += blockDim.x)
+        if (shist[k]) atomicAdd(s.hist_bins + k, shist[k]);
   }
   __shared__ bool last;
   __threadfence();
@@ -907,6 +1005,14 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
   for (int seg = warp; seg < nseg; seg += blockDim.x >> 5) {
     SelSeg ss = s.sel[seg];
     if (!ss.active) continue;
+    if (digit_known(ss, shift)) {
+      if (lane == 0) {
+        ss.prefix |= ss.kmin & ((uint64_t)(kRadixBins - 1) << shift);
+        ss.mask |= (uint64_t)(kRadixBins - 1) << shift;
+        s.sel[seg] = ss;
+      }
+      continue;
+    }
     uint32_t* row = s.hist_bins + (size_t)seg * kRadixBins;
     uint32_t v[kRadixBins / 32];
     uint32_t sum = 0;
@@ -914,14 +1020,12 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
     for (int j = 0; j < kRadixBins / 32; ++j) { v[j] = ldcg_u32(row + lane * (kRadixBins / 32) + j); sum += v[j]; }
     const uint32_t incl = warp_incl_scan(sum);
     const uint32_t excl = incl - sum;
-    // the lane whose range holds the rank-th item
-    const bool here = excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= incl;
-    const unsigned who = __ballot_sync(kFull, here);
+    const bool here = (uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl;
     if (here) {
       uint32_t run = excl;
       int d = 0;
       for (int j = 0; j < kRadixBins / 32; ++j) {
-        if ((uint64_t)ss.rank <= run + v[j]) { d = lane * (kRadixBins / 32) + j; break; }
+        if ((uint64_t)ss.rank <= (uint64_t)(run + v[j])) { d = lane * (kRadixBins / 32) + j; break; }
         run += v[j];
       }
       ss.prefix |= (uint64_t)d << shift;
@@ -929,7 +1033,6 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
       ss.rank -= run;
       s.sel[seg] = ss;
     }
-    (void)who;
 #pragma unroll
     for (int j = 0; j < kRadixBins / 32; ++j) row[lane * (kRadixBins / 32) + j] = 0;
   }
@@ -980,10 +1083,7 @@ __global__ void k_mark(DevState s, int single, int fallback) {
       }
     }
     const unsigned bits = __ballot_sync(kFull, v);
-    if (bits && lane_id() == 0) {
-      // 32 consecutive block ids share one bitmap word when b0 is 32-aligned
-      atomicOr(s.bm_victim + ((b - lane_id()) >> 5), bits);
-    }
+    if (bits && lane_id() == 0) atomicOr(s.bm_victim + ((b - lane_id()) >> 5), bits);
     marked += __popc(bits);
   }
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
@@ -1021,20 +1121,6 @@ __global__ void __launch_bounds__(1024) k_freetake(DevState s) {
       }
     }
     s.bm_alloc[w] = take | s.bm_victim[w];
-  }
-}
-
-// Evict the victims: drop their table entries and metadata.
-__global__ void k_evict(DevState s) {
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK || c->mvict == 0) return;
-  for (int64_t w = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; w < s.nwords; w += (int64_t)gridDim.x * blockDim.x) {
-    uint32_t bits = s.bm_victim[w];
-    while (bits) {
-      const int j = __ffs(bits) - 1;
-      bits &= bits - 1;
-      drop_block(s, (uint32_t)(w * 32 + j), PS_STAT_EVICTED_BLOCKS);
-    }
   }
 }
 
@@ -1081,53 +1167,63 @@ __global__ void __launch_bounds__(1024) k_bm_write(DevState s) {
   }
 }
 
-// Stage 6: place granted claims.  The allocated ids (ascending) go to the
-// granted keys in (request, position) order; each new block carries the
-// metadata OnCacheFullBlocks attached plus any in-step touches.
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_insert(DevState s) {
+// Evict the victims (thread per evicted id): drop table entries and metadata.
+__global__ void __launch_bounds__(kThreads) k_evict(DevState s) {
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int i = blockIdx.x * kWarpsPerCta + warp;
-  if (i >= s.R) return;
-  const int a = s.rq_a[i];
-  if (a == 0) return;
-  const int si = s.rq_s[i], pbase = s.rq_pbase[i], cb = s.rq_cbase[i];
-  const uint32_t g = (uint32_t)s.in_group[i];
-  const uint8_t cid = (uint8_t)s.rq_cid[i];
-  const uint64_t p = s.rq_p[i];
-  const uint8_t knew = s.rq_knew[i];
-  const uint64_t step = c->step;
-  const int64_t n_alloc = c->n_alloc;
-  bool bad = false;
-  for (int m = si + lane; m < si + a; m += 32) {
-    const int pos = pbase + m;
-    if (cb + (m - si) >= n_alloc) { bad = true; continue; }  // allocated set short: internal error
-    const uint32_t b = (uint32_t)s.out.admitted_ids[cb + (m - si)];
-    if (b >= (uint64_t)s.N) { bad = true; continue; }
-    const ClaimEntry e = s.claims[s.pos_claim[pos]];
-    const uint64_t key = s.pos_key[pos];
-    s.blk_key[b] = key;
-    s.blk_group[b] = (uint16_t)g;
-    s.blk_contract[b] = cid;
-    s.blk_prefix[b] = p;
-    s.blk_klass[b] = e.promo != kNone ? (uint8_t)kReuse : knew;
-    s.blk_stamp[b] = make_stamp(step, e.last ? e.last - 1 : (uint32_t)i, m);
-    s.blk_acc[b] = e.tcnt;
-    s.blk_freq[b] = e.tcnt;
-    s.blk_flags[b] = 1;
-    s.blk_slot[b] = table_insert(s, key, g, b);
-    atomicOr(s.res_bits + (b >> 5), 1u << (b & 31));
+  const int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  const int64_t nv = c->n_evicted;
+  const bool act = v < nv && v < s.max_blocks;
+  if (act) drop_block(s, (uint32_t)s.out.evicted_ids[v], PS_STAT_EVICTED_BLOCKS);
+  const int k = __popc(__ballot_sync(kFull, act));
+  if (lane_id() == 0 && k) atomic_add_i64(&c->n_resident, -k);
+}
+
+// Stage 6: place granted claims (thread per position).  The allocated ids
+// (ascending) go to the granted keys in (request, position) order; each new
+// block carries the metadata OnCacheFullBlocks attached plus any in-step
+// touches.
+__global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  PosRef r;
+  bool placed = false;
+  uint32_t g = 0;
+  if (pos_ref(s, pos, &r)) {
+    const uint32_t i = r.i;
+    const int si = s.rq_s[i], a = s.rq_a[i];
+    g = (uint32_t)s.in_group[i];
+    if (r.m >= si && r.m < si + a) {
+      const int64_t rank = (int64_t)s.rq_cbase[i] + (r.m - si);
+      const uint32_t b = rank < c->n_alloc ? (uint32_t)s.out.admitted_ids[rank] : kNone;
+      if (b >= (uint64_t)s.N) {
+        c->internal_error = 1;  // the allocated set is short: never expected
+      } else {
+        const ClaimEntry e = s.claims[s.pos_claim[pos]];
+        const uint64_t key = s.pos_key[pos];
+        s.blk_key[b] = key;
+        s.blk_group[b] = (uint16_t)g;
+        s.blk_contract[b] = (uint8_t)s.rq_cid[i];
+        s.blk_prefix[b] = s.rq_p[i];
+        s.blk_klass[b] = e.promo != kNone ? (uint8_t)kReuse : s.rq_knew[i];
+        s.blk_stamp[b] = make_stamp(c->step, e.last ? e.last - 1 : i, r.m);
+        s.blk_acc[b] = e.tcnt;
+        s.blk_freq[b] = e.tcnt;
+        s.blk_flags[b] = 1;
+        s.blk_slot[b] = table_insert(s, key, g, b);
+        atomicOr(s.res_bits + (b >> 5), 1u << (b & 31));
+        placed = true;
+      }
+    }
   }
-  if (__any_sync(kFull, bad) && lane == 0) c->internal_error = 1;
-  if (lane == 0) {
-    atomic_add_i64(&c->n_resident, a);
-    atomic_add_i64(&stat_ref(s, g, PS_STAT_RESIDENT_BLOCKS), a);
-  }
+  agg_stat(s, g, PS_STAT_RESIDENT_BLOCKS, placed ? 1 : 0, placed);
+  const int k = __popc(__ballot_sync(kFull, placed));
+  if (lane_id() == 0 && k) atomic_add_i64(&c->n_resident, k);
 }
 
 // OnRequest / RecordSuccessfulAdmission commit: reference counts and admitted
-// flags of the history entries.
+// flags of the history entries (thread per request).
 __global__ void k_hist_commit(DevState s) {
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
@@ -1140,21 +1236,18 @@ __global__ void k_hist_commit(DevState s) {
   if (s.rq_a[i] > 0) atomicOr(&s.hist[hs].refadm, 0x80000000u);
 }
 
-// Clear the claim-map slots this step used.
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_claim_clear(DevState s) {
-  Ctl* c = s.ctl;
+// Clear the claim-map slots this step used (thread per position).
+__global__ void __launch_bounds__(kThreads) k_claim_clear(DevState s) {
+  const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int i = blockIdx.x * kWarpsPerCta + warp;
-  if (i >= s.R) return;
-  const int n = s.rq_n[i], h = s.rq_h[i], pbase = s.rq_pbase[i];
-  for (int m = h + lane; m < n; m += 32) {
-    const uint32_t slot = s.pos_claim[pbase + m];
-    if (slot == kNone) continue;
-    ClaimEntry z{};
-    z.key = 0; z.minreq = kNone; z.last = 0; z.tcnt = 0; z.promo = kNone; z.pad0 = 0; z.pad1 = 0;
-    s.claims[slot] = z;
-  }
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  PosRef r;
+  if (!pos_ref(s, pos, &r) || r.m < s.rq_h[r.i]) return;
+  const uint32_t slot = s.pos_claim[pos];
+  if (slot == kNone) return;
+  ClaimEntry z{};
+  z.key = 0; z.minreq = kNone; z.last = 0; z.tcnt = 0; z.promo = kNone; z.pad0 = 0; z.pad1 = 0;
+  s.claims[slot] = z;
 }
 
 __global__ void k_finalize(DevState s) {
@@ -1162,12 +1255,21 @@ __global__ void k_finalize(DevState s) {
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   const int32_t st = c->internal_error ? PS_ERR_DEVICE_STATUS : c->status;
   s.out.counts[3] = st;
-  if (st != PS_OK) return;
+  if (c->status != PS_OK) return;
   s.out.counts[0] = (int32_t)c->need;
   s.out.counts[1] = (int32_t)c->n_evicted;
   s.out.counts[2] = (int32_t)c->n_inval;
   c->t_prev = s.now;
   c->step += 1;
+}
+
+// Read-only probe output: h_i per request, and the probe's status.
+__global__ void k_probe_out(DevState s, int32_t* out, int32_t* status) {
+  const Ctl* c = s.ctl;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i == 0) *status = c->status;
+  if (c->status != PS_OK || i >= s.R) return;
+  out[i] = s.rq_h[i];
 }
 
 // ===========================================================================
@@ -1180,88 +1282,115 @@ static int grid_for(int64_t items, int threads, int max_ctas) {
 }
 
 void launch_init(const DevState& s, cudaStream_t st) {
-  k_init_blocks<<<grid_for(s.N, 256, 152 * 8), 256, 0, st>>>(s);
+  k_init_blocks<<<grid_for((int64_t)kClaimWays << s.cl_nbuckets_log2, 256, 152 * 8), 256, 0, st>>>(s);
   k_init_ctl<<<1, 1024, 0, st>>>(s);
 }
 
 template <int PPB>
-static void launch_hash(const DevState& s, cudaStream_t st) {
+static void launch_hash_t(const DevState& s, cudaStream_t st) {
   const size_t smem = (size_t)kWarpsPerCta * (32 * 2 * PPB + 4) * sizeof(int32_t);
-  static bool configured = false;
-  if (!configured) {
-    cudaFuncSetAttribute(k_hash_lookup<PPB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    configured = true;
+  if (smem > 48 * 1024) cudaFuncSetAttribute(k_hash<PPB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  k_hash<PPB><<<(int)((s.max_segments + kWarpsPerCta - 1) / kWarpsPerCta), kWarpsPerCta * 32, smem, st>>>(s);
+}
+static int32_t launch_hash(const DevState& s, cudaStream_t st) {
+  switch (s.bs / 2) {
+    case 1: launch_hash_t<1>(s, st); break;
+    case 2: launch_hash_t<2>(s, st); break;
+    case 4: launch_hash_t<4>(s, st); break;
+    case 8: launch_hash_t<8>(s, st); break;
+    case 16: launch_hash_t<16>(s, st); break;
+    case 32: launch_hash_t<32>(s, st); break;
+    default: return PS_ERR_INVALID_ARG;
   }
-  k_hash_lookup<PPB><<<(s.R + kWarpsPerCta - 1) / kWarpsPerCta, kWarpsPerCta * 32, smem, st>>>(s);
+  return PS_OK;
 }
 
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   const int R = s.R;
-  const int wgrid = R > 0 ? (R + kWarpsPerCta - 1) / kWarpsPerCta : 1;
-  const int wthreads = kWarpsPerCta * 32;
+  const int rgrid = grid_for(R, 256, 1 << 20);
+  const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
+  const int prgrid = grid_for(s.max_blocks + R, kThreads, 1 << 30);
   const int ngrid = grid_for(s.N, 256, 152 * 8);
+  const int sgrid = grid_for(s.N, 256, 152 * 2);
+  const int radix_smem = (s.G <= 64 ? s.G : 1) * kRadixBins * 4;
   int launches = 0;
   auto mark = [&](int stage) {
     if (tr && tr->timing) cudaEventRecord(tr->ev[stage], st);
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
+  if (radix_smem > 48 * 1024)
+    cudaFuncSetAttribute(k_radix_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, radix_smem);
   mark(0);
-  PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s, 0));
   mark(1);
   if (R > 0) {
-    switch (s.bs / 2) {
-      case 1: PS_LAUNCH(launch_hash<1>(s, st)); break;
-      case 2: PS_LAUNCH(launch_hash<2>(s, st)); break;
-      case 4: PS_LAUNCH(launch_hash<4>(s, st)); break;
-      case 8: PS_LAUNCH(launch_hash<8>(s, st)); break;
-      case 16: PS_LAUNCH(launch_hash<16>(s, st)); break;
-      case 32: PS_LAUNCH(launch_hash<32>(s, st)); break;
-      default: return PS_ERR_INVALID_ARG;
-    }
+    if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
+    ++launches;
+    PS_LAUNCH(k_seg_carry<<<rgrid, 256, 0, st>>>(s));
+    PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
   }
+  PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
   mark(2);
-  PS_LAUNCH(k_claims<<<wgrid, wthreads, 0, st>>>(s));
+  PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
   mark(3);
   PS_LAUNCH(k_grant<<<1, 1024, 0, st>>>(s));
-  PS_LAUNCH(k_instep<<<wgrid, wthreads, 0, st>>>(s));
+  PS_LAUNCH(k_instep<<<pgrid, kThreads, 0, st>>>(s));
+  PS_LAUNCH(k_instep_fin<<<rgrid, 256, 0, st>>>(s));
   mark(4);
   PS_LAUNCH(k_meter<<<s.G, 1024, 0, st>>>(s));
   mark(5);
-  PS_LAUNCH(k_touch<<<wgrid, wthreads, 0, st>>>(s));
-  PS_LAUNCH(k_touch2<<<wgrid, wthreads, 0, st>>>(s));
+  PS_LAUNCH(k_touch<<<pgrid, kThreads, 0, st>>>(s));
+  PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
   mark(6);
   PS_LAUNCH(k_cand<<<ngrid, 256, 0, st>>>(s));
   if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));
-    for (int pass = 0; pass < 8; ++pass) PS_LAUNCH(k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 0, 0));
+    for (int pass = 0; pass < 8; ++pass)
+      PS_LAUNCH(k_radix_pass<<<sgrid, 256, radix_smem, st>>>(s, pass, 0, 0));
     PS_LAUNCH(k_tie<<<1, 1024, 0, st>>>(s));
     PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 0, 0));
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 1));
-    for (int pass = 0; pass < 8; ++pass) PS_LAUNCH(k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 1, 1));
+    for (int pass = 0; pass < 8; ++pass)
+      PS_LAUNCH(k_radix_pass<<<sgrid, 256, kRadixBins * 4, st>>>(s, pass, 1, 1));
     PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 1));
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
-    for (int pass = 0; pass < 8; ++pass) PS_LAUNCH(k_radix_pass<<<ngrid, 256, 0, st>>>(s, pass, 1, 0));
+    for (int pass = 0; pass < 8; ++pass)
+      PS_LAUNCH(k_radix_pass<<<sgrid, 256, kRadixBins * 4, st>>>(s, pass, 1, 0));
     PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 0));
   } else {
     return PS_ERR_INVALID_ARG;  // S3-FIFO: not yet
   }
   mark(7);
   PS_LAUNCH(k_freetake<<<1, 1024, 0, st>>>(s));
-  PS_LAUNCH(k_evict<<<grid_for(s.nwords, 256, 152 * 4), 256, 0, st>>>(s));
   mark(8);
   const int nchunks = (int)((s.nwords + kBmChunk - 1) / kBmChunk);
   PS_LAUNCH(k_bm_count<<<nchunks, 1024, 0, st>>>(s));
   PS_LAUNCH(k_bm_write<<<nchunks, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_evict<<<pgrid, kThreads, 0, st>>>(s));
   mark(9);
-  PS_LAUNCH(k_insert<<<wgrid, wthreads, 0, st>>>(s));
+  PS_LAUNCH(k_insert<<<pgrid, kThreads, 0, st>>>(s));
   mark(10);
-  PS_LAUNCH(k_hist_commit<<<grid_for(R, 256, 1 << 20), 256, 0, st>>>(s));
-  PS_LAUNCH(k_claim_clear<<<wgrid, wthreads, 0, st>>>(s));
+  PS_LAUNCH(k_hist_commit<<<rgrid, 256, 0, st>>>(s));
+  PS_LAUNCH(k_claim_clear<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_finalize<<<1, 32, 0, st>>>(s));
   mark(11);
 #undef PS_LAUNCH
   if (tr) tr->launches = launches;
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* status) {
+  const int R = s.R;
+  const int rgrid = grid_for(R, 256, 1 << 20);
+  const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
+  k_validate<<<1, 1024, 0, st>>>(s, 1);
+  if (R > 0) {
+    if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
+    k_seg_carry<<<rgrid, 256, 0, st>>>(s);
+    k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s);
+  }
+  k_probe_out<<<rgrid, 256, 0, st>>>(s, out, status);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 

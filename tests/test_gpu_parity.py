@@ -184,3 +184,34 @@ def test_parity_scale_full_size(policy):
                      max_requests=spec.requests_per_step, max_tokens=maxT)
     _run(gpu, orc, steps, state_every=4, label=f"scale/{policy}")
     assert orc.stats()[:, O.STAT_NAMES.index("evicted_blocks")].sum() > 0  # reclamation was exercised
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+def test_cached_prefix_probe(policy):
+    """ps_cached_prefix (read-only) equals the oracle's leading-resident count
+    before every step, leaves the state untouched, and equals the step's own
+    hit counts for requests without in-step sharing."""
+    steps = W.fuzz_steps(51, 3, 6, 40, docs_per_group=3, doc_blocks=40, fresh_max_blocks=30)
+    gpu, orc = _pair(150, 16, 3, policy, dict(rho=(3.0,), beta=(9.0,)), max_requests=6, max_tokens=8192)
+    dev = torch.device("cuda")
+    for st in steps:
+        g = torch.from_numpy(st.groups).to(dev)
+        o = torch.from_numpy(st.offsets).to(dev)
+        t = torch.from_numpy(st.tokens if st.num_tokens else np.zeros(4, np.int32)).to(dev)
+        before = gpu.export()
+        cnt, status = gpu.cached_prefix(g, o, t)
+        torch.cuda.synchronize()
+        assert int(status.item()) == 0
+        want = orc.cached_prefix(st.groups, st.offsets, st.tokens)
+        assert np.array_equal(cnt[: st.num_requests].cpu().numpy(), want)
+        compare_state(gpu.export(), before, "probe must not change state")
+        assert gpu.step(st.now, g, o, t) == 0
+        got = gpu.fetch(st.num_requests)
+        ref = orc.step(st.now, st.groups, st.offsets, st.tokens)
+        compare_outputs(got, ref, f"step {st.index}")
+    # a bad group id is reported, not a fault
+    g = torch.tensor([7], dtype=torch.int32, device=dev)
+    o = torch.tensor([0, 32], dtype=torch.int64, device=dev)
+    t = torch.zeros(32, dtype=torch.int32, device=dev)
+    _, status = gpu.cached_prefix(g, o, t)
+    assert int(status.item()) == O.ERR_INVALID_ARG

@@ -148,3 +148,49 @@ def test_stamp_layout_orders_step_request_then_reverse_position():
     assert s(1, 5, 0) > s(1, 4, 0)
     # within a request the deeper block is released first, so it is older
     assert s(1, 4, 0) > s(1, 4, 1) > s(1, 4, 1000)
+
+
+P61 = (1 << 61) - 1
+
+
+def _unmix64(z):
+    """Inverse of the SplitMix64 output function (xorshifts and odd multipliers)."""
+    def unxs(y, s):
+        x = y
+        k = s
+        while k < 64:
+            x = y ^ (x >> s)
+            k += s
+        return x & M64
+    z = unxs(z & M64, 31)
+    z = (z * pow(0x94D049BB133111EB, -1, 1 << 64)) & M64
+    z = unxs(z, 27)
+    z = (z * pow(0xBF58476D1CE4E5B9, -1, 1 << 64)) & M64
+    return unxs(z, 30)
+
+
+def test_unmix_inverts_mix():
+    for z in (0, 1, 12345, M64, 0xDEADBEEFCAFEBABE):
+        assert _unmix64(O.mix64(z)) == z
+
+
+@pytest.mark.parametrize("bs,g", [(16, 0), (16, 5), (4, 2), (32, 1)])
+def test_chain_is_the_affine_recurrence_mod_2p61m1(bs, g):
+    """Recover C_m from each key and check C_m = Kc*C_{m-1} + D_m (mod p),
+    C_{-1} = mix(seed ^ (g+1)*phi) mod p, D_m = NH0 + Kd*NH2 (mod p), with
+    the key schedule taken from the pinned SplitMix64 stream."""
+    seed = 0x1234ABCD
+    rng = np.random.default_rng(bs + 7 * g)
+    t = rng.integers(0, 32000, 9 * bs, dtype=np.int32)
+    keys = [int(k) for k in O.chain_keys(seed, g, bs, t)]
+    stream = O.splitmix64_stream(seed, bs + 4)
+    K = [w & 0xFFFFFFFF for w in stream[: bs + 2]]
+    Kc = stream[bs + 2] % P61 or 1
+    Kd = stream[bs + 3] % P61 or 1
+    C = O.mix64(seed ^ (((g + 1) * 0x9E3779B97F4A7C15) & M64)) % P61
+    for m, key in enumerate(keys):
+        Cm = _unmix64(key) ^ (((m + 1) * 0xD1B54A32D192ED03) & M64)
+        blk = t[m * bs:(m + 1) * bs]
+        D = (O.nh(K, 0, blk, bs) + Kd * (O.nh(K, 2, blk, bs) % P61)) % P61
+        assert Cm == (Kc * C + D) % P61, m
+        C = Cm
