@@ -213,6 +213,26 @@ int32_t ps_cached_prefix(ps_handle_t* h, void* stream, int32_t num_requests, con
                          const int64_t* d_token_offsets, const int32_t* d_tokens, int32_t* d_cached_blocks,
                          int32_t* d_status);
 
+/* ps_cached_prefix() for callers that cannot allocate device memory.  The
+ * paper has no counterpart: this is a deployment convenience.  Some callers
+ * may not call cudaMalloc or touch a workspace they do not own -- code inside
+ * a CUDA graph capture region, code under a framework whose allocator owns
+ * every device allocation, or a thread that only queries a cache another
+ * thread steps.  This variant computes the same counts as ps_cached_prefix()
+ * with its scratch in one fixed array compiled into the library (about
+ * 2.3 MB, held on every GPU that loads the library until the process exits).
+ * It allocates nothing; the caller passes inputs and outputs as for
+ * ps_cached_prefix().  Limits of one call: 4096 requests (more returns
+ * PS_ERR_CAPACITY at once) and 131072 full blocks (more tokens than
+ * 131072 * block_size make d_status PS_ERR_INVALID_ARG).  The first call on
+ * a device looks up the array's device address for that device; make that
+ * first call before any stream capture.  Every call on a device shares the
+ * one array: calls that overlap on the GPU (other streams, other handles,
+ * other threads) race and must be serialized by the caller. */
+int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_t num_requests, const int32_t* d_group_ids,
+                                 const int64_t* d_token_offsets, const int32_t* d_tokens, int32_t* d_cached_blocks,
+                                 int32_t* d_status);
+
 /* Profiling hook.  When enabled, ps_step() records a CUDA event on its
  * stream before each of its PS_NUM_STAGES stages and after the last one:
  *   0 validate, 1 hash + lookup, 2 claims + orphans, 3 grant + in-step hits,

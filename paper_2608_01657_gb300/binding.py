@@ -31,7 +31,8 @@ PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE = 1, 2
 
 EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_stats", "ps_clear_status",
             "ps_reset", "ps_destroy", "ps_status_string", "ps_export_state", "ps_export_history",
-            "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times", "ps_cached_prefix")
+            "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times", "ps_cached_prefix",
+            "ps_cached_prefix_noalloc")
 PS_NUM_STAGES = 11
 STAGE_NAMES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
                "freetake_evict", "id_lists", "insert", "commit")
@@ -107,6 +108,8 @@ def load():
     L.ps_export_ghost.argtypes = [vp, vp, vp, vp, vp, i64]
     L.ps_cached_prefix.restype = i32
     L.ps_cached_prefix.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
+    L.ps_cached_prefix_noalloc.restype = i32
+    L.ps_cached_prefix_noalloc.argtypes = [vp, vp, i32, vp, vp, vp, vp, vp]
     L.ps_set_stage_timing.restype = i32
     L.ps_set_stage_timing.argtypes = [vp, i32]
     L.ps_get_stage_times.restype = i32
@@ -240,6 +243,13 @@ class Cache:
         if rc != PS_OK:
             raise RuntimeError(f"ps_cached_prefix failed ({rc})")
         return out, status
+
+    def cached_prefix_noalloc(self, groups, offsets, tokens, out, status, stream=None) -> int:
+        """The same probe with the library's fixed scratch array: allocates
+        nothing (the caller supplies ``out`` and ``status``).  Returns the rc."""
+        R = int(groups.shape[0])
+        return load().ps_cached_prefix_noalloc(self._h, _stream_ptr(stream), R, _ptr(groups), _ptr(offsets),
+                                               _ptr(tokens), _ptr(out), _ptr(status))
 
     def step_host(self, now: int, groups, offsets, tokens, contracts=None, prefixes=None, stream=None,
                   out: Optional[dict] = None) -> dict:

@@ -245,6 +245,11 @@ inline cudaStream_t as_stream(void* p) { return reinterpret_cast<cudaStream_t>(p
 
 }  // namespace
 
+namespace ps {
+// Device state of a handle, for entry points defined outside this file.
+const DevState* handle_state(const ps_handle_t* h) { return &h->base; }
+}  // namespace ps
+
 extern "C" {
 
 size_t ps_workspace_bytes(int64_t capacity_blocks, int32_t block_size, int32_t num_groups, const ps_params_t* params,
