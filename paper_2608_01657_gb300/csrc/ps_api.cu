@@ -118,6 +118,9 @@ struct Carver {
 
 struct Dims {
   int64_t N, max_tokens, max_blocks, nwords, hist_cap, max_segments;
+  int64_t s3_small_cap, s3_ghost_cap;
+  uint64_t ghost_ring_cap;
+  uint32_t gh_log2;
   int32_t bs, G, C, max_requests;
   uint32_t tb_log2, cl_log2, hist_log2;
 };
@@ -138,6 +141,12 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   d.hist_log2 = log2_pow2_at_least((uint64_t)(2 * (P->history_capacity + max_requests)));
   if (d.hist_log2 < 1) d.hist_log2 = 1;
   d.hist_cap = P->history_capacity;
+  // S3-FIFO: small queue max(1, floor(N * pct / 100)); ghost holds the rest
+  d.s3_small_cap = N * P->s3_small_pct / 100 > 1 ? N * P->s3_small_pct / 100 : 1;
+  d.s3_ghost_cap = N - d.s3_small_cap;
+  d.gh_log2 = log2_pow2_at_least((uint64_t)((d.s3_ghost_cap + 3) / 4 > 1 ? (d.s3_ghost_cap + 3) / 4 : 1));
+  if (d.gh_log2 < 1) d.gh_log2 = 1;
+  d.ghost_ring_cap = 1ull << log2_pow2_at_least((uint64_t)(2 * d.s3_ghost_cap + 64));
   return d;
 }
 
@@ -163,6 +172,14 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.blk_inval = cv.take<uint32_t>(N);
   const size_t zero_end = cv.off;  // everything above starts zeroed
   t.res_bits = cv.take<uint32_t>((size_t)d.nwords);
+  t.s3_prev = cv.take<uint32_t>(N);
+  t.s3_next = cv.take<uint32_t>(N);
+  t.s3_inval = cv.take<uint32_t>(B);
+  t.ghost_map = cv.take<TableEntry>((size_t)kTableWays << d.gh_log2);
+  t.ghost_ovf = cv.take<uint32_t>((size_t)1 << d.gh_log2);
+  t.ghost_ring_key = cv.take<uint64_t>((size_t)d.ghost_ring_cap);
+  t.ghost_ring_grp = cv.take<uint32_t>((size_t)d.ghost_ring_cap);
+  t.ghost_ring_seq = cv.take<uint64_t>((size_t)d.ghost_ring_cap);
   t.table = cv.take<TableEntry>((size_t)kTableWays << d.tb_log2);
   t.table_ovf = cv.take<uint32_t>((size_t)1 << d.tb_log2);
   t.ledger = cv.take<int64_t>(G * d.C);
@@ -237,6 +254,12 @@ int32_t init_state(ps_handle* h, cudaStream_t st) {
   if (cudaMemsetAsync(h->workspace, 0, h->workspace_bytes, st) != cudaSuccess) return PS_ERR_CUDA;
   if (cudaMemsetAsync(s.table, 0xFF, sizeof(TableEntry) * ((size_t)kTableWays << s.tb_nbuckets_log2), st) != cudaSuccess)
     return PS_ERR_CUDA;
+  if (cudaMemsetAsync(s.ghost_map, 0xFF, sizeof(TableEntry) * ((size_t)kTableWays << s.gh_nbuckets_log2), st) !=
+      cudaSuccess)
+    return PS_ERR_CUDA;
+  if (cudaMemsetAsync(s.s3_prev, 0xFF, sizeof(uint32_t) * (size_t)s.N, st) != cudaSuccess ||
+      cudaMemsetAsync(s.s3_next, 0xFF, sizeof(uint32_t) * (size_t)s.N, st) != cudaSuccess)
+    return PS_ERR_CUDA;
   launch_init(s, st);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
@@ -267,7 +290,6 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   if (!out) return PS_ERR_INVALID_ARG;
   *out = nullptr;
   if (check_params(capacity_blocks, block_size, num_groups, policy, params) != PS_OK) return PS_ERR_INVALID_ARG;
-  if (policy == PS_S3FIFO) return PS_ERR_INVALID_ARG;  // not built yet
   const size_t need = ps_workspace_bytes(capacity_blocks, block_size, num_groups, params, max_requests, max_tokens);
   if (need == 0 || !d_workspace || workspace_bytes < need || (reinterpret_cast<uintptr_t>(d_workspace) & 255))
     return PS_ERR_INVALID_ARG;
@@ -288,6 +310,8 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
     if (c < s.C && params->rho_fp[c] < s.rho_min) s.rho_min = params->rho_fp[c];
   }
   s.s3_small_pct = params->s3_small_pct; s.s3_freq_cap = params->s3_freq_cap; s.s3_move_min = params->s3_move_min_freq;
+  s.s3_small_cap = d.s3_small_cap; s.s3_ghost_cap = d.s3_ghost_cap;
+  s.gh_nbuckets_log2 = d.gh_log2; s.ghost_ring_cap = d.ghost_ring_cap;
   s.max_requests = max_requests; s.max_tokens = max_tokens; s.max_blocks = d.max_blocks;
   s.history_capacity = params->history_capacity;
   s.tb_nbuckets_log2 = d.tb_log2; s.cl_nbuckets_log2 = d.cl_log2; s.hist_cap_log2 = d.hist_log2;
@@ -523,8 +547,28 @@ int64_t ps_export_history(ps_handle_t* h, void* stream, int32_t* h_group, uint64
 }
 
 int64_t ps_export_ghost(ps_handle_t* h, void* stream, int32_t* h_group, uint64_t* h_key, uint64_t* h_seq, int64_t cap) {
-  (void)h; (void)stream; (void)h_group; (void)h_key; (void)h_seq; (void)cap;
-  return 0;
+  if (!h) return PS_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream);
+  const DevState& s = h->base;
+  // copy the ghost map and the ring's sequence numbers, read them here
+  const size_t n = (size_t)kTableWays << s.gh_nbuckets_log2;
+  std::vector<TableEntry> map(n);
+  std::vector<uint64_t> seq((size_t)s.ghost_ring_cap);
+  if (cudaMemcpyAsync(map.data(), s.ghost_map, n * sizeof(TableEntry), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaMemcpyAsync(seq.data(), s.ghost_ring_seq, seq.size() * 8, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return PS_ERR_CUDA;
+  int64_t k = 0;
+  for (const TableEntry& e : map) {
+    if (e.blk == kNone) continue;
+    if (h_group && k < cap) {
+      h_group[k] = (int32_t)e.grp;
+      h_key[k] = e.key;
+      h_seq[k] = seq[e.blk];
+    }
+    ++k;
+  }
+  return k;
 }
 
 }  // extern "C"

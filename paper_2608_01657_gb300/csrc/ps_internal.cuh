@@ -67,10 +67,10 @@ struct Ctl {
   int64_t n_resident;
   int64_t hist_live;
   uint64_t s3_ctr, ghost_ctr;
-  int64_t s3_nS, s3_nM;
-  uint64_t ringS_head, ringS_tail, ringM_head, ringM_tail;
-  uint64_t ghost_head, ghost_tail;
-  int64_t ghost_live;
+  int64_t s3_nS, s3_nM;             // queue sizes (pinned members included)
+  uint32_t s3_head[2], s3_tail[2];  // small (0) and main (1) queues: tail = oldest
+  uint64_t ghost_head, ghost_tail;  // ghost FIFO ring positions
+  int64_t ghost_live;               // live ghost entries
   // per step
   int32_t status;          // this step's status
   int32_t pad1;
@@ -80,6 +80,8 @@ struct Ctl {
   int64_t n_evicted, n_alloc, n_victims_marked;
   int64_t m_fb;            // prefixshield: victims left to the global fallback
   int32_t sel_ntie, sel_k; // prefixshield tie bookkeeping
+  int64_t s3_pinned[2];    // pinned members of each S3-FIFO queue this step
+  int64_t s3_ninval;       // invalidated blocks to unlink this step
   uint32_t ticket;         // last-block-done counter for the radix passes
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
 };
@@ -107,6 +109,9 @@ struct DevState {
   int64_t rho[PS_MAX_CONTRACTS], beta[PS_MAX_CONTRACTS];
   int64_t rho_min;
   int32_t s3_small_pct, s3_freq_cap, s3_move_min;
+  int64_t s3_small_cap, s3_ghost_cap;
+  uint32_t gh_nbuckets_log2;
+  uint64_t ghost_ring_cap;  // power of two
   int32_t max_requests;
   int64_t max_tokens, max_blocks;
   int64_t history_capacity;
@@ -129,6 +134,14 @@ struct DevState {
   uint32_t* blk_pin;       // step tag: hit in this step
   uint32_t* blk_inval;     // step tag: invalidated in this step
   uint32_t* res_bits;      // resident bitmap
+  uint32_t* s3_prev;       // S3-FIFO queue links: toward the tail (older)
+  uint32_t* s3_next;       //                      toward the head (newer)
+  uint32_t* s3_inval;      // blocks invalidated this step (to unlink)
+  TableEntry* ghost_map;   // (group, key) -> ring position (in blk)
+  uint32_t* ghost_ovf;
+  uint64_t* ghost_ring_key;
+  uint32_t* ghost_ring_grp;
+  uint64_t* ghost_ring_seq;
   TableEntry* table;
   uint32_t* table_ovf;     // per bucket: live keys probing past it
   int64_t* ledger;         // B_{g,c}, fixed point
@@ -218,6 +231,9 @@ struct StepTrace {
 };
 void launch_init(const DevState& s, cudaStream_t st);
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr);
+// S3-FIFO (ps_s3fifo.cu)
+void launch_s3_evict(const DevState& s, cudaStream_t st);
+void launch_s3_insert(const DevState& s, cudaStream_t st);
 // Read-only cached-prefix probe; 'out' receives h_i per request, 'status' the outcome.
 int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* status);
 

@@ -257,6 +257,8 @@ __global__ void k_init_ctl(DevState s) {
   if (threadIdx.x == 0 && blockIdx.x == 0) {
     Ctl c{};
     c.step = 1;
+    c.s3_head[0] = c.s3_head[1] = kNone;
+    c.s3_tail[0] = c.s3_tail[1] = kNone;
     *s.ctl = c;
   }
   for (int i = threadIdx.x; i < s.G * s.C; i += blockDim.x) s.ledger[i] = s.beta[i % s.C];
@@ -325,6 +327,7 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
       c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
       c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
       c->internal_error = 0;
+      c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
     }
   }
 }
@@ -479,7 +482,9 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
     PosRef r;
     pos_ref(s, t, &r);
     if (r.m < s.rq_h[r.i]) {
-      newpin = atomicExch(s.blk_pin + s.pos_blk[t], step32) != step32;
+      const uint32_t b = s.pos_blk[t];
+      newpin = atomicExch(s.blk_pin + b, step32) != step32;
+      if (newpin && s.policy == PS_S3FIFO) atomic_add_i64(&c->s3_pinned[(s.blk_flags[b] >> 1) & 1], 1);
       s.pos_claim[t] = kNone;
     } else {
       s.pos_claim[t] = claim_insert(s, s.pos_key[t], r.i);
@@ -541,6 +546,7 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
       if (b != kNone && ldcg_u32(s.blk_pin + b) != step32 && atomicExch(s.blk_inval + b, step32) != step32) {
         drop_block(s, b, PS_STAT_INVALIDATED_BLOCKS);
         atomicOr(s.bm_inval + (b >> 5), 1u << (b & 31));
+        if (s.policy == PS_S3FIFO) s.s3_inval[atomicAdd(reinterpret_cast<unsigned long long*>(&c->s3_ninval), 1ull)] = b;
         inv = true;
       }
     }
@@ -1342,7 +1348,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   PS_LAUNCH(k_touch<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
   mark(6);
-  PS_LAUNCH(k_cand<<<ngrid, 256, 0, st>>>(s));
+  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<ngrid, 256, 0, st>>>(s));
   if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));
     for (int pass = 0; pass < 8; ++pass)
@@ -1359,7 +1365,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
       PS_LAUNCH(k_radix_pass<<<sgrid, 256, kRadixBins * 4, st>>>(s, pass, 1, 0));
     PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 0));
   } else {
-    return PS_ERR_INVALID_ARG;  // S3-FIFO: not yet
+    PS_LAUNCH(launch_s3_evict(s, st));
   }
   mark(7);
   PS_LAUNCH(k_freetake<<<1, 1024, 0, st>>>(s));
@@ -1370,6 +1376,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   PS_LAUNCH(k_evict<<<pgrid, kThreads, 0, st>>>(s));
   mark(9);
   PS_LAUNCH(k_insert<<<pgrid, kThreads, 0, st>>>(s));
+  if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));
   mark(10);
   PS_LAUNCH(k_hist_commit<<<rgrid, 256, 0, st>>>(s));
   PS_LAUNCH(k_claim_clear<<<pgrid, kThreads, 0, st>>>(s));

@@ -40,11 +40,11 @@ def _run(gpu, orc, steps, state_every=1, s3=False, label=""):
         want = orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts, st.prefixes)
         compare_outputs(got, want, f"{label} step {k}")
         if state_every and (k % state_every == 0 or k == len(steps) - 1):
-            compare_state(gpu.export(), orc.export(), f"{label} step {k}", s3=s3)
+            compare_state(gpu.export(), orc.export(), f"{label} step {k}", s3=s3 or gpu.policy == "s3fifo")
     assert np.array_equal(gpu.stats(), orc.stats()), f"{label}: stats differ"
 
 
-GPU_POLICIES = ["lru", "prefixshield"]
+GPU_POLICIES = ["lru", "s3fifo", "prefixshield"]
 
 
 @pytest.mark.parametrize("policy", GPU_POLICIES)
@@ -63,6 +63,23 @@ def test_parity_fuzz(policy, seed, N, G, R, contracts, prefixes, flags):
     kw = dict(rho=(2.0, 1.5, 1.0), beta=(6.0, 5.0, 4.0), flags=flags, contract_of_group=[g % 3 for g in range(G)])
     gpu, orc = _pair(N, 16, G, policy, kw, max_requests=R, max_tokens=4096)
     _run(gpu, orc, steps, label=f"fuzz{seed}/{policy}")
+
+
+@pytest.mark.parametrize("policy,fname", [("lru", "lru_hand_trace.txt"), ("s3fifo", "s3fifo_hand_trace.txt")])
+def test_parity_hand_traces(policy, fname):
+    """The hand-traced golden traces, GPU against oracle (which the traces pin)."""
+    from _util import make_step, obj_tokens, params_line, parse_trace
+    steps, _ = parse_trace(fname)
+    pr = params_line(fname)
+    kw = dict(rho=(1000.0,), beta=(1000.0,))
+    if policy == "s3fifo":
+        kw.update(s3_small_pct=pr["small_pct"], s3_freq_cap=pr["freq_cap"], s3_move_min_freq=pr["move_min_freq"])
+    gpu, orc = _pair(pr["N"], 16, 1, policy, kw, max_requests=4, max_tokens=256)
+    seq = []
+    for si, (reqs, _, _) in enumerate(steps):
+        g, o, t, _ = make_step([obj_tokens(n) for n in reqs])
+        seq.append(W.Step(index=si, now=si + 1, groups=g, offsets=o, tokens=t))
+    _run(gpu, orc, seq, label=fname)
 
 
 @pytest.mark.parametrize("bs", [2, 4, 8, 32, 64])
