@@ -91,7 +91,8 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            time.sleep(0.5)  # let the sampler start before the timed region
         except Exception:
             self.proc = None
         return self
@@ -99,6 +100,7 @@ class ClockSampler:
     def __exit__(self, *a):
         self.lines = []
         if self.proc is not None:
+            time.sleep(0.25)  # one more sample after the timed region
             self.proc.terminate()
             try:
                 out, _ = self.proc.communicate(timeout=5)

@@ -219,16 +219,16 @@ __device__ uint32_t claim_insert(const DevState& s, uint64_t key, uint32_t req) 
 }
 
 // ---- block state changes -----------------------------------------------------
-// Remove a resident block from the pool (eviction or invalidation).
-__device__ void drop_block(const DevState& s, uint32_t b, int stat_kind) {
+// Remove a resident block from the pool (eviction or invalidation); returns
+// its group.  Callers account the per-group statistics, warp-aggregated.
+__device__ uint32_t drop_block(const DevState& s, uint32_t b) {
   table_delete(s, b);
-  const int g = s.blk_group[b];
+  const uint32_t g = s.blk_group[b];
   const uint8_t fl = s.blk_flags[b];
   s.blk_flags[b] = 0;
   atomicAnd(s.res_bits + (b >> 5), ~(1u << (b & 31)));
-  atomic_add_i64(stat_ptr(s, g, stat_kind), 1);
-  atomic_add_i64(stat_ptr(s, g, PS_STAT_RESIDENT_BLOCKS), -1);
   if (s.policy == PS_S3FIFO) atomic_add_i64((fl & 2) ? &s.ctl->s3_nM : &s.ctl->s3_nS, -1);
+  return g;
 }
 
 // Position -> (request, position within the request).
@@ -536,6 +536,7 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const uint32_t step32 = (uint32_t)c->step;
   bool inv = false;
+  uint32_t ginv = 0;
   PosRef r;
   if (pos_ref(s, pos, &r)) {
     const int h = s.rq_h[r.i];
@@ -544,13 +545,15 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
     if (r.m > h) {
       const uint32_t b = s.pos_blk[pos];
       if (b != kNone && ldcg_u32(s.blk_pin + b) != step32 && atomicExch(s.blk_inval + b, step32) != step32) {
-        drop_block(s, b, PS_STAT_INVALIDATED_BLOCKS);
+        ginv = drop_block(s, b);
         atomicOr(s.bm_inval + (b >> 5), 1u << (b & 31));
         if (s.policy == PS_S3FIFO) s.s3_inval[atomicAdd(reinterpret_cast<unsigned long long*>(&c->s3_ninval), 1ull)] = b;
         inv = true;
       }
     }
   }
+  agg_stat(s, ginv, PS_STAT_INVALIDATED_BLOCKS, 1, inv);
+  agg_stat(s, ginv, PS_STAT_RESIDENT_BLOCKS, -1, inv);
   const int ni = __popc(__ballot_sync(kFull, inv));
   if (lane_id() == 0 && ni) {
     atomic_add_i64(&c->n_inval, ni);
@@ -1095,11 +1098,12 @@ __global__ void k_mark(DevState s, int single, int fallback) {
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
 }
 
-// TakeTrueFree (Alg. 2): the ftake smallest free block ids, plus the victims,
-// form the allocated set (one CTA, contiguous word ranges per thread).
+// TakeTrueFree (Alg. 2): the ftake smallest free block ids (one CTA,
+// contiguous word ranges per thread).  With the victims they form the
+// allocated set; the id-list compaction takes their union.
 __global__ void __launch_bounds__(1024) k_freetake(DevState s) {
   Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
+  if (c->status != PS_OK || c->ftake == 0) return;
   const int64_t ftake = c->ftake;
   const int64_t nw = s.nwords;
   const int64_t per = (nw + blockDim.x - 1) / blockDim.x;
@@ -1126,7 +1130,7 @@ __global__ void __launch_bounds__(1024) k_freetake(DevState s) {
         ++before;
       }
     }
-    s.bm_alloc[w] = take | s.bm_victim[w];
+    s.bm_alloc[w] = take;
   }
 }
 
@@ -1139,7 +1143,9 @@ __global__ void __launch_bounds__(1024) k_bm_count(DevState s) {
   const uint32_t* bms[3] = {s.bm_alloc, s.bm_victim, s.bm_inval};
   const int nchunks = gridDim.x;
   for (int k = 0; k < 3; ++k) {
-    const int v = w < s.nwords ? __popc(bms[k][w]) : 0;
+    uint32_t bits = w < s.nwords ? bms[k][w] : 0u;
+    if (k == 0 && w < s.nwords) bits |= s.bm_victim[w];
+    const int v = __popc(bits);
     const int t = block_sum(v);
     if (threadIdx.x == 0) s.bm_chunk_cnt[k * nchunks + blockIdx.x] = t;
   }
@@ -1154,7 +1160,8 @@ __global__ void __launch_bounds__(1024) k_bm_write(DevState s) {
     int base = 0;
     for (int j = threadIdx.x; j < blockIdx.x; j += blockDim.x) base += s.bm_chunk_cnt[k * nchunks + j];
     base = block_sum(base);
-    const uint32_t bits = w < s.nwords ? bms[k][w] : 0u;
+    uint32_t bits = w < s.nwords ? bms[k][w] : 0u;
+    if (k == 0 && w < s.nwords) bits |= s.bm_victim[w];
     int tot;
     const int ex = block_excl_scan(__popc(bits), &tot);
     int o = base + ex;
@@ -1180,7 +1187,10 @@ __global__ void __launch_bounds__(kThreads) k_evict(DevState s) {
   const int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const int64_t nv = c->n_evicted;
   const bool act = v < nv && v < s.max_blocks;
-  if (act) drop_block(s, (uint32_t)s.out.evicted_ids[v], PS_STAT_EVICTED_BLOCKS);
+  uint32_t g = 0;
+  if (act) g = drop_block(s, (uint32_t)s.out.evicted_ids[v]);
+  agg_stat(s, g, PS_STAT_EVICTED_BLOCKS, 1, act);
+  agg_stat(s, g, PS_STAT_RESIDENT_BLOCKS, -1, act);
   const int k = __popc(__ballot_sync(kFull, act));
   if (lane_id() == 0 && k) atomic_add_i64(&c->n_resident, -k);
 }
