@@ -82,6 +82,7 @@ struct Ctl {
   int32_t sel_ntie, sel_k; // prefixshield tie bookkeeping
   int64_t s3_pinned[2];    // pinned members of each S3-FIFO queue this step
   int64_t s3_ninval;       // invalidated blocks to unlink this step
+  uint64_t fb_kmin, fb_kmax;  // key range of candidates the debt phase left
   uint32_t ticket;         // last-block-done counter for the radix passes
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
 };

@@ -17,6 +17,7 @@ namespace ps {
 constexpr unsigned kFull = 0xFFFFFFFFu;
 constexpr int kWarpsPerCta = 8;   // warp-per-segment hashing kernel
 constexpr int kThreads = 256;     // position-parallel kernels
+constexpr int kRadixSmemRows = 48;  // radix rows counted in shared memory (48 KB)
 
 // ---------------------------------------------------------------------------
 // small device helpers
@@ -328,6 +329,7 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
       c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
       c->internal_error = 0;
       c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
+      c->fb_kmin = ~0ull; c->fb_kmax = 0;
     }
   }
 }
@@ -342,8 +344,8 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
 // pair sums are reduced with xor shuffles and routed to lane = block.  The
 // chain C_m = Kc C_{m-1} + D_m (mod 2^61-1) is a composition of affine maps,
 // so a warp scan gives every block its chain value relative to the segment
-// start (B_m, with the value before the segment taken as 0); k_seg_carry then
-// supplies the true value entering each segment.
+// start (B_m, with the value before the segment taken as 0); k_keys_lookup
+// then folds in the true value entering the segment.
 template <int PPB>
 __global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash(DevState s) {
   extern __shared__ int32_t smem_tokens[];
@@ -431,34 +433,23 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash(DevState s) {
   if (lane == 0) s.seg_tot[seg] = carry;
 }
 
-// Chain value entering each segment, serially over a request's segments
-// (thread per request): C = Kc^len C + B_end.
-__global__ void k_seg_carry(DevState s) {
-  const Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= s.R) return;
-  const int n = s.rq_n[i];
-  const int64_t sb = s.rq_sbase[i];
-  uint64_t C = red61(chain_seed(s.hash_seed, s.in_group[i]));
-  for (int j = 0; j * kSegBlocks < n; ++j) {
-    s.seg_cin[sb + j] = C;
-    const int len = tmin(kSegBlocks, n - j * kSegBlocks);
-    C = add61(mul61(s.kc_pow[len], C), s.seg_tot[sb + j]);
-  }
-}
-
 // Stage 2: block keys and the longest cached prefix (n_cached of Alg. 1),
-// thread per position: key_m = mix(C_m ^ (m+1) c), C_m = Kc^(k+1) C_in + B_m,
-// then a table probe; a miss lowers the request's h_i to its position.
+// thread per position: C_in = the chain value entering the position's
+// segment (C = Kc^256 C + B_end over the request's earlier segments),
+// key_m = mix(C_m ^ (m+1) c) with C_m = Kc^(k+1) C_in + B_m, then a table
+// probe; a miss lowers the request's h_i to its position.
 __global__ void __launch_bounds__(kThreads) k_keys_lookup(DevState s) {
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   PosRef r;
   if (!pos_ref(s, pos, &r)) return;
-  const int64_t seg = s.rq_sbase[r.i] + r.m / kSegBlocks;
-  const uint64_t C = add61(mul61(s.kc_pow[r.m % kSegBlocks + 1], s.seg_cin[seg]), s.pos_key[pos]);
+  // chain value entering this position's segment: fold the earlier segments
+  const int64_t sb = s.rq_sbase[r.i];
+  const int js = r.m / kSegBlocks;
+  uint64_t cin = red61(chain_seed(s.hash_seed, s.in_group[r.i]));
+  for (int j = 0; j < js; ++j) cin = add61(mul61(s.kc_pow[kSegBlocks], cin), s.seg_tot[sb + j]);
+  const uint64_t C = add61(mul61(s.kc_pow[r.m % kSegBlocks + 1], cin), s.pos_key[pos]);
   const uint64_t key = fix_reserved(mix64(C ^ ((uint64_t)(r.m + 1) * 0xD1B54A32D192ED03ull)));
   s.pos_key[pos] = key;
   const uint32_t blk = table_find(s, key, (uint32_t)s.in_group[r.i]);
@@ -809,41 +800,35 @@ __global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
 // the no-segmentation ablation) and the stamp for lru.  Also the smallest
 // and largest key of every segment, so the radix select can skip the bytes
 // its candidates share.
-__global__ void k_cand(DevState s) {
+__global__ void __launch_bounds__(256) k_cand(DevState s) {
+  __shared__ unsigned long long s_min[PS_MAX_GROUPS], s_max[PS_MAX_GROUPS];
+  __shared__ unsigned int s_cnt[PS_MAX_GROUPS];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const uint32_t step32 = (uint32_t)c->step;
   const bool ps = s.policy == PS_PREFIXSHIELD;
   const bool seg = ps && !(s.flags & PS_FLAG_NO_SEGMENTATION);
-  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t b = b0 + threadIdx.x;
-    bool cand = false;
-    uint32_t g = 0;
+  const int nseg = ps ? s.G : 1;
+  for (int g = threadIdx.x; g < nseg; g += blockDim.x) { s_min[g] = ~0ull; s_max[g] = 0; s_cnt[g] = 0; }
+  __syncthreads();
+  for (int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; b < s.N; b += (int64_t)gridDim.x * blockDim.x) {
     uint64_t key = ~0ull;
-    if (b < s.N) {
-      cand = (s.blk_flags[b] & 1) && s.blk_pin[b] != step32;
-      if (cand) {
-        key = s.blk_stamp[b];
-        if (seg) key |= (uint64_t)s.blk_klass[b] << 62;
-        g = ps ? s.blk_group[b] : 0;
-      }
-      s.csk[b] = key;
+    if ((s.blk_flags[b] & 1) && s.blk_pin[b] != step32) {
+      key = s.blk_stamp[b];
+      if (seg) key |= (uint64_t)s.blk_klass[b] << 62;
+      const uint32_t g = ps ? s.blk_group[b] : 0;
+      atomicMin(&s_min[g], (unsigned long long)key);
+      atomicMax(&s_max[g], (unsigned long long)key);
+      atomicAdd(&s_cnt[g], 1u);
     }
-    const unsigned act = __ballot_sync(kFull, cand);
-    if (cand) {
-      const unsigned peers = __match_any_sync(act, g);
-      uint64_t mn = key, mx = key;
-      for (unsigned m = peers; m; m &= m - 1) {
-        const uint64_t v = __shfl_sync(peers, key, __ffs(m) - 1);
-        mn = tmin(mn, v);
-        mx = tmax(mx, v);
-      }
-      if (lane_id() == __ffs(peers) - 1) {
-        if (ps) atomic_add_i64(s.grp_qsize + g, __popc(peers));
-        atomicMin(reinterpret_cast<unsigned long long*>(&s.sel[g].kmin), (unsigned long long)mn);
-        atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[g].kmax), (unsigned long long)mx);
-      }
-    }
+    s.csk[b] = key;
+  }
+  __syncthreads();
+  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+    if (!s_cnt[g]) continue;
+    if (ps) atomic_add_i64(s.grp_qsize + g, s_cnt[g]);
+    atomicMin(reinterpret_cast<unsigned long long*>(&s.sel[g].kmin), s_min[g]);
+    atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[g].kmax), s_max[g]);
   }
 }
 
@@ -857,10 +842,10 @@ __global__ void k_sel_single(DevState s, int fallback) {
   z.rank = m;
   z.active = m > 0;
   z.incl = 1;
-  // the fallback selects among the candidates the debt phase left over all
-  // groups: its key range is not known, so it starts from the top byte
-  z.kmin = fallback ? 0 : old.kmin;
-  z.kmax = fallback ? ~0ull : old.kmax;
+  // the fallback selects among the candidates the debt phase left, whose key
+  // range the debt phase's marking pass recorded
+  z.kmin = fallback ? c->fb_kmin : old.kmin;
+  z.kmax = fallback ? c->fb_kmax : old.kmax;
   s.sel[0] = z;
 }
 
@@ -921,10 +906,33 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     __syncthreads();
     pmax = s_pmax;
   }
-  int64_t lo = eps + 1, hi = pmax;  // tau = max{t > eps : count_gt(t - 1) >= m}
+  // tau = max{t in [eps+1, pmax] : count_gt(t - 1) >= m}.  Each round every
+  // thread tests one of blockDim thresholds spread over the interval.
+  __shared__ int s_best;
+  int64_t lo = eps + 1, hi = pmax;
+  const int nt = blockDim.x;
   while (lo < hi) {
-    const int64_t mid = lo + (hi - lo + 1) / 2;
-    if (count_gt(mid - 1) >= m) lo = mid; else hi = mid - 1;
+    const int64_t span = hi - lo;
+    const int64_t t = lo + 1 + (int64_t)(((__int128)(span - 1) * threadIdx.x) / (nt - 1));
+    int64_t cnt = 0;
+    for (int g = 0; g < G; ++g) {
+      const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
+      if (P > t - 1 && d > 0) cnt += tmin<int64_t>(q, (P - t) / d + 1);
+    }
+    if (threadIdx.x == 0) s_best = -1;
+    __syncthreads();
+    if (cnt >= m) atomicMax(&s_best, (int)threadIdx.x);
+    __syncthreads();
+    const int J = s_best;
+    __syncthreads();
+    if (J < 0) {
+      hi = lo;
+    } else {
+      const int64_t tj = lo + 1 + (int64_t)(((__int128)(span - 1) * J) / (nt - 1));
+      const int64_t tn = J + 1 < nt ? lo + 1 + (int64_t)(((__int128)(span - 1) * (J + 1)) / (nt - 1)) : hi + 1;
+      lo = tj;
+      hi = tn - 1;
+    }
   }
   const int64_t tau = lo;
   int64_t above = 0, ntie = 0;
@@ -963,23 +971,31 @@ __device__ __forceinline__ bool digit_known(const SelSeg& ss, int shift) {
 
 __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int single, int fallback) {
   extern __shared__ uint32_t shist[];
+  __shared__ int16_t row_of[PS_MAX_GROUPS];
+  __shared__ int16_t seg_of_row[PS_MAX_GROUPS];
+  __shared__ int s_nrows;
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const int nseg = single ? 1 : s.G;
   if (single && !s.sel[0].active) return;
   const int shift = 64 - kRadixBits * (pass + 1);
-  const bool use_smem = nseg <= 64;
-  __shared__ int s_work;
-  if (threadIdx.x == 0) s_work = 0;
-  __syncthreads();
-  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
-    const SelSeg ss = s.sel[g];
-    if (ss.active && !digit_known(ss, shift)) s_work = 1;
+  // segments that still count at this digit get a histogram row
+  if (threadIdx.x == 0) {
+    int k = 0;
+    for (int g = 0; g < nseg; ++g) {
+      const SelSeg ss = s.sel[g];
+      const bool counts = ss.active && !digit_known(ss, shift);
+      row_of[g] = counts ? (int16_t)k : (int16_t)-1;
+      if (counts) seg_of_row[k++] = (int16_t)g;
+    }
+    s_nrows = k;
   }
   __syncthreads();
-  if (s_work) {
+  const int nrows = s_nrows;
+  const bool use_smem = nrows <= kRadixSmemRows;
+  if (nrows > 0) {
     if (use_smem)
-      for (int k = threadIdx.x; k < nseg * kRadixBins; k += blockDim.x) shist[k] = 0;
+      for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x) shist[k] = 0;
     __syncthreads();
     for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
       const int64_t b = b0 + threadIdx.x;
@@ -989,10 +1005,14 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
         const uint64_t key = s.csk[b];
         if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
           const int seg = single ? 0 : s.blk_group[b];
-          const SelSeg ss = s.sel[seg];
-          if (ss.active && (key & ss.mask) == ss.prefix && !digit_known(ss, shift)) {
-            act = true;
-            idx = (uint32_t)seg * kRadixBins + (uint32_t)((key >> shift) & (kRadixBins - 1));
+          const int row = row_of[seg];
+          if (row >= 0) {
+            const SelSeg ss = s.sel[seg];
+            if ((key & ss.mask) == ss.prefix) {
+              act = true;
+              const uint32_t digit = (uint32_t)((key >> shift) & (kRadixBins - 1));
+              idx = use_smem ? (uint32_t)row * kRadixBins + digit : (uint32_t)seg * kRadixBins + digit;
+            }
           }
         }
       }
@@ -1000,8 +1020,11 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
     }
     __syncthreads();
     if (use_smem)
-      for (int k = threadIdx.x; k < nseg * kRadixBins; k += blockDim.x)
-        if (shist[k]) atomicAdd(s.hist_bins + k, shist[k]);
+      for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x) {
+        if (!shist[k]) continue;
+        const int seg = seg_of_row[k / kRadixBins];
+        atomicAdd(s.hist_bins + (size_t)seg * kRadixBins + (k % kRadixBins), shist[k]);
+      }
   }
   __shared__ bool last;
   __threadfence();
@@ -1076,11 +1099,18 @@ __global__ void __launch_bounds__(1024) k_tie(DevState s) {
 }
 
 // Mark victims: keys below (or equal to, if incl) the located threshold.
-__global__ void k_mark(DevState s, int single, int fallback) {
+// The per-group pass also records the key range of the candidates it leaves,
+// for the global fallback that may follow.
+__global__ void __launch_bounds__(256) k_mark(DevState s, int single, int fallback) {
+  __shared__ unsigned long long s_rng[2];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   if (single && !s.sel[0].active) return;
+  const bool track = !single;
+  if (threadIdx.x == 0) { s_rng[0] = ~0ull; s_rng[1] = 0; }
+  __syncthreads();
   int marked = 0;
+  uint64_t lo = ~0ull, hi = 0;
   for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
     const int64_t b = b0 + threadIdx.x;
     bool v = false;
@@ -1089,11 +1119,24 @@ __global__ void k_mark(DevState s, int single, int fallback) {
       if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
         const SelSeg ss = s.sel[single ? 0 : s.blk_group[b]];
         v = ss.active && (key < ss.prefix || (ss.incl && key == ss.prefix));
+        if (track && !v) { lo = tmin(lo, key); hi = tmax(hi, key); }
       }
     }
     const unsigned bits = __ballot_sync(kFull, v);
     if (bits && lane_id() == 0) atomicOr(s.bm_victim + ((b - lane_id()) >> 5), bits);
     marked += __popc(bits);
+  }
+  if (track) {
+    for (int o = 16; o > 0; o >>= 1) {
+      lo = tmin(lo, (uint64_t)__shfl_xor_sync(kFull, lo, o));
+      hi = tmax(hi, (uint64_t)__shfl_xor_sync(kFull, hi, o));
+    }
+    if (lane_id() == 0) { atomicMin(&s_rng[0], lo); atomicMax(&s_rng[1], hi); }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      atomicMin(reinterpret_cast<unsigned long long*>(&c->fb_kmin), s_rng[0]);
+      atomicMax(reinterpret_cast<unsigned long long*>(&c->fb_kmax), s_rng[1]);
+    }
   }
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
 }
@@ -1135,9 +1178,9 @@ __global__ void __launch_bounds__(1024) k_freetake(DevState s) {
 }
 
 // Bitmaps -> ascending id lists (allocated, evicted, invalidated).  Each CTA
-// owns 1024 bitmap words; pass 1 counts, pass 2 scans the counts and writes.
-constexpr int kBmChunk = 1024;
-__global__ void __launch_bounds__(1024) k_bm_count(DevState s) {
+// owns kBmChunk bitmap words; pass 1 counts, pass 2 scans the counts and writes.
+constexpr int kBmChunk = 256;
+__global__ void __launch_bounds__(kBmChunk) k_bm_count(DevState s) {
   if (s.ctl->status != PS_OK) return;
   const int64_t w = (int64_t)blockIdx.x * kBmChunk + threadIdx.x;
   const uint32_t* bms[3] = {s.bm_alloc, s.bm_victim, s.bm_inval};
@@ -1150,7 +1193,7 @@ __global__ void __launch_bounds__(1024) k_bm_count(DevState s) {
     if (threadIdx.x == 0) s.bm_chunk_cnt[k * nchunks + blockIdx.x] = t;
   }
 }
-__global__ void __launch_bounds__(1024) k_bm_write(DevState s) {
+__global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
   if (s.ctl->status != PS_OK) return;
   const int64_t w = (int64_t)blockIdx.x * kBmChunk + threadIdx.x;
   uint32_t* bms[3] = {s.bm_alloc, s.bm_victim, s.bm_inval};
@@ -1328,7 +1371,8 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   const int prgrid = grid_for(s.max_blocks + R, kThreads, 1 << 30);
   const int ngrid = grid_for(s.N, 256, 152 * 8);
   const int sgrid = grid_for(s.N, 256, 152 * 2);
-  const int radix_smem = (s.G <= 64 ? s.G : 1) * kRadixBins * 4;
+  const int cgrid = grid_for(s.N, 256, 152 * 2);
+  const int radix_smem = kRadixSmemRows * kRadixBins * 4;
   int launches = 0;
   auto mark = [&](int stage) {
     if (tr && tr->timing) cudaEventRecord(tr->ev[stage], st);
@@ -1342,7 +1386,6 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   if (R > 0) {
     if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
     ++launches;
-    PS_LAUNCH(k_seg_carry<<<rgrid, 256, 0, st>>>(s));
     PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
   }
   PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
@@ -1358,7 +1401,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   PS_LAUNCH(k_touch<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
   mark(6);
-  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<ngrid, 256, 0, st>>>(s));
+  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<cgrid, 256, 0, st>>>(s));
   if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));
     for (int pass = 0; pass < 8; ++pass)
@@ -1367,12 +1410,12 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
     PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 0, 0));
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 1));
     for (int pass = 0; pass < 8; ++pass)
-      PS_LAUNCH(k_radix_pass<<<sgrid, 256, kRadixBins * 4, st>>>(s, pass, 1, 1));
+      PS_LAUNCH(k_radix_pass<<<sgrid, 256, radix_smem, st>>>(s, pass, 1, 1));
     PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 1));
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
     for (int pass = 0; pass < 8; ++pass)
-      PS_LAUNCH(k_radix_pass<<<sgrid, 256, kRadixBins * 4, st>>>(s, pass, 1, 0));
+      PS_LAUNCH(k_radix_pass<<<sgrid, 256, radix_smem, st>>>(s, pass, 1, 0));
     PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 0));
   } else {
     PS_LAUNCH(launch_s3_evict(s, st));
@@ -1381,8 +1424,8 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   PS_LAUNCH(k_freetake<<<1, 1024, 0, st>>>(s));
   mark(8);
   const int nchunks = (int)((s.nwords + kBmChunk - 1) / kBmChunk);
-  PS_LAUNCH(k_bm_count<<<nchunks, 1024, 0, st>>>(s));
-  PS_LAUNCH(k_bm_write<<<nchunks, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_bm_count<<<nchunks, kBmChunk, 0, st>>>(s));
+  PS_LAUNCH(k_bm_write<<<nchunks, kBmChunk, 0, st>>>(s));
   PS_LAUNCH(k_evict<<<pgrid, kThreads, 0, st>>>(s));
   mark(9);
   PS_LAUNCH(k_insert<<<pgrid, kThreads, 0, st>>>(s));
@@ -1404,7 +1447,6 @@ int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* 
   k_validate<<<1, 1024, 0, st>>>(s, 1);
   if (R > 0) {
     if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
-    k_seg_carry<<<rgrid, 256, 0, st>>>(s);
     k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s);
   }
   k_probe_out<<<rgrid, 256, 0, st>>>(s, out, status);
