@@ -1378,8 +1378,8 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
     if (tr && tr->timing) cudaEventRecord(tr->ev[stage], st);
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
-  if (radix_smem > 48 * 1024)
-    cudaFuncSetAttribute(k_radix_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, radix_smem);
+  // dynamic plus static shared memory exceeds the 48 KB default: opt in
+  cudaFuncSetAttribute(k_radix_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, radix_smem);
   mark(0);
   PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s, 0));
   mark(1);
