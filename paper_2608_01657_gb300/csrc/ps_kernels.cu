@@ -1179,7 +1179,6 @@ __global__ void __launch_bounds__(1024) k_freetake(DevState s) {
 
 // Bitmaps -> ascending id lists (allocated, evicted, invalidated).  Each CTA
 // owns kBmChunk bitmap words; pass 1 counts, pass 2 scans the counts and writes.
-constexpr int kBmChunk = 256;
 __global__ void __launch_bounds__(kBmChunk) k_bm_count(DevState s) {
   if (s.ctl->status != PS_OK) return;
   const int64_t w = (int64_t)blockIdx.x * kBmChunk + threadIdx.x;

@@ -159,12 +159,15 @@ def test_invalid_inputs_leave_state_unchanged():
     assert both(7, [], []) == 0
 
 
-def test_step_host_matches_step():
+@pytest.mark.parametrize("N", [40, 70000])
+def test_step_host_matches_step(N):
+    """The host-buffer entry point (staging copies in the workspace) against
+    the oracle; the larger pool spans several id-list compaction chunks."""
     from paper_2608_01657_gb300 import binding as B
     steps = W.fuzz_steps(41, 3, 5, 30, docs_per_group=3, doc_blocks=6)
     kw = dict(rho=(2.0,), beta=(6.0,))
-    a = B.Cache(40, 16, 3, "prefixshield", B.Params(**kw), max_requests=5, max_tokens=2048)
-    orc = O.OracleCache(40, 16, 3, "prefixshield", O.Params(**kw))
+    a = B.Cache(N, 16, 3, "prefixshield", B.Params(**kw), max_requests=5, max_tokens=2048)
+    orc = O.OracleCache(N, 16, 3, "prefixshield", O.Params(**kw))
     for st in steps:
         out = a.step_host(st.now, st.groups, st.offsets, st.tokens)
         assert out["rc"] == 0
