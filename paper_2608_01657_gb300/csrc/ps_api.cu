@@ -221,6 +221,9 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.grp_x = cv.take<int64_t>(G);
   t.sel = cv.take<SelSeg>(G);
   t.hist_bins = cv.take<uint32_t>(G * kRadixBins);
+  t.lst_key = cv.take<uint64_t>(N);
+  t.lst_blk = cv.take<uint32_t>(N);
+  t.lst_seg = cv.take<uint16_t>(N);
   t.bm_chunk_cnt = cv.take<int32_t>(3 * (((size_t)d.nwords + kBmChunk - 1) / kBmChunk));
   // staging for ps_step_host
   int32_t* st_group = cv.take<int32_t>(R);

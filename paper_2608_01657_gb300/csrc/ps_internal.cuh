@@ -84,6 +84,7 @@ struct Ctl {
   int64_t s3_pinned[2];    // pinned members of each S3-FIFO queue this step
   int64_t s3_ninval;       // invalidated blocks to unlink this step
   uint64_t fb_kmin, fb_kmax;  // key range of candidates the debt phase left
+  int64_t lst_n;              // members of the select's split list
   uint32_t ticket;         // last-block-done counter for the radix passes
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
 };
@@ -186,6 +187,9 @@ struct DevState {
   int64_t* grp_x;          // victims taken from the group in the debt phase
   SelSeg* sel;             // [G] segments
   uint32_t* hist_bins;     // [G][256] radix histogram
+  uint64_t* lst_key;       // split list of the select: key, block, segment
+  uint32_t* lst_blk;
+  uint16_t* lst_seg;
   int32_t* bm_chunk_cnt;   // [3][chunks] bitmap compaction counts
   // current step inputs / outputs
   int64_t now;

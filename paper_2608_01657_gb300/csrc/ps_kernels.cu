@@ -832,6 +832,7 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
   }
 }
 
+__device__ __forceinline__ void sel_start(SelSeg& z);
 __global__ void k_sel_single(DevState s, int fallback) {
   Ctl* c = s.ctl;
   if (threadIdx.x != 0) return;
@@ -843,10 +844,12 @@ __global__ void k_sel_single(DevState s, int fallback) {
   z.active = m > 0;
   z.incl = 1;
   // the fallback selects among the candidates the debt phase left, whose key
-  // range the debt phase's marking pass recorded
+  // range the debt phase's split pass recorded
   z.kmin = fallback ? c->fb_kmin : old.kmin;
   z.kmax = fallback ? c->fb_kmax : old.kmax;
+  sel_start(z);
   s.sel[0] = z;
+  c->lst_n = 0;
 }
 
 // Alg. 2 in closed form (one CTA).  Group g's j-th victim would be taken at
@@ -883,11 +886,14 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
       const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
       const int64_t x = (P > eps && d > 0) ? tmin<int64_t>(q, (P - eps - 1) / d + 1) : 0;
       s.grp_x[g] = x;
-      s.sel[g].rank = x;
-      s.sel[g].active = x > 0;
-      s.sel[g].incl = 1;
+      SelSeg z = s.sel[g];
+      z.rank = x;
+      z.active = x > 0;
+      z.incl = 1;
+      sel_start(z);
+      s.sel[g] = z;
     }
-    if (threadIdx.x == 0) { c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; }
+    if (threadIdx.x == 0) { c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; c->lst_n = 0; }
     return;
   }
   int64_t pmax = 0;
@@ -944,32 +950,62 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     if (d > 0 && P >= tau && (P - tau) % d == 0 && (P - tau) / d < q) tied = true;
     above += xa;
     ntie += tied;
-    s.sel[g].rank = xa + (tied ? 1 : 0);
-    s.sel[g].active = xa + (tied ? 1 : 0) > 0;
-    s.sel[g].incl = tied ? 2 : 1;  // 2: the tie item is taken only if k_tie chooses it
+    SelSeg z = s.sel[g];
+    z.rank = xa + (tied ? 1 : 0);
+    z.active = z.rank > 0;
+    z.incl = tied ? 2 : 1;  // 2: the tie item is taken only if k_tie chooses it
+    sel_start(z);
+    s.sel[g] = z;
     s.grp_x[g] = xa + (tied ? 1 : 0);
   }
   above = block_sum(above);
   ntie = block_sum(ntie);
   if (threadIdx.x == 0) {
     c->m_fb = 0;
+    c->lst_n = 0;
     c->sel_ntie = (int32_t)ntie;
     c->sel_k = (int32_t)(m - above);  // tied items to take, 1..ntie
   }
 }
 
-// One MSB-first radix digit of the segmented select.  Every candidate of an
-// active segment whose key matches the segment's prefix adds to that
-// segment's histogram of the next 8-bit digit (a shared-memory histogram per
-// CTA, flushed as non-zero bins); the last CTA to finish picks, for every
-// segment, the digit whose cumulative count reaches the rank.  Bytes that all
-// of a segment's candidates share (from its smallest and largest key) are
-// taken without counting.
-__device__ __forceinline__ bool digit_known(const SelSeg& ss, int shift) {
-  return ((ss.kmin ^ ss.kmax) & (~0ull << shift)) == 0;
+// ---- exact segmented select -------------------------------------------------
+// Each active segment (a group in the debt phase, one global segment for lru
+// and for the fallback) looks for the rank-th smallest key among its
+// candidates, MSB-first, one byte at a time.  Bytes that all its candidates
+// share (from their smallest and largest key) are fixed without counting.
+// The first counted byte is histogrammed over the whole candidate array;
+// a split pass then marks every candidate below the chosen bucket as a
+// victim and copies the bucket's members into a short list, over which the
+// remaining bytes are counted.  A last-CTA-done resolve picks each digit.
+
+// Highest byte where kmin and kmax differ, as a shift; -1 if equal.
+__device__ __forceinline__ int first_shift(uint64_t kmin, uint64_t kmax) {
+  const uint64_t d = kmin ^ kmax;
+  return d == 0 ? -1 : ((63 - __clzll((long long)d)) / 8) * 8;
+}
+// Bytes above 'shift' (shift a multiple of 8 in [0, 56]).
+__device__ __forceinline__ uint64_t above_mask(int shift) { return shift >= 56 ? 0ull : (~0ull << (shift + 8)); }
+// The next unresolved digit under a byte-aligned prefix mask, or -1.
+__device__ __forceinline__ int next_shift(uint64_t mask) {
+  if (mask == ~0ull) return -1;
+  if (mask == 0) return 56;
+  return __ffsll((long long)mask) - 1 - 8;
+}
+// Start a segment's search from its key range (rank and activity already set).
+__device__ __forceinline__ void sel_start(SelSeg& z) {
+  const int fs = first_shift(z.kmin, z.kmax);
+  if (fs < 0) {
+    z.prefix = z.kmin;
+    z.mask = ~0ull;
+  } else {
+    z.mask = above_mask(fs);
+    z.prefix = z.kmin & z.mask;
+  }
 }
 
-__global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int single, int fallback) {
+// One digit for every segment that still has one: over the whole candidate
+// array (from_list = 0) or over the split list (from_list = 1).
+__global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int fallback, int from_list) {
   extern __shared__ uint32_t shist[];
   __shared__ int16_t row_of[PS_MAX_GROUPS];
   __shared__ int16_t seg_of_row[PS_MAX_GROUPS];
@@ -978,54 +1014,68 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
   if (c->status != PS_OK || c->mvict == 0) return;
   const int nseg = single ? 1 : s.G;
   if (single && !s.sel[0].active) return;
-  const int shift = 64 - kRadixBits * (pass + 1);
-  // segments that still count at this digit get a histogram row
-  if (threadIdx.x == 0) {
+  // rows for the segments that still count (parallel flags, scanned)
+  {
     int k = 0;
-    for (int g = 0; g < nseg; ++g) {
-      const SelSeg ss = s.sel[g];
-      const bool counts = ss.active && !digit_known(ss, shift);
-      row_of[g] = counts ? (int16_t)k : (int16_t)-1;
-      if (counts) seg_of_row[k++] = (int16_t)g;
+    for (int base = 0; base < nseg; base += blockDim.x) {
+      const int g = base + threadIdx.x;
+      bool counts = false;
+      if (g < nseg) {
+        const SelSeg ss = s.sel[g];
+        counts = ss.active && next_shift(ss.mask) >= 0;
+      }
+      int tot;
+      const int ex = block_excl_scan((int)counts, &tot);
+      if (g < nseg) row_of[g] = counts ? (int16_t)(k + ex) : (int16_t)-1;
+      if (counts) seg_of_row[k + ex] = (int16_t)g;
+      k += tot;
     }
-    s_nrows = k;
-  }
-  __syncthreads();
-  const int nrows = s_nrows;
-  const bool use_smem = nrows <= kRadixSmemRows;
-  if (nrows > 0) {
-    if (use_smem)
-      for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x) shist[k] = 0;
+    if (threadIdx.x == 0) s_nrows = k;
     __syncthreads();
-    for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
-      const int64_t b = b0 + threadIdx.x;
-      bool act = false;
-      uint32_t idx = 0;
-      if (b < s.N) {
-        const uint64_t key = s.csk[b];
-        if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
-          const int seg = single ? 0 : s.blk_group[b];
-          const int row = row_of[seg];
-          if (row >= 0) {
-            const SelSeg ss = s.sel[seg];
-            if ((key & ss.mask) == ss.prefix) {
-              act = true;
-              const uint32_t digit = (uint32_t)((key >> shift) & (kRadixBins - 1));
-              idx = use_smem ? (uint32_t)row * kRadixBins + digit : (uint32_t)seg * kRadixBins + digit;
-            }
+  }
+  const int nrows = s_nrows;
+  if (nrows == 0) return;  // uniform across CTAs: nothing counts, nothing to resolve
+  const bool use_smem = nrows <= kRadixSmemRows;
+  if (use_smem)
+    for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x) shist[k] = 0;
+  __syncthreads();
+  const int64_t n = from_list ? c->lst_n : s.N;
+  for (int64_t e0 = blockIdx.x * (int64_t)blockDim.x; e0 < n; e0 += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t e = e0 + threadIdx.x;
+    bool act = false;
+    uint32_t idx = 0;
+    if (e < n) {
+      uint64_t key;
+      int seg;
+      bool ok;
+      if (from_list) {
+        key = s.lst_key[e];
+        seg = s.lst_seg[e];
+        ok = true;
+      } else {
+        key = s.csk[e];
+        seg = single ? 0 : s.blk_group[e];
+        ok = key != ~0ull && !(fallback && ((s.bm_victim[e >> 5] >> (e & 31)) & 1));
+      }
+      if (ok) {
+        const int row = row_of[seg];
+        if (row >= 0) {
+          const SelSeg ss = s.sel[seg];
+          if ((key & ss.mask) == ss.prefix) {
+            act = true;
+            const int sh = next_shift(ss.mask);
+            const uint32_t digit = (uint32_t)((key >> sh) & (kRadixBins - 1));
+            idx = use_smem ? (uint32_t)row * kRadixBins + digit : (uint32_t)seg * kRadixBins + digit;
           }
         }
       }
-      agg_inc(use_smem ? shist : s.hist_bins, idx, act);
     }
-    __syncthreads();
-    if (use_smem)
-      for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x) {
-        if (!shist[k]) continue;
-        const int seg = seg_of_row[k / kRadixBins];
-        atomicAdd(s.hist_bins + (size_t)seg * kRadixBins + (k % kRadixBins), shist[k]);
-      }
+    agg_inc(use_smem ? shist : s.hist_bins, idx, act);
   }
+  __syncthreads();
+  if (use_smem)
+    for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x)
+      if (shist[k]) atomicAdd(s.hist_bins + (size_t)seg_of_row[k / kRadixBins] * kRadixBins + (k % kRadixBins), shist[k]);
   __shared__ bool last;
   __threadfence();
   __syncthreads();
@@ -1034,17 +1084,10 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
   if (!last) return;
   __threadfence();
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  for (int seg = warp; seg < nseg; seg += blockDim.x >> 5) {
+  for (int r = warp; r < nrows; r += blockDim.x >> 5) {
+    const int seg = seg_of_row[r];
     SelSeg ss = s.sel[seg];
-    if (!ss.active) continue;
-    if (digit_known(ss, shift)) {
-      if (lane == 0) {
-        ss.prefix |= ss.kmin & ((uint64_t)(kRadixBins - 1) << shift);
-        ss.mask |= (uint64_t)(kRadixBins - 1) << shift;
-        s.sel[seg] = ss;
-      }
-      continue;
-    }
+    const int sh = next_shift(ss.mask);
     uint32_t* row = s.hist_bins + (size_t)seg * kRadixBins;
     uint32_t v[kRadixBins / 32];
     uint32_t sum = 0;
@@ -1060,8 +1103,8 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
         if ((uint64_t)ss.rank <= (uint64_t)(run + v[j])) { d = lane * (kRadixBins / 32) + j; break; }
         run += v[j];
       }
-      ss.prefix |= (uint64_t)d << shift;
-      ss.mask |= (uint64_t)(kRadixBins - 1) << shift;
+      ss.prefix |= (uint64_t)d << sh;
+      ss.mask |= (uint64_t)(kRadixBins - 1) << sh;
       ss.rank -= run;
       s.sel[seg] = ss;
     }
@@ -1069,6 +1112,69 @@ __global__ void __launch_bounds__(256) k_radix_pass(DevState s, int pass, int si
     for (int j = 0; j < kRadixBins / 32; ++j) row[lane * (kRadixBins / 32) + j] = 0;
   }
   if (threadIdx.x == 0) c->ticket = 0;
+}
+
+// Split: candidates below their segment's chosen bucket are victims; the
+// bucket's members go to the list for the remaining digits.  The per-group
+// pass also records the key range of every candidate it does not mark, for
+// the global fallback.
+__global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallback) {
+  __shared__ unsigned long long s_rng[2];
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK || c->mvict == 0) return;
+  if (single && !s.sel[0].active) return;
+  const bool track = !single;
+  if (threadIdx.x == 0) { s_rng[0] = ~0ull; s_rng[1] = 0; }
+  __syncthreads();
+  int marked = 0;
+  uint64_t lo = ~0ull, hi = 0;
+  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t b = b0 + threadIdx.x;
+    bool v = false, to_list = false;
+    uint64_t key = ~0ull;
+    int seg = 0;
+    if (b < s.N) {
+      key = s.csk[b];
+      if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
+        seg = single ? 0 : s.blk_group[b];
+        const SelSeg ss = s.sel[seg];
+        if (ss.active) {
+          const uint64_t k = key & ss.mask;
+          v = k < ss.prefix;
+          to_list = k == ss.prefix;
+        }
+        if (track && !v) { lo = tmin(lo, key); hi = tmax(hi, key); }
+      }
+    }
+    const unsigned bits = __ballot_sync(kFull, v);
+    if (bits && lane_id() == 0) atomicOr(s.bm_victim + ((b - lane_id()) >> 5), bits);
+    marked += __popc(bits);
+    const unsigned lm = __ballot_sync(kFull, to_list);
+    if (lm) {
+      unsigned long long base = 0;
+      if (lane_id() == 0) base = atomicAdd(reinterpret_cast<unsigned long long*>(&c->lst_n), (unsigned long long)__popc(lm));
+      base = __shfl_sync(kFull, base, 0);
+      if (to_list) {
+        const int64_t slot = (int64_t)base + __popc(lm & ((1u << lane_id()) - 1));
+        s.lst_key[slot] = key;
+        s.lst_blk[slot] = (uint32_t)b;
+        s.lst_seg[slot] = (uint16_t)seg;
+      }
+    }
+  }
+  if (track) {
+    for (int o = 16; o > 0; o >>= 1) {
+      lo = tmin(lo, (uint64_t)__shfl_xor_sync(kFull, lo, o));
+      hi = tmax(hi, (uint64_t)__shfl_xor_sync(kFull, hi, o));
+    }
+    if (lane_id() == 0) { atomicMin(&s_rng[0], lo); atomicMax(&s_rng[1], hi); }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      atomicMin(reinterpret_cast<unsigned long long*>(&c->fb_kmin), s_rng[0]);
+      atomicMax(reinterpret_cast<unsigned long long*>(&c->fb_kmax), s_rng[1]);
+    }
+  }
+  if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
 }
 
 // Ties at tau (Eq. 7's tie rule: equal projected debt is broken by the
@@ -1098,47 +1204,21 @@ __global__ void __launch_bounds__(1024) k_tie(DevState s) {
   }
 }
 
-// Mark victims: keys below (or equal to, if incl) the located threshold.
-// The per-group pass also records the key range of the candidates it leaves,
-// for the global fallback that may follow.
-__global__ void __launch_bounds__(256) k_mark(DevState s, int single, int fallback) {
-  __shared__ unsigned long long s_rng[2];
+// Mark the list's victims: keys below (or equal to, if incl) the located
+// threshold of their segment.
+__global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   if (single && !s.sel[0].active) return;
-  const bool track = !single;
-  if (threadIdx.x == 0) { s_rng[0] = ~0ull; s_rng[1] = 0; }
-  __syncthreads();
-  int marked = 0;
-  uint64_t lo = ~0ull, hi = 0;
-  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t b = b0 + threadIdx.x;
-    bool v = false;
-    if (b < s.N) {
-      const uint64_t key = s.csk[b];
-      if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
-        const SelSeg ss = s.sel[single ? 0 : s.blk_group[b]];
-        v = ss.active && (key < ss.prefix || (ss.incl && key == ss.prefix));
-        if (track && !v) { lo = tmin(lo, key); hi = tmax(hi, key); }
-      }
-    }
-    const unsigned bits = __ballot_sync(kFull, v);
-    if (bits && lane_id() == 0) atomicOr(s.bm_victim + ((b - lane_id()) >> 5), bits);
-    marked += __popc(bits);
-  }
-  if (track) {
-    for (int o = 16; o > 0; o >>= 1) {
-      lo = tmin(lo, (uint64_t)__shfl_xor_sync(kFull, lo, o));
-      hi = tmax(hi, (uint64_t)__shfl_xor_sync(kFull, hi, o));
-    }
-    if (lane_id() == 0) { atomicMin(&s_rng[0], lo); atomicMax(&s_rng[1], hi); }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      atomicMin(reinterpret_cast<unsigned long long*>(&c->fb_kmin), s_rng[0]);
-      atomicMax(reinterpret_cast<unsigned long long*>(&c->fb_kmax), s_rng[1]);
+  const int64_t n = c->lst_n;
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+    const uint64_t key = s.lst_key[e];
+    const SelSeg ss = s.sel[s.lst_seg[e]];
+    if (ss.active && (key < ss.prefix || (ss.incl && key == ss.prefix))) {
+      const uint32_t b = s.lst_blk[e];
+      atomicOr(s.bm_victim + (b >> 5), 1u << (b & 31));
     }
   }
-  if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
 }
 
 // TakeTrueFree (Alg. 2): the ftake smallest free block ids (one CTA,
@@ -1371,6 +1451,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   const int ngrid = grid_for(s.N, 256, 152 * 8);
   const int sgrid = grid_for(s.N, 256, 152 * 2);
   const int cgrid = grid_for(s.N, 256, 152 * 2);
+  const int lgrid = 152;  // list passes: the split list is short
   const int radix_smem = kRadixSmemRows * kRadixBins * 4;
   int launches = 0;
   auto mark = [&](int stage) {
@@ -1378,7 +1459,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
   // dynamic plus static shared memory exceeds the 48 KB default: opt in
-  cudaFuncSetAttribute(k_radix_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, radix_smem);
+  cudaFuncSetAttribute(k_digit_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, radix_smem);
   mark(0);
   PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s, 0));
   mark(1);
@@ -1401,21 +1482,23 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
   mark(6);
   if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<cgrid, 256, 0, st>>>(s));
+  // one exact segmented select: a digit over the candidates, the split, then
+  // the remaining digits over the list, then the list's victims
+  auto select = [&](int single, int fallback) {
+    PS_LAUNCH(k_digit_pass<<<sgrid, 256, radix_smem, st>>>(s, single, fallback, 0));
+    PS_LAUNCH(k_split<<<sgrid, 256, 0, st>>>(s, single, fallback));
+    for (int d = 0; d < 7; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, st>>>(s, single, fallback, 1));
+    if (!single) PS_LAUNCH(k_tie<<<1, 1024, 0, st>>>(s));
+    PS_LAUNCH(k_mark_list<<<lgrid, 256, 0, st>>>(s, single));
+  };
   if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));
-    for (int pass = 0; pass < 8; ++pass)
-      PS_LAUNCH(k_radix_pass<<<sgrid, 256, radix_smem, st>>>(s, pass, 0, 0));
-    PS_LAUNCH(k_tie<<<1, 1024, 0, st>>>(s));
-    PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 0, 0));
+    select(0, 0);
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 1));
-    for (int pass = 0; pass < 8; ++pass)
-      PS_LAUNCH(k_radix_pass<<<sgrid, 256, radix_smem, st>>>(s, pass, 1, 1));
-    PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 1));
+    select(1, 1);
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
-    for (int pass = 0; pass < 8; ++pass)
-      PS_LAUNCH(k_radix_pass<<<sgrid, 256, radix_smem, st>>>(s, pass, 1, 0));
-    PS_LAUNCH(k_mark<<<ngrid, 256, 0, st>>>(s, 1, 0));
+    select(1, 0);
   } else {
     PS_LAUNCH(launch_s3_evict(s, st));
   }
