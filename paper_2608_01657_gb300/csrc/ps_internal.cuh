@@ -25,7 +25,7 @@ constexpr int kTableWays = 8;    // native prefix table: 8 x 16 B entries per 12
 constexpr int kClaimWays = 4;    // per-step claim map: 4 x 32 B entries per bucket
 constexpr int kRadixBits = 8;
 constexpr int kRadixBins = 1 << kRadixBits;
-constexpr int kSegBlocks = 256;  // blocks of one prompt hashed by one warp
+constexpr int kSegBlocks = 128;  // blocks of one prompt hashed by one warp
 constexpr int kBmChunk = 256;    // bitmap words per CTA of the id-list compaction
 constexpr uint64_t kP61 = (1ull << 61) - 1;  // chain modulus, a Mersenne prime
 

@@ -15,7 +15,6 @@
 namespace ps {
 
 constexpr unsigned kFull = 0xFFFFFFFFu;
-constexpr int kWarpsPerCta = 8;   // warp-per-segment hashing kernel
 constexpr int kThreads = 256;     // position-parallel kernels
 constexpr int kRadixSmemRows = 48;  // radix rows counted in shared memory (48 KB)
 
@@ -338,25 +337,43 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
 // Stage 1: chained block hashing (Sec. III-B native content key), one warp
 // per segment of up to kSegBlocks blocks of one prompt.
 //
-// Tokens of 32 blocks at a time are staged in shared memory with coalesced
-// 16-byte loads.  NH products are spread over the warp: lane l takes pair
-// (l % PPB) of block (l / PPB + (32 / PPB) r) in round r, PPB = bs / 2; the
-// pair sums are reduced with xor shuffles and routed to lane = block.  The
-// chain C_m = Kc C_{m-1} + D_m (mod 2^61-1) is a composition of affine maps,
-// so a warp scan gives every block its chain value relative to the segment
-// start (B_m, with the value before the segment taken as 0); k_keys_lookup
-// then folds in the true value entering the segment.
+// The segment's tokens arrive in shared memory with one TMA bulk copy
+// (cp.async.bulk, completion counted on an mbarrier) of the 16-byte aligned
+// window around them, so each warp has its whole segment in flight at once;
+// a window that would end past the token buffer, or an unaligned buffer, is
+// loaded with plain coalesced loads instead.  NH products are spread over the
+// warp: lane l takes pair (l % PPB) of block (l / PPB + (32 / PPB) r) in
+// round r, PPB = bs / 2; the pair sums are reduced with xor shuffles and
+// routed to lane = block.  The chain C_m = Kc C_{m-1} + D_m (mod 2^61-1) is a
+// composition of affine maps, so a warp scan gives every block its chain
+// value relative to the segment start (B_m, with the value before the segment
+// taken as 0); k_keys_lookup then folds in the true value entering it.
 template <int PPB>
-__global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash(DevState s) {
-  extern __shared__ int32_t smem_tokens[];
+struct HashCfg {
+  static constexpr int BS = 2 * PPB;
+  static constexpr int kWindow = kSegBlocks * BS + 8;  // tokens staged per warp (+ alignment slack)
+  static constexpr int kWarps = (64 * 1024) / (kWindow * 4) < 1 ? 1
+                                : ((64 * 1024) / (kWindow * 4) > 8 ? 8 : (64 * 1024) / (kWindow * 4));
+  static constexpr size_t kSmem = (size_t)kWarps * kWindow * 4 + (size_t)kWarps * 8;
+};
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+template <int PPB>
+__global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) {
+  extern __shared__ __align__(16) int32_t smem_tokens[];
+  using Cfg = HashCfg<PPB>;
+  constexpr int BS = Cfg::BS;
+  constexpr int G32 = 32 / PPB;
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
-  constexpr int BS = 2 * PPB;
-  constexpr int G32 = 32 / PPB;
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int64_t seg = (int64_t)blockIdx.x * kWarpsPerCta + warp;
+  const int64_t seg = (int64_t)blockIdx.x * Cfg::kWarps + warp;
   if (seg >= c->nsegs) return;
-  int32_t* buf = smem_tokens + warp * (32 * BS + 4);
+  int32_t* buf = smem_tokens + warp * Cfg::kWindow;
+  uint64_t* mbar = reinterpret_cast<uint64_t*>(smem_tokens + Cfg::kWarps * Cfg::kWindow) + warp;
   const uint32_t i = s.seg_req[seg];
   const int n = s.rq_n[i];
   const int m0 = (int)(seg - s.rq_sbase[i]) * kSegBlocks;
@@ -364,6 +381,51 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash(DevState s) {
   const int64_t o0 = s.in_offsets[i];
   const int pbase = s.rq_pbase[i];
   const int64_t T = c->T;
+  // the segment's tokens [cs, ce) and their 16-byte aligned window [ws, we)
+  const int64_t cs = o0 + (int64_t)m0 * BS, ce = o0 + (int64_t)m1 * BS;
+  const int64_t ws = cs & ~3ll, we = (ce + 3) & ~3ll;
+  const int off = (int)(cs - ws);
+  bool staged = false;
+  if (s.tokens_aligned16 && we <= T) {
+    const uint32_t bytes = (uint32_t)((we - ws) * 4);
+    if (lane == 0) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(mbar)) : "memory");
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(mbar)), "r"(bytes)
+                   : "memory");
+      asm volatile(
+          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+              smem_addr(buf)),
+          "l"(s.in_tokens + ws), "r"(bytes), "r"(smem_addr(mbar))
+          : "memory");
+    }
+    __syncwarp();
+    // bounded wait for the copy (phase 0); a copy that does not land in time
+    // is reported, and waited for once more (again bounded) before the warp
+    // leaves, so it never writes into released shared memory
+    auto wait_copy = [&](int limit) -> bool {
+      uint32_t done = 0;
+      for (int it = 0; it < limit && !done; ++it)
+        asm volatile(
+            "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+            : "=r"(done)
+            : "r"(smem_addr(mbar))
+            : "memory");
+      return __all_sync(kFull, done != 0);
+    };
+    if (!wait_copy(1 << 22)) {
+      if (lane == 0) s.ctl->internal_error = 1;
+      wait_copy(1 << 22);
+      return;
+    }
+    staged = true;
+  }
+  const int64_t base_tok = staged ? ws : cs;
+  if (!staged) {
+    for (int64_t t = cs + lane; t < ce; t += 32) buf[t - cs] = s.in_tokens[t];
+    __syncwarp();
+  }
+  const int shift_tok = (int)(cs - base_tok);  // 0..3 when staged, 0 otherwise
   const int k = lane % PPB;
   const uint32_t K0 = s.key_words[2 * k], K1 = s.key_words[2 * k + 1];
   const uint32_t K2 = s.key_words[2 * k + 2], K3 = s.key_words[2 * k + 3];
@@ -375,55 +437,34 @@ __global__ void __launch_bounds__(kWarpsPerCta * 32) k_hash(DevState s) {
   uint64_t carry = 0;  // local chain value at the block before the chunk
   for (int c0 = m0; c0 < m1; c0 += 32) {
     const int nb = tmin(32, m1 - c0);
-    const int64_t cs = o0 + (int64_t)c0 * BS, ce = cs + (int64_t)nb * BS;
-    if (s.tokens_aligned16) {
-      const int64_t q1 = (ce + 3) >> 2;
-      for (int64_t q = (cs >> 2) + lane; q < q1; q += 32) {
-        const int64_t t0 = q << 2;
-        int v[4];
-        if (t0 + 3 < T) {
-          const int4 w = __ldcs(reinterpret_cast<const int4*>(s.in_tokens) + q);
-          v[0] = w.x; v[1] = w.y; v[2] = w.z; v[3] = w.w;
-        } else {
-#pragma unroll
-          for (int j = 0; j < 4; ++j) v[j] = (t0 + j < T) ? s.in_tokens[t0 + j] : 0;
-        }
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (t0 + j >= cs && t0 + j < ce) buf[t0 + j - cs] = v[j];
-      }
-    } else {
-      for (int64_t t = cs + lane; t < ce; t += 32) buf[t - cs] = s.in_tokens[t];
-    }
-    __syncwarp();
+    const int32_t* cb = buf + shift_tok + (c0 - m0) * BS;
     uint64_t d1 = 0, d2 = 0;
 #pragma unroll
     for (int r = 0; r < PPB; ++r) {
       const int b = lane / PPB + G32 * r;
       uint64_t p1 = 0, p2 = 0;
       if (b < nb) {
-        const int2 t = *reinterpret_cast<const int2*>(buf + b * BS + 2 * k);
-        p1 = (uint64_t)((uint32_t)t.x + K0) * (uint64_t)((uint32_t)t.y + K1);
-        p2 = (uint64_t)((uint32_t)t.x + K2) * (uint64_t)((uint32_t)t.y + K3);
+        const int32_t tx = cb[b * BS + 2 * k], ty = cb[b * BS + 2 * k + 1];
+        p1 = (uint64_t)((uint32_t)tx + K0) * (uint64_t)((uint32_t)ty + K1);
+        p2 = (uint64_t)((uint32_t)tx + K2) * (uint64_t)((uint32_t)ty + K3);
       }
 #pragma unroll
-      for (int off = 1; off < PPB; off <<= 1) {
-        p1 += __shfl_xor_sync(kFull, p1, off);
-        p2 += __shfl_xor_sync(kFull, p2, off);
+      for (int o = 1; o < PPB; o <<= 1) {
+        p1 += __shfl_xor_sync(kFull, p1, o);
+        p2 += __shfl_xor_sync(kFull, p2, o);
       }
       const int src = (lane % G32) * PPB;
       const uint64_t q1 = __shfl_sync(kFull, p1, src), q2 = __shfl_sync(kFull, p2, src);
       if (lane / G32 == r) { d1 = q1; d2 = q2; }
     }
-    __syncwarp();
     // D_m, then the inclusive scan of the affine maps x -> Kc x + D
-    uint64_t b = lane < nb ? add61(red61(d1), mul61(Kd, red61(d2))) : 0;
+    uint64_t bb = lane < nb ? add61(red61(d1), mul61(Kd, red61(d2))) : 0;
 #pragma unroll
     for (int j = 0; j < 5; ++j) {
-      const uint64_t t = __shfl_up_sync(kFull, b, 1 << j);
-      if (lane >= (1 << j)) b = add61(b, mul61(kp[j], t));
+      const uint64_t t = __shfl_up_sync(kFull, bb, 1 << j);
+      if (lane >= (1 << j)) bb = add61(bb, mul61(kp[j], t));
     }
-    const uint64_t B = add61(mul61(kpl, carry), b);
+    const uint64_t B = add61(mul61(kpl, carry), bb);
     if (lane < nb) {
       s.pos_key[pbase + c0 + lane] = B;
       s.pos_req[pbase + c0 + lane] = i;
@@ -801,15 +842,16 @@ __global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
 // and largest key of every segment, so the radix select can skip the bytes
 // its candidates share.
 __global__ void __launch_bounds__(256) k_cand(DevState s) {
-  __shared__ unsigned long long s_min[PS_MAX_GROUPS], s_max[PS_MAX_GROUPS];
-  __shared__ unsigned int s_cnt[PS_MAX_GROUPS];
+  // per segment: candidates, and the range of the keys' top 32 bits (class,
+  // step, request's top bits); the bytes below are treated as differing
+  __shared__ unsigned int s_min[PS_MAX_GROUPS], s_max[PS_MAX_GROUPS], s_cnt[PS_MAX_GROUPS];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const uint32_t step32 = (uint32_t)c->step;
   const bool ps = s.policy == PS_PREFIXSHIELD;
   const bool seg = ps && !(s.flags & PS_FLAG_NO_SEGMENTATION);
   const int nseg = ps ? s.G : 1;
-  for (int g = threadIdx.x; g < nseg; g += blockDim.x) { s_min[g] = ~0ull; s_max[g] = 0; s_cnt[g] = 0; }
+  for (int g = threadIdx.x; g < nseg; g += blockDim.x) { s_min[g] = ~0u; s_max[g] = 0; s_cnt[g] = 0; }
   __syncthreads();
   for (int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; b < s.N; b += (int64_t)gridDim.x * blockDim.x) {
     uint64_t key = ~0ull;
@@ -817,8 +859,9 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
       key = s.blk_stamp[b];
       if (seg) key |= (uint64_t)s.blk_klass[b] << 62;
       const uint32_t g = ps ? s.blk_group[b] : 0;
-      atomicMin(&s_min[g], (unsigned long long)key);
-      atomicMax(&s_max[g], (unsigned long long)key);
+      const uint32_t hi = (uint32_t)(key >> 32);
+      atomicMin(&s_min[g], hi);
+      atomicMax(&s_max[g], hi);
       atomicAdd(&s_cnt[g], 1u);
     }
     s.csk[b] = key;
@@ -827,8 +870,8 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
   for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
     if (!s_cnt[g]) continue;
     if (ps) atomic_add_i64(s.grp_qsize + g, s_cnt[g]);
-    atomicMin(reinterpret_cast<unsigned long long*>(&s.sel[g].kmin), s_min[g]);
-    atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[g].kmax), s_max[g]);
+    atomicMin(reinterpret_cast<unsigned long long*>(&s.sel[g].kmin), (unsigned long long)s_min[g] << 32);
+    atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[g].kmax), ((unsigned long long)s_max[g] << 32) | 0xFFFFFFFFull);
   }
 }
 
@@ -863,7 +906,9 @@ __global__ void k_sel_single(DevState s, int fallback) {
 // to the global fallback in (class, stamp) order.
 __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
   Ctl* c = s.ctl;
+  __shared__ int64_t sP[PS_MAX_GROUPS], sD[PS_MAX_GROUPS], sQ[PS_MAX_GROUPS];
   __shared__ int64_t s_pmax;
+  __shared__ int s_best;
   const int G = s.G;
   const int64_t eps = s.eps;
   const int64_t m = (c->status == PS_OK) ? c->mvict : 0;
@@ -872,19 +917,22 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     if (threadIdx.x == 0) c->m_fb = 0;
     return;
   }
-  auto count_gt = [&](int64_t t) -> int64_t {  // items with value > t over all groups
-    int64_t tot = 0;
-    for (int g = threadIdx.x; g < G; g += blockDim.x) {
-      const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
-      if (P > t && d > 0) tot += tmin<int64_t>(q, (P - t - 1) / d + 1);
-    }
-    return block_sum(tot);
+  for (int g = threadIdx.x; g < G; g += blockDim.x) { sP[g] = s.grp_P[g]; sD[g] = s.grp_delta[g]; sQ[g] = s.grp_qsize[g]; }
+  if (threadIdx.x == 0) s_pmax = 0;
+  __syncthreads();
+  // items of group g with value > t: min(q, floor((P - t - 1) / d) + 1) if P > t
+  auto items_gt = [&](int g, int64_t t) -> int64_t {
+    const int64_t P = sP[g], d = sD[g];
+    return (P > t && d > 0) ? tmin<int64_t>(sQ[g], (P - t - 1) / d + 1) : 0;
   };
-  const int64_t E = count_gt(eps);
+  int64_t e = 0, pm = 0;
+  for (int g = threadIdx.x; g < G; g += blockDim.x) { e += items_gt(g, eps); pm = tmax(pm, sP[g]); }
+  const int64_t E = block_sum(e);
+  if (pm) atomicMax(reinterpret_cast<unsigned long long*>(&s_pmax), (unsigned long long)pm);
+  __syncthreads();
   if (E <= m) {
     for (int g = threadIdx.x; g < G; g += blockDim.x) {
-      const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
-      const int64_t x = (P > eps && d > 0) ? tmin<int64_t>(q, (P - eps - 1) / d + 1) : 0;
+      const int64_t x = items_gt(g, eps);
       s.grp_x[g] = x;
       SelSeg z = s.sel[g];
       z.rank = x;
@@ -896,35 +944,17 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     if (threadIdx.x == 0) { c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; c->lst_n = 0; }
     return;
   }
-  int64_t pmax = 0;
-  for (int g = threadIdx.x; g < G; g += blockDim.x) pmax = tmax(pmax, s.grp_P[g]);
-  {
-    __shared__ int64_t red[32];
-    int64_t v = pmax;
-    for (int o = 16; o > 0; o >>= 1) v = tmax(v, (int64_t)__shfl_xor_sync(kFull, v, o));
-    if (lane_id() == 0) red[threadIdx.x >> 5] = v;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      int64_t rr = 0;
-      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) rr = tmax(rr, red[w]);
-      s_pmax = rr;
-    }
-    __syncthreads();
-    pmax = s_pmax;
-  }
-  // tau = max{t in [eps+1, pmax] : count_gt(t - 1) >= m}.  Each round every
-  // thread tests one of blockDim thresholds spread over the interval.
-  __shared__ int s_best;
-  int64_t lo = eps + 1, hi = pmax;
+  // tau = max{t in [eps+1, pmax] : items_gt(t - 1) summed >= m}.  Each round
+  // every thread tests one of blockDim thresholds spread over the interval.
+  int64_t lo = eps + 1, hi = s_pmax;
   const int nt = blockDim.x;
   while (lo < hi) {
-    const int64_t span = hi - lo;
-    const int64_t t = lo + 1 + (int64_t)(((__int128)(span - 1) * threadIdx.x) / (nt - 1));
+    const int64_t span = hi - lo;  // >= 1
+    const int64_t stride = tmax<int64_t>(1, (span - 1) / (nt - 1));
+    auto thr = [&](int j) -> int64_t { return j == nt - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * j); };
+    const int64_t t = thr(threadIdx.x);
     int64_t cnt = 0;
-    for (int g = 0; g < G; ++g) {
-      const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
-      if (P > t - 1 && d > 0) cnt += tmin<int64_t>(q, (P - t) / d + 1);
-    }
+    for (int g = 0; g < G; ++g) cnt += items_gt(g, t - 1);
     if (threadIdx.x == 0) s_best = -1;
     __syncthreads();
     if (cnt >= m) atomicMax(&s_best, (int)threadIdx.x);
@@ -934,20 +964,17 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     if (J < 0) {
       hi = lo;
     } else {
-      const int64_t tj = lo + 1 + (int64_t)(((__int128)(span - 1) * J) / (nt - 1));
-      const int64_t tn = J + 1 < nt ? lo + 1 + (int64_t)(((__int128)(span - 1) * (J + 1)) / (nt - 1)) : hi + 1;
-      lo = tj;
-      hi = tn - 1;
+      lo = thr(J);
+      hi = J + 1 < nt ? thr(J + 1) - 1 : hi;
+      if (hi < lo) hi = lo;
     }
   }
   const int64_t tau = lo;
   int64_t above = 0, ntie = 0;
   for (int g = threadIdx.x; g < G; g += blockDim.x) {
-    const int64_t P = s.grp_P[g], d = s.grp_delta[g], q = s.grp_qsize[g];
-    int64_t xa = 0;
-    bool tied = false;
-    if (P > tau && d > 0) xa = tmin<int64_t>(q, (P - tau - 1) / d + 1);
-    if (d > 0 && P >= tau && (P - tau) % d == 0 && (P - tau) / d < q) tied = true;
+    const int64_t P = sP[g], d = sD[g], q = sQ[g];
+    const int64_t xa = items_gt(g, tau);
+    const bool tied = d > 0 && P >= tau && (P - tau) % d == 0 && (P - tau) / d < q;
     above += xa;
     ntie += tied;
     SelSeg z = s.sel[g];
@@ -1426,9 +1453,9 @@ void launch_init(const DevState& s, cudaStream_t st) {
 
 template <int PPB>
 static void launch_hash_t(const DevState& s, cudaStream_t st) {
-  const size_t smem = (size_t)kWarpsPerCta * (32 * 2 * PPB + 4) * sizeof(int32_t);
-  if (smem > 48 * 1024) cudaFuncSetAttribute(k_hash<PPB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  k_hash<PPB><<<(int)((s.max_segments + kWarpsPerCta - 1) / kWarpsPerCta), kWarpsPerCta * 32, smem, st>>>(s);
+  using Cfg = HashCfg<PPB>;
+  cudaFuncSetAttribute(k_hash<PPB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmem);
+  k_hash<PPB><<<(int)((s.max_segments + Cfg::kWarps - 1) / Cfg::kWarps), Cfg::kWarps * 32, Cfg::kSmem, st>>>(s);
 }
 static int32_t launch_hash(const DevState& s, cudaStream_t st) {
   switch (s.bs / 2) {
