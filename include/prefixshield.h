@@ -45,7 +45,8 @@ extern "C" {
 #define PS_MAX_CONTRACTS 8
 #define PS_MAX_GROUPS 1024
 #define PS_NUM_STATS 15
-/* Limits of the recency stamp (step:26 | request:18 | reversed position:18). */
+/* Limits of one step (a step with more is rejected as PS_ERR_INVALID_ARG);
+ * after 2^31 - 1 steps a handle reports PS_ERR_CAPACITY until ps_reset(). */
 #define PS_MAX_REQUESTS_PER_STEP ((1 << 18) - 1)
 #define PS_MAX_BLOCKS_PER_REQUEST ((1 << 18) - 1)
 

@@ -99,7 +99,7 @@ def lib():
         L.orc_chain_keys.restype = i64
         L.orc_chain_keys.argtypes = [u64, i32, i32, vp, i64, vp]
         L.orc_make_stamp.restype = u64
-        L.orc_make_stamp.argtypes = [u64, u64, u64]
+        L.orc_make_stamp.argtypes = [u64, u64, u64, u64]
         L.orc_alg2_loop.restype = i64
         L.orc_alg2_loop.argtypes = [i32, vp, vp, i64, vp, vp, i64, vp, vp]
         _lib = L
@@ -268,8 +268,8 @@ def chain_keys(seed: int, group: int, bs: int, tokens) -> np.ndarray:
     return out[:n].copy()
 
 
-def make_stamp(step: int, req: int, pos: int) -> int:
-    return int(lib().orc_make_stamp(step, req, pos))
+def make_stamp(base: int, blocks_before: int, n: int, m: int) -> int:
+    return int(lib().orc_make_stamp(base, blocks_before, n, m))
 
 
 def alg2_loop(P, delta, eps, queues, m):

@@ -63,14 +63,18 @@ enum Stat {
   S_DEBT_RAW, S_DEBT_NORM
 };
 
-// Recency stamp: (step, request, reversed position), 62 bits in all.  A
-// request releases its blocks tail first, so within a request the deeper block
-// is older.  Limits: 2^18-1 requests per step and full blocks per request,
-// 2^26-1 steps.
-constexpr uint64_t POS_BITS = 18, REQ_BITS = 18, STEP_BITS = 26;
-constexpr uint64_t MAX_POS = (1ull << POS_BITS) - 1;
-uint64_t make_stamp(uint64_t step, uint64_t req, uint64_t pos) {
-  return (step << (REQ_BITS + POS_BITS)) | (req << POS_BITS) | (MAX_POS - pos);
+// Recency stamp (native free-queue order, Sec. III-D).  Every touch or
+// admission of a step gets the next value of one running counter, in request
+// order and, within a request, deepest block first: a request releases its
+// blocks tail first, so its deeper blocks are older.  With `base` the number
+// of full blocks of all earlier steps (plus one), request i's block m gets
+//   base + (full blocks of requests 0..i-1) + (n_i - 1 - m).
+// Limits: 2^18-1 requests per step and full blocks per request, 2^31-1 steps.
+constexpr uint64_t MAX_POS = (1ull << 18) - 1;
+constexpr uint64_t MAX_REQ = (1ull << 18) - 1;
+constexpr uint64_t MAX_STEP = (1ull << 31) - 1;
+uint64_t make_stamp(uint64_t base, uint64_t blocks_before, uint64_t n, uint64_t m) {
+  return base + blocks_before + (n - 1 - m);
 }
 
 }  // namespace
@@ -228,6 +232,7 @@ struct Oracle {
   std::vector<int64_t> B;                        // B_{g,c}, fixed point
   int64_t t_prev = 0;                            // last refill time t0
   uint64_t step = 1;                             // index of the next step
+  uint64_t stamp_base = 1;                       // first recency stamp of the next step
   std::map<GKey, History> history;               // keyed by (g, p)
   // S3-FIFO queues keyed by sequence number (head = largest).
   std::map<uint64_t, int32_t> s3_small, s3_main;
@@ -310,8 +315,8 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
   // ---- input validation (state is left unchanged on any error) -----------
   if (sticky != OK) return sticky;
   if (now < t_prev) return ERR_CLOCK;
-  if (R < 0 || (uint64_t)R > (1ull << REQ_BITS) - 1) return ERR_INVALID_ARG;
-  if (step >= (1ull << STEP_BITS)) return ERR_CAPACITY;
+  if (R < 0 || (uint64_t)R > MAX_REQ) return ERR_INVALID_ARG;
+  if (step > MAX_STEP) return ERR_CAPACITY;
   if (R > 0 && offsets[0] != 0) return ERR_INVALID_ARG;
   for (int32_t i = 0; i < R; ++i) {
     if (offsets[i + 1] < offsets[i]) return ERR_INVALID_ARG;
@@ -325,12 +330,13 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
   std::vector<std::vector<uint64_t>> keys(R);
   std::vector<int32_t> g(R), c(R);
   std::vector<uint64_t> p(R);
-  std::vector<int64_t> n(R);
+  std::vector<int64_t> n(R), before(R);  // before[i]: full blocks of requests 0..i-1
   for (int32_t i = 0; i < R; ++i) {
     g[i] = group[i];
     c[i] = contract_ids ? contract_ids[i] : P.contract_of_group[g[i]];
     keys[i] = chain_keys(P.hash_seed, g[i], bs, tokens + offsets[i], offsets[i + 1] - offsets[i]);
     n[i] = (int64_t)keys[i].size();
+    before[i] = i ? before[i - 1] + n[i - 1] : 0;
     // The logical prefix id defaults to the key of the first full block.
     p[i] = prefix_ids ? prefix_ids[i] : (n[i] > 0 ? keys[i][0] : 0);
   }
@@ -447,7 +453,7 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
     const int64_t d = raw_debt(gi);  // D_g(t) before this request's charge
     const bool gate_open = (P.flags & FLAG_NO_DEBT_GATE) || d <= eps;
     for (int64_t m = 0; m < hit[i]; ++m) {
-      const uint64_t st = make_stamp(step, (uint64_t)i, (uint64_t)m);
+      const uint64_t st = make_stamp(stamp_base, (uint64_t)before[i], (uint64_t)n[i], (uint64_t)m);
       int32_t owner_g, owner_c, *klass;
       uint64_t owner_p, *stamp;
       uint32_t* acc;
@@ -494,7 +500,7 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
         Pending pb;
         pb.owner_req = i; pb.pos = (int32_t)m; pb.group = gi; pb.contract = c[i];
         pb.key = keys[i][m]; pb.prefix = p[i]; pb.klass = k_new;
-        pb.stamp = make_stamp(step, (uint64_t)i, (uint64_t)m);
+        pb.stamp = make_stamp(stamp_base, (uint64_t)before[i], (uint64_t)n[i], (uint64_t)m);
         pending[{gi, keys[i][m]}] = pb;
       }
     }
@@ -661,6 +667,7 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
   }
   if (out) out->status = OK;
   step += 1;
+  stamp_base += R ? (uint64_t)(before[R - 1] + n[R - 1]) : 0;
   return OK;
 }
 
@@ -779,7 +786,9 @@ int64_t orc_chain_keys(uint64_t seed, int32_t group, int32_t bs, const int32_t* 
   for (size_t i = 0; i < k.size(); ++i) out[i] = k[i];
   return (int64_t)k.size();
 }
-uint64_t orc_make_stamp(uint64_t step, uint64_t req, uint64_t pos) { return make_stamp(step, req, pos); }
+uint64_t orc_make_stamp(uint64_t base, uint64_t blocks_before, uint64_t n, uint64_t m) {
+  return make_stamp(base, blocks_before, n, m);
+}
 
 // The literal Alg. 2 victim loop on abstract inputs: G groups with projected
 // scores P[g], decrements delta[g], and candidate keys per group (ascending,

@@ -18,9 +18,8 @@ namespace ps {
 // ---- constants -------------------------------------------------------------
 constexpr uint32_t kNone = 0xFFFFFFFFu;           // empty slot / no block
 constexpr int kProb = 0, kNormal = 1, kReuse = 2;  // retention classes (Eq. 9 order)
-constexpr int kStampPosBits = 18, kStampReqBits = 18, kStampStepBits = 26;
-constexpr uint64_t kMaxPos = (1ull << kStampPosBits) - 1;
-constexpr uint64_t kMaxStep = (1ull << kStampStepBits) - 1;
+constexpr uint64_t kMaxPos = (1ull << 18) - 1;   // full blocks per request
+constexpr uint64_t kMaxStep = (1ull << 31) - 1;  // steps (step tags keep 32 bits)
 constexpr int kTableWays = 8;    // native prefix table: 8 x 16 B entries per 128 B bucket
 constexpr int kClaimWays = 4;    // per-step claim map: 4 x 32 B entries per bucket
 constexpr int kRadixBits = 8;
@@ -30,8 +29,11 @@ constexpr int kBmChunk = 256;    // bitmap words per CTA of the id-list compacti
 constexpr uint64_t kP61 = (1ull << 61) - 1;  // chain modulus, a Mersenne prime
 
 // Recency stamp (native free-queue order): larger = more recently released.
-__host__ __device__ __forceinline__ uint64_t make_stamp(uint64_t step, uint64_t req, uint64_t pos) {
-  return (step << (kStampReqBits + kStampPosBits)) | (req << kStampPosBits) | (kMaxPos - pos);
+// One running counter over the steps: request i's block m gets
+// base + (full blocks of the step's earlier requests) + (n_i - 1 - m), so a
+// request's deeper blocks (released first) are older.
+__host__ __device__ __forceinline__ uint64_t make_stamp(uint64_t base, uint64_t pbase, uint64_t n, uint64_t m) {
+  return base + pbase + (n - 1 - m);
 }
 
 // ---- table entries ---------------------------------------------------------
@@ -64,6 +66,7 @@ struct Ctl {
   int32_t sticky;          // PS_OK or PS_ERR_CAPACITY
   int32_t pad0;
   uint64_t step;           // index of the step being / next to be processed (from 1)
+  uint64_t stamp_base;     // first recency stamp of this step (from 1)
   int64_t t_prev;          // last refill time
   int64_t n_resident;
   int64_t hist_live;

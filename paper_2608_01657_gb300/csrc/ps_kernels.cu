@@ -257,6 +257,7 @@ __global__ void k_init_ctl(DevState s) {
   if (threadIdx.x == 0 && blockIdx.x == 0) {
     Ctl c{};
     c.step = 1;
+    c.stamp_base = 1;
     c.s3_head[0] = c.s3_head[1] = kNone;
     c.s3_tail[0] = c.s3_tail[1] = kNone;
     *s.ctl = c;
@@ -789,7 +790,8 @@ __global__ void __launch_bounds__(kThreads) k_touch(DevState s) {
   bool elig;
   if (m < h) {
     const uint32_t b = s.pos_blk[pos];
-    atomicMax(reinterpret_cast<unsigned long long*>(s.blk_stamp + b), (unsigned long long)make_stamp(step, i, m));
+    atomicMax(reinterpret_cast<unsigned long long*>(s.blk_stamp + b),
+              (unsigned long long)make_stamp(c->stamp_base, s.rq_pbase[i], s.rq_n[i], m));
     atomicAdd(s.blk_acc + b, 1u);
     atomicAdd(s.blk_freq + b, 1u);
     elig = proven && s.blk_contract[b] == cid && s.blk_prefix[b] == p && s.blk_klass[b] != kReuse;
@@ -907,6 +909,7 @@ __global__ void k_sel_single(DevState s, int fallback) {
 __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
   Ctl* c = s.ctl;
   __shared__ int64_t sP[PS_MAX_GROUPS], sD[PS_MAX_GROUPS], sQ[PS_MAX_GROUPS];
+  __shared__ uint64_t sRcp[PS_MAX_GROUPS];  // floor((2^64 - 1) / d) for the division below
   __shared__ int64_t s_pmax;
   __shared__ int s_best;
   const int G = s.G;
@@ -917,13 +920,27 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     if (threadIdx.x == 0) c->m_fb = 0;
     return;
   }
-  for (int g = threadIdx.x; g < G; g += blockDim.x) { sP[g] = s.grp_P[g]; sD[g] = s.grp_delta[g]; sQ[g] = s.grp_qsize[g]; }
+  for (int g = threadIdx.x; g < G; g += blockDim.x) {
+    sP[g] = s.grp_P[g];
+    sD[g] = s.grp_delta[g];
+    sQ[g] = s.grp_qsize[g];
+    sRcp[g] = sD[g] > 1 ? ~0ull / (uint64_t)sD[g] : 0;
+  }
   if (threadIdx.x == 0) s_pmax = 0;
   __syncthreads();
+  // floor(x / d) for x >= 0 from the reciprocal: the estimate is at most two
+  // below the quotient, and the correction makes it exact
+  auto div_d = [&](int g, uint64_t x) -> uint64_t {
+    const uint64_t d = (uint64_t)sD[g];
+    if (d == 1) return x;
+    uint64_t q = __umul64hi(x, sRcp[g]);
+    while (x - q * d >= d) ++q;
+    return q;
+  };
   // items of group g with value > t: min(q, floor((P - t - 1) / d) + 1) if P > t
   auto items_gt = [&](int g, int64_t t) -> int64_t {
     const int64_t P = sP[g], d = sD[g];
-    return (P > t && d > 0) ? tmin<int64_t>(sQ[g], (P - t - 1) / d + 1) : 0;
+    return (P > t && d > 0) ? tmin<int64_t>(sQ[g], (int64_t)div_d(g, (uint64_t)(P - t - 1)) + 1) : 0;
   };
   int64_t e = 0, pm = 0;
   for (int g = threadIdx.x; g < G; g += blockDim.x) { e += items_gt(g, eps); pm = tmax(pm, sP[g]); }
@@ -1372,7 +1389,8 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
         s.blk_contract[b] = (uint8_t)s.rq_cid[i];
         s.blk_prefix[b] = s.rq_p[i];
         s.blk_klass[b] = e.promo != kNone ? (uint8_t)kReuse : s.rq_knew[i];
-        s.blk_stamp[b] = make_stamp(c->step, e.last ? e.last - 1 : i, r.m);
+        const uint32_t toucher = e.last ? e.last - 1 : i;  // the last request that touched it
+        s.blk_stamp[b] = make_stamp(c->stamp_base, s.rq_pbase[toucher], s.rq_n[toucher], r.m);
         s.blk_acc[b] = e.tcnt;
         s.blk_freq[b] = e.tcnt;
         s.blk_flags[b] = 1;
@@ -1426,6 +1444,7 @@ __global__ void k_finalize(DevState s) {
   s.out.counts[2] = (int32_t)c->n_inval;
   c->t_prev = s.now;
   c->step += 1;
+  c->stamp_base += c->nblocks;
 }
 
 // Read-only probe output: h_i per request, and the probe's status.

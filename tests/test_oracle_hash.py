@@ -142,12 +142,20 @@ def test_chain_keys_avoid_reserved_values():
     assert len(np.unique(k)) == len(k)
 
 
-def test_stamp_layout_orders_step_request_then_reverse_position():
+def test_stamps_order_step_request_then_reverse_position():
+    """Stamps follow (step, request, deepest block first) and are dense: a step
+    of requests with n = (3, 0, 2) full blocks from base 10 uses 10..14."""
     s = O.make_stamp
-    assert s(2, 0, 0) > s(1, 999, 0)
-    assert s(1, 5, 0) > s(1, 4, 0)
+    n = [3, 0, 2]
+    before = [0, 3, 3]
+    got = {(i, m): s(10, before[i], n[i], m) for i in range(3) for m in range(n[i])}
+    assert sorted(got.values()) == list(range(10, 15))
     # within a request the deeper block is released first, so it is older
-    assert s(1, 4, 0) > s(1, 4, 1) > s(1, 4, 1000)
+    assert got[(0, 0)] > got[(0, 1)] > got[(0, 2)]
+    # a later request is newer than every block of an earlier one
+    assert min(got[(2, m)] for m in range(2)) > max(got[(0, m)] for m in range(3))
+    # the next step starts after all of this step's stamps
+    assert s(15, 0, 1, 0) > max(got.values())
 
 
 P61 = (1 << 61) - 1
