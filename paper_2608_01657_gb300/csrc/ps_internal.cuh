@@ -99,7 +99,8 @@ struct __align__(16) SelSeg {
   int64_t rank;      // 1-based rank still to locate inside the prefix class
   int32_t active;    // 1 while this segment selects
   int32_t incl;      // 1: victims are keys <= prefix; 0: keys < prefix
-  uint64_t kmin, kmax;  // smallest / largest candidate key of the segment
+  uint64_t kmin, kmax;  // a range holding every candidate key of the segment
+  uint32_t hmin, hmax, lmin, lmax;  // ranges of the keys' top / bottom 32 bits
 };
 
 struct DevState {

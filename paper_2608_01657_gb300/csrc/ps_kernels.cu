@@ -761,6 +761,8 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s) {
     SelSeg z{};
     z.kmin = ~0ull;
     z.kmax = 0;
+    z.hmin = z.lmin = ~0u;
+    z.hmax = z.lmax = 0;
     s.sel[g] = z;
   }
 }
@@ -844,16 +846,21 @@ __global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
 // and largest key of every segment, so the radix select can skip the bytes
 // its candidates share.
 __global__ void __launch_bounds__(256) k_cand(DevState s) {
-  // per segment: candidates, and the range of the keys' top 32 bits (class,
-  // step, request's top bits); the bytes below are treated as differing
-  __shared__ unsigned int s_min[PS_MAX_GROUPS], s_max[PS_MAX_GROUPS], s_cnt[PS_MAX_GROUPS];
+  // per segment: candidates, and the ranges of the keys' top and bottom 32
+  // bits (native 32-bit shared atomics); sel_range() combines them
+  __shared__ unsigned int s_hmin[PS_MAX_GROUPS], s_hmax[PS_MAX_GROUPS];
+  __shared__ unsigned int s_lmin[PS_MAX_GROUPS], s_lmax[PS_MAX_GROUPS], s_cnt[PS_MAX_GROUPS];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const uint32_t step32 = (uint32_t)c->step;
   const bool ps = s.policy == PS_PREFIXSHIELD;
   const bool seg = ps && !(s.flags & PS_FLAG_NO_SEGMENTATION);
   const int nseg = ps ? s.G : 1;
-  for (int g = threadIdx.x; g < nseg; g += blockDim.x) { s_min[g] = ~0u; s_max[g] = 0; s_cnt[g] = 0; }
+  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+    s_hmin[g] = s_lmin[g] = ~0u;
+    s_hmax[g] = s_lmax[g] = 0;
+    s_cnt[g] = 0;
+  }
   __syncthreads();
   for (int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; b < s.N; b += (int64_t)gridDim.x * blockDim.x) {
     uint64_t key = ~0ull;
@@ -861,9 +868,11 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
       key = s.blk_stamp[b];
       if (seg) key |= (uint64_t)s.blk_klass[b] << 62;
       const uint32_t g = ps ? s.blk_group[b] : 0;
-      const uint32_t hi = (uint32_t)(key >> 32);
-      atomicMin(&s_min[g], hi);
-      atomicMax(&s_max[g], hi);
+      const uint32_t hi = (uint32_t)(key >> 32), lo = (uint32_t)key;
+      atomicMin(&s_hmin[g], hi);
+      atomicMax(&s_hmax[g], hi);
+      atomicMin(&s_lmin[g], lo);
+      atomicMax(&s_lmax[g], lo);
       atomicAdd(&s_cnt[g], 1u);
     }
     s.csk[b] = key;
@@ -872,9 +881,20 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
   for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
     if (!s_cnt[g]) continue;
     if (ps) atomic_add_i64(s.grp_qsize + g, s_cnt[g]);
-    atomicMin(reinterpret_cast<unsigned long long*>(&s.sel[g].kmin), (unsigned long long)s_min[g] << 32);
-    atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[g].kmax), ((unsigned long long)s_max[g] << 32) | 0xFFFFFFFFull);
+    atomicMin(&s.sel[g].hmin, s_hmin[g]);
+    atomicMax(&s.sel[g].hmax, s_hmax[g]);
+    atomicMin(&s.sel[g].lmin, s_lmin[g]);
+    atomicMax(&s.sel[g].lmax, s_lmax[g]);
   }
+}
+
+// A key range from the two half ranges: exact below the top half when every
+// candidate shares its top 32 bits, conservative otherwise.
+__device__ __forceinline__ void sel_range(SelSeg& z) {
+  if (z.hmin > z.hmax) return;  // no candidate
+  const bool same_hi = z.hmin == z.hmax;
+  z.kmin = ((uint64_t)z.hmin << 32) | (same_hi ? z.lmin : 0u);
+  z.kmax = ((uint64_t)z.hmax << 32) | (same_hi ? z.lmax : 0xFFFFFFFFu);
 }
 
 __device__ __forceinline__ void sel_start(SelSeg& z);
@@ -890,8 +910,15 @@ __global__ void k_sel_single(DevState s, int fallback) {
   z.incl = 1;
   // the fallback selects among the candidates the debt phase left, whose key
   // range the debt phase's split pass recorded
-  z.kmin = fallback ? c->fb_kmin : old.kmin;
-  z.kmax = fallback ? c->fb_kmax : old.kmax;
+  if (fallback) {
+    z.kmin = c->fb_kmin;
+    z.kmax = c->fb_kmax;
+  } else {
+    SelSeg r = old;
+    sel_range(r);
+    z.kmin = r.kmin;
+    z.kmax = r.kmax;
+  }
   sel_start(z);
   s.sel[0] = z;
   c->lst_n = 0;
@@ -955,6 +982,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
       z.rank = x;
       z.active = x > 0;
       z.incl = 1;
+      sel_range(z);
       sel_start(z);
       s.sel[g] = z;
     }
@@ -962,27 +990,34 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     return;
   }
   // tau = max{t in [eps+1, pmax] : items_gt(t - 1) summed >= m}.  Each round
-  // every thread tests one of blockDim thresholds spread over the interval.
+  // tests kThr thresholds spread over the interval; the 16 lanes of a
+  // half-warp split the groups of one threshold.
+  constexpr int kThr = 64, kLanes = 16;
+  __shared__ int s_ok[kThr];
   int64_t lo = eps + 1, hi = s_pmax;
-  const int nt = blockDim.x;
+  const int j = threadIdx.x / kLanes, gl = threadIdx.x % kLanes;
   while (lo < hi) {
     const int64_t span = hi - lo;  // >= 1
-    const int64_t stride = tmax<int64_t>(1, (span - 1) / (nt - 1));
-    auto thr = [&](int j) -> int64_t { return j == nt - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * j); };
-    const int64_t t = thr(threadIdx.x);
+    const int64_t stride = tmax<int64_t>(1, (span - 1) / (kThr - 1));
+    auto thr = [&](int jj) -> int64_t { return jj == kThr - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * jj); };
     int64_t cnt = 0;
-    for (int g = 0; g < G; ++g) cnt += items_gt(g, t - 1);
-    if (threadIdx.x == 0) s_best = -1;
+    if (j < kThr) {
+      const int64_t t = thr(j);
+      for (int g = gl; g < G; g += kLanes) cnt += items_gt(g, t - 1);
+    }
+#pragma unroll
+    for (int o = kLanes / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
+    if (j < kThr && gl == 0) s_ok[j] = cnt >= m;
     __syncthreads();
-    if (cnt >= m) atomicMax(&s_best, (int)threadIdx.x);
-    __syncthreads();
-    const int J = s_best;
+    int J = -1;
+    for (int jj = kThr - 1; jj >= 0; --jj)
+      if (s_ok[jj]) { J = jj; break; }
     __syncthreads();
     if (J < 0) {
       hi = lo;
     } else {
       lo = thr(J);
-      hi = J + 1 < nt ? thr(J + 1) - 1 : hi;
+      hi = J + 1 < kThr ? thr(J + 1) - 1 : hi;
       if (hi < lo) hi = lo;
     }
   }
@@ -998,6 +1033,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     z.rank = xa + (tied ? 1 : 0);
     z.active = z.rank > 0;
     z.incl = tied ? 2 : 1;  // 2: the tie item is taken only if k_tie chooses it
+    sel_range(z);
     sel_start(z);
     s.sel[g] = z;
     s.grp_x[g] = xa + (tied ? 1 : 0);
