@@ -26,6 +26,13 @@ struct ps_handle {
   ps_step_out_t st_out;
   StepTrace trace;
   std::vector<int32_t> contract_of_group;
+  // the step as one CUDA graph, captured on a private stream at first use
+  StepArgs* step_args;
+  cudaStream_t cap_stream = nullptr;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  bool exec_timing = false;
+  bool use_graph = true;
 };
 
 namespace {
@@ -225,6 +232,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.lst_blk = cv.take<uint32_t>(N);
   t.lst_seg = cv.take<uint16_t>(N);
   t.bm_chunk_cnt = cv.take<int32_t>(3 * (((size_t)d.nwords + kBmChunk - 1) / kBmChunk));
+  StepArgs* step_args = cv.take<StepArgs>(1);
   // staging for ps_step_host
   int32_t* st_group = cv.take<int32_t>(R);
   int64_t* st_offsets = cv.take<int64_t>(R + 1);
@@ -246,6 +254,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
     *s = t;
     h->st_group = st_group; h->st_offsets = st_offsets; h->st_tokens = st_tokens;
     h->st_contract = st_contract; h->st_prefix = st_prefix; h->st_out = so;
+    h->step_args = step_args;
   }
   (void)zero_end;
   return total;
@@ -268,6 +277,42 @@ int32_t init_state(ps_handle* h, cudaStream_t st) {
 }
 
 inline cudaStream_t as_stream(void* p) { return reinterpret_cast<cudaStream_t>(p); }
+
+void drop_graph(ps_handle* h) {
+  if (h->exec) cudaGraphExecDestroy(h->exec);
+  if (h->graph) cudaGraphDestroy(h->graph);
+  h->exec = nullptr;
+  h->graph = nullptr;
+}
+
+// Capture the step's launch sequence once (its kernels read the per-step
+// arguments from h->step_args, and every grid depends on the handle's bounds
+// only); on any failure the handle keeps launching kernel by kernel.
+void capture_step(ps_handle* h) {
+  drop_graph(h);
+  DevState tmpl = h->base;
+  tmpl.args = h->step_args;
+  tmpl.R = 0;
+  bool ok = cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+  if (ok) {
+    const int32_t rc = launch_step(tmpl, h->cap_stream, &h->trace);
+    cudaGraph_t g = nullptr;
+    const bool ended = cudaStreamEndCapture(h->cap_stream, &g) == cudaSuccess;
+    ok = rc == PS_OK && ended && g;
+    if (ok) {
+      h->graph = g;
+      ok = cudaGraphInstantiate(&h->exec, g, 0) == cudaSuccess;
+    } else if (g) {
+      cudaGraphDestroy(g);
+    }
+  }
+  cudaGetLastError();  // a failed capture leaves no sticky launch error behind
+  if (!ok) {
+    drop_graph(h);
+    h->use_graph = false;
+  }
+  h->exec_timing = h->trace.timing;
+}
 
 }  // namespace
 
@@ -323,11 +368,14 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   const KeySchedule ks = key_schedule(params->hash_seed, block_size);
   s.chain_mul = ks.kc;
   s.digest_mul = ks.kd;
+  s.args = h->step_args;
   h->base = s;
   h->contract_of_group.assign(params->contract_of_group, params->contract_of_group + num_groups);
   cudaStream_t st = as_stream(stream);
+  configure_kernels(s);  // per device: attributes are set on the current one
   int32_t rc = init_state(h, st);
   if (rc == PS_OK) rc = upload_constants(h, st);
+  if (rc == PS_OK && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess) rc = PS_ERR_CUDA;
   if (rc != PS_OK) {
     delete h;
     return rc;
@@ -354,7 +402,14 @@ int32_t ps_step(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t num_req
   s.in_prefix = d_prefix_ids;
   s.tokens_aligned16 = (reinterpret_cast<uintptr_t>(d_tokens) & 15) == 0;
   s.out = *out;
-  return launch_step(s, as_stream(stream), &h->trace);
+  s.args = h->step_args;
+  cudaStream_t st = as_stream(stream);
+  const StepArgs a = args_of(s);
+  if (cudaMemcpyAsync(h->step_args, &a, sizeof(a), cudaMemcpyHostToDevice, st) != cudaSuccess) return PS_ERR_CUDA;
+  if (h->use_graph && (!h->exec || h->exec_timing != h->trace.timing)) capture_step(h);
+  if (h->use_graph && h->exec)
+    return cudaGraphLaunch(h->exec, st) == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+  return launch_step(s, st, &h->trace);
 }
 
 int32_t ps_step_host(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t num_requests, const int32_t* h_group_ids,
@@ -440,6 +495,8 @@ int32_t ps_cached_prefix(ps_handle_t* h, void* stream, int32_t num_requests, con
 
 void ps_destroy(ps_handle_t* h) {
   if (!h) return;
+  drop_graph(h);
+  if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   if (h->trace.timing)
     for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
   delete h;
@@ -452,6 +509,7 @@ int32_t ps_set_stage_timing(ps_handle_t* h, int32_t enable) {
       if (cudaEventCreate(&e) != cudaSuccess) return PS_ERR_CUDA;
     h->trace.timing = true;
   } else if (!enable && h->trace.timing) {
+    drop_graph(h);  // its event nodes refer to the events
     for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
     h->trace.timing = false;
   }

@@ -103,6 +103,20 @@ struct __align__(16) SelSeg {
   uint32_t hmin, hmax, lmin, lmax;  // ranges of the keys' top / bottom 32 bits
 };
 
+// Per-call arguments of a step or probe, in device memory: the step's kernels
+// read them at entry, so one captured CUDA graph serves every step.
+struct StepArgs {
+  int64_t now;
+  int32_t R;
+  int32_t tokens_aligned16;
+  const int32_t* in_group;
+  const int64_t* in_offsets;
+  const int32_t* in_tokens;
+  const int32_t* in_contract;
+  const uint64_t* in_prefix;
+  ps_step_out_t out;
+};
+
 struct DevState {
   // constants
   int64_t N;
@@ -195,7 +209,8 @@ struct DevState {
   uint32_t* lst_blk;
   uint16_t* lst_seg;
   int32_t* bm_chunk_cnt;   // [3][chunks] bitmap compaction counts
-  // current step inputs / outputs
+  StepArgs* args;          // this call's arguments (device memory)
+  // current step inputs / outputs (kernels refresh them from *args)
   int64_t now;
   int32_t R;
   const int32_t* in_group;
@@ -239,6 +254,33 @@ struct StepTrace {
   bool timing = false;
   int launches = 0;
 };
+
+// Copy the call's arguments from device memory into the kernel's DevState.
+__device__ __forceinline__ DevState with_args(DevState s) {
+  const StepArgs* a = s.args;
+  if (a == nullptr) return s;  // launched directly with its arguments by value
+  s.now = a->now;
+  s.R = a->R;
+  s.tokens_aligned16 = a->tokens_aligned16;
+  s.in_group = a->in_group;
+  s.in_offsets = a->in_offsets;
+  s.in_tokens = a->in_tokens;
+  s.in_contract = a->in_contract;
+  s.in_prefix = a->in_prefix;
+  s.out = a->out;
+  return s;
+}
+// The host-side argument block of a DevState.
+inline StepArgs args_of(const DevState& s) {
+  StepArgs a{};
+  a.now = s.now; a.R = s.R; a.tokens_aligned16 = s.tokens_aligned16;
+  a.in_group = s.in_group; a.in_offsets = s.in_offsets; a.in_tokens = s.in_tokens;
+  a.in_contract = s.in_contract; a.in_prefix = s.in_prefix; a.out = s.out;
+  return a;
+}
+// Kernel attributes (shared-memory opt-ins), set once per process before
+// any launch or capture.
+void configure_kernels(const DevState& s);
 void launch_init(const DevState& s, cudaStream_t st);
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr);
 // S3-FIFO (ps_s3fifo.cu)

@@ -269,6 +269,7 @@ __global__ void k_init_ctl(DevState s) {
 // Stage 0: validation of the step's inputs; n_i, block positions, hashing
 // segments.  One CTA.  'probe' skips the clock and step checks.
 __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   __shared__ int s_bad;
   if (threadIdx.x == 0) s_bad = 0;
@@ -364,6 +365,7 @@ __device__ __forceinline__ uint32_t smem_addr(const void* p) {
 
 template <int PPB>
 __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) {
+  s = with_args(s);
   extern __shared__ __align__(16) int32_t smem_tokens[];
   using Cfg = HashCfg<PPB>;
   constexpr int BS = Cfg::BS;
@@ -481,6 +483,7 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
 // key_m = mix(C_m ^ (m+1) c) with C_m = Kc^(k+1) C_in + B_m, then a table
 // probe; a miss lowers the request's h_i to its position.
 __global__ void __launch_bounds__(kThreads) k_keys_lookup(DevState s) {
+  s = with_args(s);
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -505,6 +508,7 @@ __global__ void __launch_bounds__(kThreads) k_keys_lookup(DevState s) {
 // Threads past the positions record each request's history entry
 // (OnRequest of Alg. 1) under its prefix id.
 __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -560,6 +564,7 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
 // resident block past a request's first miss cannot be reached by lookup; it
 // is dropped (invalidated) unless some request pinned it.
 __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   if (c->hist_live + c->hist_new > s.history_capacity) {  // history capacity is sticky
@@ -599,6 +604,7 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
 // resident = N - pinned; claims are ranked in (request, position) order; the
 // first avail ranks are materialized.  One CTA.
 __global__ void __launch_bounds__(1024) k_grant(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int R = s.R;
@@ -638,6 +644,7 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
 // the leading granted ones are hits.  A position whose owner's rank is past
 // avail lowers the request's first-ungranted mark.
 __global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
+  s = with_args(s);
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -652,6 +659,7 @@ __global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
 // hit_i = h_i + e_i per request; records the first admitting request of each
 // (group, prefix) history entry of the step.
 __global__ void k_instep_fin(DevState s) {
+  s = with_args(s);
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -676,6 +684,7 @@ __global__ void k_instep_fin(DevState s) {
 // the start of the step and the first request of the step that referenced /
 // admitted it.  Also writes the group's statistics, balances and debts.
 __global__ void __launch_bounds__(1024) k_meter(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int g = blockIdx.x;
@@ -775,6 +784,7 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s) {
 // promotion (or all of them when none promotes) and applies the promotion of
 // resident blocks.
 __global__ void __launch_bounds__(kThreads) k_touch(DevState s) {
+  s = with_args(s);
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -811,6 +821,7 @@ __global__ void __launch_bounds__(kThreads) k_touch(DevState s) {
 }
 
 __global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
+  s = with_args(s);
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -846,6 +857,7 @@ __global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
 // and largest key of every segment, so the radix select can skip the bytes
 // its candidates share.
 __global__ void __launch_bounds__(256) k_cand(DevState s) {
+  s = with_args(s);
   // per segment: candidates, and the ranges of the keys' top and bottom 32
   // bits (native 32-bit shared atomics); sel_range() combines them
   __shared__ unsigned int s_hmin[PS_MAX_GROUPS], s_hmax[PS_MAX_GROUPS];
@@ -899,6 +911,7 @@ __device__ __forceinline__ void sel_range(SelSeg& z) {
 
 __device__ __forceinline__ void sel_start(SelSeg& z);
 __global__ void k_sel_single(DevState s, int fallback) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (threadIdx.x != 0) return;
   int64_t m = 0;
@@ -934,6 +947,7 @@ __global__ void k_sel_single(DevState s, int fallback) {
 // the radix select finds those keys).  What the debt phase cannot cover goes
 // to the global fallback in (class, stamp) order.
 __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   __shared__ int64_t sP[PS_MAX_GROUPS], sD[PS_MAX_GROUPS], sQ[PS_MAX_GROUPS];
   __shared__ uint64_t sRcp[PS_MAX_GROUPS];  // floor((2^64 - 1) / d) for the division below
@@ -1086,6 +1100,7 @@ __device__ __forceinline__ void sel_start(SelSeg& z) {
 // One digit for every segment that still has one: over the whole candidate
 // array (from_list = 0) or over the split list (from_list = 1).
 __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int fallback, int from_list) {
+  s = with_args(s);
   extern __shared__ uint32_t shist[];
   __shared__ int16_t row_of[PS_MAX_GROUPS];
   __shared__ int16_t seg_of_row[PS_MAX_GROUPS];
@@ -1199,6 +1214,7 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
 // pass also records the key range of every candidate it does not mark, for
 // the global fallback.
 __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallback) {
+  s = with_args(s);
   __shared__ unsigned long long s_rng[2];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
@@ -1262,6 +1278,7 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
 // among the groups holding an item at exactly tau (incl == 2 after the
 // water-filling), the k with the smallest candidate keys take it.
 __global__ void __launch_bounds__(1024) k_tie(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0 || c->sel_ntie == 0) return;
   const int G = s.G;
@@ -1287,6 +1304,7 @@ __global__ void __launch_bounds__(1024) k_tie(DevState s) {
 // Mark the list's victims: keys below (or equal to, if incl) the located
 // threshold of their segment.
 __global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   if (single && !s.sel[0].active) return;
@@ -1305,6 +1323,7 @@ __global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
 // contiguous word ranges per thread).  With the victims they form the
 // allocated set; the id-list compaction takes their union.
 __global__ void __launch_bounds__(1024) k_freetake(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->ftake == 0) return;
   const int64_t ftake = c->ftake;
@@ -1340,6 +1359,7 @@ __global__ void __launch_bounds__(1024) k_freetake(DevState s) {
 // Bitmaps -> ascending id lists (allocated, evicted, invalidated).  Each CTA
 // owns kBmChunk bitmap words; pass 1 counts, pass 2 scans the counts and writes.
 __global__ void __launch_bounds__(kBmChunk) k_bm_count(DevState s) {
+  s = with_args(s);
   if (s.ctl->status != PS_OK) return;
   const int64_t w = (int64_t)blockIdx.x * kBmChunk + threadIdx.x;
   const uint32_t* bms[3] = {s.bm_alloc, s.bm_victim, s.bm_inval};
@@ -1353,6 +1373,7 @@ __global__ void __launch_bounds__(kBmChunk) k_bm_count(DevState s) {
   }
 }
 __global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
+  s = with_args(s);
   if (s.ctl->status != PS_OK) return;
   const int64_t w = (int64_t)blockIdx.x * kBmChunk + threadIdx.x;
   uint32_t* bms[3] = {s.bm_alloc, s.bm_victim, s.bm_inval};
@@ -1384,6 +1405,7 @@ __global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
 
 // Evict the victims (thread per evicted id): drop table entries and metadata.
 __global__ void __launch_bounds__(kThreads) k_evict(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -1402,6 +1424,7 @@ __global__ void __launch_bounds__(kThreads) k_evict(DevState s) {
 // block carries the metadata OnCacheFullBlocks attached plus any in-step
 // touches.
 __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -1444,6 +1467,7 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
 // OnRequest / RecordSuccessfulAdmission commit: reference counts and admitted
 // flags of the history entries (thread per request).
 __global__ void k_hist_commit(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -1457,6 +1481,7 @@ __global__ void k_hist_commit(DevState s) {
 
 // Clear the claim-map slots this step used (thread per position).
 __global__ void __launch_bounds__(kThreads) k_claim_clear(DevState s) {
+  s = with_args(s);
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -1470,6 +1495,7 @@ __global__ void __launch_bounds__(kThreads) k_claim_clear(DevState s) {
 }
 
 __global__ void k_finalize(DevState s) {
+  s = with_args(s);
   Ctl* c = s.ctl;
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   const int32_t st = c->internal_error ? PS_ERR_DEVICE_STATUS : c->status;
@@ -1485,6 +1511,7 @@ __global__ void k_finalize(DevState s) {
 
 // Read-only probe output: h_i per request, and the probe's status.
 __global__ void k_probe_out(DevState s, int32_t* out, int32_t* status) {
+  s = with_args(s);
   const Ctl* c = s.ctl;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i == 0) *status = c->status;
@@ -1509,7 +1536,6 @@ void launch_init(const DevState& s, cudaStream_t st) {
 template <int PPB>
 static void launch_hash_t(const DevState& s, cudaStream_t st) {
   using Cfg = HashCfg<PPB>;
-  cudaFuncSetAttribute(k_hash<PPB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Cfg::kSmem);
   k_hash<PPB><<<(int)((s.max_segments + Cfg::kWarps - 1) / Cfg::kWarps), Cfg::kWarps * 32, Cfg::kSmem, st>>>(s);
 }
 static int32_t launch_hash(const DevState& s, cudaStream_t st) {
@@ -1525,8 +1551,20 @@ static int32_t launch_hash(const DevState& s, cudaStream_t st) {
   return PS_OK;
 }
 
+void configure_kernels(const DevState& s) {
+  (void)s;
+  cudaFuncSetAttribute(k_digit_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, kRadixSmemRows * kRadixBins * 4);
+  cudaFuncSetAttribute(k_hash<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<1>::kSmem);
+  cudaFuncSetAttribute(k_hash<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<2>::kSmem);
+  cudaFuncSetAttribute(k_hash<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<4>::kSmem);
+  cudaFuncSetAttribute(k_hash<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<8>::kSmem);
+  cudaFuncSetAttribute(k_hash<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<16>::kSmem);
+  cudaFuncSetAttribute(k_hash<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<32>::kSmem);
+}
+
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
-  const int R = s.R;
+  // grids depend only on the handle's bounds (a captured graph serves any step)
+  const int R = s.max_requests;
   const int rgrid = grid_for(R, 256, 1 << 20);
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
   const int prgrid = grid_for(s.max_blocks + R, kThreads, 1 << 30);
@@ -1537,19 +1575,16 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   const int radix_smem = kRadixSmemRows * kRadixBins * 4;
   int launches = 0;
   auto mark = [&](int stage) {
-    if (tr && tr->timing) cudaEventRecord(tr->ev[stage], st);
+    // external: under capture the record becomes a node of the graph
+    if (tr && tr->timing) cudaEventRecordWithFlags(tr->ev[stage], st, cudaEventRecordExternal);
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
-  // dynamic plus static shared memory exceeds the 48 KB default: opt in
-  cudaFuncSetAttribute(k_digit_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, radix_smem);
   mark(0);
   PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s, 0));
   mark(1);
-  if (R > 0) {
-    if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
-    ++launches;
-    PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
-  }
+  if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
+  ++launches;
+  PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
   mark(2);
   PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
@@ -1605,15 +1640,16 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
 }
 
 int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* status) {
-  const int R = s.R;
-  const int rgrid = grid_for(R, 256, 1 << 20);
+  const int rgrid = grid_for(s.R, 256, 1 << 20);
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
-  k_validate<<<1, 1024, 0, st>>>(s, 1);
-  if (R > 0) {
-    if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
-    k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s);
+  DevState p = s;
+  p.args = nullptr;  // the probe's kernels take every argument by value
+  k_validate<<<1, 1024, 0, st>>>(p, 1);
+  if (s.R > 0) {
+    if (launch_hash(p, st) != PS_OK) return PS_ERR_INVALID_ARG;
+    k_keys_lookup<<<pgrid, kThreads, 0, st>>>(p);
   }
-  k_probe_out<<<rgrid, 256, 0, st>>>(s, out, status);
+  k_probe_out<<<rgrid, 256, 0, st>>>(p, out, status);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 

@@ -144,6 +144,7 @@ __device__ bool ghost_push(const DevState& s, Ctl* c, uint64_t key, uint32_t g) 
 
 // Unlink the step's invalidated blocks, then choose the step's m victims.
 __global__ void k_s3_evict(DevState s) {
+  s = with_args(s);
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
@@ -222,6 +223,7 @@ __global__ void k_s3_evict(DevState s) {
 // Link the step's new blocks in rank order: a key found in the ghost enters
 // the main queue (and leaves the ghost), any other the small queue.
 __global__ void k_s3_insert(DevState s) {
+  s = with_args(s);
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;

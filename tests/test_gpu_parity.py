@@ -235,3 +235,34 @@ def test_cached_prefix_probe(policy):
     t = torch.zeros(32, dtype=torch.int32, device=dev)
     _, status = gpu.cached_prefix(g, o, t)
     assert int(status.item()) == O.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+def test_parity_graph_replay_streams_and_timing(policy):
+    """The step replays one captured graph: steps of every size (empty ones
+    included) on a side stream, stage timing switched on and off (which
+    captures the step again), with every output and the state checked."""
+    steps = W.fuzz_steps(21, 3, 6, 48, docs_per_group=3, doc_blocks=7, fresh_max_blocks=2,
+                         with_contracts=3, with_prefixes=True, now_stride=2, empty_every=5)
+    kw = dict(rho=(2.0, 1.5, 1.0), beta=(6.0, 5.0, 4.0), contract_of_group=[0, 1, 2])
+    gpu, orc = _pair(40, 16, 3, policy, kw, max_requests=6, max_tokens=4096)
+    dev = torch.device("cuda")
+    side = torch.cuda.Stream()
+    for k, st in enumerate(steps):
+        if k % 7 == 3:
+            gpu.set_stage_timing(k % 14 == 3)
+        with torch.cuda.stream(side):
+            g = torch.from_numpy(st.groups).to(dev)
+            o = torch.from_numpy(st.offsets).to(dev)
+            t = torch.from_numpy(st.tokens if st.num_tokens else np.zeros(4, np.int32)).to(dev)
+            c = torch.from_numpy(st.contracts).to(dev)
+            p = torch.from_numpy(st.prefixes.view(np.int64)).to(dev)
+            assert gpu.step(st.now, g, o, t, c, p, stream=side) == 0
+        got = gpu.fetch(st.num_requests, stream=side)
+        want = orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts, st.prefixes)
+        compare_outputs(got, want, f"graph/{policy} step {k}")
+        if k % 7 == 3 and k % 14 == 3:
+            ms, launches = gpu.stage_times()
+            assert launches > 0 and np.all(ms >= 0)
+    compare_state(gpu.export(), orc.export(), f"graph/{policy}", s3=policy == "s3fifo")
+    assert np.array_equal(gpu.stats(), orc.stats())
