@@ -683,8 +683,10 @@ __global__ void k_instep_fin(DevState s) {
 // q_r >= 1 and "(g,p) was admitted" come from the history entry as it stood at
 // the start of the step and the first request of the step that referenced /
 // admitted it.  Also writes the group's statistics, balances and debts.
-__global__ void __launch_bounds__(1024) k_meter(DevState s) {
-  s = with_args(s);
+__global__ void __launch_bounds__(1024) k_meter(DevState s0) {
+  // Contract arrays are read from the parameter block: indexing the per-step
+  // copy by a run-time contract would move the whole copy to local memory.
+  const DevState s = with_args(s0);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int g = blockIdx.x;
@@ -694,7 +696,7 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s) {
   __shared__ int64_t B0[PS_MAX_CONTRACTS];
   if (threadIdx.x < C) {
     const int cc = threadIdx.x;
-    B0[cc] = refill(s.ledger[g * C + cc], s.beta[cc], s.rho[cc], s.now - c->t_prev);
+    B0[cc] = refill(s.ledger[g * C + cc], s0.beta[cc], s0.rho[cc], s.now - c->t_prev);
   }
   __syncthreads();
   int64_t carry[PS_MAX_CONTRACTS];
@@ -708,23 +710,22 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s) {
     int n = 0, a = 0, cid = 0;
     if (member) { n = s.rq_n[i]; a = s.rq_a[i]; cid = s.rq_cid[i]; }
     const bool pol = member && n > 0;
-    int64_t S[PS_MAX_CONTRACTS];
+    // charges of this group's earlier requests, per contract; then the raw
+    // debt before this request's charge (Eq. 3) and the balance after it
+    int64_t d = 0, b_after = 0;
 #pragma unroll
     for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
       if (cc < C) {
         int64_t tot;
         const int64_t ex = block_excl_scan<int64_t>((pol && cid == cc) ? a : 0, &tot);
-        S[cc] = carry[cc] + ex;
+        const int64_t Sx = carry[cc] + ex;
         carry[cc] += tot;
-      } else {
-        S[cc] = 0;
+        d += tmax<int64_t>(0, -(B0[cc] - Sx * unit));
+        if (cid == cc) b_after = B0[cc] - (Sx + a) * unit;
       }
     }
     if (pol) {
-      int64_t d = 0;
-      for (int cc = 0; cc < C; ++cc) d += tmax<int64_t>(0, -(B0[cc] - S[cc] * unit));
       const bool gate = (s.flags & PS_FLAG_NO_DEBT_GATE) || d <= s.eps;
-      const int64_t b_after = B0[cid] - (S[cid] + a) * unit;
       const uint32_t hs = s.rq_hs[i];
       HistEntry he{};
       if (hs != kNone) he = s.hist[hs];
@@ -752,13 +753,16 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s) {
     row[PS_STAT_ADMITTED_BLOCKS] += st_adm;
     row[PS_STAT_UNGRANTED_BLOCKS] += st_ungr;
     int64_t raw = 0, norm = 0, rmax = 0;
-    for (int cc = 0; cc < C; ++cc) {
-      const int64_t b = B0[cc] - carry[cc] * unit;  // Eq. 2 over the step's charges
-      s.ledger[g * C + cc] = b;
-      const int64_t def = tmax<int64_t>(0, -b);
-      raw += def;                                    // Eq. 3
-      norm += muldiv(def, s.rho_min, s.rho[cc]);     // Eq. 5
-      if (b < 0) rmax = tmax(rmax, s.rho[cc]);
+#pragma unroll
+    for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
+      if (cc < C) {
+        const int64_t b = B0[cc] - carry[cc] * unit;  // Eq. 2 over the step's charges
+        s.ledger[g * C + cc] = b;
+        const int64_t def = tmax<int64_t>(0, -b);
+        raw += def;                                    // Eq. 3
+        norm += muldiv(def, s.rho_min, s0.rho[cc]);    // Eq. 5
+        if (b < 0) rmax = tmax(rmax, s0.rho[cc]);
+      }
     }
     row[PS_STAT_DEBT_RAW] = raw;
     row[PS_STAT_DEBT_NORM] = norm;
