@@ -101,6 +101,7 @@ struct __align__(16) SelSeg {
   int32_t incl;      // 1: victims are keys <= prefix; 0: keys < prefix
   uint64_t kmin, kmax;  // a range holding every candidate key of the segment
   uint32_t hmin, hmax, lmin, lmax;  // ranges of the keys' top / bottom 32 bits
+  uint64_t qmin, qmax;  // range of the segment's keys on the split list
 };
 
 // Per-call arguments of a step or probe, in device memory: the step's kernels

@@ -776,6 +776,8 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s0) {
     z.kmax = 0;
     z.hmin = z.lmin = ~0u;
     z.hmax = z.lmax = 0;
+    z.qmin = ~0ull;
+    z.qmax = 0;
     s.sel[g] = z;
   }
 }
@@ -878,20 +880,31 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
     s_cnt[g] = 0;
   }
   __syncthreads();
-  for (int64_t b = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; b < s.N; b += (int64_t)gridDim.x * blockDim.x) {
+  // warp-uniform trip count; lanes of one group combine their ranges and
+  // counts with warp reductions, and one lane per group updates shared memory
+  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t b = b0 + threadIdx.x;
     uint64_t key = ~0ull;
-    if ((s.blk_flags[b] & 1) && s.blk_pin[b] != step32) {
+    uint32_t g = ~0u;
+    if (b < s.N && (s.blk_flags[b] & 1) && s.blk_pin[b] != step32) {
       key = s.blk_stamp[b];
       if (seg) key |= (uint64_t)s.blk_klass[b] << 62;
-      const uint32_t g = ps ? s.blk_group[b] : 0;
-      const uint32_t hi = (uint32_t)(key >> 32), lo = (uint32_t)key;
-      atomicMin(&s_hmin[g], hi);
-      atomicMax(&s_hmax[g], hi);
-      atomicMin(&s_lmin[g], lo);
-      atomicMax(&s_lmax[g], lo);
-      atomicAdd(&s_cnt[g], 1u);
+      g = ps ? s.blk_group[b] : 0;
     }
-    s.csk[b] = key;
+    const unsigned peers = __match_any_sync(kFull, g);
+    if (g != ~0u) {
+      const uint32_t hi = (uint32_t)(key >> 32), lo = (uint32_t)key;
+      const uint32_t hmin = __reduce_min_sync(peers, hi), hmax = __reduce_max_sync(peers, hi);
+      const uint32_t lmin = __reduce_min_sync(peers, lo), lmax = __reduce_max_sync(peers, lo);
+      if (lane_id() == __ffs(peers) - 1) {
+        atomicMin(&s_hmin[g], hmin);
+        atomicMax(&s_hmax[g], hmax);
+        atomicMin(&s_lmin[g], lmin);
+        atomicMax(&s_lmax[g], lmax);
+        atomicAdd(&s_cnt[g], (unsigned)__popc(peers));
+      }
+    }
+    if (b < s.N) s.csk[b] = key;
   }
   __syncthreads();
   for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
@@ -925,6 +938,8 @@ __global__ void k_sel_single(DevState s, int fallback) {
   z.rank = m;
   z.active = m > 0;
   z.incl = 1;
+  z.qmin = ~0ull;
+  z.qmax = 0;
   // the fallback selects among the candidates the debt phase left, whose key
   // range the debt phase's split pass recorded
   if (fallback) {
@@ -1101,6 +1116,18 @@ __device__ __forceinline__ void sel_start(SelSeg& z) {
   }
 }
 
+// A segment as the list passes see it: the list's members of the segment all
+// share the bits above the highest byte where the list's smallest and largest
+// key differ, so those bytes are fixed without counting.
+__device__ __forceinline__ SelSeg list_view(SelSeg z) {
+  if (z.qmin > z.qmax) return z;  // no member on the list
+  const int fs = first_shift(z.qmin, z.qmax);
+  const uint64_t cm = fs < 0 ? ~0ull : above_mask(fs);
+  z.mask |= cm;
+  z.prefix |= z.qmin & cm;
+  return z;
+}
+
 // One digit for every segment that still has one: over the whole candidate
 // array (from_list = 0) or over the split list (from_list = 1).
 __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int fallback, int from_list) {
@@ -1120,7 +1147,7 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
       const int g = base + threadIdx.x;
       bool counts = false;
       if (g < nseg) {
-        const SelSeg ss = s.sel[g];
+        const SelSeg ss = from_list ? list_view(s.sel[g]) : s.sel[g];
         counts = ss.active && next_shift(ss.mask) >= 0;
       }
       int tot;
@@ -1159,7 +1186,7 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
       if (ok) {
         const int row = row_of[seg];
         if (row >= 0) {
-          const SelSeg ss = s.sel[seg];
+          const SelSeg ss = from_list ? list_view(s.sel[seg]) : s.sel[seg];
           if ((key & ss.mask) == ss.prefix) {
             act = true;
             const int sh = next_shift(ss.mask);
@@ -1185,7 +1212,7 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
   const int warp = threadIdx.x >> 5, lane = lane_id();
   for (int r = warp; r < nrows; r += blockDim.x >> 5) {
     const int seg = seg_of_row[r];
-    SelSeg ss = s.sel[seg];
+    SelSeg ss = from_list ? list_view(s.sel[seg]) : s.sel[seg];
     const int sh = next_shift(ss.mask);
     uint32_t* row = s.hist_bins + (size_t)seg * kRadixBins;
     uint32_t v[kRadixBins / 32];
@@ -1260,6 +1287,18 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
         s.lst_blk[slot] = (uint32_t)b;
         s.lst_seg[slot] = (uint16_t)seg;
       }
+      // the list's key range per segment (lanes of one segment combined)
+      const unsigned peers = __match_any_sync(kFull, to_list ? (uint32_t)seg : ~0u);
+      if (to_list) {
+        const uint32_t hi = (uint32_t)(key >> 32), lo = (uint32_t)key;
+        const uint32_t hmin = __reduce_min_sync(peers, hi), hmax = __reduce_max_sync(peers, hi);
+        const uint32_t lmin = __reduce_min_sync(peers, hi == hmin ? lo : ~0u);
+        const uint32_t lmax = __reduce_max_sync(peers, hi == hmax ? lo : 0u);
+        if (lane_id() == __ffs(peers) - 1) {
+          atomicMin(reinterpret_cast<unsigned long long*>(&s.sel[seg].qmin), ((unsigned long long)hmin << 32) | lmin);
+          atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[seg].qmax), ((unsigned long long)hmax << 32) | lmax);
+        }
+      }
     }
   }
   if (track) {
@@ -1290,7 +1329,7 @@ __global__ void __launch_bounds__(1024) k_tie(DevState s) {
   __shared__ uint64_t tkey[PS_MAX_GROUPS];
   __shared__ int tied[PS_MAX_GROUPS];
   for (int g = threadIdx.x; g < G; g += blockDim.x) {
-    const SelSeg sg = s.sel[g];
+    const SelSeg sg = list_view(s.sel[g]);
     tied[g] = sg.active && sg.incl == 2;
     tkey[g] = sg.prefix;
   }
@@ -1315,7 +1354,7 @@ __global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
   const int64_t n = c->lst_n;
   for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
     const uint64_t key = s.lst_key[e];
-    const SelSeg ss = s.sel[s.lst_seg[e]];
+    const SelSeg ss = list_view(s.sel[s.lst_seg[e]]);
     if (ss.active && (key < ss.prefix || (ss.incl && key == ss.prefix))) {
       const uint32_t b = s.lst_blk[e];
       atomicOr(s.bm_victim + (b >> 5), 1u << (b & 31));
