@@ -17,6 +17,8 @@ namespace ps {
 constexpr unsigned kFull = 0xFFFFFFFFu;
 constexpr int kThreads = 256;     // position-parallel kernels
 constexpr int kRadixSmemRows = 48;  // radix rows counted in shared memory (48 KB)
+constexpr int64_t kListSmall = 16384;  // split lists up to this size are finished by one CTA
+constexpr int kFinRows = 32;           // rows k_list_finish counts at once (32 KB)
 
 // ---------------------------------------------------------------------------
 // small device helpers
@@ -886,10 +888,16 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
     const int64_t b = b0 + threadIdx.x;
     uint64_t key = ~0ull;
     uint32_t g = ~0u;
-    if (b < s.N && (s.blk_flags[b] & 1) && s.blk_pin[b] != step32) {
-      key = s.blk_stamp[b];
-      if (seg) key |= (uint64_t)s.blk_klass[b] << 62;
-      g = ps ? s.blk_group[b] : 0;
+    if (b < s.N) {
+      // every load issued at once (no dependent round trips)
+      const uint8_t fl = s.blk_flags[b], kl = s.blk_klass[b];
+      const uint32_t pin = s.blk_pin[b];
+      const uint64_t st = s.blk_stamp[b];
+      const uint16_t grp = s.blk_group[b];
+      if ((fl & 1) && pin != step32) {
+        key = seg ? (st | (uint64_t)kl << 62) : st;
+        g = ps ? grp : 0;
+      }
     }
     const unsigned peers = __match_any_sync(kFull, g);
     if (g != ~0u) {
@@ -1042,9 +1050,11 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     for (int o = kLanes / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
     if (j < kThr && gl == 0) s_ok[j] = cnt >= m;
     __syncthreads();
-    int J = -1;
-    for (int jj = kThr - 1; jj >= 0; --jj)
-      if (s_ok[jj]) { J = jj; break; }
+    // J = the largest threshold that still holds m items (counts fall as the
+    // threshold rises, so the flags are a prefix): two ballots per warp
+    const unsigned lo32 = __ballot_sync(kFull, s_ok[lane_id()] != 0);
+    const unsigned hi32 = __ballot_sync(kFull, s_ok[32 + lane_id()] != 0);
+    const int J = hi32 ? 63 - __clz((int)hi32) : (lo32 ? 31 - __clz((int)lo32) : -1);
     __syncthreads();
     if (J < 0) {
       hi = lo;
@@ -1065,7 +1075,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     SelSeg z = s.sel[g];
     z.rank = xa + (tied ? 1 : 0);
     z.active = z.rank > 0;
-    z.incl = tied ? 2 : 1;  // 2: the tie item is taken only if k_tie chooses it
+    z.incl = tied ? 2 : 1;  // 2: the tie item is taken only if the tie rule chooses it
     sel_range(z);
     sel_start(z);
     s.sel[g] = z;
@@ -1140,6 +1150,7 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
   if (c->status != PS_OK || c->mvict == 0) return;
   const int nseg = single ? 1 : s.G;
   if (single && !s.sel[0].active) return;
+  if (from_list && c->lst_n <= kListSmall) return;  // k_list_finish takes short lists whole
   // rows for the segments that still count (parallel flags, scanned)
   {
     int k = 0;
@@ -1180,7 +1191,7 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
         ok = true;
       } else {
         key = s.csk[e];
-        seg = single ? 0 : s.blk_group[e];
+        seg = single ? 0 : s.blk_group[e];  // issued with the key load
         ok = key != ~0ull && !(fallback && ((s.bm_victim[e >> 5] >> (e & 31)) & 1));
       }
       if (ok) {
@@ -1262,8 +1273,9 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
     int seg = 0;
     if (b < s.N) {
       key = s.csk[b];
+      const int grp = single ? 0 : s.blk_group[b];
       if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
-        seg = single ? 0 : s.blk_group[b];
+        seg = grp;
         const SelSeg ss = s.sel[seg];
         if (ss.active) {
           const uint64_t k = key & ss.mask;
@@ -1316,43 +1328,117 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
 }
 
-// Ties at tau (Eq. 7's tie rule: equal projected debt is broken by the
-// retention segment and native queue order of each group's next candidate):
-// among the groups holding an item at exactly tau (incl == 2 after the
-// water-filling), the k with the smallest candidate keys take it.
-__global__ void __launch_bounds__(1024) k_tie(DevState s) {
+// The rest of a select on one CTA: every remaining digit of every segment
+// over the split list (shared-memory histograms, up to kFinRows segments per
+// sweep), then the tie rule at tau for the debt phase, then the list's victims.
+// Long lists have been narrowed by the multi-CTA list passes before this.
+__global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
   s = with_args(s);
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK || c->mvict == 0 || c->sel_ntie == 0) return;
-  const int G = s.G;
-  const int64_t k = c->sel_k;
-  __shared__ uint64_t tkey[PS_MAX_GROUPS];
-  __shared__ int tied[PS_MAX_GROUPS];
-  for (int g = threadIdx.x; g < G; g += blockDim.x) {
-    const SelSeg sg = list_view(s.sel[g]);
-    tied[g] = sg.active && sg.incl == 2;
-    tkey[g] = sg.prefix;
-  }
-  __syncthreads();
-  for (int g = threadIdx.x; g < G; g += blockDim.x) {
-    if (!tied[g]) continue;
-    int rank = 0;
-    for (int h = 0; h < G; ++h) rank += tied[h] && tkey[h] < tkey[g];
-    const bool chosen = rank < k;
-    s.sel[g].incl = chosen ? 1 : 0;
-    if (!chosen) s.grp_x[g] -= 1;
-  }
-}
-
-// Mark the list's victims: keys below (or equal to, if incl) the located
-// threshold of their segment.
-__global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
-  s = with_args(s);
+  __shared__ __align__(16) uint32_t fh[kFinRows * kRadixBins];
+  __shared__ int16_t row_of[PS_MAX_GROUPS];
+  __shared__ int16_t seg_of_row[PS_MAX_GROUPS];
+  __shared__ int s_nrows;
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   if (single && !s.sel[0].active) return;
+  const int nseg = single ? 1 : s.G;
   const int64_t n = c->lst_n;
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  for (int iter = 0; iter < 8; ++iter) {  // at most 8 digits in a 64-bit key
+    {
+      int k = 0;
+      for (int base = 0; base < nseg; base += blockDim.x) {
+        const int g = base + threadIdx.x;
+        bool counts = false;
+        if (g < nseg) {
+          const SelSeg ss = list_view(s.sel[g]);
+          counts = ss.active && next_shift(ss.mask) >= 0;
+        }
+        int tot;
+        const int ex = block_excl_scan((int)counts, &tot);
+        if (g < nseg) row_of[g] = counts ? (int16_t)(k + ex) : (int16_t)-1;
+        if (counts) seg_of_row[k + ex] = (int16_t)g;
+        k += tot;
+      }
+      if (threadIdx.x == 0) s_nrows = k;
+      __syncthreads();
+    }
+    const int nrows = s_nrows;
+    if (nrows == 0) break;
+    for (int r0 = 0; r0 < nrows; r0 += kFinRows) {
+      const int rn = tmin(kFinRows, nrows - r0);
+      for (int k = threadIdx.x; k < rn * kRadixBins; k += blockDim.x) fh[k] = 0;
+      __syncthreads();
+      for (int64_t e0 = 0; e0 < n; e0 += blockDim.x) {
+        const int64_t e = e0 + threadIdx.x;
+        bool act = false;
+        uint32_t idx = 0;
+        if (e < n) {
+          const int seg = s.lst_seg[e];
+          const int row = row_of[seg];
+          if (row >= r0 && row < r0 + rn) {
+            const SelSeg ss = list_view(s.sel[seg]);
+            const uint64_t key = s.lst_key[e];
+            if ((key & ss.mask) == ss.prefix) {
+              act = true;
+              const int sh = next_shift(ss.mask);
+              idx = (uint32_t)(row - r0) * kRadixBins + (uint32_t)((key >> sh) & (kRadixBins - 1));
+            }
+          }
+        }
+        agg_inc(fh, idx, act);
+      }
+      __syncthreads();
+      for (int r = warp; r < rn; r += blockDim.x >> 5) {
+        const int seg = seg_of_row[r0 + r];
+        SelSeg ss = list_view(s.sel[seg]);
+        const int sh = next_shift(ss.mask);
+        uint32_t v[kRadixBins / 32];
+        uint32_t sum = 0;
+#pragma unroll
+        for (int j = 0; j < kRadixBins / 32; ++j) { v[j] = fh[r * kRadixBins + lane * (kRadixBins / 32) + j]; sum += v[j]; }
+        const uint32_t incl = warp_incl_scan(sum);
+        const uint32_t excl = incl - sum;
+        if ((uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl) {
+          uint32_t run = excl;
+          int d = 0;
+          for (int j = 0; j < kRadixBins / 32; ++j) {
+            if ((uint64_t)ss.rank <= (uint64_t)(run + v[j])) { d = lane * (kRadixBins / 32) + j; break; }
+            run += v[j];
+          }
+          ss.prefix |= (uint64_t)d << sh;
+          ss.mask |= (uint64_t)(kRadixBins - 1) << sh;
+          ss.rank -= run;
+          s.sel[seg] = ss;
+        }
+      }
+      __syncthreads();
+    }
+  }
+  // Eq. 7's tie rule at tau: among the groups holding an item at exactly tau,
+  // the sel_k with the smallest candidate keys take it
+  if (!single && c->sel_ntie > 0) {
+    uint64_t* tkey = reinterpret_cast<uint64_t*>(fh);                  // G <= 1024: 8 KB
+    int* tied = reinterpret_cast<int*>(fh + 2 * PS_MAX_GROUPS);        // 4 KB after it
+    const int64_t k = c->sel_k;
+    for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+      const SelSeg sg = list_view(s.sel[g]);
+      tied[g] = sg.active && sg.incl == 2;
+      tkey[g] = sg.prefix;
+    }
+    __syncthreads();
+    for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+      if (!tied[g]) continue;
+      int rank = 0;
+      for (int h = 0; h < nseg; ++h) rank += tied[h] && tkey[h] < tkey[g];
+      const bool chosen = rank < k;
+      s.sel[g].incl = chosen ? 1 : 0;
+      if (!chosen) s.grp_x[g] -= 1;
+    }
+    __syncthreads();
+  }
+  // the list's victims: keys below (or at, if incl) their segment's threshold
+  for (int64_t e = threadIdx.x; e < n; e += blockDim.x) {
     const uint64_t key = s.lst_key[e];
     const SelSeg ss = list_view(s.sel[s.lst_seg[e]]);
     if (ss.active && (key < ss.prefix || (ss.incl && key == ss.prefix))) {
@@ -1612,8 +1698,8 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
   const int prgrid = grid_for(s.max_blocks + R, kThreads, 1 << 30);
   const int ngrid = grid_for(s.N, 256, 152 * 8);
-  const int sgrid = grid_for(s.N, 256, 152 * 2);
-  const int cgrid = grid_for(s.N, 256, 152 * 2);
+  const int sgrid = grid_for(s.N, 256, 152 * 4);  // 48 KB histograms: 4 CTAs per SM
+  const int cgrid = grid_for(s.N, 256, 152 * 8);
   const int lgrid = 152;  // list passes: the split list is short
   const int radix_smem = kRadixSmemRows * kRadixBins * 4;
   int launches = 0;
@@ -1646,10 +1732,9 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   // the remaining digits over the list, then the list's victims
   auto select = [&](int single, int fallback) {
     PS_LAUNCH(k_digit_pass<<<sgrid, 256, radix_smem, st>>>(s, single, fallback, 0));
-    PS_LAUNCH(k_split<<<sgrid, 256, 0, st>>>(s, single, fallback));
-    for (int d = 0; d < 7; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, st>>>(s, single, fallback, 1));
-    if (!single) PS_LAUNCH(k_tie<<<1, 1024, 0, st>>>(s));
-    PS_LAUNCH(k_mark_list<<<lgrid, 256, 0, st>>>(s, single));
+    PS_LAUNCH(k_split<<<cgrid, 256, 0, st>>>(s, single, fallback));
+    for (int d = 0; d < 3; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, st>>>(s, single, fallback, 1));
+    PS_LAUNCH(k_list_finish<<<1, 1024, 0, st>>>(s, single));
   };
   if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));
