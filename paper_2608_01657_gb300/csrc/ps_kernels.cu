@@ -17,8 +17,8 @@ namespace ps {
 constexpr unsigned kFull = 0xFFFFFFFFu;
 constexpr int kThreads = 256;     // position-parallel kernels
 constexpr int kRadixSmemRows = 48;  // radix rows counted in shared memory (48 KB)
-constexpr int64_t kListSmall = 16384;  // split lists up to this size are finished by one CTA
-constexpr int kFinRows = 32;           // rows k_list_finish counts at once (32 KB)
+constexpr int kFinCap = 8192;  // split lists up to this size are finished by one CTA in shared memory
+constexpr int kFinRows = 32;   // rows k_list_finish counts at once (32 KB)
 
 // ---------------------------------------------------------------------------
 // small device helpers
@@ -1150,7 +1150,7 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
   if (c->status != PS_OK || c->mvict == 0) return;
   const int nseg = single ? 1 : s.G;
   if (single && !s.sel[0].active) return;
-  if (from_list && c->lst_n <= kListSmall) return;  // k_list_finish takes short lists whole
+  if (from_list && c->lst_n <= kFinCap) return;  // k_list_finish takes short lists whole
   // rows for the segments that still count (parallel flags, scanned)
   {
     int k = 0;
@@ -1328,13 +1328,26 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
 }
 
-// The rest of a select on one CTA: every remaining digit of every segment
-// over the split list (shared-memory histograms, up to kFinRows segments per
-// sweep), then the tie rule at tau for the debt phase, then the list's victims.
-// Long lists have been narrowed by the multi-CTA list passes before this.
+// The rest of a select on one CTA.  A short split list (at most kFinCap
+// members) is staged in shared memory with every segment's state, and every
+// remaining digit, Eq. 7's tie rule and the marking of the list's victims run
+// there.  A longer list has had all its digits located by the multi-CTA list
+// passes; here it gets only the tie rule, and k_mark_list marks it.
+struct FinSeg {
+  uint64_t prefix, mask;
+  int64_t rank;
+  int32_t active, incl;
+};
+constexpr size_t kFinSmem = (size_t)kFinCap * 8 + (size_t)kFinCap * 2 + (size_t)kFinRows * kRadixBins * 4 +
+                            (size_t)PS_MAX_GROUPS * sizeof(FinSeg);
+
 __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
   s = with_args(s);
-  __shared__ __align__(16) uint32_t fh[kFinRows * kRadixBins];
+  extern __shared__ __align__(16) unsigned char fin_smem[];
+  FinSeg* sl = reinterpret_cast<FinSeg*>(fin_smem);
+  uint64_t* lkey = reinterpret_cast<uint64_t*>(sl + PS_MAX_GROUPS);
+  uint32_t* fh = reinterpret_cast<uint32_t*>(lkey + kFinCap);
+  uint16_t* lseg = reinterpret_cast<uint16_t*>(fh + kFinRows * kRadixBins);
   __shared__ int16_t row_of[PS_MAX_GROUPS];
   __shared__ int16_t seg_of_row[PS_MAX_GROUPS];
   __shared__ int s_nrows;
@@ -1343,17 +1356,21 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
   if (single && !s.sel[0].active) return;
   const int nseg = single ? 1 : s.G;
   const int64_t n = c->lst_n;
+  const bool small = n <= kFinCap;
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  for (int iter = 0; iter < 8; ++iter) {  // at most 8 digits in a 64-bit key
+  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+    const SelSeg v = list_view(s.sel[g]);
+    sl[g] = FinSeg{v.prefix, v.mask, v.rank, v.active, v.incl};
+  }
+  if (small)
+    for (int64_t e = threadIdx.x; e < n; e += blockDim.x) { lkey[e] = s.lst_key[e]; lseg[e] = s.lst_seg[e]; }
+  __syncthreads();
+  for (int iter = 0; small && iter < 8; ++iter) {  // at most 8 digits in a 64-bit key
     {
       int k = 0;
       for (int base = 0; base < nseg; base += blockDim.x) {
         const int g = base + threadIdx.x;
-        bool counts = false;
-        if (g < nseg) {
-          const SelSeg ss = list_view(s.sel[g]);
-          counts = ss.active && next_shift(ss.mask) >= 0;
-        }
+        const bool counts = g < nseg && sl[g].active && next_shift(sl[g].mask) >= 0;
         int tot;
         const int ex = block_excl_scan((int)counts, &tot);
         if (g < nseg) row_of[g] = counts ? (int16_t)(k + ex) : (int16_t)-1;
@@ -1369,19 +1386,18 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
       const int rn = tmin(kFinRows, nrows - r0);
       for (int k = threadIdx.x; k < rn * kRadixBins; k += blockDim.x) fh[k] = 0;
       __syncthreads();
-      for (int64_t e0 = 0; e0 < n; e0 += blockDim.x) {
-        const int64_t e = e0 + threadIdx.x;
+      for (int e0 = 0; e0 < n; e0 += blockDim.x) {
+        const int e = e0 + threadIdx.x;
         bool act = false;
         uint32_t idx = 0;
         if (e < n) {
-          const int seg = s.lst_seg[e];
+          const int seg = lseg[e];
           const int row = row_of[seg];
           if (row >= r0 && row < r0 + rn) {
-            const SelSeg ss = list_view(s.sel[seg]);
-            const uint64_t key = s.lst_key[e];
-            if ((key & ss.mask) == ss.prefix) {
+            const uint64_t key = lkey[e];
+            if ((key & sl[seg].mask) == sl[seg].prefix) {
               act = true;
-              const int sh = next_shift(ss.mask);
+              const int sh = next_shift(sl[seg].mask);
               idx = (uint32_t)(row - r0) * kRadixBins + (uint32_t)((key >> sh) & (kRadixBins - 1));
             }
           }
@@ -1391,25 +1407,24 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
       __syncthreads();
       for (int r = warp; r < rn; r += blockDim.x >> 5) {
         const int seg = seg_of_row[r0 + r];
-        SelSeg ss = list_view(s.sel[seg]);
-        const int sh = next_shift(ss.mask);
+        const int sh = next_shift(sl[seg].mask);
+        const int64_t rank = sl[seg].rank;
         uint32_t v[kRadixBins / 32];
         uint32_t sum = 0;
 #pragma unroll
         for (int j = 0; j < kRadixBins / 32; ++j) { v[j] = fh[r * kRadixBins + lane * (kRadixBins / 32) + j]; sum += v[j]; }
         const uint32_t incl = warp_incl_scan(sum);
         const uint32_t excl = incl - sum;
-        if ((uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl) {
+        if ((uint64_t)excl < (uint64_t)rank && (uint64_t)rank <= (uint64_t)incl) {
           uint32_t run = excl;
           int d = 0;
           for (int j = 0; j < kRadixBins / 32; ++j) {
-            if ((uint64_t)ss.rank <= (uint64_t)(run + v[j])) { d = lane * (kRadixBins / 32) + j; break; }
+            if ((uint64_t)rank <= (uint64_t)(run + v[j])) { d = lane * (kRadixBins / 32) + j; break; }
             run += v[j];
           }
-          ss.prefix |= (uint64_t)d << sh;
-          ss.mask |= (uint64_t)(kRadixBins - 1) << sh;
-          ss.rank -= run;
-          s.sel[seg] = ss;
+          sl[seg].prefix |= (uint64_t)d << sh;
+          sl[seg].mask |= (uint64_t)(kRadixBins - 1) << sh;
+          sl[seg].rank = rank - run;
         }
       }
       __syncthreads();
@@ -1418,27 +1433,51 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
   // Eq. 7's tie rule at tau: among the groups holding an item at exactly tau,
   // the sel_k with the smallest candidate keys take it
   if (!single && c->sel_ntie > 0) {
-    uint64_t* tkey = reinterpret_cast<uint64_t*>(fh);                  // G <= 1024: 8 KB
-    int* tied = reinterpret_cast<int*>(fh + 2 * PS_MAX_GROUPS);        // 4 KB after it
     const int64_t k = c->sel_k;
     for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
-      const SelSeg sg = list_view(s.sel[g]);
-      tied[g] = sg.active && sg.incl == 2;
-      tkey[g] = sg.prefix;
+      if (!(sl[g].active && sl[g].incl == 2)) continue;
+      int rank = 0;
+      for (int h = 0; h < nseg; ++h) rank += sl[h].active && sl[h].incl == 2 && sl[h].prefix < sl[g].prefix;
+      const bool chosen = rank < k;
+      s.grp_x[g] -= chosen ? 0 : 1;
+      fh[g] = chosen ? 1 : 0;  // applied after every thread has read the flags
     }
     __syncthreads();
-    for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
-      if (!tied[g]) continue;
-      int rank = 0;
-      for (int h = 0; h < nseg; ++h) rank += tied[h] && tkey[h] < tkey[g];
-      const bool chosen = rank < k;
-      s.sel[g].incl = chosen ? 1 : 0;
-      if (!chosen) s.grp_x[g] -= 1;
-    }
+    for (int g = threadIdx.x; g < nseg; g += blockDim.x)
+      if (sl[g].active && sl[g].incl == 2) sl[g].incl = (int32_t)fh[g];
     __syncthreads();
   }
-  // the list's victims: keys below (or at, if incl) their segment's threshold
-  for (int64_t e = threadIdx.x; e < n; e += blockDim.x) {
+  if (small) {  // the list's victims: keys below (or at, if incl) the threshold
+    for (int e = threadIdx.x; e < n; e += blockDim.x) {
+      const uint64_t key = lkey[e];
+      const FinSeg& f = sl[lseg[e]];
+      if (f.active && (key < f.prefix || (f.incl && key == f.prefix))) {
+        const uint32_t b = s.lst_blk[e];
+        atomicOr(s.bm_victim + (b >> 5), 1u << (b & 31));
+      }
+    }
+  } else {  // k_mark_list marks a long list from the segments' final state
+    for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+      SelSeg v = s.sel[g];
+      v.prefix = sl[g].prefix;
+      v.mask = sl[g].mask;
+      v.rank = sl[g].rank;
+      v.incl = sl[g].incl;
+      s.sel[g] = v;
+    }
+  }
+}
+
+// Mark a long list's victims (multi-CTA): keys below (or at, if incl) their
+// segment's located threshold.
+__global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
+  s = with_args(s);
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK || c->mvict == 0) return;
+  if (single && !s.sel[0].active) return;
+  const int64_t n = c->lst_n;
+  if (n <= kFinCap) return;  // marked by k_list_finish
+  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
     const uint64_t key = s.lst_key[e];
     const SelSeg ss = list_view(s.sel[s.lst_seg[e]]);
     if (ss.active && (key < ss.prefix || (ss.incl && key == ss.prefix))) {
@@ -1683,6 +1722,7 @@ static int32_t launch_hash(const DevState& s, cudaStream_t st) {
 void configure_kernels(const DevState& s) {
   (void)s;
   cudaFuncSetAttribute(k_digit_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, kRadixSmemRows * kRadixBins * 4);
+  cudaFuncSetAttribute(k_list_finish, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFinSmem);
   cudaFuncSetAttribute(k_hash<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<1>::kSmem);
   cudaFuncSetAttribute(k_hash<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<2>::kSmem);
   cudaFuncSetAttribute(k_hash<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<4>::kSmem);
@@ -1733,8 +1773,9 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   auto select = [&](int single, int fallback) {
     PS_LAUNCH(k_digit_pass<<<sgrid, 256, radix_smem, st>>>(s, single, fallback, 0));
     PS_LAUNCH(k_split<<<cgrid, 256, 0, st>>>(s, single, fallback));
-    for (int d = 0; d < 3; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, st>>>(s, single, fallback, 1));
-    PS_LAUNCH(k_list_finish<<<1, 1024, 0, st>>>(s, single));
+    for (int d = 0; d < 7; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, st>>>(s, single, fallback, 1));
+    PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, st>>>(s, single));
+    PS_LAUNCH(k_mark_list<<<lgrid, 256, 0, st>>>(s, single));
   };
   if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));

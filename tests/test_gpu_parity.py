@@ -266,3 +266,20 @@ def test_parity_graph_replay_streams_and_timing(policy):
             assert launches > 0 and np.all(ms >= 0)
     compare_state(gpu.export(), orc.export(), f"graph/{policy}", s3=policy == "s3fifo")
     assert np.array_equal(gpu.stats(), orc.stats())
+
+
+def test_parity_long_split_list():
+    """A select whose split list is longer than one CTA finishes in shared
+    memory: one indebted group holds 12,001 Probationary and 12,000 Normal
+    candidates, and 5,425 victims fall inside the Probationary class, so the
+    first digit (the class byte) leaves the whole class on the list."""
+    rng = np.random.default_rng(77)
+    steps = []
+    for k, (pid, nb) in enumerate([(7, 1), (7, 12000), (9, 12000), (11, 6000)]):
+        toks = rng.integers(0, W.VOCAB, size=nb * 16, dtype=np.int32)
+        steps.append(W.Step(k, k, np.zeros(1, np.int32), np.array([0, nb * 16], np.int64), toks,
+                            None, np.array([pid], np.uint64)))
+    gpu, orc = _pair(24576, 16, 2, "prefixshield", dict(rho=(1.0,), beta=(13000.0,)),
+                     max_requests=1, max_tokens=12000 * 16)
+    _run(gpu, orc, steps, label="long list")
+    assert int(gpu.stats()[0][8]) == 5425  # evicted blocks of group 0
