@@ -86,7 +86,6 @@ struct Ctl {
   int32_t sel_ntie, sel_k; // prefixshield tie bookkeeping
   int64_t s3_pinned[2];    // pinned members of each S3-FIFO queue this step
   int64_t s3_ninval;       // invalidated blocks to unlink this step
-  uint64_t fb_kmin, fb_kmax;  // key range of candidates the debt phase left
   int64_t lst_n;              // members of the select's split list
   uint32_t ticket;         // last-block-done counter for the radix passes
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
@@ -100,9 +99,15 @@ struct __align__(16) SelSeg {
   int32_t active;    // 1 while this segment selects
   int32_t incl;      // 1: victims are keys <= prefix; 0: keys < prefix
   uint64_t kmin, kmax;  // a range holding every candidate key of the segment
-  uint32_t hmin, hmax, lmin, lmax;  // ranges of the keys' top / bottom 32 bits
   uint64_t qmin, qmax;  // range of the segment's keys on the split list
 };
+
+// Candidates of one (segment, retention class): their number and the ranges
+// of their stamps' top and bottom 32 bits.
+struct ClsRange {
+  uint32_t cnt, hmin, hmax, lmin, lmax;
+};
+constexpr int kClasses = 3;
 
 // Per-call arguments of a step or probe, in device memory: the step's kernels
 // read them at entry, so one captured CUDA graph serves every step.
@@ -205,6 +210,7 @@ struct DevState {
   int64_t* grp_delta;      // Eq. 8 decrement
   int64_t* grp_x;          // victims taken from the group in the debt phase
   SelSeg* sel;             // [G] segments
+  ClsRange* cls;           // [G * kClasses] candidates per (segment, class)
   uint32_t* hist_bins;     // [G][256] radix histogram
   uint64_t* lst_key;       // split list of the select: key, block, segment
   uint32_t* lst_blk;

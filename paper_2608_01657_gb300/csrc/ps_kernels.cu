@@ -332,7 +332,6 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
       c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
       c->internal_error = 0;
       c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
-      c->fb_kmin = ~0ull; c->fb_kmax = 0;
     }
   }
 }
@@ -776,11 +775,10 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s0) {
     SelSeg z{};
     z.kmin = ~0ull;
     z.kmax = 0;
-    z.hmin = z.lmin = ~0u;
-    z.hmax = z.lmax = 0;
     z.qmin = ~0ull;
     z.qmax = 0;
     s.sel[g] = z;
+    for (int k = 0; k < kClasses; ++k) s.cls[g * kClasses + k] = ClsRange{0, ~0u, 0, ~0u, 0};
   }
 }
 
@@ -861,105 +859,160 @@ __global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
 // ===========================================================================
 // Stage 5: reclamation.  Candidates are resident blocks not hit in this step.
 // The order key is (class, stamp) for prefixshield (Eq. 9; stamp only with
-// the no-segmentation ablation) and the stamp for lru.  Also the smallest
-// and largest key of every segment, so the radix select can skip the bytes
-// its candidates share.
+// the no-segmentation ablation) and the stamp for lru.  Per (segment, class):
+// the candidates and their stamp range, so the radix select can start inside
+// the class that holds its rank and skip the bytes the class's stamps share.
 __global__ void __launch_bounds__(256) k_cand(DevState s) {
   s = with_args(s);
-  // per segment: candidates, and the ranges of the keys' top and bottom 32
-  // bits (native 32-bit shared atomics); sel_range() combines them
-  __shared__ unsigned int s_hmin[PS_MAX_GROUPS], s_hmax[PS_MAX_GROUPS];
-  __shared__ unsigned int s_lmin[PS_MAX_GROUPS], s_lmax[PS_MAX_GROUPS], s_cnt[PS_MAX_GROUPS];
+  extern __shared__ uint32_t cand_smem[];  // 5 arrays of nseg * kClasses
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const uint32_t step32 = (uint32_t)c->step;
   const bool ps = s.policy == PS_PREFIXSHIELD;
   const bool seg = ps && !(s.flags & PS_FLAG_NO_SEGMENTATION);
-  const int nseg = ps ? s.G : 1;
-  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
-    s_hmin[g] = s_lmin[g] = ~0u;
-    s_hmax[g] = s_lmax[g] = 0;
-    s_cnt[g] = 0;
+  const int nrow = (ps ? s.G : 1) * kClasses;
+  uint32_t* s_cnt = cand_smem;
+  uint32_t* s_hmin = s_cnt + nrow;
+  uint32_t* s_hmax = s_hmin + nrow;
+  uint32_t* s_lmin = s_hmax + nrow;
+  uint32_t* s_lmax = s_lmin + nrow;
+  for (int r = threadIdx.x; r < nrow; r += blockDim.x) {
+    s_cnt[r] = 0;
+    s_hmin[r] = s_lmin[r] = ~0u;
+    s_hmax[r] = s_lmax[r] = 0;
   }
   __syncthreads();
-  // warp-uniform trip count; lanes of one group combine their ranges and
-  // counts with warp reductions, and one lane per group updates shared memory
+  // warp-uniform trip count; lanes of one (segment, class) combine their
+  // ranges and counts with warp reductions, one lane updates shared memory
   for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
     const int64_t b = b0 + threadIdx.x;
-    uint64_t key = ~0ull;
-    uint32_t g = ~0u;
+    uint64_t key = ~0ull, st = 0;
+    uint32_t row = ~0u;
     if (b < s.N) {
       // every load issued at once (no dependent round trips)
       const uint8_t fl = s.blk_flags[b], kl = s.blk_klass[b];
       const uint32_t pin = s.blk_pin[b];
-      const uint64_t st = s.blk_stamp[b];
       const uint16_t grp = s.blk_group[b];
+      st = s.blk_stamp[b];
       if ((fl & 1) && pin != step32) {
         key = seg ? (st | (uint64_t)kl << 62) : st;
-        g = ps ? grp : 0;
+        row = (ps ? (uint32_t)grp : 0u) * kClasses + (seg ? kl : 0u);
       }
     }
-    const unsigned peers = __match_any_sync(kFull, g);
-    if (g != ~0u) {
-      const uint32_t hi = (uint32_t)(key >> 32), lo = (uint32_t)key;
+    const unsigned peers = __match_any_sync(kFull, row);
+    if (row != ~0u) {
+      const uint32_t hi = (uint32_t)(st >> 32), lo = (uint32_t)st;
       const uint32_t hmin = __reduce_min_sync(peers, hi), hmax = __reduce_max_sync(peers, hi);
       const uint32_t lmin = __reduce_min_sync(peers, lo), lmax = __reduce_max_sync(peers, lo);
       if (lane_id() == __ffs(peers) - 1) {
-        atomicMin(&s_hmin[g], hmin);
-        atomicMax(&s_hmax[g], hmax);
-        atomicMin(&s_lmin[g], lmin);
-        atomicMax(&s_lmax[g], lmax);
-        atomicAdd(&s_cnt[g], (unsigned)__popc(peers));
+        atomicAdd(&s_cnt[row], (unsigned)__popc(peers));
+        atomicMin(&s_hmin[row], hmin);
+        atomicMax(&s_hmax[row], hmax);
+        atomicMin(&s_lmin[row], lmin);
+        atomicMax(&s_lmax[row], lmax);
       }
     }
     if (b < s.N) s.csk[b] = key;
   }
   __syncthreads();
-  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
-    if (!s_cnt[g]) continue;
-    if (ps) atomic_add_i64(s.grp_qsize + g, s_cnt[g]);
-    atomicMin(&s.sel[g].hmin, s_hmin[g]);
-    atomicMax(&s.sel[g].hmax, s_hmax[g]);
-    atomicMin(&s.sel[g].lmin, s_lmin[g]);
-    atomicMax(&s.sel[g].lmax, s_lmax[g]);
+  for (int r = threadIdx.x; r < nrow; r += blockDim.x) {
+    if (!s_cnt[r]) continue;
+    if (ps) atomic_add_i64(s.grp_qsize + r / kClasses, s_cnt[r]);
+    ClsRange* d = s.cls + r;
+    atomicAdd(&d->cnt, s_cnt[r]);
+    atomicMin(&d->hmin, s_hmin[r]);
+    atomicMax(&d->hmax, s_hmax[r]);
+    atomicMin(&d->lmin, s_lmin[r]);
+    atomicMax(&d->lmax, s_lmax[r]);
   }
 }
 
-// A key range from the two half ranges: exact below the top half when every
-// candidate shares its top 32 bits, conservative otherwise.
-__device__ __forceinline__ void sel_range(SelSeg& z) {
-  if (z.hmin > z.hmax) return;  // no candidate
-  const bool same_hi = z.hmin == z.hmax;
-  z.kmin = ((uint64_t)z.hmin << 32) | (same_hi ? z.lmin : 0u);
-  z.kmax = ((uint64_t)z.hmax << 32) | (same_hi ? z.lmax : 0xFFFFFFFFu);
+// Stamp range of a class from its two half ranges: exact below the top half
+// when every member shares its top 32 bits, conservative otherwise.
+__device__ __forceinline__ void cls_stamp_range(const ClsRange& r, uint64_t* lo, uint64_t* hi) {
+  const bool same_hi = r.hmin == r.hmax;
+  *lo = ((uint64_t)r.hmin << 32) | (same_hi ? r.lmin : 0u);
+  *hi = ((uint64_t)r.hmax << 32) | (same_hi ? r.lmax : 0xFFFFFFFFu);
 }
 
 __device__ __forceinline__ void sel_start(SelSeg& z);
-__global__ void k_sel_single(DevState s, int fallback) {
+// Start a segment's search from its per-class candidates: the class holding
+// the rank-th smallest key is fixed (lower classes are all below it), the rank
+// becomes a rank inside that class, and the key range is the class's.
+// cnt[k] and [lo[k], hi[k]] describe class k (unsegmented keys: class 0 only).
+__device__ __forceinline__ void sel_start_cls(SelSeg& z, const int64_t* cnt, const uint64_t* lo, const uint64_t* hi,
+                                              bool segmented) {
+  int k = 0;
+  int64_t below = 0;
+  if (segmented)
+    while (k < kClasses - 1 && z.rank > below + cnt[k]) below += cnt[k++];
+  const uint64_t cb = segmented ? (uint64_t)k << 62 : 0ull;
+  if (z.active && cnt[k] > 0) {
+    z.rank -= below;
+    z.kmin = cb | lo[k];
+    z.kmax = cb | hi[k];
+  } else {
+    z.kmin = z.kmax = cb;
+  }
+  sel_start(z);
+}
+__device__ __forceinline__ void sel_start_group(const DevState& s, int g, SelSeg& z, bool segmented) {
+  int64_t cnt[kClasses];
+  uint64_t lo[kClasses], hi[kClasses];
+  for (int k = 0; k < kClasses; ++k) {
+    const ClsRange r = s.cls[g * kClasses + k];
+    cnt[k] = r.cnt;
+    cls_stamp_range(r, &lo[k], &hi[k]);
+  }
+  sel_start_cls(z, cnt, lo, hi, segmented);
+}
+
+// One global segment: all candidates for lru, or (fallback) the candidates
+// the debt phase of prefixshield left, in (class, stamp) order (Eq. 9).  The
+// debt phase took group g's x_g smallest keys, so of class k it took
+// clamp(x_g - (members of lower classes), 0, members of class k).
+__global__ void __launch_bounds__(32) k_sel_single(DevState s, int fallback) {
   s = with_args(s);
   Ctl* c = s.ctl;
-  if (threadIdx.x != 0) return;
+  const int lane = lane_id();
   int64_t m = 0;
   if (c->status == PS_OK) m = fallback ? c->m_fb : c->mvict;
-  const SelSeg old = s.sel[0];
+  const bool segmented = s.policy == PS_PREFIXSHIELD && !(s.flags & PS_FLAG_NO_SEGMENTATION);
+  int64_t cnt[kClasses];
+  uint64_t lo[kClasses], hi[kClasses];
+  for (int k = 0; k < kClasses; ++k) { cnt[k] = 0; lo[k] = ~0ull; hi[k] = 0; }
+  if (m > 0) {
+    const int nseg = fallback ? s.G : 1;
+    for (int g = lane; g < nseg; g += 32) {
+      int64_t taken = fallback ? s.grp_x[g] : 0;
+      for (int k = 0; k < kClasses; ++k) {
+        const ClsRange r = s.cls[g * kClasses + k];
+        const int64_t t = tmin<int64_t>(taken, (int64_t)r.cnt);
+        taken -= t;
+        if ((int64_t)r.cnt > t) {
+          uint64_t a, b;
+          cls_stamp_range(r, &a, &b);
+          cnt[k] += (int64_t)r.cnt - t;
+          lo[k] = tmin(lo[k], a);
+          hi[k] = tmax(hi[k], b);
+        }
+      }
+    }
+    for (int k = 0; k < kClasses; ++k)
+      for (int o = 16; o > 0; o >>= 1) {
+        cnt[k] += __shfl_xor_sync(kFull, cnt[k], o);
+        lo[k] = tmin(lo[k], (uint64_t)__shfl_xor_sync(kFull, lo[k], o));
+        hi[k] = tmax(hi[k], (uint64_t)__shfl_xor_sync(kFull, hi[k], o));
+      }
+  }
+  if (lane != 0) return;
   SelSeg z{};
   z.rank = m;
   z.active = m > 0;
   z.incl = 1;
   z.qmin = ~0ull;
   z.qmax = 0;
-  // the fallback selects among the candidates the debt phase left, whose key
-  // range the debt phase's split pass recorded
-  if (fallback) {
-    z.kmin = c->fb_kmin;
-    z.kmax = c->fb_kmax;
-  } else {
-    SelSeg r = old;
-    sel_range(r);
-    z.kmin = r.kmin;
-    z.kmax = r.kmax;
-  }
-  sel_start(z);
+  sel_start_cls(z, cnt, lo, hi, segmented);
   s.sel[0] = z;
   c->lst_n = 0;
 }
@@ -982,6 +1035,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
   __shared__ int s_best;
   const int G = s.G;
   const int64_t eps = s.eps;
+  const bool seg = !(s.flags & PS_FLAG_NO_SEGMENTATION);
   const int64_t m = (c->status == PS_OK) ? c->mvict : 0;
   if (m == 0) {
     for (int g = threadIdx.x; g < G; g += blockDim.x) { s.sel[g].active = 0; s.grp_x[g] = 0; }
@@ -1023,8 +1077,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
       z.rank = x;
       z.active = x > 0;
       z.incl = 1;
-      sel_range(z);
-      sel_start(z);
+      sel_start_group(s, g, z, seg);
       s.sel[g] = z;
     }
     if (threadIdx.x == 0) { c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; c->lst_n = 0; }
@@ -1076,8 +1129,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
     z.rank = xa + (tied ? 1 : 0);
     z.active = z.rank > 0;
     z.incl = tied ? 2 : 1;  // 2: the tie item is taken only if the tie rule chooses it
-    sel_range(z);
-    sel_start(z);
+    sel_start_group(s, g, z, seg);
     s.sel[g] = z;
     s.grp_x[g] = xa + (tied ? 1 : 0);
   }
@@ -1252,20 +1304,14 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
 }
 
 // Split: candidates below their segment's chosen bucket are victims; the
-// bucket's members go to the list for the remaining digits.  The per-group
-// pass also records the key range of every candidate it does not mark, for
-// the global fallback.
+// bucket's members go to the list for the remaining digits, with the list's
+// key range per segment.
 __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallback) {
   s = with_args(s);
-  __shared__ unsigned long long s_rng[2];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   if (single && !s.sel[0].active) return;
-  const bool track = !single;
-  if (threadIdx.x == 0) { s_rng[0] = ~0ull; s_rng[1] = 0; }
-  __syncthreads();
   int marked = 0;
-  uint64_t lo = ~0ull, hi = 0;
   for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
     const int64_t b = b0 + threadIdx.x;
     bool v = false, to_list = false;
@@ -1282,7 +1328,6 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
           v = k < ss.prefix;
           to_list = k == ss.prefix;
         }
-        if (track && !v) { lo = tmin(lo, key); hi = tmax(hi, key); }
       }
     }
     const unsigned bits = __ballot_sync(kFull, v);
@@ -1311,18 +1356,6 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
           atomicMax(reinterpret_cast<unsigned long long*>(&s.sel[seg].qmax), ((unsigned long long)hmax << 32) | lmax);
         }
       }
-    }
-  }
-  if (track) {
-    for (int o = 16; o > 0; o >>= 1) {
-      lo = tmin(lo, (uint64_t)__shfl_xor_sync(kFull, lo, o));
-      hi = tmax(hi, (uint64_t)__shfl_xor_sync(kFull, hi, o));
-    }
-    if (lane_id() == 0) { atomicMin(&s_rng[0], lo); atomicMax(&s_rng[1], hi); }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      atomicMin(reinterpret_cast<unsigned long long*>(&c->fb_kmin), s_rng[0]);
-      atomicMax(reinterpret_cast<unsigned long long*>(&c->fb_kmax), s_rng[1]);
     }
   }
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
@@ -1723,6 +1756,7 @@ void configure_kernels(const DevState& s) {
   (void)s;
   cudaFuncSetAttribute(k_digit_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, kRadixSmemRows * kRadixBins * 4);
   cudaFuncSetAttribute(k_list_finish, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFinSmem);
+  cudaFuncSetAttribute(k_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, PS_MAX_GROUPS * kClasses * 5 * 4);
   cudaFuncSetAttribute(k_hash<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<1>::kSmem);
   cudaFuncSetAttribute(k_hash<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<2>::kSmem);
   cudaFuncSetAttribute(k_hash<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<4>::kSmem);
@@ -1767,7 +1801,8 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   PS_LAUNCH(k_touch<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
   mark(6);
-  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<cgrid, 256, 0, st>>>(s));
+  const int cand_smem = (s.policy == PS_PREFIXSHIELD ? s.G : 1) * kClasses * 5 * 4;
+  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<cgrid, 256, cand_smem, st>>>(s));
   // one exact segmented select: a digit over the candidates, the split, then
   // the remaining digits over the list, then the list's victims
   auto select = [&](int single, int fallback) {
