@@ -29,6 +29,7 @@ struct ps_handle {
   // the step as one CUDA graph, captured on a private stream at first use
   StepArgs* step_args;
   cudaStream_t cap_stream = nullptr;
+  cudaStream_t cap_aux = nullptr;  // conditional bodies are captured here
   cudaGraph_t graph = nullptr;
   cudaGraphExec_t exec = nullptr;
   bool exec_timing = false;
@@ -296,7 +297,14 @@ void capture_step(ps_handle* h) {
   tmpl.R = 0;
   bool ok = cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
   if (ok) {
-    const int32_t rc = launch_step(tmpl, h->cap_stream, &h->trace);
+    const CaptureCtx ctx{h->cap_aux};
+    const int32_t rc = launch_step(tmpl, h->cap_stream, &h->trace, &ctx);
+    // a body whose capture did not close leaves the auxiliary stream capturing
+    cudaStreamCaptureStatus aux_cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(h->cap_aux, &aux_cs) == cudaSuccess && aux_cs != cudaStreamCaptureStatusNone) {
+      cudaGraph_t body = nullptr;
+      cudaStreamEndCapture(h->cap_aux, &body);
+    }
     cudaGraph_t g = nullptr;
     const bool ended = cudaStreamEndCapture(h->cap_stream, &g) == cudaSuccess;
     ok = rc == PS_OK && ended && g;
@@ -376,7 +384,9 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   configure_kernels(s);  // per device: attributes are set on the current one
   int32_t rc = init_state(h, st);
   if (rc == PS_OK) rc = upload_constants(h, st);
-  if (rc == PS_OK && cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess) rc = PS_ERR_CUDA;
+  if (rc == PS_OK && (cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess ||
+                      cudaStreamCreateWithFlags(&h->cap_aux, cudaStreamNonBlocking) != cudaSuccess))
+    rc = PS_ERR_CUDA;
   if (rc != PS_OK) {
     delete h;
     return rc;
@@ -498,6 +508,7 @@ void ps_destroy(ps_handle_t* h) {
   if (!h) return;
   drop_graph(h);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
+  if (h->cap_aux) cudaStreamDestroy(h->cap_aux);
   if (h->trace.timing)
     for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
   delete h;
@@ -522,6 +533,9 @@ int32_t ps_get_stage_times(ps_handle_t* h, float* h_ms, int32_t max_stages, int3
   if (h_launches) *h_launches = h->trace.launches;
   if (!h->trace.timing) return 0;
   if (cudaEventSynchronize(h->trace.ev[PS_NUM_STAGES]) != cudaSuccess) return PS_ERR_CUDA;
+  // kernels the step actually launched (conditional bodies included or not)
+  if (h_launches && cudaMemcpy(h_launches, &h->base.ctl->nlaunch, 4, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return PS_ERR_CUDA;
   const int n = max_stages < PS_NUM_STAGES ? max_stages : PS_NUM_STAGES;
   for (int k = 0; k < n; ++k)
     if (cudaEventElapsedTime(h_ms + k, h->trace.ev[k], h->trace.ev[k + 1]) != cudaSuccess) return PS_ERR_CUDA;

@@ -87,7 +87,8 @@ struct Ctl {
   int64_t s3_pinned[2];    // pinned members of each S3-FIFO queue this step
   int64_t s3_ninval;       // invalidated blocks to unlink this step
   int64_t lst_n;              // members of the select's split list
-  uint32_t ticket;         // last-block-done counter for the radix passes
+  uint32_t ticket;         // last-block-done counter for the radix passes and the split
+  int32_t nlaunch;         // kernels launched by the step (conditional bodies run or not)
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
 };
 
@@ -262,10 +263,17 @@ struct StepTrace {
   int launches = 0;
 };
 
+// Stream capture of a step: a second private stream on which the bodies of
+// conditional graph nodes are captured (phases that many steps skip).
+struct CaptureCtx {
+  cudaStream_t aux;
+};
+
 // Copy the call's arguments from device memory into the kernel's DevState.
 __device__ __forceinline__ DevState with_args(DevState s) {
   const StepArgs* a = s.args;
   if (a == nullptr) return s;  // launched directly with its arguments by value
+  if (blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(&s.ctl->nlaunch, 1);
   s.now = a->now;
   s.R = a->R;
   s.tokens_aligned16 = a->tokens_aligned16;
@@ -289,7 +297,7 @@ inline StepArgs args_of(const DevState& s) {
 // any launch or capture.
 void configure_kernels(const DevState& s);
 void launch_init(const DevState& s, cudaStream_t st);
-int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr);
+int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const CaptureCtx* cap = nullptr);
 // S3-FIFO (ps_s3fifo.cu)
 void launch_s3_evict(const DevState& s, cudaStream_t st);
 void launch_s3_insert(const DevState& s, cudaStream_t st);

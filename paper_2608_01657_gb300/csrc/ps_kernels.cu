@@ -10,6 +10,8 @@
 #include <climits>
 #include <cstdio>
 
+#include <vector>
+
 #include "ps_internal.cuh"
 
 namespace ps {
@@ -331,6 +333,7 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
       c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
       c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
       c->internal_error = 0;
+      c->nlaunch = 1;  // this kernel; every later kernel of the step adds itself
       c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
     }
   }
@@ -1026,7 +1029,7 @@ __global__ void __launch_bounds__(32) k_sel_single(DevState s, int fallback) {
 // each) the ones with the smallest candidate keys are taken (resolved after
 // the radix select finds those keys).  What the debt phase cannot cover goes
 // to the global fallback in (class, stamp) order.
-__global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
+__global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditionalHandle fb_cond, int has_cond) {
   s = with_args(s);
   Ctl* c = s.ctl;
   __shared__ int64_t sP[PS_MAX_GROUPS], sD[PS_MAX_GROUPS], sQ[PS_MAX_GROUPS];
@@ -1080,7 +1083,10 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s) {
       sel_start_group(s, g, z, seg);
       s.sel[g] = z;
     }
-    if (threadIdx.x == 0) { c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; c->lst_n = 0; }
+    if (threadIdx.x == 0) {
+      c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; c->lst_n = 0;
+      if (has_cond && m > E) cudaGraphSetConditional(fb_cond, 1);  // the fallback phase runs
+    }
     return;
   }
   // tau = max{t in [eps+1, pmax] : items_gt(t - 1) summed >= m}.  Each round
@@ -1306,7 +1312,8 @@ __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int 
 // Split: candidates below their segment's chosen bucket are victims; the
 // bucket's members go to the list for the remaining digits, with the list's
 // key range per segment.
-__global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallback) {
+__global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallback, cudaGraphConditionalHandle long_cond,
+                                                int has_cond) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
@@ -1359,13 +1366,27 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
     }
   }
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
+  if (!has_cond) return;
+  // the last CTA to finish knows the list's length: the multi-CTA list
+  // passes run only for a long list
+  __shared__ bool last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(&c->ticket, 1u) == gridDim.x - 1;
+  __syncthreads();
+  if (last && threadIdx.x == 0) {
+    __threadfence();
+    c->ticket = 0;
+    if (ldcg_u64(reinterpret_cast<const uint64_t*>(&c->lst_n)) > (uint64_t)kFinCap) cudaGraphSetConditional(long_cond, 1);
+  }
 }
 
 // The rest of a select on one CTA.  A short split list (at most kFinCap
-// members) is staged in shared memory with every segment's state, and every
-// remaining digit, Eq. 7's tie rule and the marking of the list's victims run
-// there.  A longer list has had all its digits located by the multi-CTA list
-// passes; here it gets only the tie rule, and k_mark_list marks it.
+// members; long_list = 0) is staged in shared memory with every segment's
+// state, and every remaining digit, Eq. 7's tie rule and the marking of the
+// list's victims run there.  A longer list (long_list = 1) has had all its
+// digits located by the multi-CTA list passes; here it gets only the tie
+// rule, and k_mark_list marks it.
 struct FinSeg {
   uint64_t prefix, mask;
   int64_t rank;
@@ -1374,7 +1395,7 @@ struct FinSeg {
 constexpr size_t kFinSmem = (size_t)kFinCap * 8 + (size_t)kFinCap * 2 + (size_t)kFinRows * kRadixBins * 4 +
                             (size_t)PS_MAX_GROUPS * sizeof(FinSeg);
 
-__global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
+__global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, int long_list) {
   s = with_args(s);
   extern __shared__ __align__(16) unsigned char fin_smem[];
   FinSeg* sl = reinterpret_cast<FinSeg*>(fin_smem);
@@ -1390,6 +1411,7 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
   const int nseg = single ? 1 : s.G;
   const int64_t n = c->lst_n;
   const bool small = n <= kFinCap;
+  if (small == (long_list != 0)) return;  // the other launch's list
   const int warp = threadIdx.x >> 5, lane = lane_id();
   for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
     const SelSeg v = list_view(s.sel[g]);
@@ -1765,7 +1787,35 @@ void configure_kernels(const DevState& s) {
   cudaFuncSetAttribute(k_hash<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<32>::kSmem);
 }
 
-int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
+// Under stream capture: append an 'if' conditional node to the graph being
+// captured on st, and start capturing its body on aux.  Returns false (and
+// the capture then fails as a whole) if any step is refused.
+static bool cond_open(cudaStream_t st, cudaStream_t aux, cudaGraphConditionalHandle h) {
+  cudaStreamCaptureStatus cs;
+  cudaGraph_t g = nullptr;
+  const cudaGraphNode_t* deps = nullptr;
+  size_t nd = 0;
+  if (cudaStreamGetCaptureInfo(st, &cs, nullptr, &g, &deps, nullptr, &nd) != cudaSuccess ||
+      cs != cudaStreamCaptureStatusActive)
+    return false;
+  std::vector<cudaGraphNode_t> dv(deps, deps + nd);
+  cudaGraphNodeParams p{};
+  p.type = cudaGraphNodeTypeConditional;
+  p.conditional.handle = h;
+  p.conditional.type = cudaGraphCondTypeIf;
+  p.conditional.size = 1;
+  cudaGraphNode_t node;
+  return cudaGraphAddNode(&node, g, dv.data(), nullptr, nd, &p) == cudaSuccess &&
+         cudaStreamUpdateCaptureDependencies(st, &node, nullptr, 1, cudaStreamSetCaptureDependencies) == cudaSuccess &&
+         cudaStreamBeginCaptureToGraph(aux, p.conditional.phGraph_out[0], nullptr, nullptr, 0,
+                                       cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+}
+static bool cond_close(cudaStream_t aux) {
+  cudaGraph_t body = nullptr;
+  return cudaStreamEndCapture(aux, &body) == cudaSuccess;
+}
+
+int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const CaptureCtx* cap) {
   // grids depend only on the handle's bounds (a captured graph serves any step)
   const int R = s.max_requests;
   const int rgrid = grid_for(R, 256, 1 << 20);
@@ -1803,23 +1853,53 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr) {
   mark(6);
   const int cand_smem = (s.policy == PS_PREFIXSHIELD ? s.G : 1) * kClasses * 5 * 4;
   if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<cgrid, 256, cand_smem, st>>>(s));
-  // one exact segmented select: a digit over the candidates, the split, then
-  // the remaining digits over the list, then the list's victims
-  auto select = [&](int single, int fallback) {
-    PS_LAUNCH(k_digit_pass<<<sgrid, 256, radix_smem, st>>>(s, single, fallback, 0));
-    PS_LAUNCH(k_split<<<cgrid, 256, 0, st>>>(s, single, fallback));
-    for (int d = 0; d < 7; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, st>>>(s, single, fallback, 1));
-    PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, st>>>(s, single));
-    PS_LAUNCH(k_mark_list<<<lgrid, 256, 0, st>>>(s, single));
+  // Under capture, phases that many steps skip become conditional bodies:
+  // the long-list passes of a select, and the global fallback of Alg. 2.
+  cudaGraphConditionalHandle h_fb = 0, h_long = 0;
+  bool conds = false, cond_ok = true;
+  if (cap) {
+    cudaStreamCaptureStatus cs;
+    cudaGraph_t g = nullptr;
+    conds = cudaStreamGetCaptureInfo(st, &cs, nullptr, &g) == cudaSuccess && cs == cudaStreamCaptureStatusActive &&
+            cudaGraphConditionalHandleCreate(&h_fb, g, 0, cudaGraphCondAssignDefault) == cudaSuccess &&
+            cudaGraphConditionalHandleCreate(&h_long, g, 0, cudaGraphCondAssignDefault) == cudaSuccess;
+    if (!conds) return PS_ERR_CUDA;
+  }
+  // One exact segmented select: a digit over the candidates, the split, then
+  // the list: a long one through the multi-CTA digit passes, the tie rule
+  // and the multi-CTA marking; a short one finished by one CTA.
+  // (a body is launched only once its capture has started: a kernel launched
+  // on the auxiliary stream outside a capture would run)
+  auto select = [&](cudaStream_t q, int single, int fallback, bool cond) {
+    PS_LAUNCH(k_digit_pass<<<sgrid, 256, radix_smem, q>>>(s, single, fallback, 0));
+    PS_LAUNCH(k_split<<<cgrid, 256, 0, q>>>(s, single, fallback, h_long, cond ? 1 : 0));
+    cudaStream_t b = q;
+    if (cond) {
+      if (!cond_open(q, cap->aux, h_long)) { cond_ok = false; return; }
+      b = cap->aux;
+    }
+    for (int d = 0; d < 7; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, b>>>(s, single, fallback, 1));
+    PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, b>>>(s, single, 1));
+    PS_LAUNCH(k_mark_list<<<lgrid, 256, 0, b>>>(s, single));
+    if (cond && !cond_close(cap->aux)) { cond_ok = false; return; }
+    PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, q>>>(s, single, 0));
   };
   if (s.policy == PS_PREFIXSHIELD) {
-    PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s));
-    select(0, 0);
-    PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 1));
-    select(1, 1);
+    PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s, h_fb, conds ? 1 : 0));
+    select(st, 0, 0, conds);
+    if (!cond_ok) return PS_ERR_CUDA;
+    cudaStream_t f = st;
+    if (conds) {
+      if (!cond_open(st, cap->aux, h_fb)) return PS_ERR_CUDA;
+      f = cap->aux;
+    }
+    PS_LAUNCH(k_sel_single<<<1, 32, 0, f>>>(s, 1));
+    select(f, 1, 1, false);  // no nested body: the fallback is itself one
+    if (conds && !cond_close(cap->aux)) return PS_ERR_CUDA;
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
-    select(1, 0);
+    select(st, 1, 0, conds);
+    if (!cond_ok) return PS_ERR_CUDA;
   } else {
     PS_LAUNCH(launch_s3_evict(s, st));
   }
