@@ -249,6 +249,14 @@ int32_t ps_set_stage_timing(ps_handle_t* h, int32_t enable);
  * the number of stages written, or an error. */
 int32_t ps_get_stage_times(ps_handle_t* h, float* h_ms, int32_t max_stages, int32_t* h_launches);
 
+/* 1 if the handle replays its step as one captured CUDA graph (the step's
+ * per-call arguments live in a device block that every kernel reads, so one
+ * graph serves every step; phases many steps skip are conditional nodes), 0
+ * if it launches kernel by kernel (the graph could not be captured or
+ * instantiated: results are the same).  Known after the first ps_step().
+ * Measurement hook; the paper has no counterpart. */
+int32_t ps_uses_graph(const ps_handle_t* h);
+
 #ifdef __cplusplus
 }
 #endif

@@ -32,7 +32,7 @@ PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE = 1, 2
 EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_stats", "ps_clear_status",
             "ps_reset", "ps_destroy", "ps_status_string", "ps_export_state", "ps_export_history",
             "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times", "ps_cached_prefix",
-            "ps_cached_prefix_noalloc")
+            "ps_cached_prefix_noalloc", "ps_uses_graph")
 PS_NUM_STAGES = 11
 STAGE_NAMES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
                "freetake_evict", "id_lists", "insert", "commit")
@@ -114,6 +114,8 @@ def load():
     L.ps_set_stage_timing.argtypes = [vp, i32]
     L.ps_get_stage_times.restype = i32
     L.ps_get_stage_times.argtypes = [vp, vp, i32, vp]
+    L.ps_uses_graph.restype = i32
+    L.ps_uses_graph.argtypes = [C.c_void_p]
     _lib = L
     return L
 
@@ -292,6 +294,13 @@ class Cache:
         rc = load().ps_set_stage_timing(self._h, int(enable))
         if rc != PS_OK:
             raise RuntimeError(f"ps_set_stage_timing failed ({rc})")
+
+    def uses_graph(self) -> bool:
+        """True once the step replays one captured CUDA graph."""
+        rc = load().ps_uses_graph(self._h)
+        if rc < 0:
+            raise RuntimeError(f"ps_uses_graph failed ({rc})")
+        return rc == 1
 
     def stage_times(self):
         """(per-stage ms of the last timed step, kernel launches of that step)."""

@@ -542,6 +542,11 @@ int32_t ps_get_stage_times(ps_handle_t* h, float* h_ms, int32_t max_stages, int3
   return n;
 }
 
+int32_t ps_uses_graph(const ps_handle_t* h) {
+  if (!h) return PS_ERR_INVALID_ARG;
+  return h->use_graph && h->exec ? 1 : 0;
+}
+
 const char* ps_status_string(int32_t status) {
   switch (status) {
     case PS_OK: return "ok";

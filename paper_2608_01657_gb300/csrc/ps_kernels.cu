@@ -1828,8 +1828,12 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   const int radix_smem = kRadixSmemRows * kRadixBins * 4;
   int launches = 0;
   auto mark = [&](int stage) {
-    // external: under capture the record becomes a node of the graph
-    if (tr && tr->timing) cudaEventRecordWithFlags(tr->ev[stage], st, cudaEventRecordExternal);
+    // under capture an external record becomes an event-record node of the
+    // graph (the flag is refused outside a capture)
+    if (tr && tr->timing) {
+      if (cap) cudaEventRecordWithFlags(tr->ev[stage], st, cudaEventRecordExternal);
+      else cudaEventRecord(tr->ev[stage], st);
+    }
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
   mark(0);
@@ -1860,10 +1864,15 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   if (cap) {
     cudaStreamCaptureStatus cs;
     cudaGraph_t g = nullptr;
-    conds = cudaStreamGetCaptureInfo(st, &cs, nullptr, &g) == cudaSuccess && cs == cudaStreamCaptureStatusActive &&
-            cudaGraphConditionalHandleCreate(&h_fb, g, 0, cudaGraphCondAssignDefault) == cudaSuccess &&
-            cudaGraphConditionalHandleCreate(&h_long, g, 0, cudaGraphCondAssignDefault) == cudaSuccess;
-    if (!conds) return PS_ERR_CUDA;
+    // a handle that no conditional node uses can make instantiation fail:
+    // create only the ones this policy's sequence uses
+    conds = s.policy != PS_S3FIFO;
+    if (conds &&
+        !(cudaStreamGetCaptureInfo(st, &cs, nullptr, &g) == cudaSuccess && cs == cudaStreamCaptureStatusActive &&
+          cudaGraphConditionalHandleCreate(&h_long, g, 0, cudaGraphCondAssignDefault) == cudaSuccess &&
+          (s.policy != PS_PREFIXSHIELD ||
+           cudaGraphConditionalHandleCreate(&h_fb, g, 0, cudaGraphCondAssignDefault) == cudaSuccess)))
+      return PS_ERR_CUDA;
   }
   // One exact segmented select: a digit over the candidates, the split, then
   // the list: a long one through the multi-CTA digit passes, the tie rule

@@ -36,6 +36,7 @@ def _run(gpu, orc, steps, state_every=1, s3=False, label=""):
         p = None if st.prefixes is None else torch.from_numpy(st.prefixes.view(np.int64)).to(dev)
         rc = gpu.step(st.now, g, o, t, c, p)
         assert rc == 0, f"{label} step {k}: launch rc {rc}"
+        assert gpu.uses_graph(), f"{label} step {k}: the step is not replayed as a graph"
         got = gpu.fetch(st.num_requests)
         want = orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts, st.prefixes)
         compare_outputs(got, want, f"{label} step {k}")
@@ -258,6 +259,7 @@ def test_parity_graph_replay_streams_and_timing(policy):
             c = torch.from_numpy(st.contracts).to(dev)
             p = torch.from_numpy(st.prefixes.view(np.int64)).to(dev)
             assert gpu.step(st.now, g, o, t, c, p, stream=side) == 0
+            assert gpu.uses_graph()
         got = gpu.fetch(st.num_requests, stream=side)
         want = orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts, st.prefixes)
         compare_outputs(got, want, f"graph/{policy} step {k}")
