@@ -230,6 +230,12 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.sel = cv.take<SelSeg>(G);
   t.cls = cv.take<ClsRange>(G * kClasses);
   t.hist_bins = cv.take<uint32_t>(G * kRadixBins);
+  {
+    const size_t wrows = G < (size_t)kWideRows ? G : (size_t)kWideRows;
+    const size_t wb = wrows * kWideBins > G * kRadixBins ? wrows * kWideBins : G * kRadixBins;
+    t.wide_bins = cv.take<uint32_t>(wb);
+  }
+  t.wide_seg = cv.take<int16_t>(G);
   t.lst_key = cv.take<uint64_t>(N);
   t.lst_blk = cv.take<uint32_t>(N);
   t.lst_seg = cv.take<uint16_t>(N);

@@ -89,6 +89,7 @@ struct Ctl {
   int64_t lst_n;              // members of the select's split list
   uint32_t ticket;         // last-block-done counter for the radix passes and the split
   int32_t nlaunch;         // kernels launched by the step (conditional bodies run or not)
+  int32_t wide_nrows;      // segments counted by the last first-digit pass
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
 };
 
@@ -109,6 +110,10 @@ struct ClsRange {
   uint32_t cnt, hmin, hmax, lmin, lmax;
 };
 constexpr int kClasses = 3;
+// The first digit of a select is 16 bits wide while at most kWideRows
+// segments count (8 bits otherwise).
+constexpr int kWideRows = 64;
+constexpr int kWideBins = 1 << 16;
 
 // Per-call arguments of a step or probe, in device memory: the step's kernels
 // read them at entry, so one captured CUDA graph serves every step.
@@ -213,6 +218,8 @@ struct DevState {
   SelSeg* sel;             // [G] segments
   ClsRange* cls;           // [G * kClasses] candidates per (segment, class)
   uint32_t* hist_bins;     // [G][256] radix histogram
+  uint32_t* wide_bins;     // [kWideRows][65536] first-digit histograms (or [G][256])
+  int16_t* wide_seg;       // [G] segment of each first-digit row
   uint64_t* lst_key;       // split list of the select: key, block, segment
   uint32_t* lst_blk;
   uint16_t* lst_seg;

@@ -1196,6 +1196,139 @@ __device__ __forceinline__ SelSeg list_view(SelSeg z) {
   return z;
 }
 
+// The first counted digit of every segment, over the whole candidate array:
+// 16 bits wide (two bytes) while at most kWideRows segments count, one byte
+// otherwise, into global histograms (warp-aggregated atomics).  CTA 0 records
+// the rows' segments for k_wide_resolve.
+__device__ __forceinline__ void wide_digit(int nrows, uint64_t mask, int* dshift, uint32_t* nbins) {
+  const int sh = next_shift(mask);
+  const bool w16 = nrows <= kWideRows && sh >= 8;
+  *dshift = w16 ? sh - 8 : sh;
+  *nbins = w16 ? (uint32_t)kWideBins : (uint32_t)kRadixBins;
+}
+__global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int fallback) {
+  s = with_args(s);
+  __shared__ int16_t row_of[PS_MAX_GROUPS];
+  __shared__ int s_nrows;
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK || c->mvict == 0) return;
+  const int nseg = single ? 1 : s.G;
+  if (single && !s.sel[0].active) return;
+  {
+    int k = 0;
+    for (int base = 0; base < nseg; base += blockDim.x) {
+      const int g = base + threadIdx.x;
+      bool counts = false;
+      if (g < nseg) {
+        const SelSeg ss = s.sel[g];
+        counts = ss.active && next_shift(ss.mask) >= 0;
+      }
+      int tot;
+      const int ex = block_excl_scan((int)counts, &tot);
+      if (g < nseg) row_of[g] = counts ? (int16_t)(k + ex) : (int16_t)-1;
+      if (counts && blockIdx.x == 0) s.wide_seg[k + ex] = (int16_t)g;
+      k += tot;
+    }
+    if (threadIdx.x == 0) {
+      s_nrows = k;
+      if (blockIdx.x == 0) c->wide_nrows = k;
+    }
+    __syncthreads();
+  }
+  const int nrows = s_nrows;
+  if (nrows == 0) return;
+  const uint32_t stride = nrows <= kWideRows ? (uint32_t)kWideBins : (uint32_t)kRadixBins;
+  for (int64_t e0 = blockIdx.x * (int64_t)blockDim.x; e0 < s.N; e0 += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t e = e0 + threadIdx.x;
+    bool act = false;
+    uint32_t idx = 0;
+    if (e < s.N) {
+      const uint64_t key = s.csk[e];
+      const int seg = single ? 0 : s.blk_group[e];  // issued with the key load
+      if (key != ~0ull && !(fallback && ((s.bm_victim[e >> 5] >> (e & 31)) & 1))) {
+        const int row = row_of[seg];
+        if (row >= 0) {
+          const SelSeg ss = s.sel[seg];
+          if ((key & ss.mask) == ss.prefix) {
+            int dsh;
+            uint32_t nb;
+            wide_digit(nrows, ss.mask, &dsh, &nb);
+            act = true;
+            idx = (uint32_t)row * stride + (uint32_t)((key >> dsh) & (nb - 1));
+          }
+        }
+      }
+    }
+    agg_inc(s.wide_bins, idx, act);
+  }
+}
+
+// One CTA per counted segment: the bucket holding the segment's rank-th key
+// fixes the digit; the row's bins are cleared for the next pass.
+__global__ void __launch_bounds__(1024) k_wide_resolve(DevState s, int single) {
+  s = with_args(s);
+  __shared__ uint32_t s_warp[32];
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK || c->mvict == 0) return;
+  if (single && !s.sel[0].active) return;
+  const int nrows = c->wide_nrows;
+  const int r = blockIdx.x;
+  if (r >= nrows) return;
+  const int seg = s.wide_seg[r];
+  SelSeg ss = s.sel[seg];
+  int dsh;
+  uint32_t nb;
+  wide_digit(nrows, ss.mask, &dsh, &nb);
+  const uint32_t stride = nrows <= kWideRows ? (uint32_t)kWideBins : (uint32_t)kRadixBins;
+  uint32_t* row = s.wide_bins + (size_t)r * stride;
+  // thread t owns bins [t * per, (t + 1) * per): 64 (16-bit digit) or 1 (8-bit, t < 256)
+  const uint32_t per = nb / blockDim.x ? nb / blockDim.x : 1;
+  const uint32_t b0 = threadIdx.x * per;
+  uint32_t sum = 0;
+  if (b0 < nb) {
+    if (per >= 4) {
+      for (uint32_t j = 0; j < per; j += 4) {
+        const uint4 v = __ldcg(reinterpret_cast<const uint4*>(row + b0 + j));
+        sum += v.x + v.y + v.z + v.w;
+      }
+    } else {
+      sum = __ldcg(row + b0);
+    }
+  }
+  // block-wide inclusive scan of the per-thread sums
+  const int lane = lane_id(), warp = threadIdx.x >> 5;
+  const uint32_t wincl = warp_incl_scan(sum);
+  if (lane == 31) s_warp[warp] = wincl;
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t t = lane < (int)(blockDim.x >> 5) ? s_warp[lane] : 0;
+    s_warp[lane] = warp_incl_scan(t) - t;
+  }
+  __syncthreads();
+  const uint32_t incl = s_warp[warp] + wincl;
+  const uint32_t excl = incl - sum;
+  if (b0 < nb && (uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl) {
+    uint32_t run = excl, d = b0;
+    for (uint32_t j = 0; j < per; ++j) {
+      const uint32_t v = __ldcg(row + b0 + j);
+      if ((uint64_t)ss.rank <= (uint64_t)(run + v)) { d = b0 + j; break; }
+      run += v;
+    }
+    ss.prefix |= (uint64_t)d << dsh;
+    ss.mask |= (uint64_t)(nb - 1) << dsh;
+    ss.rank -= run;
+    s.sel[seg] = ss;
+  }
+  __syncthreads();
+  if (b0 < nb) {
+    if (per >= 4) {
+      for (uint32_t j = 0; j < per; j += 4) *reinterpret_cast<uint4*>(row + b0 + j) = make_uint4(0, 0, 0, 0);
+    } else {
+      row[b0] = 0;
+    }
+  }
+}
+
 // One digit for every segment that still has one: over the whole candidate
 // array (from_list = 0) or over the split list (from_list = 1).
 __global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int fallback, int from_list) {
@@ -1880,7 +2013,8 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   // (a body is launched only once its capture has started: a kernel launched
   // on the auxiliary stream outside a capture would run)
   auto select = [&](cudaStream_t q, int single, int fallback, bool cond) {
-    PS_LAUNCH(k_digit_pass<<<sgrid, 256, radix_smem, q>>>(s, single, fallback, 0));
+    PS_LAUNCH(k_wide_pass<<<cgrid, 256, 0, q>>>(s, single, fallback));
+    PS_LAUNCH(k_wide_resolve<<<single ? 1 : s.G, 1024, 0, q>>>(s, single));
     PS_LAUNCH(k_split<<<cgrid, 256, 0, q>>>(s, single, fallback, h_long, cond ? 1 : 0));
     cudaStream_t b = q;
     if (cond) {
