@@ -52,6 +52,8 @@ def parse_args():
     ap.add_argument("--cpu-steps", type=int, default=3, help="timed oracle steps for cpu_baseline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="launch the step kernel by kernel (profilers cannot see inside its graph)")
     return ap.parse_args()
 
 
@@ -242,6 +244,7 @@ def run_own(args, ws, rank, local):
     cache = B.Cache(spec.capacity_blocks, spec.block_size, spec.num_groups, args.policy, params,
                     max_requests=R, max_tokens=maxT)
     cache.set_stage_timing(True)
+    cache.set_graph(not args.no_graph)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
 
     def run(k):
@@ -323,7 +326,8 @@ def run_own(args, ws, rank, local):
         "config": {"workload": WORKLOAD, "policy": args.policy, "prefill_steps": args.prefill,
                    "requests_per_step": R, "block_size": spec.block_size, "capacity_blocks": spec.capacity_blocks,
                    "groups": spec.num_groups, "l2": "flushed (256 MiB write) between timed steps",
-                   "parallelism": f"replicas x{ws}"},
+                   "parallelism": f"replicas x{ws}",
+                   "launch": "cuda graph" if cache.uses_graph() else "kernel by kernel"},
         "kv_blocks_per_s": blk_all / total_max,
         "step_roofline": {"bound": "hbm", "achieved": step_gbs, "peak": peak, "unit": "GB/s",
                           "frac": step_gbs / peak, "algorithmic_bytes_per_step": alg / args.steps,

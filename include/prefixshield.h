@@ -257,6 +257,13 @@ int32_t ps_get_stage_times(ps_handle_t* h, float* h_ms, int32_t max_stages, int3
  * Measurement hook; the paper has no counterpart. */
 int32_t ps_uses_graph(const ps_handle_t* h);
 
+/* Launch mode of ps_step(): enable = 1 (the default) replays the step as one
+ * captured CUDA graph, enable = 0 launches its kernels one by one on the
+ * caller's stream (for profilers that cannot see inside graphs with
+ * conditional nodes).  The same kernels do the same work either way.
+ * Measurement hook; the paper has no counterpart. */
+int32_t ps_set_graph(ps_handle_t* h, int32_t enable);
+
 #ifdef __cplusplus
 }
 #endif

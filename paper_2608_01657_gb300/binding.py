@@ -32,7 +32,7 @@ PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE = 1, 2
 EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_stats", "ps_clear_status",
             "ps_reset", "ps_destroy", "ps_status_string", "ps_export_state", "ps_export_history",
             "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times", "ps_cached_prefix",
-            "ps_cached_prefix_noalloc", "ps_uses_graph")
+            "ps_cached_prefix_noalloc", "ps_uses_graph", "ps_set_graph")
 PS_NUM_STAGES = 11
 STAGE_NAMES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
                "freetake_evict", "id_lists", "insert", "commit")
@@ -116,6 +116,8 @@ def load():
     L.ps_get_stage_times.argtypes = [vp, vp, i32, vp]
     L.ps_uses_graph.restype = i32
     L.ps_uses_graph.argtypes = [C.c_void_p]
+    L.ps_set_graph.restype = i32
+    L.ps_set_graph.argtypes = [C.c_void_p, i32]
     _lib = L
     return L
 
@@ -294,6 +296,12 @@ class Cache:
         rc = load().ps_set_stage_timing(self._h, int(enable))
         if rc != PS_OK:
             raise RuntimeError(f"ps_set_stage_timing failed ({rc})")
+
+    def set_graph(self, enable: bool = True):
+        """Replay the step as one CUDA graph (default) or launch kernel by kernel."""
+        rc = load().ps_set_graph(self._h, int(enable))
+        if rc != PS_OK:
+            raise RuntimeError(f"ps_set_graph failed ({rc})")
 
     def uses_graph(self) -> bool:
         """True once the step replays one captured CUDA graph."""

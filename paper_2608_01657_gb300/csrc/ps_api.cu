@@ -548,6 +548,13 @@ int32_t ps_get_stage_times(ps_handle_t* h, float* h_ms, int32_t max_stages, int3
   return n;
 }
 
+int32_t ps_set_graph(ps_handle_t* h, int32_t enable) {
+  if (!h) return PS_ERR_INVALID_ARG;
+  if (!enable) drop_graph(h);
+  h->use_graph = enable != 0;  // captured (again) at the next step
+  return PS_OK;
+}
+
 int32_t ps_uses_graph(const ps_handle_t* h) {
   if (!h) return PS_ERR_INVALID_ARG;
   return h->use_graph && h->exec ? 1 : 0;

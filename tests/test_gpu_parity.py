@@ -285,3 +285,30 @@ def test_parity_long_split_list():
                      max_requests=1, max_tokens=12000 * 16)
     _run(gpu, orc, steps, label="long list")
     assert int(gpu.stats()[0][8]) == 5425  # evicted blocks of group 0
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+def test_parity_kernel_by_kernel(policy):
+    """The same step launched kernel by kernel (no graph), stage timing on and
+    off, matches the oracle too."""
+    steps = W.fuzz_steps(23, 3, 6, 40, docs_per_group=3, doc_blocks=7, fresh_max_blocks=2,
+                         with_contracts=3, with_prefixes=True, now_stride=2, empty_every=5)
+    kw = dict(rho=(2.0, 1.5, 1.0), beta=(6.0, 5.0, 4.0), contract_of_group=[0, 1, 2])
+    gpu, orc = _pair(40, 16, 3, policy, kw, max_requests=6, max_tokens=4096)
+    gpu.set_graph(False)
+    dev = torch.device("cuda")
+    for k, st in enumerate(steps):
+        if k % 10 == 5:
+            gpu.set_stage_timing(k % 20 == 5)
+        g = torch.from_numpy(st.groups).to(dev)
+        o = torch.from_numpy(st.offsets).to(dev)
+        t = torch.from_numpy(st.tokens if st.num_tokens else np.zeros(4, np.int32)).to(dev)
+        c = torch.from_numpy(st.contracts).to(dev)
+        p = torch.from_numpy(st.prefixes.view(np.int64)).to(dev)
+        assert gpu.step(st.now, g, o, t, c, p) == 0
+        assert not gpu.uses_graph()
+        compare_outputs(gpu.fetch(st.num_requests),
+                        orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts, st.prefixes),
+                        f"direct/{policy} step {k}")
+    compare_state(gpu.export(), orc.export(), f"direct/{policy}", s3=policy == "s3fifo")
+    assert np.array_equal(gpu.stats(), orc.stats())
