@@ -1307,17 +1307,36 @@ __global__ void __launch_bounds__(1024) k_wide_resolve(DevState s, int single) {
   __syncthreads();
   const uint32_t incl = s_warp[warp] + wincl;
   const uint32_t excl = incl - sum;
-  if (b0 < nb && (uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl) {
-    uint32_t run = excl, d = b0;
-    for (uint32_t j = 0; j < per; ++j) {
-      const uint32_t v = __ldcg(row + b0 + j);
-      if ((uint64_t)ss.rank <= (uint64_t)(run + v)) { d = b0 + j; break; }
-      run += v;
+  const bool here = b0 < nb && (uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl;
+  // the owning thread's warp searches its bins together (2 per lane): one
+  // round of independent loads and a warp scan instead of a chain of loads
+  const unsigned hw = __ballot_sync(kFull, here);
+  if (hw) {
+    const int src = __ffs(hw) - 1;
+    const uint32_t sb0 = __shfl_sync(kFull, b0, src), sexcl = __shfl_sync(kFull, excl, src);
+    uint32_t d = sb0, run = sexcl;
+    if (per == 1) {
+      // 8-bit digit: the owner's single bin is the digit
+    } else {
+      const uint32_t i0 = sb0 + 2 * lane;  // per == 64: 32 lanes x 2 bins
+      const uint32_t v0 = __ldcg(row + i0), v1 = __ldcg(row + i0 + 1);
+      const uint32_t pair = v0 + v1;
+      const uint32_t pincl = warp_incl_scan(pair) + sexcl;
+      const uint32_t pexcl = pincl - pair;
+      const bool mine = (uint64_t)pexcl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)pincl;
+      const unsigned mw = __ballot_sync(kFull, mine);
+      const int ml = mw ? __ffs(mw) - 1 : 0;
+      const uint32_t me = __shfl_sync(kFull, pexcl, ml), mv0 = __shfl_sync(kFull, v0, ml);
+      const bool first = (uint64_t)ss.rank <= (uint64_t)(me + mv0);
+      d = sb0 + 2 * ml + (first ? 0 : 1);
+      run = first ? me : me + mv0;
     }
-    ss.prefix |= (uint64_t)d << dsh;
-    ss.mask |= (uint64_t)(nb - 1) << dsh;
-    ss.rank -= run;
-    s.sel[seg] = ss;
+    if (lane == src) {
+      ss.prefix |= (uint64_t)d << dsh;
+      ss.mask |= (uint64_t)(nb - 1) << dsh;
+      ss.rank -= run;
+      s.sel[seg] = ss;
+    }
   }
   __syncthreads();
   if (b0 < nb) {
