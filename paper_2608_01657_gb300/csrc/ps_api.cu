@@ -235,6 +235,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
     const size_t wb = wrows * kWideBins > G * kRadixBins ? wrows * kWideBins : G * kRadixBins;
     t.wide_bins = cv.take<uint32_t>(wb);
   }
+  t.wide_coarse = cv.take<uint32_t>((size_t)kWideRows * kRadixBins);
   t.wide_seg = cv.take<int16_t>(G);
   t.lst_key = cv.take<uint64_t>(N);
   t.lst_blk = cv.take<uint32_t>(N);

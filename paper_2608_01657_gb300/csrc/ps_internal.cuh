@@ -219,6 +219,7 @@ struct DevState {
   ClsRange* cls;           // [G * kClasses] candidates per (segment, class)
   uint32_t* hist_bins;     // [G][256] radix histogram
   uint32_t* wide_bins;     // [kWideRows][65536] first-digit histograms (or [G][256])
+  uint32_t* wide_coarse;   // [kWideRows][256] the 16-bit histograms summed by their top byte
   int16_t* wide_seg;       // [G] segment of each first-digit row
   uint64_t* lst_key;       // split list of the select: key, block, segment
   uint32_t* lst_blk;

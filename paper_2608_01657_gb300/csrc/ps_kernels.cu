@@ -1089,37 +1089,53 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
     }
     return;
   }
-  // tau = max{t in [eps+1, pmax] : items_gt(t - 1) summed >= m}.  Each round
-  // tests kThr thresholds spread over the interval; the 16 lanes of a
-  // half-warp split the groups of one threshold.
-  constexpr int kThr = 64, kLanes = 16;
-  __shared__ int s_ok[kThr];
-  int64_t lo = eps + 1, hi = s_pmax;
-  const int j = threadIdx.x / kLanes, gl = threadIdx.x % kLanes;
-  while (lo < hi) {
-    const int64_t span = hi - lo;  // >= 1
-    const int64_t stride = tmax<int64_t>(1, (span - 1) / (kThr - 1));
-    auto thr = [&](int jj) -> int64_t { return jj == kThr - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * jj); };
-    int64_t cnt = 0;
-    if (j < kThr) {
-      const int64_t t = thr(j);
-      for (int g = gl; g < G; g += kLanes) cnt += items_gt(g, t - 1);
+  // tau = max{t in [eps+1, pmax] : items_gt(t - 1) summed >= m}.  Only the
+  // groups that can hold an item above eps count (d > 0, q > 0, P > eps);
+  // each round tests T thresholds spread over the interval, L lanes (a power
+  // of two covering those groups, at most 32) splitting the groups of one.
+  __shared__ int16_t s_gid[PS_MAX_GROUPS];
+  __shared__ int s_ng;
+  __shared__ int s_J[3];
+  {
+    int k = 0;
+    for (int base = 0; base < G; base += blockDim.x) {
+      const int g = base + threadIdx.x;
+      const bool holds = g < G && sD[g] > 0 && sQ[g] > 0 && sP[g] > eps;
+      int tot;
+      const int ex = block_excl_scan((int)holds, &tot);
+      if (holds) s_gid[k + ex] = (int16_t)g;
+      k += tot;
     }
-#pragma unroll
-    for (int o = kLanes / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
-    if (j < kThr && gl == 0) s_ok[j] = cnt >= m;
+    if (threadIdx.x == 0) s_ng = k;
+    if (threadIdx.x < 3) s_J[threadIdx.x] = -1;
     __syncthreads();
-    // J = the largest threshold that still holds m items (counts fall as the
-    // threshold rises, so the flags are a prefix): two ballots per warp
-    const unsigned lo32 = __ballot_sync(kFull, s_ok[lane_id()] != 0);
-    const unsigned hi32 = __ballot_sync(kFull, s_ok[32 + lane_id()] != 0);
-    const int J = hi32 ? 63 - __clz((int)hi32) : (lo32 ? 31 - __clz((int)lo32) : -1);
+  }
+  const int ng = s_ng;
+  int L = 1, logT = 10;  // blockDim.x == 1024 == T * L
+  while (L < ng && L < 32) { L <<= 1; --logT; }
+  const int T = 1 << logT;
+  int64_t lo = eps + 1, hi = s_pmax;
+  const int jt = threadIdx.x / L, gl = threadIdx.x % L;
+  for (int r = 0; lo < hi; ++r) {
+    const int64_t span = hi - lo;  // >= 1
+    const int64_t stride = tmax<int64_t>(1, (span + T - 1) >> logT);
+    auto thr = [&](int jj) -> int64_t { return jj == T - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * jj); };
+    const int64_t t = thr(jt);
+    int64_t cnt = 0;
+    for (int k = gl; k < ng; k += L) cnt += items_gt(s_gid[k], t - 1);
+    for (int o = L / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
+    // J = the largest threshold still holding m items (counts fall as the
+    // threshold rises); slots rotate over three rounds, so one barrier a
+    // round separates every slot's reset, updates and reads
+    if (threadIdx.x == 0) s_J[(r + 1) % 3] = -1;
+    if (gl == 0 && cnt >= m) atomicMax(&s_J[r % 3], jt);
     __syncthreads();
+    const int J = s_J[r % 3];
     if (J < 0) {
       hi = lo;
     } else {
       lo = thr(J);
-      hi = J + 1 < kThr ? thr(J + 1) - 1 : hi;
+      hi = J + 1 < T ? thr(J + 1) - 1 : hi;
       if (hi < lo) hi = lo;
     }
   }
@@ -1240,7 +1256,7 @@ __global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int f
   const uint32_t stride = nrows <= kWideRows ? (uint32_t)kWideBins : (uint32_t)kRadixBins;
   for (int64_t e0 = blockIdx.x * (int64_t)blockDim.x; e0 < s.N; e0 += (int64_t)gridDim.x * blockDim.x) {
     const int64_t e = e0 + threadIdx.x;
-    bool act = false;
+    bool act = false, act16 = false;
     uint32_t idx = 0;
     if (e < s.N) {
       const uint64_t key = s.csk[e];
@@ -1254,97 +1270,80 @@ __global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int f
             uint32_t nb;
             wide_digit(nrows, ss.mask, &dsh, &nb);
             act = true;
+            act16 = nb == (uint32_t)kWideBins;
             idx = (uint32_t)row * stride + (uint32_t)((key >> dsh) & (nb - 1));
           }
         }
       }
     }
     agg_inc(s.wide_bins, idx, act);
+    // 16-bit digits also by their top byte (row-major, 256 a row)
+    if (stride == (uint32_t)kWideBins) agg_inc(s.wide_coarse, (idx >> 16) * kRadixBins + ((idx >> 8) & 0xFF), act16);
   }
 }
 
-// One CTA per counted segment: the bucket holding the segment's rank-th key
-// fixes the digit; the row's bins are cleared for the next pass.
-__global__ void __launch_bounds__(1024) k_wide_resolve(DevState s, int single) {
+// One warp per counted segment: the bucket holding the segment's rank-th key
+// fixes the digit.  A 16-bit digit is found in two short scans (its top byte
+// from the coarse histogram, then the 256 bins under it); the coarse bins are
+// cleared here and the fine ones by the split that follows.
+__global__ void __launch_bounds__(32) k_wide_resolve(DevState s, int single) {
   s = with_args(s);
-  __shared__ uint32_t s_warp[32];
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   if (single && !s.sel[0].active) return;
   const int nrows = c->wide_nrows;
   const int r = blockIdx.x;
   if (r >= nrows) return;
+  const int lane = lane_id();
   const int seg = s.wide_seg[r];
   SelSeg ss = s.sel[seg];
   int dsh;
   uint32_t nb;
   wide_digit(nrows, ss.mask, &dsh, &nb);
+  const bool w16 = nb == (uint32_t)kWideBins;
   const uint32_t stride = nrows <= kWideRows ? (uint32_t)kWideBins : (uint32_t)kRadixBins;
   uint32_t* row = s.wide_bins + (size_t)r * stride;
-  // thread t owns bins [t * per, (t + 1) * per): 64 (16-bit digit) or 1 (8-bit, t < 256)
-  const uint32_t per = nb / blockDim.x ? nb / blockDim.x : 1;
-  const uint32_t b0 = threadIdx.x * per;
-  uint32_t sum = 0;
-  if (b0 < nb) {
-    if (per >= 4) {
-      for (uint32_t j = 0; j < per; j += 4) {
-        const uint4 v = __ldcg(reinterpret_cast<const uint4*>(row + b0 + j));
-        sum += v.x + v.y + v.z + v.w;
+  // locate rank among 256 consecutive bins (8 a lane); returns the bin and
+  // the count before it
+  auto locate = [&](const uint32_t* bins, uint64_t rank, uint32_t* before) -> uint32_t {
+    uint32_t v[8], sum = 0;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) { v[k] = __ldcg(bins + lane * 8 + k); sum += v[k]; }
+    const uint32_t incl = warp_incl_scan(sum), excl = incl - sum;
+    const bool mine = (uint64_t)excl < rank && rank <= (uint64_t)incl;
+    const unsigned mw = __ballot_sync(kFull, mine);
+    const int ml = mw ? __ffs(mw) - 1 : 0;
+    uint32_t d = 0, run = excl;
+    if (mine) {
+      for (int k = 0; k < 8; ++k) {
+        if (rank <= (uint64_t)(run + v[k])) { d = lane * 8 + k; break; }
+        run += v[k];
       }
-    } else {
-      sum = __ldcg(row + b0);
     }
+    *before = __shfl_sync(kFull, run, ml);
+    return __shfl_sync(kFull, d, ml);
+  };
+  uint32_t d, run;
+  if (w16) {
+    uint32_t* coarse = s.wide_coarse + (size_t)r * kRadixBins;
+    uint32_t cb_before;
+    const uint32_t cb = locate(coarse, (uint64_t)ss.rank, &cb_before);
+    uint32_t fb_before;
+    const uint32_t fb = locate(row + cb * kRadixBins, (uint64_t)ss.rank - cb_before, &fb_before);
+    d = cb * kRadixBins + fb;
+    run = cb_before + fb_before;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) coarse[lane * 8 + k] = 0;
+  } else {
+    d = locate(row, (uint64_t)ss.rank, &run);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) row[lane * 8 + k] = 0;
   }
-  // block-wide inclusive scan of the per-thread sums
-  const int lane = lane_id(), warp = threadIdx.x >> 5;
-  const uint32_t wincl = warp_incl_scan(sum);
-  if (lane == 31) s_warp[warp] = wincl;
-  __syncthreads();
-  if (warp == 0) {
-    const uint32_t t = lane < (int)(blockDim.x >> 5) ? s_warp[lane] : 0;
-    s_warp[lane] = warp_incl_scan(t) - t;
-  }
-  __syncthreads();
-  const uint32_t incl = s_warp[warp] + wincl;
-  const uint32_t excl = incl - sum;
-  const bool here = b0 < nb && (uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl;
-  // the owning thread's warp searches its bins together (2 per lane): one
-  // round of independent loads and a warp scan instead of a chain of loads
-  const unsigned hw = __ballot_sync(kFull, here);
-  if (hw) {
-    const int src = __ffs(hw) - 1;
-    const uint32_t sb0 = __shfl_sync(kFull, b0, src), sexcl = __shfl_sync(kFull, excl, src);
-    uint32_t d = sb0, run = sexcl;
-    if (per == 1) {
-      // 8-bit digit: the owner's single bin is the digit
-    } else {
-      const uint32_t i0 = sb0 + 2 * lane;  // per == 64: 32 lanes x 2 bins
-      const uint32_t v0 = __ldcg(row + i0), v1 = __ldcg(row + i0 + 1);
-      const uint32_t pair = v0 + v1;
-      const uint32_t pincl = warp_incl_scan(pair) + sexcl;
-      const uint32_t pexcl = pincl - pair;
-      const bool mine = (uint64_t)pexcl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)pincl;
-      const unsigned mw = __ballot_sync(kFull, mine);
-      const int ml = mw ? __ffs(mw) - 1 : 0;
-      const uint32_t me = __shfl_sync(kFull, pexcl, ml), mv0 = __shfl_sync(kFull, v0, ml);
-      const bool first = (uint64_t)ss.rank <= (uint64_t)(me + mv0);
-      d = sb0 + 2 * ml + (first ? 0 : 1);
-      run = first ? me : me + mv0;
-    }
-    if (lane == src) {
-      ss.prefix |= (uint64_t)d << dsh;
-      ss.mask |= (uint64_t)(nb - 1) << dsh;
-      ss.rank -= run;
-      s.sel[seg] = ss;
-    }
-  }
-  __syncthreads();
-  if (b0 < nb) {
-    if (per >= 4) {
-      for (uint32_t j = 0; j < per; j += 4) *reinterpret_cast<uint4*>(row + b0 + j) = make_uint4(0, 0, 0, 0);
-    } else {
-      row[b0] = 0;
-    }
+  if (lane == 0) {
+    ss.prefix |= (uint64_t)d << dsh;
+    ss.mask |= (uint64_t)(nb - 1) << dsh;
+    ss.rank -= run;
+    s.sel[seg] = ss;
   }
 }
 
@@ -1470,6 +1469,16 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   if (single && !s.sel[0].active) return;
+  {
+    // the first digit's 16-bit rows are read: clear them for the next select
+    const int nrows = c->wide_nrows;
+    if (nrows <= kWideRows) {
+      uint4* w = reinterpret_cast<uint4*>(s.wide_bins);
+      const int64_t n4 = (int64_t)nrows * kWideBins / 4;
+      for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n4; k += (int64_t)gridDim.x * blockDim.x)
+        w[k] = make_uint4(0, 0, 0, 0);
+    }
+  }
   int marked = 0;
   for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
     const int64_t b = b0 + threadIdx.x;
@@ -2033,7 +2042,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   // on the auxiliary stream outside a capture would run)
   auto select = [&](cudaStream_t q, int single, int fallback, bool cond) {
     PS_LAUNCH(k_wide_pass<<<cgrid, 256, 0, q>>>(s, single, fallback));
-    PS_LAUNCH(k_wide_resolve<<<single ? 1 : s.G, 1024, 0, q>>>(s, single));
+    PS_LAUNCH(k_wide_resolve<<<single ? 1 : s.G, 32, 0, q>>>(s, single));
     PS_LAUNCH(k_split<<<cgrid, 256, 0, q>>>(s, single, fallback, h_long, cond ? 1 : 0));
     cudaStream_t b = q;
     if (cond) {
