@@ -22,6 +22,7 @@ path).
 from __future__ import annotations
 
 import argparse
+import gc
 import json
 import os
 import statistics
@@ -264,6 +265,8 @@ def run_own(args, ws, rank, local):
     launches = 0
     barrier(ws)
     torch.cuda.synchronize()
+    gc.collect()
+    gc.disable()
     with ClockSampler(local) as clk:
         for j in range(args.steps):
             flush.zero_()
@@ -275,6 +278,7 @@ def run_own(args, ws, rank, local):
             stage_ms[: len(ms)] += ms
             launches += nl
         torch.cuda.synchronize()
+    gc.enable()
     barrier(ws)
     step_ms = [e0.elapsed_time(e1) for e0, e1 in evs]
     total_s = sum(step_ms) / 1e3
@@ -367,21 +371,27 @@ def run_e2e(args, cache, steps, dsteps, flush, R):
     out = B.host_outputs(R, cache.max_blocks, cache.G, pinned=True)
     h2d = d2h = 0
     t_sum = 0.0
+    per = []
+    gc.collect()
+    gc.disable()  # no collector pauses inside the timed host loop
     for (now, g, o, t) in host:
         flush.zero_()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         r = cache.step_host(now, g, o, t, out=out)
-        t_sum += time.perf_counter() - t0
+        per.append(time.perf_counter() - t0)
+        t_sum += per[-1]
         if r["rc"] != 0:
             raise RuntimeError(f"ps_step_host rc={r['rc']}")
         cnt = out["counts"]
         h2d += g.nbytes + o.nbytes + t.nbytes
         d2h += 16 + 4 * (2 * len(g) + len(g) + 1) + 16 * cache.G + 4 * int(cnt[0] + cnt[1] + cnt[2])
+    gc.enable()
     n = len(host)
     return {"value": sum(len(h[1]) for h in host) / t_sum, "unit": "requests/s",
             "h2d_bytes_per_step": h2d // n, "d2h_bytes_per_step": d2h // n,
-            "ms_per_step": 1e3 * t_sum / n}
+            "ms_per_step": 1e3 * t_sum / n,
+            "step_ms": {"min": 1e3 * min(per), "median": 1e3 * statistics.median(per), "max": 1e3 * max(per)}}
 
 
 def main():
