@@ -943,17 +943,28 @@ __device__ __forceinline__ void sel_start(SelSeg& z);
 // the rank-th smallest key is fixed (lower classes are all below it), the rank
 // becomes a rank inside that class, and the key range is the class's.
 // cnt[k] and [lo[k], hi[k]] describe class k (unsegmented keys: class 0 only).
-__device__ __forceinline__ void sel_start_cls(SelSeg& z, const int64_t* cnt, const uint64_t* lo, const uint64_t* hi,
-                                              bool segmented) {
+// Classes are picked without run-time array indexing (registers only).
+__device__ __forceinline__ void sel_start_cls(SelSeg& z, const int64_t (&cnt)[kClasses], const uint64_t (&lo)[kClasses],
+                                              const uint64_t (&hi)[kClasses], bool segmented) {
+  static_assert(kClasses == 3, "class choice below is written for three classes");
   int k = 0;
   int64_t below = 0;
-  if (segmented)
-    while (k < kClasses - 1 && z.rank > below + cnt[k]) below += cnt[k++];
+  if (segmented && z.rank > cnt[0]) {
+    below = cnt[0];
+    k = 1;
+    if (z.rank > cnt[0] + cnt[1]) {
+      below += cnt[1];
+      k = 2;
+    }
+  }
+  const int64_t ck = k == 0 ? cnt[0] : k == 1 ? cnt[1] : cnt[2];
+  const uint64_t lk = k == 0 ? lo[0] : k == 1 ? lo[1] : lo[2];
+  const uint64_t hk = k == 0 ? hi[0] : k == 1 ? hi[1] : hi[2];
   const uint64_t cb = segmented ? (uint64_t)k << 62 : 0ull;
-  if (z.active && cnt[k] > 0) {
+  if (z.active && ck > 0) {
     z.rank -= below;
-    z.kmin = cb | lo[k];
-    z.kmax = cb | hi[k];
+    z.kmin = cb | lk;
+    z.kmax = cb | hk;
   } else {
     z.kmin = z.kmax = cb;
   }
@@ -962,6 +973,7 @@ __device__ __forceinline__ void sel_start_cls(SelSeg& z, const int64_t* cnt, con
 __device__ __forceinline__ void sel_start_group(const DevState& s, int g, SelSeg& z, bool segmented) {
   int64_t cnt[kClasses];
   uint64_t lo[kClasses], hi[kClasses];
+#pragma unroll
   for (int k = 0; k < kClasses; ++k) {
     const ClsRange r = s.cls[g * kClasses + k];
     cnt[k] = r.cnt;
@@ -1806,12 +1818,15 @@ __global__ void __launch_bounds__(kThreads) k_evict(DevState s) {
 // Stage 6: place granted claims (thread per position).  The allocated ids
 // (ascending) go to the granted keys in (request, position) order; each new
 // block carries the metadata OnCacheFullBlocks attached plus any in-step
-// touches.
+// touches.  Each claim's owning position then clears its claim-map slot (no
+// other thread reads it here), and each request's first position commits its
+// OnRequest / RecordSuccessfulAdmission history update.
 __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  if (pos == 0) c->hist_live += c->hist_new;
   PosRef r;
   bool placed = false;
   uint32_t g = 0;
@@ -1819,6 +1834,14 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
     const uint32_t i = r.i;
     const int si = s.rq_s[i], a = s.rq_a[i];
     g = (uint32_t)s.in_group[i];
+    if (r.m == 0) {  // history commit of request i (it has a full block)
+      const uint32_t hs = s.rq_hs[i];
+      if (hs != kNone) {
+        atomicAdd(&s.hist[hs].refadm, 1u);
+        if (a > 0) atomicOr(&s.hist[hs].refadm, 0x80000000u);
+      }
+    }
+    const uint32_t slot = r.m >= si ? s.pos_claim[pos] : kNone;  // an own claim
     if (r.m >= si && r.m < si + a) {
       const int64_t rank = (int64_t)s.rq_cbase[i] + (r.m - si);
       const uint32_t b = rank < c->n_alloc ? (uint32_t)s.out.admitted_ids[rank] : kNone;
@@ -1842,42 +1865,19 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
         placed = true;
       }
     }
+    if (slot != kNone) {
+      ClaimEntry z{};
+      z.key = 0; z.minreq = kNone; z.last = 0; z.tcnt = 0; z.promo = kNone; z.pad0 = 0; z.pad1 = 0;
+      s.claims[slot] = z;
+    }
   }
   agg_stat(s, g, PS_STAT_RESIDENT_BLOCKS, placed ? 1 : 0, placed);
   const int k = __popc(__ballot_sync(kFull, placed));
   if (lane_id() == 0 && k) atomic_add_i64(&c->n_resident, k);
 }
 
-// OnRequest / RecordSuccessfulAdmission commit: reference counts and admitted
-// flags of the history entries (thread per request).
-__global__ void k_hist_commit(DevState s) {
-  s = with_args(s);
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i == 0) c->hist_live += c->hist_new;
-  if (i >= s.R || s.rq_n[i] == 0) return;
-  const uint32_t hs = s.rq_hs[i];
-  if (hs == kNone) return;
-  atomicAdd(&s.hist[hs].refadm, 1u);
-  if (s.rq_a[i] > 0) atomicOr(&s.hist[hs].refadm, 0x80000000u);
-}
-
-// Clear the claim-map slots this step used (thread per position).
-__global__ void __launch_bounds__(kThreads) k_claim_clear(DevState s) {
-  s = with_args(s);
-  const Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  PosRef r;
-  if (!pos_ref(s, pos, &r) || r.m < s.rq_h[r.i]) return;
-  const uint32_t slot = s.pos_claim[pos];
-  if (slot == kNone) return;
-  ClaimEntry z{};
-  z.key = 0; z.minreq = kNone; z.last = 0; z.tcnt = 0; z.promo = kNone; z.pad0 = 0; z.pad1 = 0;
-  s.claims[slot] = z;
-}
-
+// Step end: the outputs' counts and status, then the clock, the step index
+// and the next step's first recency stamp.
 __global__ void k_finalize(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
@@ -2085,8 +2085,6 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(k_insert<<<pgrid, kThreads, 0, st>>>(s));
   if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));
   mark(10);
-  PS_LAUNCH(k_hist_commit<<<rgrid, 256, 0, st>>>(s));
-  PS_LAUNCH(k_claim_clear<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_finalize<<<1, 32, 0, st>>>(s));
   mark(11);
 #undef PS_LAUNCH
