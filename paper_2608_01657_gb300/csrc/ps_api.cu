@@ -29,7 +29,8 @@ struct ps_handle {
   // the step as one CUDA graph, captured on a private stream at first use
   StepArgs* step_args;
   cudaStream_t cap_stream = nullptr;
-  cudaStream_t cap_aux = nullptr;  // conditional bodies are captured here
+  cudaStream_t cap_aux = nullptr;   // conditional bodies are captured here
+  cudaStream_t cap_aux2 = nullptr;  // and bodies nested in them here
   cudaGraph_t graph = nullptr;
   cudaGraphExec_t exec = nullptr;
   bool exec_timing = false;
@@ -304,13 +305,15 @@ void capture_step(ps_handle* h) {
   tmpl.R = 0;
   bool ok = cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
   if (ok) {
-    const CaptureCtx ctx{h->cap_aux};
+    const CaptureCtx ctx{h->cap_aux, h->cap_aux2};
     const int32_t rc = launch_step(tmpl, h->cap_stream, &h->trace, &ctx);
-    // a body whose capture did not close leaves the auxiliary stream capturing
-    cudaStreamCaptureStatus aux_cs = cudaStreamCaptureStatusNone;
-    if (cudaStreamIsCapturing(h->cap_aux, &aux_cs) == cudaSuccess && aux_cs != cudaStreamCaptureStatusNone) {
-      cudaGraph_t body = nullptr;
-      cudaStreamEndCapture(h->cap_aux, &body);
+    // a body whose capture did not close leaves an auxiliary stream capturing
+    for (cudaStream_t a : {h->cap_aux2, h->cap_aux}) {
+      cudaStreamCaptureStatus aux_cs = cudaStreamCaptureStatusNone;
+      if (cudaStreamIsCapturing(a, &aux_cs) == cudaSuccess && aux_cs != cudaStreamCaptureStatusNone) {
+        cudaGraph_t body = nullptr;
+        cudaStreamEndCapture(a, &body);
+      }
     }
     cudaGraph_t g = nullptr;
     const bool ended = cudaStreamEndCapture(h->cap_stream, &g) == cudaSuccess;
@@ -392,7 +395,8 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   int32_t rc = init_state(h, st);
   if (rc == PS_OK) rc = upload_constants(h, st);
   if (rc == PS_OK && (cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess ||
-                      cudaStreamCreateWithFlags(&h->cap_aux, cudaStreamNonBlocking) != cudaSuccess))
+                      cudaStreamCreateWithFlags(&h->cap_aux, cudaStreamNonBlocking) != cudaSuccess ||
+                      cudaStreamCreateWithFlags(&h->cap_aux2, cudaStreamNonBlocking) != cudaSuccess))
     rc = PS_ERR_CUDA;
   if (rc != PS_OK) {
     delete h;
@@ -516,6 +520,7 @@ void ps_destroy(ps_handle_t* h) {
   drop_graph(h);
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   if (h->cap_aux) cudaStreamDestroy(h->cap_aux);
+  if (h->cap_aux2) cudaStreamDestroy(h->cap_aux2);
   if (h->trace.timing)
     for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
   delete h;

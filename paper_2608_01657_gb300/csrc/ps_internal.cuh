@@ -274,7 +274,8 @@ struct StepTrace {
 // Stream capture of a step: a second private stream on which the bodies of
 // conditional graph nodes are captured (phases that many steps skip).
 struct CaptureCtx {
-  cudaStream_t aux;
+  cudaStream_t aux;   // bodies of top-level conditional nodes
+  cudaStream_t aux2;  // bodies of conditional nodes inside those
 };
 
 // Copy the call's arguments from device memory into the kernel's DevState.

@@ -1104,7 +1104,9 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   // tau = max{t in [eps+1, pmax] : items_gt(t - 1) summed >= m}.  Only the
   // groups that can hold an item above eps count (d > 0, q > 0, P > eps);
   // each round tests T thresholds spread over the interval, L lanes (a power
-  // of two covering those groups, at most 32) splitting the groups of one.
+  // of two) splitting the groups of one so that no thread evaluates more than
+  // 32 (a thread's evaluations are independent and overlap; fewer, wider
+  // rounds beat more lanes with shuffles).
   __shared__ int16_t s_gid[PS_MAX_GROUPS];
   __shared__ int s_ng;
   __shared__ int s_J[3];
@@ -1124,7 +1126,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   }
   const int ng = s_ng;
   int L = 1, logT = 10;  // blockDim.x == 1024 == T * L
-  while (L < ng && L < 32) { L <<= 1; --logT; }
+  while (L * 32 < ng && L < 32) { L <<= 1; --logT; }
   const int T = 1 << logT;
   int64_t lo = eps + 1, hi = s_pmax;
   const int jt = threadIdx.x / L, gl = threadIdx.x % L;
@@ -1134,6 +1136,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
     auto thr = [&](int jj) -> int64_t { return jj == T - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * jj); };
     const int64_t t = thr(jt);
     int64_t cnt = 0;
+#pragma unroll 4
     for (int k = gl; k < ng; k += L) cnt += items_gt(s_gid[k], t - 1);
     for (int o = L / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
     // J = the largest threshold still holding m items (counts fall as the
@@ -1951,7 +1954,7 @@ void configure_kernels(const DevState& s) {
 // Under stream capture: append an 'if' conditional node to the graph being
 // captured on st, and start capturing its body on aux.  Returns false (and
 // the capture then fails as a whole) if any step is refused.
-static bool cond_open(cudaStream_t st, cudaStream_t aux, cudaGraphConditionalHandle h) {
+static bool cond_open(cudaStream_t st, cudaStream_t aux, cudaGraphConditionalHandle h, cudaGraph_t* body_out = nullptr) {
   cudaStreamCaptureStatus cs;
   cudaGraph_t g = nullptr;
   const cudaGraphNode_t* deps = nullptr;
@@ -1966,10 +1969,13 @@ static bool cond_open(cudaStream_t st, cudaStream_t aux, cudaGraphConditionalHan
   p.conditional.type = cudaGraphCondTypeIf;
   p.conditional.size = 1;
   cudaGraphNode_t node;
-  return cudaGraphAddNode(&node, g, dv.data(), nullptr, nd, &p) == cudaSuccess &&
-         cudaStreamUpdateCaptureDependencies(st, &node, nullptr, 1, cudaStreamSetCaptureDependencies) == cudaSuccess &&
-         cudaStreamBeginCaptureToGraph(aux, p.conditional.phGraph_out[0], nullptr, nullptr, 0,
-                                       cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+  const bool ok = cudaGraphAddNode(&node, g, dv.data(), nullptr, nd, &p) == cudaSuccess &&
+                  cudaStreamUpdateCaptureDependencies(st, &node, nullptr, 1, cudaStreamSetCaptureDependencies) ==
+                      cudaSuccess &&
+                  cudaStreamBeginCaptureToGraph(aux, p.conditional.phGraph_out[0], nullptr, nullptr, 0,
+                                                cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+  if (ok && body_out) *body_out = p.conditional.phGraph_out[0];
+  return ok;
 }
 static bool cond_close(cudaStream_t aux) {
   cudaGraph_t body = nullptr;
@@ -2040,36 +2046,44 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   // and the multi-CTA marking; a short one finished by one CTA.
   // (a body is launched only once its capture has started: a kernel launched
   // on the auxiliary stream outside a capture would run)
-  auto select = [&](cudaStream_t q, int single, int fallback, bool cond) {
+  auto select = [&](cudaStream_t q, int single, int fallback, bool cond, cudaGraphConditionalHandle hl,
+                    cudaStream_t body) {
     PS_LAUNCH(k_wide_pass<<<cgrid, 256, 0, q>>>(s, single, fallback));
     PS_LAUNCH(k_wide_resolve<<<single ? 1 : s.G, 32, 0, q>>>(s, single));
-    PS_LAUNCH(k_split<<<cgrid, 256, 0, q>>>(s, single, fallback, h_long, cond ? 1 : 0));
+    PS_LAUNCH(k_split<<<cgrid, 256, 0, q>>>(s, single, fallback, hl, cond ? 1 : 0));
     cudaStream_t b = q;
     if (cond) {
-      if (!cond_open(q, cap->aux, h_long)) { cond_ok = false; return; }
-      b = cap->aux;
+      if (!cond_open(q, body, hl)) { cond_ok = false; return; }
+      b = body;
     }
     for (int d = 0; d < 7; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, b>>>(s, single, fallback, 1));
     PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, b>>>(s, single, 1));
     PS_LAUNCH(k_mark_list<<<lgrid, 256, 0, b>>>(s, single));
-    if (cond && !cond_close(cap->aux)) { cond_ok = false; return; }
+    if (cond && !cond_close(body)) { cond_ok = false; return; }
     PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, q>>>(s, single, 0));
   };
   if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s, h_fb, conds ? 1 : 0));
-    select(st, 0, 0, conds);
+    select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
     cudaStream_t f = st;
+    cudaGraphConditionalHandle h_fb_long = 0;
     if (conds) {
-      if (!cond_open(st, cap->aux, h_fb)) return PS_ERR_CUDA;
+      // the fallback's own long-list body nests inside the fallback's body;
+      // its handle belongs to that body graph
+      cudaGraph_t fb_body = nullptr;
+      if (!cond_open(st, cap->aux, h_fb, &fb_body) ||
+          cudaGraphConditionalHandleCreate(&h_fb_long, fb_body, 0, cudaGraphCondAssignDefault) != cudaSuccess)
+        return PS_ERR_CUDA;
       f = cap->aux;
     }
     PS_LAUNCH(k_sel_single<<<1, 32, 0, f>>>(s, 1));
-    select(f, 1, 1, false);  // no nested body: the fallback is itself one
+    select(f, 1, 1, conds, h_fb_long, conds ? cap->aux2 : f);
+    if (!cond_ok) return PS_ERR_CUDA;
     if (conds && !cond_close(cap->aux)) return PS_ERR_CUDA;
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
-    select(st, 1, 0, conds);
+    select(st, 1, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
   } else {
     PS_LAUNCH(launch_s3_evict(s, st));
