@@ -865,7 +865,7 @@ __global__ void __launch_bounds__(kThreads) k_touch2(DevState s) {
 // the no-segmentation ablation) and the stamp for lru.  Per (segment, class):
 // the candidates and their stamp range, so the radix select can start inside
 // the class that holds its rank and skip the bytes the class's stamps share.
-__global__ void __launch_bounds__(256) k_cand(DevState s) {
+__global__ void __launch_bounds__(1024) k_cand(DevState s) {
   s = with_args(s);
   extern __shared__ uint32_t cand_smem[];  // 5 arrays of nseg * kClasses
   Ctl* c = s.ctl;
@@ -885,37 +885,52 @@ __global__ void __launch_bounds__(256) k_cand(DevState s) {
     s_hmax[r] = s_lmax[r] = 0;
   }
   __syncthreads();
-  // warp-uniform trip count; lanes of one (segment, class) combine their
-  // ranges and counts with warp reductions, one lane updates shared memory
-  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t b = b0 + threadIdx.x;
-    uint64_t key = ~0ull, st = 0;
-    uint32_t row = ~0u;
-    if (b < s.N) {
-      // every load issued at once (no dependent round trips)
-      const uint8_t fl = s.blk_flags[b], kl = s.blk_klass[b];
-      const uint32_t pin = s.blk_pin[b];
-      const uint16_t grp = s.blk_group[b];
-      st = s.blk_stamp[b];
-      if ((fl & 1) && pin != step32) {
-        key = seg ? (st | (uint64_t)kl << 62) : st;
-        row = (ps ? (uint32_t)grp : 0u) * kClasses + (seg ? kl : 0u);
+  // kU blocks a thread per iteration, their loads issued together; the trip
+  // count is warp-uniform.  Lanes of one (segment, class) combine their
+  // ranges and counts with warp reductions; one lane updates shared memory.
+  constexpr int kU = 4;
+  const int64_t span = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += span * kU) {
+    uint8_t fl[kU], kl[kU];
+    uint32_t pin[kU];
+    uint16_t grp[kU];
+    uint64_t st[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t b = b0 + u * span + threadIdx.x;
+      fl[u] = 0;
+      if (b < s.N) {
+        fl[u] = s.blk_flags[b];
+        kl[u] = s.blk_klass[b];
+        pin[u] = s.blk_pin[b];
+        grp[u] = s.blk_group[b];
+        st[u] = s.blk_stamp[b];
       }
     }
-    const unsigned peers = __match_any_sync(kFull, row);
-    if (row != ~0u) {
-      const uint32_t hi = (uint32_t)(st >> 32), lo = (uint32_t)st;
-      const uint32_t hmin = __reduce_min_sync(peers, hi), hmax = __reduce_max_sync(peers, hi);
-      const uint32_t lmin = __reduce_min_sync(peers, lo), lmax = __reduce_max_sync(peers, lo);
-      if (lane_id() == __ffs(peers) - 1) {
-        atomicAdd(&s_cnt[row], (unsigned)__popc(peers));
-        atomicMin(&s_hmin[row], hmin);
-        atomicMax(&s_hmax[row], hmax);
-        atomicMin(&s_lmin[row], lmin);
-        atomicMax(&s_lmax[row], lmax);
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t b = b0 + u * span + threadIdx.x;
+      uint64_t key = ~0ull;
+      uint32_t row = ~0u;
+      if ((fl[u] & 1) && pin[u] != step32) {
+        key = seg ? (st[u] | (uint64_t)kl[u] << 62) : st[u];
+        row = (ps ? (uint32_t)grp[u] : 0u) * kClasses + (seg ? kl[u] : 0u);
       }
+      const unsigned peers = __match_any_sync(kFull, row);
+      if (row != ~0u) {
+        const uint32_t hi = (uint32_t)(st[u] >> 32), lo = (uint32_t)st[u];
+        const uint32_t hmin = __reduce_min_sync(peers, hi), hmax = __reduce_max_sync(peers, hi);
+        const uint32_t lmin = __reduce_min_sync(peers, lo), lmax = __reduce_max_sync(peers, lo);
+        if (lane_id() == __ffs(peers) - 1) {
+          atomicAdd(&s_cnt[row], (unsigned)__popc(peers));
+          atomicMin(&s_hmin[row], hmin);
+          atomicMax(&s_hmax[row], hmax);
+          atomicMin(&s_lmin[row], lmin);
+          atomicMax(&s_lmax[row], lmax);
+        }
+      }
+      if (b < s.N) s.csk[b] = key;
     }
-    if (b < s.N) s.csk[b] = key;
   }
   __syncthreads();
   for (int r = threadIdx.x; r < nrow; r += blockDim.x) {
@@ -1240,6 +1255,7 @@ __device__ __forceinline__ void wide_digit(int nrows, uint64_t mask, int* dshift
 __global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int fallback) {
   s = with_args(s);
   __shared__ int16_t row_of[PS_MAX_GROUPS];
+  __shared__ uint64_t s_pre[PS_MAX_GROUPS], s_msk[PS_MAX_GROUPS];  // the segments' prefix and mask
   __shared__ int s_nrows;
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
@@ -1253,6 +1269,8 @@ __global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int f
       if (g < nseg) {
         const SelSeg ss = s.sel[g];
         counts = ss.active && next_shift(ss.mask) >= 0;
+        s_pre[g] = ss.prefix;
+        s_msk[g] = ss.mask;
       }
       int tot;
       const int ex = block_excl_scan((int)counts, &tot);
@@ -1279,11 +1297,11 @@ __global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int f
       if (key != ~0ull && !(fallback && ((s.bm_victim[e >> 5] >> (e & 31)) & 1))) {
         const int row = row_of[seg];
         if (row >= 0) {
-          const SelSeg ss = s.sel[seg];
-          if ((key & ss.mask) == ss.prefix) {
+          const uint64_t msk = s_msk[seg];
+          if ((key & msk) == s_pre[seg]) {
             int dsh;
             uint32_t nb;
-            wide_digit(nrows, ss.mask, &dsh, &nb);
+            wide_digit(nrows, msk, &dsh, &nb);
             act = true;
             act16 = nb == (uint32_t)kWideBins;
             idx = (uint32_t)row * stride + (uint32_t)((key >> dsh) & (nb - 1));
@@ -1494,6 +1512,17 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
         w[k] = make_uint4(0, 0, 0, 0);
     }
   }
+  // the segments' state, once per CTA
+  __shared__ uint64_t s_pre[PS_MAX_GROUPS], s_msk[PS_MAX_GROUPS];
+  __shared__ uint8_t s_act[PS_MAX_GROUPS];
+  const int nseg = single ? 1 : s.G;
+  for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
+    const SelSeg ss = s.sel[g];
+    s_pre[g] = ss.prefix;
+    s_msk[g] = ss.mask;
+    s_act[g] = ss.active ? 1 : 0;
+  }
+  __syncthreads();
   int marked = 0;
   for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += (int64_t)gridDim.x * blockDim.x) {
     const int64_t b = b0 + threadIdx.x;
@@ -1505,11 +1534,10 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
       const int grp = single ? 0 : s.blk_group[b];
       if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
         seg = grp;
-        const SelSeg ss = s.sel[seg];
-        if (ss.active) {
-          const uint64_t k = key & ss.mask;
-          v = k < ss.prefix;
-          to_list = k == ss.prefix;
+        if (s_act[seg]) {
+          const uint64_t k = key & s_msk[seg];
+          v = k < s_pre[seg];
+          to_list = k == s_pre[seg];
         }
       }
     }
@@ -2023,7 +2051,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
   mark(6);
   const int cand_smem = (s.policy == PS_PREFIXSHIELD ? s.G : 1) * kClasses * 5 * 4;
-  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<cgrid, 256, cand_smem, st>>>(s));
+  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, st>>>(s));
   // Under capture, phases that many steps skip become conditional bodies:
   // the long-list passes of a select, and the global fallback of Alg. 2.
   cudaGraphConditionalHandle h_fb = 0, h_long = 0;
