@@ -446,23 +446,56 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
     const int nb = tmin(32, m1 - c0);
     const int32_t* cb = buf + shift_tok + (c0 - m0) * BS;
     uint64_t d1 = 0, d2 = 0;
+    if constexpr (PPB <= 8) {
+      // Round r: the PPB lanes of group q = lane / PPB each take one token
+      // pair of block q + G32 r.  Every lane keeps its PPB partial products;
+      // a reduce-scatter over the group's lanes (recursive halving) leaves
+      // lane k of the group with round k's full sums, and one shuffle moves
+      // block b's sums to lane b.
+      uint64_t a1[PPB], a2[PPB];
 #pragma unroll
-    for (int r = 0; r < PPB; ++r) {
-      const int b = lane / PPB + G32 * r;
-      uint64_t p1 = 0, p2 = 0;
-      if (b < nb) {
-        const int32_t tx = cb[b * BS + 2 * k], ty = cb[b * BS + 2 * k + 1];
-        p1 = (uint64_t)((uint32_t)tx + K0) * (uint64_t)((uint32_t)ty + K1);
-        p2 = (uint64_t)((uint32_t)tx + K2) * (uint64_t)((uint32_t)ty + K3);
+      for (int r = 0; r < PPB; ++r) {
+        const int b = lane / PPB + G32 * r;
+        a1[r] = a2[r] = 0;
+        if (b < nb) {
+          const int32_t tx = cb[b * BS + 2 * k], ty = cb[b * BS + 2 * k + 1];
+          a1[r] = (uint64_t)((uint32_t)tx + K0) * (uint64_t)((uint32_t)ty + K1);
+          a2[r] = (uint64_t)((uint32_t)tx + K2) * (uint64_t)((uint32_t)ty + K3);
+        }
       }
 #pragma unroll
-      for (int o = 1; o < PPB; o <<= 1) {
-        p1 += __shfl_xor_sync(kFull, p1, o);
-        p2 += __shfl_xor_sync(kFull, p2, o);
+      for (int d = PPB / 2; d >= 1; d >>= 1) {
+        const bool up = (k & d) != 0;
+#pragma unroll
+        for (int j = 0; j < d; ++j) {
+          const uint64_t s1 = up ? a1[j] : a1[j + d], s2 = up ? a2[j] : a2[j + d];
+          const uint64_t k1 = up ? a1[j + d] : a1[j], k2 = up ? a2[j + d] : a2[j];
+          a1[j] = k1 + __shfl_xor_sync(kFull, s1, d);
+          a2[j] = k2 + __shfl_xor_sync(kFull, s2, d);
+        }
       }
-      const int src = (lane % G32) * PPB;
-      const uint64_t q1 = __shfl_sync(kFull, p1, src), q2 = __shfl_sync(kFull, p2, src);
-      if (lane / G32 == r) { d1 = q1; d2 = q2; }
+      const int src = (lane % G32) * PPB + lane / G32;  // holder of block `lane`
+      d1 = __shfl_sync(kFull, a1[0], src);
+      d2 = __shfl_sync(kFull, a2[0], src);
+    } else {
+#pragma unroll
+      for (int r = 0; r < PPB; ++r) {
+        const int b = lane / PPB + G32 * r;
+        uint64_t p1 = 0, p2 = 0;
+        if (b < nb) {
+          const int32_t tx = cb[b * BS + 2 * k], ty = cb[b * BS + 2 * k + 1];
+          p1 = (uint64_t)((uint32_t)tx + K0) * (uint64_t)((uint32_t)ty + K1);
+          p2 = (uint64_t)((uint32_t)tx + K2) * (uint64_t)((uint32_t)ty + K3);
+        }
+#pragma unroll
+        for (int o = 1; o < PPB; o <<= 1) {
+          p1 += __shfl_xor_sync(kFull, p1, o);
+          p2 += __shfl_xor_sync(kFull, p2, o);
+        }
+        const int src = (lane % G32) * PPB;
+        const uint64_t q1 = __shfl_sync(kFull, p1, src), q2 = __shfl_sync(kFull, p2, src);
+        if (lane / G32 == r) { d1 = q1; d2 = q2; }
+      }
     }
     // D_m, then the inclusive scan of the affine maps x -> Kc x + D
     uint64_t bb = lane < nb ? add61(red61(d1), mul61(Kd, red61(d2))) : 0;
