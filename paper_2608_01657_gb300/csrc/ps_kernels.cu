@@ -98,6 +98,15 @@ __device__ __forceinline__ void agg_inc(uint32_t* bins, uint32_t idx, bool activ
   const unsigned peers = __match_any_sync(act, idx);
   if (lane_id() == __ffs(peers) - 1) atomicAdd(bins + idx, (uint32_t)__popc(peers));
 }
+// atomicMin of v into base[i], lanes of the warp with equal i combined first
+// (every lane of the warp must call it).
+__device__ __forceinline__ void agg_min_u32(uint32_t* base, uint32_t i, uint32_t v, bool active) {
+  const unsigned act = __ballot_sync(kFull, active);
+  if (!active) return;
+  const unsigned peers = __match_any_sync(act, i);
+  const uint32_t m = __reduce_min_sync(peers, v);
+  if (lane_id() == __ffs(peers) - 1) atomicMin(base + i, m);
+}
 __device__ __forceinline__ uint64_t ldcg_u64(const uint64_t* p) { return __ldcg(reinterpret_cast<const unsigned long long*>(p)); }
 __device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
 
@@ -525,18 +534,23 @@ __global__ void __launch_bounds__(kThreads) k_keys_lookup(DevState s) {
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   PosRef r;
-  if (!pos_ref(s, pos, &r)) return;
-  // chain value entering this position's segment: fold the earlier segments
-  const int64_t sb = s.rq_sbase[r.i];
-  const int js = r.m / kSegBlocks;
-  uint64_t cin = red61(chain_seed(s.hash_seed, s.in_group[r.i]));
-  for (int j = 0; j < js; ++j) cin = add61(mul61(s.kc_pow[kSegBlocks], cin), s.seg_tot[sb + j]);
-  const uint64_t C = add61(mul61(s.kc_pow[r.m % kSegBlocks + 1], cin), s.pos_key[pos]);
-  const uint64_t key = fix_reserved(mix64(C ^ ((uint64_t)(r.m + 1) * 0xD1B54A32D192ED03ull)));
-  s.pos_key[pos] = key;
-  const uint32_t blk = table_find(s, key, (uint32_t)s.in_group[r.i]);
-  s.pos_blk[pos] = blk;
-  if (blk == kNone) atomicMin(reinterpret_cast<uint32_t*>(s.rq_h) + r.i, (uint32_t)r.m);
+  const bool valid = pos_ref(s, pos, &r);
+  bool miss = false;
+  if (valid) {
+    // chain value entering this position's segment: fold the earlier segments
+    const int64_t sb = s.rq_sbase[r.i];
+    const int js = r.m / kSegBlocks;
+    uint64_t cin = red61(chain_seed(s.hash_seed, s.in_group[r.i]));
+    for (int j = 0; j < js; ++j) cin = add61(mul61(s.kc_pow[kSegBlocks], cin), s.seg_tot[sb + j]);
+    const uint64_t C = add61(mul61(s.kc_pow[r.m % kSegBlocks + 1], cin), s.pos_key[pos]);
+    const uint64_t key = fix_reserved(mix64(C ^ ((uint64_t)(r.m + 1) * 0xD1B54A32D192ED03ull)));
+    s.pos_key[pos] = key;
+    const uint32_t blk = table_find(s, key, (uint32_t)s.in_group[r.i]);
+    s.pos_blk[pos] = blk;
+    miss = blk == kNone;
+  }
+  // h_i = the first miss: one atomic per request per warp
+  agg_min_u32(reinterpret_cast<uint32_t*>(s.rq_h), valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, miss);
 }
 
 // Stage 2 (cont.): blocks of the cached prefix are pinned for the step;
@@ -613,10 +627,11 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
   bool inv = false;
   uint32_t ginv = 0;
   PosRef r;
-  if (pos_ref(s, pos, &r)) {
+  bool own = false;
+  const bool valid = pos_ref(s, pos, &r);
+  if (valid) {
     const int h = s.rq_h[r.i];
-    if (r.m >= h && ldcg_u32(&s.claims[s.pos_claim[pos]].minreq) == r.i)
-      atomicMin(reinterpret_cast<uint32_t*>(s.rq_s) + r.i, (uint32_t)r.m);
+    own = r.m >= h && ldcg_u32(&s.claims[s.pos_claim[pos]].minreq) == r.i;
     if (r.m > h) {
       const uint32_t b = s.pos_blk[pos];
       if (b != kNone && ldcg_u32(s.blk_pin + b) != step32 && atomicExch(s.blk_inval + b, step32) != step32) {
@@ -627,6 +642,8 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
       }
     }
   }
+  // s_i = the first own claim: one atomic per request per warp
+  agg_min_u32(reinterpret_cast<uint32_t*>(s.rq_s), valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, own);
   agg_stat(s, ginv, PS_STAT_INVALIDATED_BLOCKS, 1, inv);
   agg_stat(s, ginv, PS_STAT_RESIDENT_BLOCKS, -1, inv);
   const int ni = __popc(__ballot_sync(kFull, inv));
@@ -686,11 +703,14 @@ __global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
   if (c->status != PS_OK) return;
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   PosRef r;
-  if (!pos_ref(s, pos, &r)) return;
-  if (r.m < s.rq_h[r.i] || r.m >= s.rq_s[r.i]) return;
-  const uint32_t j = s.claims[s.pos_claim[pos]].minreq;
-  const int64_t rank = (int64_t)s.rq_cbase[j] + (r.m - s.rq_s[j]);
-  if (rank >= c->avail) atomicMin(s.rq_fu + r.i, (uint32_t)r.m);
+  bool past = false;
+  const bool valid = pos_ref(s, pos, &r);
+  if (valid && r.m >= s.rq_h[r.i] && r.m < s.rq_s[r.i]) {
+    const uint32_t j = s.claims[s.pos_claim[pos]].minreq;
+    const int64_t rank = (int64_t)s.rq_cbase[j] + (r.m - s.rq_s[j]);
+    past = rank >= c->avail;
+  }
+  agg_min_u32(s.rq_fu, valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, past);
 }
 
 // hit_i = h_i + e_i per request; records the first admitting request of each
