@@ -181,6 +181,9 @@ __device__ uint32_t table_find(const DevState& s, uint64_t key, uint32_t g) {
   return kNone;
 }
 
+// Returns the slot, with kDisplaced set when it lies past the home bucket
+// (then a delete must repair the overflow counters on the way).
+constexpr uint32_t kDisplaced = 0x80000000u;
 __device__ uint32_t table_insert(const DevState& s, uint64_t key, uint32_t g, uint32_t blk) {
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
   uint32_t b = table_home(key, g, s.tb_nbuckets_log2);
@@ -190,7 +193,7 @@ __device__ uint32_t table_insert(const DevState& s, uint64_t key, uint32_t g, ui
       if (ldcg_u32(&e->blk) == kNone && atomicCAS(&e->blk, kNone, blk) == kNone) {
         e->key = key;
         e->grp = g;
-        return b * kTableWays + w;
+        return (b * kTableWays + w) | (it ? kDisplaced : 0u);
       }
     }
     atomicAdd(s.table_ovf + b, 1u);
@@ -201,13 +204,15 @@ __device__ uint32_t table_insert(const DevState& s, uint64_t key, uint32_t g, ui
 
 __device__ void table_delete(const DevState& s, uint32_t blk) {
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
-  const uint32_t slot = s.blk_slot[blk];
-  const uint32_t bucket = slot / kTableWays;
-  uint32_t x = table_home(s.blk_key[blk], s.blk_group[blk], s.tb_nbuckets_log2);
+  const uint32_t tagged = s.blk_slot[blk];
+  const uint32_t slot = tagged & ~kDisplaced;
   TableEntry* e = s.table + slot;
   e->key = 0;
   e->grp = 0;
   e->blk = kNone;
+  if (!(tagged & kDisplaced)) return;  // in its home bucket: no counter passed
+  const uint32_t bucket = slot / kTableWays;
+  uint32_t x = table_home(s.blk_key[blk], s.blk_group[blk], s.tb_nbuckets_log2);
   for (uint32_t it = 0; x != bucket && it <= mask; ++it, x = (x + 1) & mask) atomicSub(s.table_ovf + x, 1u);
 }
 
@@ -234,12 +239,14 @@ __device__ uint32_t claim_insert(const DevState& s, uint64_t key, uint32_t req) 
 // ---- block state changes -----------------------------------------------------
 // Remove a resident block from the pool (eviction or invalidation); returns
 // its group.  Callers account the per-group statistics, warp-aggregated.
-__device__ uint32_t drop_block(const DevState& s, uint32_t b) {
+// clear_res: also clear the resident bit (evictions leave it: the id is
+// allocated again in the same step, and k_bm_write sets the allocated bits).
+__device__ uint32_t drop_block(const DevState& s, uint32_t b, bool clear_res = true) {
   table_delete(s, b);
   const uint32_t g = s.blk_group[b];
   const uint8_t fl = s.blk_flags[b];
   s.blk_flags[b] = 0;
-  atomicAnd(s.res_bits + (b >> 5), ~(1u << (b & 31)));
+  if (clear_res) atomicAnd(s.res_bits + (b >> 5), ~(1u << (b & 31)));
   if (s.policy == PS_S3FIFO) atomic_add_i64((fl & 2) ? &s.ctl->s3_nM : &s.ctl->s3_nS, -1);
   return g;
 }
@@ -1172,9 +1179,9 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   // tau = max{t in [eps+1, pmax] : items_gt(t - 1) summed >= m}.  Only the
   // groups that can hold an item above eps count (d > 0, q > 0, P > eps);
   // each round tests T thresholds spread over the interval, L lanes (a power
-  // of two) splitting the groups of one so that no thread evaluates more than
-  // 32 (a thread's evaluations are independent and overlap; fewer, wider
-  // rounds beat more lanes with shuffles).
+  // of two covering them, at most 32) splitting the groups of one: each
+  // evaluation is a chain of dependent 64-bit steps, so one per thread and
+  // more rounds beat several per thread and fewer rounds.
   __shared__ int16_t s_gid[PS_MAX_GROUPS];
   __shared__ int s_ng;
   __shared__ int s_J[3];
@@ -1194,7 +1201,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   }
   const int ng = s_ng;
   int L = 1, logT = 10;  // blockDim.x == 1024 == T * L
-  while (L * 32 < ng && L < 32) { L <<= 1; --logT; }
+  while (L < ng && L < 32) { L <<= 1; --logT; }
   const int T = 1 << logT;
   int64_t lo = eps + 1, hi = s_pmax;
   const int jt = threadIdx.x / L, gl = threadIdx.x % L;
@@ -1204,7 +1211,6 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
     auto thr = [&](int jj) -> int64_t { return jj == T - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * jj); };
     const int64_t t = thr(jt);
     int64_t cnt = 0;
-#pragma unroll 4
     for (int k = gl; k < ng; k += L) cnt += items_gt(s_gid[k], t - 1);
     for (int o = L / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
     // J = the largest threshold still holding m items (counts fall as the
@@ -1846,7 +1852,10 @@ __global__ void __launch_bounds__(kBmChunk) k_bm_count(DevState s) {
   const int nchunks = gridDim.x;
   for (int k = 0; k < 3; ++k) {
     uint32_t bits = w < s.nwords ? bms[k][w] : 0u;
-    if (k == 0 && w < s.nwords) bits |= s.bm_victim[w];
+    if (k == 0 && w < s.nwords) {
+      bits |= s.bm_victim[w];
+      s.res_bits[w] |= bits;  // every allocated id is resident after the step
+    }
     const int v = __popc(bits);
     const int t = block_sum(v);
     if (threadIdx.x == 0) s.bm_chunk_cnt[k * nchunks + blockIdx.x] = t;
@@ -1864,7 +1873,10 @@ __global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
     for (int j = threadIdx.x; j < blockIdx.x; j += blockDim.x) base += s.bm_chunk_cnt[k * nchunks + j];
     base = block_sum(base);
     uint32_t bits = w < s.nwords ? bms[k][w] : 0u;
-    if (k == 0 && w < s.nwords) bits |= s.bm_victim[w];
+    if (k == 0 && w < s.nwords) {
+      bits |= s.bm_victim[w];
+      s.res_bits[w] |= bits;  // every allocated id is resident after the step
+    }
     int tot;
     const int ex = block_excl_scan(__popc(bits), &tot);
     int o = base + ex;
@@ -1892,7 +1904,7 @@ __global__ void __launch_bounds__(kThreads) k_evict(DevState s) {
   const int64_t nv = c->n_evicted;
   const bool act = v < nv && v < s.max_blocks;
   uint32_t g = 0;
-  if (act) g = drop_block(s, (uint32_t)s.out.evicted_ids[v]);
+  if (act) g = drop_block(s, (uint32_t)s.out.evicted_ids[v], false);
   agg_stat(s, g, PS_STAT_EVICTED_BLOCKS, 1, act);
   agg_stat(s, g, PS_STAT_RESIDENT_BLOCKS, -1, act);
   const int k = __popc(__ballot_sync(kFull, act));
@@ -1945,8 +1957,7 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
         s.blk_freq[b] = e.tcnt;
         s.blk_flags[b] = 1;
         s.blk_slot[b] = table_insert(s, key, g, b);
-        atomicOr(s.res_bits + (b >> 5), 1u << (b & 31));
-        placed = true;
+        placed = true;  // its resident bit was set with the allocated set
       }
     }
     if (slot != kNone) {
