@@ -25,7 +25,7 @@ STAT_NAMES = (
     "invalidated_blocks", "promotions", "gated_reuses", "resident_blocks",
     "debt_raw", "debt_norm",
 )
-POLICIES = {"lru": 0, "s3fifo": 1, "prefixshield": 2}
+POLICIES = {"lru": 0, "s3fifo": 1, "prefixshield": 2, "staticquota": 3}
 OK, ERR_INVALID_ARG, ERR_CAPACITY, ERR_CLOCK = 0, -1, -2, -3
 FLAG_NO_SEGMENTATION, FLAG_NO_DEBT_GATE = 1, 2
 

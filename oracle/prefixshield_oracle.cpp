@@ -19,7 +19,9 @@
 //        OnTouch (debt-gated promotion)     Alg. 1, Eq. 4
 //        OnCacheFullBlocks (metering)       Alg. 1, Eq. 2
 //   S5 reclamation                         Alg. 2, Eq. 5-9 (prefixshield);
-//                                          global recency (lru); S3-FIFO
+//                                          global recency (lru); S3-FIFO;
+//                                          per-group recency inside equal
+//                                          partitions (staticquota)
 //   S6 eviction, id assignment, insertion
 //
 // Parity status of each function is listed in the design doc; every function below
@@ -44,6 +46,7 @@ constexpr int32_t ERR_CLOCK = -3;
 constexpr int32_t POLICY_LRU = 0;
 constexpr int32_t POLICY_S3FIFO = 1;
 constexpr int32_t POLICY_PREFIXSHIELD = 2;
+constexpr int32_t POLICY_STATICQUOTA = 3;  // equal per-group partition, no borrowing (Sec. V-A)
 
 // Retention classes, Sec. III-A: Probationary < Normal < Reuse (Eq. 9).
 constexpr int32_t PROBATIONARY = 0;
@@ -408,9 +411,22 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
   }
 
   // ---- S3: grant new blocks against the pool ------------------------------
-  int64_t avail = N - (int64_t)pinned.size();  // free + unpinned resident
+  // Claims are granted in (request, position) rank order while the pool
+  // holds them: the whole pool (free + unpinned resident) for the shared
+  // policies; for StaticQuota each group's own partition of Q = floor(N/G)
+  // blocks minus its pinned blocks, ranked among its own requests.
+  const int64_t quota = N / G;
   std::vector<int64_t> base(R), a(R), e(R), hit(R);
-  {
+  if (policy == POLICY_STATICQUOTA) {
+    std::vector<int64_t> pinned_g(G, 0), run_g(G, 0);
+    for (int32_t id : pinned) pinned_g[blocks[id].group] += 1;
+    for (int32_t i = 0; i < R; ++i) {
+      base[i] = run_g[g[i]];
+      run_g[g[i]] += cl[i];
+      a[i] = std::min<int64_t>(cl[i], std::max<int64_t>(0, quota - pinned_g[g[i]] - base[i]));
+    }
+  } else {
+    const int64_t avail = N - (int64_t)pinned.size();  // free + unpinned resident
     int64_t run = 0;
     for (int32_t i = 0; i < R; ++i) {
       base[i] = run;
@@ -418,16 +434,18 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
       a[i] = std::min<int64_t>(cl[i], std::max<int64_t>(0, avail - base[i]));
     }
   }
-  auto granted_rank = [&](int32_t j, int64_t m) { return base[j] + (m - s[j]); };
+  // Request j's claims are ranked consecutively, so its key at position m is
+  // granted iff it is among the first a_j of them.
+  auto granted = [&](int32_t j, int64_t m) { return m - s[j] < a[j]; };
   for (int32_t i = 0; i < R; ++i) {
     e[i] = 0;
     for (int64_t m = h[i]; m < s[i]; ++m) {
       int32_t j = owner[{g[i], keys[i][m]}];
-      if (granted_rank(j, m) < avail) ++e[i]; else break;
+      if (granted(j, m)) ++e[i]; else break;
     }
-    // When e_i < s_i - h_i some earlier rank r >= avail is not granted, and
-    // base_i > r, so a_i is already 0: no block is materialized past an
-    // ungranted one.
+    // When e_i < s_i - h_i some earlier claim is not granted, so neither is
+    // any claim ranked after it in the same pool, and a_i is already 0: no
+    // block is materialized past an ungranted one.
     hit[i] = h[i] + e[i];
   }
 
@@ -509,14 +527,38 @@ int32_t Oracle::step_once(int64_t now, int32_t R, const int32_t* group, const in
   // ---- S5: reclamation (Alg. 2 for prefixshield) -------------------------
   int64_t need = 0;
   for (int32_t i = 0; i < R; ++i) need += a[i];
+  // StaticQuota: group g's new blocks first fill its partition's free part
+  // (Q - resident_g); only the rest, m_g, evicts its own blocks.
+  std::vector<int64_t> m_g(G, 0);
+  int64_t quota_victims = 0;
+  if (policy == POLICY_STATICQUOTA) {
+    std::vector<int64_t> need_g(G, 0), res_g(G, 0);
+    for (int32_t i = 0; i < R; ++i) need_g[g[i]] += a[i];
+    for (int64_t id = 0; id < N; ++id)
+      if (blocks[id].resident) res_g[blocks[id].group] += 1;
+    for (int gg = 0; gg < G; ++gg) {
+      m_g[gg] = std::max<int64_t>(0, need_g[gg] - (quota - res_g[gg]));
+      quota_victims += m_g[gg];
+    }
+  }
   // TakeTrueFree: the smallest free ids first (work conservation, Sec. III-E).
   std::vector<int32_t> take;
-  for (int64_t id = 0; id < N && (int64_t)take.size() < need; ++id)
+  const int64_t want_free = need - quota_victims;
+  for (int64_t id = 0; id < N && (int64_t)take.size() < want_free; ++id)
     if (!blocks[id].resident) take.push_back((int32_t)id);
   int64_t mvict = need - (int64_t)take.size();
   std::vector<int32_t> victims;
   if (mvict > 0) {
-    if (policy == POLICY_LRU) {
+    if (policy == POLICY_STATICQUOTA) {
+      // Each group reclaims its own m_g least recently released blocks.
+      std::vector<std::set<std::pair<uint64_t, int32_t>>> q(G);
+      for (int64_t id = 0; id < N; ++id)
+        if (blocks[id].resident && !pinned.count((int32_t)id)) q[blocks[id].group].insert({blocks[id].stamp, (int32_t)id});
+      for (int gg = 0; gg < G; ++gg) {
+        auto it = q[gg].begin();
+        for (int64_t v = 0; v < m_g[gg]; ++v, ++it) victims.push_back(it->second);
+      }
+    } else if (policy == POLICY_LRU) {
       // Global free-queue order: least recently released first.
       std::set<std::pair<uint64_t, int32_t>> q;
       for (int64_t id = 0; id < N; ++id)
@@ -679,7 +721,7 @@ extern "C" {
 
 int32_t orc_check_params(int64_t N, int32_t bs, int32_t G, int32_t policy, const orc_params_t* P) {
   if (!P || N <= 0 || N > (1ll << 30) || bs < 2 || bs > 256 || (bs & 1)) return ERR_INVALID_ARG;
-  if (G <= 0 || G > MAX_GROUPS || policy < 0 || policy > 2) return ERR_INVALID_ARG;
+  if (G <= 0 || G > MAX_GROUPS || policy < 0 || policy > 3) return ERR_INVALID_ARG;
   if (P->num_contracts < 1 || P->num_contracts > MAX_CONTRACTS) return ERR_INVALID_ARG;
   if (P->fp_shift < 0 || P->fp_shift > 30 || P->epsilon_fp < 0) return ERR_INVALID_ARG;
   int64_t rmin = P->rho_fp[0], rmax = P->rho_fp[0];
