@@ -48,7 +48,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--prefill", type=int, default=6, help="untimed steps that fill the empty pool")
     ap.add_argument("--impl", choices=("own", "reference"), default="own")
-    ap.add_argument("--policy", choices=("prefixshield", "lru"), default="prefixshield")
+    ap.add_argument("--policy", choices=("prefixshield", "lru", "staticquota"), default="prefixshield")
     ap.add_argument("--seed", type=int, default=1)
     ap.add_argument("--cpu-steps", type=int, default=3, help="timed oracle steps for cpu_baseline")
     ap.add_argument("--no-e2e", action="store_true")

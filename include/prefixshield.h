@@ -53,7 +53,9 @@ extern "C" {
 typedef enum {
   PS_LRU = 0,          /* global recency (vLLM free queue), Sec. V-A */
   PS_S3FIFO = 1,       /* S3-FIFO baseline, Sec. V-A */
-  PS_PREFIXSHIELD = 2  /* Alg. 1 + Alg. 2 */
+  PS_PREFIXSHIELD = 2, /* Alg. 1 + Alg. 2 */
+  PS_STATICQUOTA = 3   /* equal per-group partitions of floor(N / G) blocks, no
+                          borrowing; recency inside a partition (Sec. V-A) */
 } ps_policy_t;
 
 enum {

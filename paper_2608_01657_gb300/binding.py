@@ -25,7 +25,7 @@ STAT_NAMES = (
     "invalidated_blocks", "promotions", "gated_reuses", "resident_blocks",
     "debt_raw", "debt_norm",
 )
-POLICIES = {"lru": 0, "s3fifo": 1, "prefixshield": 2}
+POLICIES = {"lru": 0, "s3fifo": 1, "prefixshield": 2, "staticquota": 3}
 PS_OK, PS_ERR_INVALID_ARG, PS_ERR_CAPACITY, PS_ERR_CLOCK, PS_ERR_CUDA = 0, -1, -2, -3, -4
 PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE = 1, 2
 

@@ -90,7 +90,7 @@ int32_t upload_constants(ps_handle* h, cudaStream_t st) {
 int32_t check_params(int64_t N, int32_t bs, int32_t G, int32_t policy, const ps_params_t* P) {
   if (!P || N <= 0 || N > (1ll << 30)) return PS_ERR_INVALID_ARG;
   if (bs != 2 && bs != 4 && bs != 8 && bs != 16 && bs != 32 && bs != 64) return PS_ERR_INVALID_ARG;
-  if (G <= 0 || G > PS_MAX_GROUPS || policy < 0 || policy > 2) return PS_ERR_INVALID_ARG;
+  if (G <= 0 || G > PS_MAX_GROUPS || policy < 0 || policy > 3) return PS_ERR_INVALID_ARG;
   if (P->num_contracts < 1 || P->num_contracts > PS_MAX_CONTRACTS) return PS_ERR_INVALID_ARG;
   if (P->fp_shift < 0 || P->fp_shift > 30 || P->epsilon_fp < 0) return PS_ERR_INVALID_ARG;
   int64_t rmin = P->rho_fp[0], rmax = P->rho_fp[0];
@@ -228,6 +228,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.grp_P = cv.take<int64_t>(G);
   t.grp_delta = cv.take<int64_t>(G);
   t.grp_x = cv.take<int64_t>(G);
+  t.grp_pinned = cv.take<int64_t>(G);
   t.sel = cv.take<SelSeg>(G);
   t.cls = cv.take<ClsRange>(G * kClasses);
   t.hist_bins = cv.take<uint32_t>(G * kRadixBins);

@@ -214,7 +214,8 @@ struct DevState {
   int64_t* grp_qsize;      // candidates per group
   int64_t* grp_P;          // projected score P^(0)_g = normalized debt
   int64_t* grp_delta;      // Eq. 8 decrement
-  int64_t* grp_x;          // victims taken from the group in the debt phase
+  int64_t* grp_x;          // victims taken from the group in the debt phase (StaticQuota: its overflow)
+  int64_t* grp_pinned;     // blocks pinned this step, per group (StaticQuota grants)
   SelSeg* sel;             // [G] segments
   ClsRange* cls;           // [G * kClasses] candidates per (segment, class)
   uint32_t* hist_bins;     // [G][256] radix histogram

@@ -98,6 +98,16 @@ __device__ __forceinline__ void agg_inc(uint32_t* bins, uint32_t idx, bool activ
   const unsigned peers = __match_any_sync(act, idx);
   if (lane_id() == __ffs(peers) - 1) atomicAdd(bins + idx, (uint32_t)__popc(peers));
 }
+// base[i] += v, lanes of the warp with equal i combined first (every lane of
+// the warp must call it).
+__device__ __forceinline__ void agg_add_i64(int64_t* base, uint32_t i, int64_t v, bool active) {
+  const unsigned act = __ballot_sync(kFull, active);
+  if (!active) return;
+  const unsigned peers = __match_any_sync(act, i);
+  int64_t sum = 0;
+  for (unsigned m = peers; m; m &= m - 1) sum += __shfl_sync(peers, v, __ffs(m) - 1);
+  if (lane_id() == __ffs(peers) - 1) atomicAdd(reinterpret_cast<unsigned long long*>(base + i), (unsigned long long)sum);
+}
 // atomicMin of v into base[i], lanes of the warp with equal i combined first
 // (every lane of the warp must call it).
 __device__ __forceinline__ void agg_min_u32(uint32_t* base, uint32_t i, uint32_t v, bool active) {
@@ -353,6 +363,8 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
       c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
     }
   }
+  if (!probe && s.policy == PS_STATICQUOTA)
+    for (int g = threadIdx.x; g < s.G; g += blockDim.x) s.grp_pinned[g] = 0;
 }
 
 // ===========================================================================
@@ -573,12 +585,14 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
   const int64_t nb = c->nblocks;
   const uint32_t step32 = (uint32_t)c->step;
   bool newpin = false;
+  uint32_t pin_group = 0;
   if (t < nb) {
     PosRef r;
     pos_ref(s, t, &r);
     if (r.m < s.rq_h[r.i]) {
       const uint32_t b = s.pos_blk[t];
       newpin = atomicExch(s.blk_pin + b, step32) != step32;
+      pin_group = (uint32_t)s.in_group[r.i];  // the owner: hits are namespaced by group
       if (newpin && s.policy == PS_S3FIFO) atomic_add_i64(&c->s3_pinned[(s.blk_flags[b] >> 1) & 1], 1);
       s.pos_claim[t] = kNone;
     } else {
@@ -616,6 +630,7 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
   }
   const int np = __popc(__ballot_sync(kFull, newpin));
   if (lane_id() == 0 && np) atomic_add_i64(&c->pinned, np);
+  if (s.policy == PS_STATICQUOTA) agg_add_i64(s.grp_pinned, pin_group, 1, newpin);
 }
 
 // Stage 2 (cont.): the first own claim s_i of each request, and orphans.  A
@@ -669,41 +684,83 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int R = s.R;
+  const bool quota = s.policy == PS_STATICQUOTA;  // a_i already granted per group
   const int64_t avail = s.N - c->pinned;
-  int32_t carry = 0;
+  int64_t carry_c = 0, carry_a = 0;
   for (int t0 = 0; t0 < R; t0 += blockDim.x) {
     const int i = t0 + threadIdx.x;
     int32_t cl = 0;
     if (i < R) cl = s.rq_n[i] - s.rq_s[i];
-    int32_t tot;
-    const int32_t ex = block_excl_scan(cl, &tot);
+    int32_t tot_c;
+    const int32_t ex_c = block_excl_scan(cl, &tot_c);
+    int32_t a = 0;
+    if (i < R) a = quota ? s.rq_a[i] : (int32_t)tmin<int64_t>(cl, tmax<int64_t>(0, avail - (carry_c + ex_c)));
+    int32_t tot_a;
+    const int32_t ex_a = block_excl_scan(a, &tot_a);
     if (i < R) {
-      const int64_t cb = carry + ex;
-      s.rq_cbase[i] = (int32_t)cb;
-      const int64_t a = tmin<int64_t>(cl, tmax<int64_t>(0, avail - cb));
-      s.rq_a[i] = (int32_t)a;
-      s.out.admitted_blocks[i] = (int32_t)a;
+      // granted keys are paired with the allocated ids in (request, position)
+      // order: request i's first granted key is the (carry_a + ex_a)-th
+      s.rq_cbase[i] = (int32_t)(carry_a + ex_a);
+      s.rq_a[i] = a;
+      s.out.admitted_blocks[i] = a;
+      s.out.admitted_offsets[i] = (int32_t)(carry_a + ex_a);
     }
-    carry += tot;
+    carry_c += tot_c;
+    carry_a += tot_a;
   }
-  const int64_t need = tmin<int64_t>(avail, carry);
-  for (int i = threadIdx.x; i < R; i += blockDim.x)
-    s.out.admitted_offsets[i] = (int32_t)tmin<int64_t>(s.rq_cbase[i], need);
+  int64_t qv = 0;  // StaticQuota: the groups' overflows are the victims
+  if (quota)
+    for (int g = threadIdx.x; g < s.G; g += blockDim.x) qv += s.grp_x[g];
+  qv = block_sum(qv);
   if (threadIdx.x == 0) {
+    const int64_t need = carry_a;
     s.out.admitted_offsets[R] = (int32_t)need;
     const int64_t nfree = s.N - c->n_resident;
     c->avail = avail;
-    c->total_claims = carry;
+    c->total_claims = carry_c;
     c->need = need;
     c->nfree = nfree;
-    c->ftake = tmin(need, nfree);
-    c->mvict = need - tmin(need, nfree);
+    c->ftake = quota ? need - qv : tmin(need, nfree);
+    c->mvict = need - c->ftake;
+  }
+}
+
+// StaticQuota (Sec. V-A) grants, one CTA per group: the group's claims, in
+// (request, position) order, while its partition of Q = floor(N / G) blocks
+// minus its pinned ones holds them; its overflow m_g = granted - (Q -
+// resident) is what it must reclaim from its own blocks.
+__global__ void __launch_bounds__(1024) k_grant_quota(DevState s) {
+  s = with_args(s);
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  const int g = blockIdx.x;
+  const int64_t Q = s.N / s.G;
+  const int64_t avail = Q - s.grp_pinned[g];
+  const int R = s.R;
+  int64_t carry = 0, granted = 0;
+  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
+    const int i = t0 + threadIdx.x;
+    const bool member = i < R && s.in_group[i] == g;
+    const int32_t cl = member ? s.rq_n[i] - s.rq_s[i] : 0;
+    int32_t tot;
+    const int32_t ex = block_excl_scan(cl, &tot);
+    if (member) {
+      const int64_t a = tmin<int64_t>(cl, tmax<int64_t>(0, avail - (carry + ex)));
+      s.rq_a[i] = (int32_t)a;
+      granted += a;
+    }
+    carry += tot;
+  }
+  granted = block_sum(granted);
+  if (threadIdx.x == 0) {
+    const int64_t resident = s.stats[(int64_t)g * PS_NUM_STATS + PS_STAT_RESIDENT_BLOCKS];
+    s.grp_x[g] = tmax<int64_t>(0, granted - (Q - resident));
   }
 }
 
 // In-step hits: positions of [h_i, s_i) belong to earlier requests' claims;
-// the leading granted ones are hits.  A position whose owner's rank is past
-// avail lowers the request's first-ungranted mark.
+// the leading granted ones are hits.  A position whose owner's key was not
+// granted lowers the request's first-ungranted mark.
 __global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
   s = with_args(s);
   const Ctl* c = s.ctl;
@@ -713,9 +770,10 @@ __global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
   bool past = false;
   const bool valid = pos_ref(s, pos, &r);
   if (valid && r.m >= s.rq_h[r.i] && r.m < s.rq_s[r.i]) {
+    // the owner's claims are ranked consecutively: its key here is granted
+    // iff it is among the owner's first a_j
     const uint32_t j = s.claims[s.pos_claim[pos]].minreq;
-    const int64_t rank = (int64_t)s.rq_cbase[j] + (r.m - s.rq_s[j]);
-    past = rank >= c->avail;
+    past = r.m - s.rq_s[j] >= s.rq_a[j];
   }
   agg_min_u32(s.rq_fu, valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, past);
 }
@@ -931,8 +989,10 @@ __global__ void __launch_bounds__(1024) k_cand(DevState s) {
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
   const uint32_t step32 = (uint32_t)c->step;
-  const bool ps = s.policy == PS_PREFIXSHIELD;
-  const bool seg = ps && !(s.flags & PS_FLAG_NO_SEGMENTATION);
+  // segments: groups for prefixshield and staticquota, one for lru; retention
+  // classes only for prefixshield
+  const bool ps = s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA;
+  const bool seg = s.policy == PS_PREFIXSHIELD && !(s.flags & PS_FLAG_NO_SEGMENTATION);
   const int nrow = (ps ? s.G : 1) * kClasses;
   uint32_t* s_cnt = cand_smem;
   uint32_t* s_hmin = s_cnt + nrow;
@@ -1105,6 +1165,23 @@ __global__ void __launch_bounds__(32) k_sel_single(DevState s, int fallback) {
   sel_start_cls(z, cnt, lo, hi, segmented);
   s.sel[0] = z;
   c->lst_n = 0;
+}
+
+// StaticQuota: each group reclaims its overflow m_g from its own blocks, in
+// recency order (one segment per group, no global fallback).
+__global__ void __launch_bounds__(1024) k_quota_sel(DevState s) {
+  s = with_args(s);
+  Ctl* c = s.ctl;
+  const int64_t m = c->status == PS_OK ? c->mvict : 0;
+  for (int g = threadIdx.x; g < s.G; g += blockDim.x) {
+    SelSeg z = s.sel[g];
+    z.rank = m > 0 ? s.grp_x[g] : 0;
+    z.active = z.rank > 0;
+    z.incl = 1;
+    sel_start_group(s, g, z, false);
+    s.sel[g] = z;
+  }
+  if (threadIdx.x == 0) { c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->lst_n = 0; }
 }
 
 // Alg. 2 in closed form (one CTA).  Group g's j-th victim would be taken at
@@ -2105,6 +2182,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(2);
   PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
   mark(3);
+  if (s.policy == PS_STATICQUOTA) PS_LAUNCH(k_grant_quota<<<s.G, 1024, 0, st>>>(s));
   PS_LAUNCH(k_grant<<<1, 1024, 0, st>>>(s));
   PS_LAUNCH(k_instep<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_instep_fin<<<rgrid, 256, 0, st>>>(s));
@@ -2114,7 +2192,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(k_touch<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
   mark(6);
-  const int cand_smem = (s.policy == PS_PREFIXSHIELD ? s.G : 1) * kClasses * 5 * 4;
+  const int cand_smem = (s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA ? s.G : 1) * kClasses * 5 * 4;
   if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, st>>>(s));
   // Under capture, phases that many steps skip become conditional bodies:
   // the long-list passes of a select, and the global fallback of Alg. 2.
@@ -2173,6 +2251,10 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
     select(f, 1, 1, conds, h_fb_long, conds ? cap->aux2 : f);
     if (!cond_ok) return PS_ERR_CUDA;
     if (conds && !cond_close(cap->aux)) return PS_ERR_CUDA;
+  } else if (s.policy == PS_STATICQUOTA) {
+    PS_LAUNCH(k_quota_sel<<<1, 1024, 0, st>>>(s));
+    select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
+    if (!cond_ok) return PS_ERR_CUDA;
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
     select(st, 1, 0, conds, h_long, conds ? cap->aux : st);

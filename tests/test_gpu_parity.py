@@ -45,7 +45,7 @@ def _run(gpu, orc, steps, state_every=1, s3=False, label=""):
     assert np.array_equal(gpu.stats(), orc.stats()), f"{label}: stats differ"
 
 
-GPU_POLICIES = ["lru", "s3fifo", "prefixshield"]
+GPU_POLICIES = ["lru", "s3fifo", "prefixshield", "staticquota"]
 
 
 @pytest.mark.parametrize("policy", GPU_POLICIES)
@@ -312,3 +312,18 @@ def test_parity_kernel_by_kernel(policy):
                         f"direct/{policy} step {k}")
     compare_state(gpu.export(), orc.export(), f"direct/{policy}", s3=policy == "s3fifo")
     assert np.array_equal(gpu.stats(), orc.stats())
+
+
+def test_parity_staticquota_borrowing_trace():
+    """The borrowing trace (Table III) on the GPU: one group idle, the other
+    capped at its equal share, every output and the state as the oracle's."""
+    from _util import obj_tokens, make_step
+    N, G = 511, 2
+    gpu, orc = _pair(N, 16, G, "staticquota", dict(rho=(64.0,), beta=(4096.0,)), max_requests=8, max_tokens=8 * 64)
+    steps = []
+    for t in range(40):
+        grp, offs, toks, _ = make_step([obj_tokens(f"borrow-{t}-{j}", blocks=4) for j in range(8)], groups=[0] * 8)
+        steps.append(W.Step(t, t, grp, offs, toks))
+    _run(gpu, orc, steps, state_every=5, label="borrowing")
+    e = gpu.export()
+    assert int(((e["resident"] == 1) & (e["group"] == 0)).sum()) == N // G
