@@ -267,6 +267,29 @@ class Scale(Workload):
         return _pack(s, [int(g) for g in gs], pieces)
 
 
+class LowAndSlow(Workload):
+    """Low-and-slow rotation (Sec. V-A): the victim (group 0) sends one
+    request per step, cycling through four 1536-token hot prefixes (96
+    blocks each) plus a 32-token fresh suffix; the attacker (group 1) spreads
+    one-touch pressure over time, one fresh 1536-token prompt every third
+    step.  A prefix's reuse distance is three other victim requests (294
+    blocks with their suffixes)."""
+
+    def __init__(self, spec, seed, n_hot=4, hot_len=1536, suffix=32, atk_len=1536, atk_every=3):
+        super().__init__(spec, seed)
+        self.hot = [_tokens(_rng(seed, "hot", 0, j), hot_len) for j in range(n_hot)]
+        self.suffix, self.atk_len, self.atk_every = suffix, atk_len, atk_every
+
+    def make_step(self, s: int) -> Step:
+        fresh = _Fresh(self.seed, s, self.suffix + self.atk_len)
+        groups = [0]
+        pieces = [[self.hot[s % len(self.hot)], fresh.take(self.suffix)]]
+        if s % self.atk_every == self.atk_every - 1:
+            groups.append(1)
+            pieces.append([fresh.take(self.atk_len)])
+        return _pack(s, groups, pieces)
+
+
 def _lognormal_2048(r):
     return _lognormal_len(r, np.log(2048.0), 0.5, 256, 8192)
 
@@ -284,12 +307,16 @@ CONFIGS = {
                     description="4 system prompts U[256,1024] per group, multi-turn histories; 256 req/step"),
     4: WorkloadSpec("scale", 64, 1 << 20, 16, 4096, 2000000, rho=(2000,), beta=(6000,),
                     description="8 victim, 8 attacker, 48 benign groups; 4096 req/step"),
+    5: WorkloadSpec("low-and-slow rotation", 2, 511, 16, 2, 600, rho=(64, 16), beta=(256, 128),
+                    contract_of_group=(0, 1),
+                    description="victim: 4 hot 1536-token prefixes in rotation + 32 fresh, one a step; "
+                                "attacker: one fresh 1536-token prompt every third step; 511 usable blocks"),
 }
 
 
 def make_workload(config: int, seed: int = 1, requests_per_step: Optional[int] = None,
                   total_requests: Optional[int] = None) -> Workload:
-    """The seeded trace of one configuration (0..4).  ``requests_per_step``
+    """The seeded trace of one configuration (0..5).  ``requests_per_step``
     overrides the batch size (e.g. the discriminative 8-request variants)."""
     spec = CONFIGS[config]
     if requests_per_step is not None or total_requests is not None:
@@ -310,6 +337,8 @@ def make_workload(config: int, seed: int = 1, requests_per_step: Optional[int] =
         return BenignChat(spec, seed)
     if config == 4:
         return Scale(spec, seed)
+    if config == 5:
+        return LowAndSlow(spec, seed)
     raise KeyError(config)
 
 

@@ -101,13 +101,16 @@ def test_parity_tiny_one_touch(policy):
 
 
 @pytest.mark.parametrize("policy", GPU_POLICIES)
-@pytest.mark.parametrize("cfg,nsteps,rps", [(1, 40, None), (1, 60, 8), (2, 40, 8), (3, 30, None)])
+@pytest.mark.parametrize("cfg,nsteps,rps", [(1, 40, None), (1, 60, 8), (2, 40, 8), (3, 30, None), (5, 120, None)])
 def test_parity_configs(policy, cfg, nsteps, rps):
     wl = W.make_workload(cfg, seed=2, requests_per_step=rps)
     sp = wl.spec
     steps = list(wl.steps(nsteps))
     maxT = max(s.num_tokens for s in steps)
-    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, dict(rho=sp.rho, beta=sp.beta),
+    kw = dict(rho=sp.rho, beta=sp.beta)
+    if sp.contract_of_group is not None:
+        kw["contract_of_group"] = list(sp.contract_of_group)
+    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, kw,
                      max_requests=sp.requests_per_step, max_tokens=maxT)
     _run(gpu, orc, steps, state_every=10, label=f"cfg{cfg}/{policy}")
 
