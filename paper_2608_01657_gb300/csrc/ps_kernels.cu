@@ -298,63 +298,76 @@ __global__ void k_init_ctl(DevState s) {
 // ===========================================================================
 // Stage 0: validation of the step's inputs; n_i, block positions, hashing
 // segments.  One CTA.  'probe' skips the clock and step checks.
-__global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
+__global__ void __launch_bounds__(512) k_validate(DevState s, int probe) {
   s = with_args(s);
   Ctl* c = s.ctl;
-  __shared__ int s_bad;
-  if (threadIdx.x == 0) s_bad = 0;
-  __syncthreads();
   const int R = s.R;
-  for (int i = threadIdx.x; i < R; i += blockDim.x) {
-    const int64_t o0 = s.in_offsets[i], o1 = s.in_offsets[i + 1];
-    const int g = s.in_group[i];
-    bool bad = o1 < o0 || g < 0 || g >= s.G || (o1 - o0) / s.bs > (int64_t)kMaxPos;
-    if (s.in_contract) bad |= s.in_contract[i] < 0 || s.in_contract[i] >= s.C;
-    if (s.in_prefix) bad |= s.in_prefix[i] == 0;
-    if (bad) atomicOr(&s_bad, 1);
+  // One pass: each thread takes kPer consecutive requests, checks them, and
+  // one block scan of (segments << 32 | blocks) places them.  Writes are
+  // bounds-checked, because the input is validated in the same pass (a step
+  // with any bad request is a no-op: every later kernel sees the status).
+  constexpr int kPer = 8;
+  int bad = 0;
+  int64_t carry = 0, scarry = 0;
+  for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
+    const int i0 = base + (int)threadIdx.x * kPer;
+    int32_t n[kPer], ns[kPer];
+    int64_t tn = 0, ts = 0;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      n[u] = ns[u] = 0;
+      if (i < R) {
+        const int64_t o0 = s.in_offsets[i], o1 = s.in_offsets[i + 1];
+        const int g = s.in_group[i];
+        bool b = o1 < o0 || g < 0 || g >= s.G || (o1 - o0) / s.bs > (int64_t)kMaxPos;
+        if (s.in_contract) b |= s.in_contract[i] < 0 || s.in_contract[i] >= s.C;
+        if (s.in_prefix) b |= s.in_prefix[i] == 0;
+        bad |= b;
+        if (!b) {
+          n[u] = (int32_t)((o1 - o0) / s.bs);
+          ns[u] = (n[u] + kSegBlocks - 1) / kSegBlocks;
+        }
+        s.rq_n[i] = n[u];
+        s.rq_h[i] = n[u];
+        s.rq_s[i] = n[u];
+        s.rq_fu[i] = kNone;
+        if (!probe && !b) s.rq_cid[i] = s.in_contract ? s.in_contract[i] : s.contract_of_group[g];
+      }
+      tn += n[u];
+      ts += ns[u];
+    }
+    int64_t tot;
+    const int64_t ex = block_excl_scan<int64_t>((ts << 32) | tn, &tot);
+    int64_t pb = carry + (ex & 0xFFFFFFFFll), sb = scarry + (ex >> 32);
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      if (i < R) {
+        s.rq_pbase[i] = (int32_t)pb;
+        s.rq_sbase[i] = (int32_t)sb;
+        for (int j = 0; j < ns[u]; ++j)
+          if (sb + j < s.max_segments) s.seg_req[sb + j] = (uint32_t)i;
+      }
+      pb += n[u];
+      sb += ns[u];
+    }
+    carry += tot & 0xFFFFFFFFll;
+    scarry += tot >> 32;
   }
-  __syncthreads();
+  bad = __syncthreads_or(bad);
   int32_t st = PS_OK;
   const int64_t T = R > 0 ? s.in_offsets[R] : 0;
   if (!probe && c->sticky != PS_OK) st = c->sticky;
   else if (!probe && s.now < c->t_prev) st = PS_ERR_CLOCK;
   else if (!probe && c->step > kMaxStep) st = PS_ERR_CAPACITY;
-  else if (s_bad || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens) st = PS_ERR_INVALID_ARG;
-  if (st != PS_OK) {
-    __syncthreads();
-    if (threadIdx.x == 0) { c->status = st; c->nblocks = 0; c->nsegs = 0; }
-    return;
-  }
-  int32_t carry = 0, scarry = 0;
-  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
-    const int i = t0 + threadIdx.x;
-    int32_t n = 0, nseg = 0;
-    if (i < R) {
-      n = (int32_t)((s.in_offsets[i + 1] - s.in_offsets[i]) / s.bs);
-      nseg = (n + kSegBlocks - 1) / kSegBlocks;
-      s.rq_n[i] = n;
-      s.rq_h[i] = n;
-      s.rq_s[i] = n;
-      s.rq_fu[i] = kNone;
-      if (!probe) s.rq_cid[i] = s.in_contract ? s.in_contract[i] : s.contract_of_group[s.in_group[i]];
-    }
-    int32_t tot, stot;
-    const int32_t ex = block_excl_scan(n, &tot);
-    const int32_t sex = block_excl_scan(nseg, &stot);
-    if (i < R) {
-      s.rq_pbase[i] = carry + ex;
-      s.rq_sbase[i] = scarry + sex;
-      for (int j = 0; j < nseg; ++j) s.seg_req[scarry + sex + j] = (uint32_t)i;
-    }
-    carry += tot;
-    scarry += stot;
-  }
+  else if (bad || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens || carry > s.max_blocks) st = PS_ERR_INVALID_ARG;
   if (threadIdx.x == 0) {
-    c->status = PS_OK;
-    c->T = T;
-    c->nblocks = carry;
-    c->nsegs = scarry;
-    if (!probe) {
+    c->status = st;
+    c->T = st == PS_OK ? T : 0;
+    c->nblocks = st == PS_OK ? carry : 0;
+    c->nsegs = st == PS_OK ? scarry : 0;
+    if (!probe && st == PS_OK) {
       c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
       c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
       c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
@@ -363,7 +376,7 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
       c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
     }
   }
-  if (!probe && s.policy == PS_STATICQUOTA)
+  if (st == PS_OK && !probe && s.policy == PS_STATICQUOTA)
     for (int g = threadIdx.x; g < s.G; g += blockDim.x) s.grp_pinned[g] = 0;
 }
 
@@ -679,7 +692,7 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
 // Stage 3: grant new blocks against the pool.  avail = free + unpinned
 // resident = N - pinned; claims are ranked in (request, position) order; the
 // first avail ranks are materialized.  One CTA.
-__global__ void __launch_bounds__(1024) k_grant(DevState s) {
+__global__ void __launch_bounds__(512) k_grant(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
@@ -687,23 +700,45 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
   const bool quota = s.policy == PS_STATICQUOTA;  // a_i already granted per group
   const int64_t avail = s.N - c->pinned;
   int64_t carry_c = 0, carry_a = 0;
-  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
-    const int i = t0 + threadIdx.x;
-    int32_t cl = 0;
-    if (i < R) cl = s.rq_n[i] - s.rq_s[i];
-    int32_t tot_c;
-    const int32_t ex_c = block_excl_scan(cl, &tot_c);
-    int32_t a = 0;
-    if (i < R) a = quota ? s.rq_a[i] : (int32_t)tmin<int64_t>(cl, tmax<int64_t>(0, avail - (carry_c + ex_c)));
-    int32_t tot_a;
-    const int32_t ex_a = block_excl_scan(a, &tot_a);
-    if (i < R) {
-      // granted keys are paired with the allocated ids in (request, position)
-      // order: request i's first granted key is the (carry_a + ex_a)-th
-      s.rq_cbase[i] = (int32_t)(carry_a + ex_a);
-      s.rq_a[i] = a;
-      s.out.admitted_blocks[i] = a;
-      s.out.admitted_offsets[i] = (int32_t)(carry_a + ex_a);
+  // each thread takes kPer consecutive requests: one scan of the claims and
+  // one of the grants place kPer * blockDim requests
+  constexpr int kPer = 8;
+  for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
+    const int i0 = base + (int)threadIdx.x * kPer;
+    int32_t cl[kPer];
+    int64_t mine_c = 0;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      cl[u] = i < R ? s.rq_n[i] - s.rq_s[i] : 0;
+      mine_c += cl[u];
+    }
+    int64_t tot_c;
+    int64_t cb = carry_c + block_excl_scan<int64_t>(mine_c, &tot_c);
+    int32_t a[kPer];
+    int64_t mine_a = 0;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      a[u] = 0;
+      if (i < R) a[u] = quota ? s.rq_a[i] : (int32_t)tmin<int64_t>(cl[u], tmax<int64_t>(0, avail - cb));
+      cb += cl[u];
+      mine_a += a[u];
+    }
+    int64_t tot_a;
+    int64_t ab = carry_a + block_excl_scan<int64_t>(mine_a, &tot_a);
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      if (i < R) {
+        // granted keys are paired with the allocated ids in (request,
+        // position) order: request i's first granted key is the ab-th
+        s.rq_cbase[i] = (int32_t)ab;
+        s.rq_a[i] = a[u];
+        s.out.admitted_blocks[i] = a[u];
+        s.out.admitted_offsets[i] = (int32_t)ab;
+      }
+      ab += a[u];
     }
     carry_c += tot_c;
     carry_a += tot_a;
@@ -805,7 +840,7 @@ __global__ void k_instep_fin(DevState s) {
 // q_r >= 1 and "(g,p) was admitted" come from the history entry as it stood at
 // the start of the step and the first request of the step that referenced /
 // admitted it.  Also writes the group's statistics, balances and debts.
-__global__ void __launch_bounds__(1024) k_meter(DevState s0) {
+__global__ void __launch_bounds__(512) k_meter(DevState s0) {
   // Contract arrays are read from the parameter block: indexing the per-step
   // copy by a run-time contract would move the whole copy to local memory.
   const DevState s = with_args(s0);
@@ -816,54 +851,93 @@ __global__ void __launch_bounds__(1024) k_meter(DevState s0) {
   const int64_t unit = (int64_t)1 << s.fp_shift;
   const uint64_t step = c->step;
   __shared__ int64_t B0[PS_MAX_CONTRACTS];
+  __shared__ unsigned long long s_st[7];  // the group's request statistics
   if (threadIdx.x < C) {
     const int cc = threadIdx.x;
     B0[cc] = refill(s.ledger[g * C + cc], s0.beta[cc], s0.rho[cc], s.now - c->t_prev);
   }
+  if (threadIdx.x < 7) s_st[threadIdx.x] = 0;
   __syncthreads();
   int64_t carry[PS_MAX_CONTRACTS];
 #pragma unroll
   for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) carry[cc] = 0;
   int64_t st_req = 0, st_ptok = 0, st_full = 0, st_hit = 0, st_inst = 0, st_adm = 0, st_ungr = 0;
   const int R = s.R;
-  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
-    const int i = t0 + threadIdx.x;
-    const bool member = i < R && s.in_group[i] == g;
-    int n = 0, a = 0, cid = 0;
-    if (member) { n = s.rq_n[i]; a = s.rq_a[i]; cid = s.rq_cid[i]; }
-    const bool pol = member && n > 0;
-    // charges of this group's earlier requests, per contract; then the raw
-    // debt before this request's charge (Eq. 3) and the balance after it
-    int64_t d = 0, b_after = 0;
+  // each thread takes kPer consecutive requests, so one block scan per
+  // contract places kPer * blockDim requests
+  constexpr int kPer = 4;
+  for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
+    const int i0 = base + (int)threadIdx.x * kPer;
+    bool mem[kPer];
+    int n[kPer], a[kPer], cid[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      mem[u] = i < R && s.in_group[i] == g;
+      n[u] = a[u] = cid[u] = 0;
+      if (mem[u]) { n[u] = s.rq_n[i]; a[u] = s.rq_a[i]; cid[u] = s.rq_cid[i]; }
+    }
+    // charges of this group's earlier requests, per contract: the thread's
+    // base from a block scan, then its own requests in order
+    int64_t S[PS_MAX_CONTRACTS];
 #pragma unroll
     for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
+      S[cc] = 0;
       if (cc < C) {
+        int64_t mine = 0;
+#pragma unroll
+        for (int u = 0; u < kPer; ++u) mine += (mem[u] && n[u] > 0 && cid[u] == cc) ? a[u] : 0;
         int64_t tot;
-        const int64_t ex = block_excl_scan<int64_t>((pol && cid == cc) ? a : 0, &tot);
-        const int64_t Sx = carry[cc] + ex;
+        const int64_t ex = block_excl_scan<int64_t>(mine, &tot);
+        S[cc] = carry[cc] + ex;
         carry[cc] += tot;
-        d += tmax<int64_t>(0, -(B0[cc] - Sx * unit));
-        if (cid == cc) b_after = B0[cc] - (Sx + a) * unit;
       }
     }
-    if (pol) {
-      const bool gate = (s.flags & PS_FLAG_NO_DEBT_GATE) || d <= s.eps;
-      const uint32_t hs = s.rq_hs[i];
-      HistEntry he{};
-      if (hs != kNone) he = s.hist[hs];
-      const uint32_t refadm = he.refadm;
-      const bool q_ge1 = (refadm & 0x7FFFFFFFu) >= 1 || tag_req(he.ftag, step) < (uint32_t)i;
-      const bool adm_before = (refadm >> 31) || tag_req(he.atag, step) < (uint32_t)i;
-      const bool proven = q_ge1 && adm_before;
-      s.rq_flags[i] = (uint8_t)((proven ? 1 : 0) | (gate ? 2 : 0));
-      s.rq_knew[i] = (uint8_t)((b_after < -s.eps || !adm_before) ? kProb : kNormal);
-      const int h = s.rq_h[i], e = s.rq_e[i];
-      st_full += n; st_hit += h + e; st_inst += e; st_adm += a; st_ungr += (n - s.rq_s[i]) - a;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      const bool pol = mem[u] && n[u] > 0;
+      // the raw debt before this request's charge (Eq. 3) and its balance after
+      int64_t d = 0, b_after = 0;
+#pragma unroll
+      for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
+        if (cc < C) {
+          d += tmax<int64_t>(0, -(B0[cc] - S[cc] * unit));
+          if (cid[u] == cc) b_after = B0[cc] - (S[cc] + a[u]) * unit;
+        }
+      }
+      if (pol) {
+        const bool gate = (s.flags & PS_FLAG_NO_DEBT_GATE) || d <= s.eps;
+        const uint32_t hs = s.rq_hs[i];
+        HistEntry he{};
+        if (hs != kNone) he = s.hist[hs];
+        const uint32_t refadm = he.refadm;
+        const bool q_ge1 = (refadm & 0x7FFFFFFFu) >= 1 || tag_req(he.ftag, step) < (uint32_t)i;
+        const bool adm_before = (refadm >> 31) || tag_req(he.atag, step) < (uint32_t)i;
+        const bool proven = q_ge1 && adm_before;
+        s.rq_flags[i] = (uint8_t)((proven ? 1 : 0) | (gate ? 2 : 0));
+        s.rq_knew[i] = (uint8_t)((b_after < -s.eps || !adm_before) ? kProb : kNormal);
+        const int h = s.rq_h[i], e = s.rq_e[i];
+        st_full += n[u]; st_hit += h + e; st_inst += e; st_adm += a[u]; st_ungr += (n[u] - s.rq_s[i]) - a[u];
+        // this request's own charge, for the requests after it in the thread
+#pragma unroll
+        for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc)
+          if (cc < C && cid[u] == cc) S[cc] += a[u];
+      }
+      if (mem[u]) { st_req += 1; st_ptok += s.in_offsets[i + 1] - s.in_offsets[i]; }
     }
-    if (member) { st_req += 1; st_ptok += s.in_offsets[i + 1] - s.in_offsets[i]; }
   }
-  st_req = block_sum(st_req); st_ptok = block_sum(st_ptok); st_full = block_sum(st_full);
-  st_hit = block_sum(st_hit); st_inst = block_sum(st_inst); st_adm = block_sum(st_adm); st_ungr = block_sum(st_ungr);
+  {
+    const int64_t v[7] = {st_req, st_ptok, st_full, st_hit, st_inst, st_adm, st_ungr};
+#pragma unroll
+    for (int k = 0; k < 7; ++k) {
+      const int64_t w = warp_sum(v[k]);
+      if (lane_id() == 0 && w) atomicAdd(&s_st[k], (unsigned long long)w);
+    }
+  }
+  __syncthreads();
+  st_req = (int64_t)s_st[0]; st_ptok = (int64_t)s_st[1]; st_full = (int64_t)s_st[2]; st_hit = (int64_t)s_st[3];
+  st_inst = (int64_t)s_st[4]; st_adm = (int64_t)s_st[5]; st_ungr = (int64_t)s_st[6];
   if (threadIdx.x == 0) {
     int64_t* row = s.stats + (int64_t)g * PS_NUM_STATS;
     row[PS_STAT_REQUESTS] += st_req;
@@ -2173,7 +2247,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
   mark(0);
-  PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s, 0));
+  PS_LAUNCH(k_validate<<<1, 512, 0, st>>>(s, 0));
   mark(1);
   if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
   ++launches;
@@ -2183,11 +2257,11 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
   mark(3);
   if (s.policy == PS_STATICQUOTA) PS_LAUNCH(k_grant_quota<<<s.G, 1024, 0, st>>>(s));
-  PS_LAUNCH(k_grant<<<1, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_grant<<<1, 512, 0, st>>>(s));
   PS_LAUNCH(k_instep<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_instep_fin<<<rgrid, 256, 0, st>>>(s));
   mark(4);
-  PS_LAUNCH(k_meter<<<s.G, 1024, 0, st>>>(s));
+  PS_LAUNCH(k_meter<<<s.G, 512, 0, st>>>(s));
   mark(5);
   PS_LAUNCH(k_touch<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
@@ -2285,7 +2359,7 @@ int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* 
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
   DevState p = s;
   p.args = nullptr;  // the probe's kernels take every argument by value
-  k_validate<<<1, 1024, 0, st>>>(p, 1);
+  k_validate<<<1, 512, 0, st>>>(p, 1);
   if (s.R > 0) {
     if (launch_hash(p, st) != PS_OK) return PS_ERR_INVALID_ARG;
     k_keys_lookup<<<pgrid, kThreads, 0, st>>>(p);
