@@ -311,31 +311,55 @@ __global__ void __launch_bounds__(512) k_validate(DevState s, int probe) {
   int64_t carry = 0, scarry = 0;
   for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
     const int i0 = base + (int)threadIdx.x * kPer;
-    int32_t n[kPer], ns[kPer];
+    // loads first (the stores below could alias them for the compiler)
+    int64_t o[kPer + 1];
+    int32_t gr[kPer], ct[kPer];
+    uint64_t px[kPer];
+#pragma unroll
+    for (int u = 0; u <= kPer; ++u) o[u] = i0 + u <= R ? s.in_offsets[i0 + u] : 0;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      gr[u] = i < R ? s.in_group[i] : 0;
+      ct[u] = (i < R && s.in_contract) ? s.in_contract[i] : 0;
+      px[u] = (i < R && s.in_prefix) ? s.in_prefix[i] : 1;
+    }
+    int32_t n[kPer], ns[kPer], cid[kPer];
+    bool bq[kPer];
     int64_t tn = 0, ts = 0;
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
       const int i = i0 + u;
       n[u] = ns[u] = 0;
+      bq[u] = false;
       if (i < R) {
-        const int64_t o0 = s.in_offsets[i], o1 = s.in_offsets[i + 1];
-        const int g = s.in_group[i];
-        bool b = o1 < o0 || g < 0 || g >= s.G || (o1 - o0) / s.bs > (int64_t)kMaxPos;
-        if (s.in_contract) b |= s.in_contract[i] < 0 || s.in_contract[i] >= s.C;
-        if (s.in_prefix) b |= s.in_prefix[i] == 0;
+        const int g = gr[u];
+        bool b = o[u + 1] < o[u] || g < 0 || g >= s.G || (o[u + 1] - o[u]) / s.bs > (int64_t)kMaxPos;
+        if (s.in_contract) b |= ct[u] < 0 || ct[u] >= s.C;
+        if (s.in_prefix) b |= px[u] == 0;
         bad |= b;
+        bq[u] = b;
         if (!b) {
-          n[u] = (int32_t)((o1 - o0) / s.bs);
+          n[u] = (int32_t)((o[u + 1] - o[u]) / s.bs);
           ns[u] = (n[u] + kSegBlocks - 1) / kSegBlocks;
         }
+      }
+      tn += n[u];
+      ts += ns[u];
+    }
+#pragma unroll
+    for (int u = 0; u < kPer; ++u)
+      cid[u] = (i0 + u < R && !probe && !bq[u]) ? (s.in_contract ? ct[u] : s.contract_of_group[gr[u]]) : 0;
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      if (i < R) {
         s.rq_n[i] = n[u];
         s.rq_h[i] = n[u];
         s.rq_s[i] = n[u];
         s.rq_fu[i] = kNone;
-        if (!probe && !b) s.rq_cid[i] = s.in_contract ? s.in_contract[i] : s.contract_of_group[g];
+        if (!probe && !bq[u]) s.rq_cid[i] = cid[u];
       }
-      tn += n[u];
-      ts += ns[u];
     }
     int64_t tot;
     const int64_t ex = block_excl_scan<int64_t>((ts << 32) | tn, &tot);
@@ -705,12 +729,13 @@ __global__ void __launch_bounds__(512) k_grant(DevState s) {
   constexpr int kPer = 8;
   for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
     const int i0 = base + (int)threadIdx.x * kPer;
-    int32_t cl[kPer];
+    int32_t cl[kPer], qa[kPer];
     int64_t mine_c = 0;
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
       const int i = i0 + u;
       cl[u] = i < R ? s.rq_n[i] - s.rq_s[i] : 0;
+      qa[u] = (quota && i < R) ? s.rq_a[i] : 0;
       mine_c += cl[u];
     }
     int64_t tot_c;
@@ -721,7 +746,7 @@ __global__ void __launch_bounds__(512) k_grant(DevState s) {
     for (int u = 0; u < kPer; ++u) {
       const int i = i0 + u;
       a[u] = 0;
-      if (i < R) a[u] = quota ? s.rq_a[i] : (int32_t)tmin<int64_t>(cl[u], tmax<int64_t>(0, avail - cb));
+      if (i < R) a[u] = quota ? qa[u] : (int32_t)tmin<int64_t>(cl[u], tmax<int64_t>(0, avail - cb));
       cb += cl[u];
       mine_a += a[u];
     }
@@ -893,6 +918,25 @@ __global__ void __launch_bounds__(512) k_meter(DevState s0) {
         carry[cc] += tot;
       }
     }
+    // the requests' other inputs, loaded before any store below
+    HistEntry he[kPer];
+    int rh[kPer], re[kPer], rs[kPer];
+    int64_t ptok[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int i = i0 + u;
+      he[u] = HistEntry{};
+      rh[u] = re[u] = rs[u] = 0;
+      ptok[u] = 0;
+      if (mem[u]) {
+        const uint32_t hs = s.rq_hs[i];
+        if (n[u] > 0 && hs != kNone) he[u] = s.hist[hs];
+        rh[u] = s.rq_h[i];
+        re[u] = s.rq_e[i];
+        rs[u] = s.rq_s[i];
+        ptok[u] = s.in_offsets[i + 1] - s.in_offsets[i];
+      }
+    }
 #pragma unroll
     for (int u = 0; u < kPer; ++u) {
       const int i = i0 + u;
@@ -908,23 +952,20 @@ __global__ void __launch_bounds__(512) k_meter(DevState s0) {
       }
       if (pol) {
         const bool gate = (s.flags & PS_FLAG_NO_DEBT_GATE) || d <= s.eps;
-        const uint32_t hs = s.rq_hs[i];
-        HistEntry he{};
-        if (hs != kNone) he = s.hist[hs];
-        const uint32_t refadm = he.refadm;
-        const bool q_ge1 = (refadm & 0x7FFFFFFFu) >= 1 || tag_req(he.ftag, step) < (uint32_t)i;
-        const bool adm_before = (refadm >> 31) || tag_req(he.atag, step) < (uint32_t)i;
+        const uint32_t refadm = he[u].refadm;
+        const bool q_ge1 = (refadm & 0x7FFFFFFFu) >= 1 || tag_req(he[u].ftag, step) < (uint32_t)i;
+        const bool adm_before = (refadm >> 31) || tag_req(he[u].atag, step) < (uint32_t)i;
         const bool proven = q_ge1 && adm_before;
         s.rq_flags[i] = (uint8_t)((proven ? 1 : 0) | (gate ? 2 : 0));
         s.rq_knew[i] = (uint8_t)((b_after < -s.eps || !adm_before) ? kProb : kNormal);
-        const int h = s.rq_h[i], e = s.rq_e[i];
-        st_full += n[u]; st_hit += h + e; st_inst += e; st_adm += a[u]; st_ungr += (n[u] - s.rq_s[i]) - a[u];
+        const int h = rh[u], e = re[u];
+        st_full += n[u]; st_hit += h + e; st_inst += e; st_adm += a[u]; st_ungr += (n[u] - rs[u]) - a[u];
         // this request's own charge, for the requests after it in the thread
 #pragma unroll
         for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc)
           if (cc < C && cid[u] == cc) S[cc] += a[u];
       }
-      if (mem[u]) { st_req += 1; st_ptok += s.in_offsets[i + 1] - s.in_offsets[i]; }
+      if (mem[u]) { st_req += 1; st_ptok += ptok[u]; }
     }
   }
   {
