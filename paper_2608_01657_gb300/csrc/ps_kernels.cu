@@ -298,100 +298,63 @@ __global__ void k_init_ctl(DevState s) {
 // ===========================================================================
 // Stage 0: validation of the step's inputs; n_i, block positions, hashing
 // segments.  One CTA.  'probe' skips the clock and step checks.
-__global__ void __launch_bounds__(512) k_validate(DevState s, int probe) {
+__global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
   s = with_args(s);
   Ctl* c = s.ctl;
+  __shared__ int s_bad;
+  if (threadIdx.x == 0) s_bad = 0;
+  __syncthreads();
   const int R = s.R;
-  // One pass: each thread takes kPer consecutive requests, checks them, and
-  // one block scan of (segments << 32 | blocks) places them.  Writes are
-  // bounds-checked, because the input is validated in the same pass (a step
-  // with any bad request is a no-op: every later kernel sees the status).
-  constexpr int kPer = 8;
-  int bad = 0;
-  int64_t carry = 0, scarry = 0;
-  for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
-    const int i0 = base + (int)threadIdx.x * kPer;
-    // loads first (the stores below could alias them for the compiler)
-    int64_t o[kPer + 1];
-    int32_t gr[kPer], ct[kPer];
-    uint64_t px[kPer];
-#pragma unroll
-    for (int u = 0; u <= kPer; ++u) o[u] = i0 + u <= R ? s.in_offsets[i0 + u] : 0;
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      gr[u] = i < R ? s.in_group[i] : 0;
-      ct[u] = (i < R && s.in_contract) ? s.in_contract[i] : 0;
-      px[u] = (i < R && s.in_prefix) ? s.in_prefix[i] : 1;
-    }
-    int32_t n[kPer], ns[kPer], cid[kPer];
-    bool bq[kPer];
-    int64_t tn = 0, ts = 0;
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      n[u] = ns[u] = 0;
-      bq[u] = false;
-      if (i < R) {
-        const int g = gr[u];
-        bool b = o[u + 1] < o[u] || g < 0 || g >= s.G || (o[u + 1] - o[u]) / s.bs > (int64_t)kMaxPos;
-        if (s.in_contract) b |= ct[u] < 0 || ct[u] >= s.C;
-        if (s.in_prefix) b |= px[u] == 0;
-        bad |= b;
-        bq[u] = b;
-        if (!b) {
-          n[u] = (int32_t)((o[u + 1] - o[u]) / s.bs);
-          ns[u] = (n[u] + kSegBlocks - 1) / kSegBlocks;
-        }
-      }
-      tn += n[u];
-      ts += ns[u];
-    }
-#pragma unroll
-    for (int u = 0; u < kPer; ++u)
-      cid[u] = (i0 + u < R && !probe && !bq[u]) ? (s.in_contract ? ct[u] : s.contract_of_group[gr[u]]) : 0;
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      if (i < R) {
-        s.rq_n[i] = n[u];
-        s.rq_h[i] = n[u];
-        s.rq_s[i] = n[u];
-        s.rq_fu[i] = kNone;
-        if (!probe && !bq[u]) s.rq_cid[i] = cid[u];
-      }
-    }
-    int64_t tot;
-    const int64_t ex = block_excl_scan<int64_t>((ts << 32) | tn, &tot);
-    int64_t pb = carry + (ex & 0xFFFFFFFFll), sb = scarry + (ex >> 32);
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      if (i < R) {
-        s.rq_pbase[i] = (int32_t)pb;
-        s.rq_sbase[i] = (int32_t)sb;
-        for (int j = 0; j < ns[u]; ++j)
-          if (sb + j < s.max_segments) s.seg_req[sb + j] = (uint32_t)i;
-      }
-      pb += n[u];
-      sb += ns[u];
-    }
-    carry += tot & 0xFFFFFFFFll;
-    scarry += tot >> 32;
+  for (int i = threadIdx.x; i < R; i += blockDim.x) {
+    const int64_t o0 = s.in_offsets[i], o1 = s.in_offsets[i + 1];
+    const int g = s.in_group[i];
+    bool bad = o1 < o0 || g < 0 || g >= s.G || (o1 - o0) / s.bs > (int64_t)kMaxPos;
+    if (s.in_contract) bad |= s.in_contract[i] < 0 || s.in_contract[i] >= s.C;
+    if (s.in_prefix) bad |= s.in_prefix[i] == 0;
+    if (bad) atomicOr(&s_bad, 1);
   }
-  bad = __syncthreads_or(bad);
+  __syncthreads();
   int32_t st = PS_OK;
   const int64_t T = R > 0 ? s.in_offsets[R] : 0;
   if (!probe && c->sticky != PS_OK) st = c->sticky;
   else if (!probe && s.now < c->t_prev) st = PS_ERR_CLOCK;
   else if (!probe && c->step > kMaxStep) st = PS_ERR_CAPACITY;
-  else if (bad || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens || carry > s.max_blocks) st = PS_ERR_INVALID_ARG;
+  else if (s_bad || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens) st = PS_ERR_INVALID_ARG;
+  if (st != PS_OK) {
+    __syncthreads();
+    if (threadIdx.x == 0) { c->status = st; c->nblocks = 0; c->nsegs = 0; }
+    return;
+  }
+  int32_t carry = 0, scarry = 0;
+  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
+    const int i = t0 + threadIdx.x;
+    int32_t n = 0, nseg = 0;
+    if (i < R) {
+      n = (int32_t)((s.in_offsets[i + 1] - s.in_offsets[i]) / s.bs);
+      nseg = (n + kSegBlocks - 1) / kSegBlocks;
+      s.rq_n[i] = n;
+      s.rq_h[i] = n;
+      s.rq_s[i] = n;
+      s.rq_fu[i] = kNone;
+      if (!probe) s.rq_cid[i] = s.in_contract ? s.in_contract[i] : s.contract_of_group[s.in_group[i]];
+    }
+    int32_t tot, stot;
+    const int32_t ex = block_excl_scan(n, &tot);
+    const int32_t sex = block_excl_scan(nseg, &stot);
+    if (i < R) {
+      s.rq_pbase[i] = carry + ex;
+      s.rq_sbase[i] = scarry + sex;
+      for (int j = 0; j < nseg; ++j) s.seg_req[scarry + sex + j] = (uint32_t)i;
+    }
+    carry += tot;
+    scarry += stot;
+  }
   if (threadIdx.x == 0) {
-    c->status = st;
-    c->T = st == PS_OK ? T : 0;
-    c->nblocks = st == PS_OK ? carry : 0;
-    c->nsegs = st == PS_OK ? scarry : 0;
-    if (!probe && st == PS_OK) {
+    c->status = PS_OK;
+    c->T = T;
+    c->nblocks = carry;
+    c->nsegs = scarry;
+    if (!probe) {
       c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
       c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
       c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
@@ -400,7 +363,7 @@ __global__ void __launch_bounds__(512) k_validate(DevState s, int probe) {
       c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
     }
   }
-  if (st == PS_OK && !probe && s.policy == PS_STATICQUOTA)
+  if (!probe && s.policy == PS_STATICQUOTA)
     for (int g = threadIdx.x; g < s.G; g += blockDim.x) s.grp_pinned[g] = 0;
 }
 
@@ -716,7 +679,7 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
 // Stage 3: grant new blocks against the pool.  avail = free + unpinned
 // resident = N - pinned; claims are ranked in (request, position) order; the
 // first avail ranks are materialized.  One CTA.
-__global__ void __launch_bounds__(512) k_grant(DevState s) {
+__global__ void __launch_bounds__(1024) k_grant(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
@@ -724,46 +687,23 @@ __global__ void __launch_bounds__(512) k_grant(DevState s) {
   const bool quota = s.policy == PS_STATICQUOTA;  // a_i already granted per group
   const int64_t avail = s.N - c->pinned;
   int64_t carry_c = 0, carry_a = 0;
-  // each thread takes kPer consecutive requests: one scan of the claims and
-  // one of the grants place kPer * blockDim requests
-  constexpr int kPer = 8;
-  for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
-    const int i0 = base + (int)threadIdx.x * kPer;
-    int32_t cl[kPer], qa[kPer];
-    int64_t mine_c = 0;
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      cl[u] = i < R ? s.rq_n[i] - s.rq_s[i] : 0;
-      qa[u] = (quota && i < R) ? s.rq_a[i] : 0;
-      mine_c += cl[u];
-    }
-    int64_t tot_c;
-    int64_t cb = carry_c + block_excl_scan<int64_t>(mine_c, &tot_c);
-    int32_t a[kPer];
-    int64_t mine_a = 0;
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      a[u] = 0;
-      if (i < R) a[u] = quota ? qa[u] : (int32_t)tmin<int64_t>(cl[u], tmax<int64_t>(0, avail - cb));
-      cb += cl[u];
-      mine_a += a[u];
-    }
-    int64_t tot_a;
-    int64_t ab = carry_a + block_excl_scan<int64_t>(mine_a, &tot_a);
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      if (i < R) {
-        // granted keys are paired with the allocated ids in (request,
-        // position) order: request i's first granted key is the ab-th
-        s.rq_cbase[i] = (int32_t)ab;
-        s.rq_a[i] = a[u];
-        s.out.admitted_blocks[i] = a[u];
-        s.out.admitted_offsets[i] = (int32_t)ab;
-      }
-      ab += a[u];
+  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
+    const int i = t0 + threadIdx.x;
+    int32_t cl = 0;
+    if (i < R) cl = s.rq_n[i] - s.rq_s[i];
+    int32_t tot_c;
+    const int32_t ex_c = block_excl_scan(cl, &tot_c);
+    int32_t a = 0;
+    if (i < R) a = quota ? s.rq_a[i] : (int32_t)tmin<int64_t>(cl, tmax<int64_t>(0, avail - (carry_c + ex_c)));
+    int32_t tot_a;
+    const int32_t ex_a = block_excl_scan(a, &tot_a);
+    if (i < R) {
+      // granted keys are paired with the allocated ids in (request, position)
+      // order: request i's first granted key is the (carry_a + ex_a)-th
+      s.rq_cbase[i] = (int32_t)(carry_a + ex_a);
+      s.rq_a[i] = a;
+      s.out.admitted_blocks[i] = a;
+      s.out.admitted_offsets[i] = (int32_t)(carry_a + ex_a);
     }
     carry_c += tot_c;
     carry_a += tot_a;
@@ -2288,7 +2228,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
   mark(0);
-  PS_LAUNCH(k_validate<<<1, 512, 0, st>>>(s, 0));
+  PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s, 0));
   mark(1);
   if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
   ++launches;
@@ -2298,7 +2238,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
   mark(3);
   if (s.policy == PS_STATICQUOTA) PS_LAUNCH(k_grant_quota<<<s.G, 1024, 0, st>>>(s));
-  PS_LAUNCH(k_grant<<<1, 512, 0, st>>>(s));
+  PS_LAUNCH(k_grant<<<1, 1024, 0, st>>>(s));
   PS_LAUNCH(k_instep<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_instep_fin<<<rgrid, 256, 0, st>>>(s));
   mark(4);
@@ -2400,7 +2340,7 @@ int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* 
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
   DevState p = s;
   p.args = nullptr;  // the probe's kernels take every argument by value
-  k_validate<<<1, 512, 0, st>>>(p, 1);
+  k_validate<<<1, 1024, 0, st>>>(p, 1);
   if (s.R > 0) {
     if (launch_hash(p, st) != PS_OK) return PS_ERR_INVALID_ARG;
     k_keys_lookup<<<pgrid, kThreads, 0, st>>>(p);
