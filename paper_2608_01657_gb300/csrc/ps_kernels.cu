@@ -189,12 +189,13 @@ __device__ uint32_t table_find(const DevState& s, uint64_t key, uint32_t g) {
   uint32_t b = table_home(key, g, s.tb_nbuckets_log2);
   for (uint32_t it = 0; it <= mask; ++it) {
     const uint4* e = reinterpret_cast<const uint4*>(s.table + (size_t)b * kTableWays);
+    const uint32_t ovf = __ldg(s.table_ovf + b);  // issued with the bucket: a miss needs no second trip
 #pragma unroll
     for (int w = 0; w < kTableWays; ++w) {
       const uint4 raw = __ldg(e + w);
       if (raw.z != kNone && raw.x == (uint32_t)key && raw.y == (uint32_t)(key >> 32) && raw.w == g) return raw.z;
     }
-    if (__ldg(s.table_ovf + b) == 0) return kNone;
+    if (ovf == 0) return kNone;
     b = (b + 1) & mask;
   }
   return kNone;
@@ -395,8 +396,8 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
 // composition of affine maps, so a warp scan gives every block its chain
 // value relative to the segment start (B_m, with the value before the segment
 // taken as 0).  A decoupled look-back over the request's earlier segments
-// gives the value entering the segment; the warp then finishes its blocks'
-// keys and probes the table for them (n_cached of Alg. 1).
+// gives the value entering the segment, and the warp finishes its blocks'
+// keys; k_lookup probes the table for them.
 template <int PPB>
 struct HashCfg {
   static constexpr int BS = 2 * PPB;
@@ -602,25 +603,36 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
     st_relaxed_u64(st, add61(mul61(A, cin), carry) | (2ull << 61));
   }
   cin = __shfl_sync(kFull, cin, 0);
-  // Keys, then the longest cached prefix (n_cached of Alg. 1): each block's
-  // table probe; the request's first miss is its h_i.
-  uint32_t first_miss = kNone;
+  // the blocks' keys: key_m = mix(C_m ^ (m+1) c), C_m = Kc^(k+1) C_in + B_m
 #pragma unroll
   for (int cc = 0; cc < kChunks; ++cc) {
     const int k = cc * 32 + lane;
     const int m = m0 + k;
     if (m < m1) {
       const uint64_t C = add61(mul61(s.kc_pow[k + 1], cin), Bv[cc]);
-      const uint64_t key = fix_reserved(mix64(C ^ ((uint64_t)(m + 1) * 0xD1B54A32D192ED03ull)));
-      s.pos_key[pbase + m] = key;
+      s.pos_key[pbase + m] = fix_reserved(mix64(C ^ ((uint64_t)(m + 1) * 0xD1B54A32D192ED03ull)));
       s.pos_req[pbase + m] = i;
-      const uint32_t blk = table_find(s, key, g);
-      s.pos_blk[pbase + m] = blk;
-      if (blk == kNone) first_miss = tmin(first_miss, (uint32_t)m);
     }
   }
-  first_miss = __reduce_min_sync(kFull, first_miss);
-  if (lane == 0 && first_miss != kNone) atomicMin(reinterpret_cast<uint32_t*>(s.rq_h) + i, first_miss);
+}
+
+// Stage 2: the longest cached prefix (n_cached of Alg. 1), thread per
+// position: a table probe; a miss lowers the request's h_i to its position
+// (one atomic per request per warp).
+__global__ void __launch_bounds__(kThreads) k_lookup(DevState s) {
+  s = with_args(s);
+  const Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+  PosRef r;
+  const bool valid = pos_ref(s, pos, &r);
+  bool miss = false;
+  if (valid) {
+    const uint32_t blk = table_find(s, s.pos_key[pos], (uint32_t)s.in_group[r.i]);
+    s.pos_blk[pos] = blk;
+    miss = blk == kNone;
+  }
+  agg_min_u32(reinterpret_cast<uint32_t*>(s.rq_h), valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, miss);
 }
 
 // Stage 2 (cont.): blocks of the cached prefix are pinned for the step;
@@ -2283,6 +2295,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(1);
   if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
   ++launches;
+  PS_LAUNCH(k_lookup<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
   mark(2);
   PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
@@ -2390,7 +2403,10 @@ int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* 
   DevState p = s;
   p.args = nullptr;  // the probe's kernels take every argument by value
   k_validate<<<1, 1024, 0, st>>>(p, 1);
-  if (s.R > 0 && launch_hash(p, st) != PS_OK) return PS_ERR_INVALID_ARG;
+  if (s.R > 0) {
+    if (launch_hash(p, st) != PS_OK) return PS_ERR_INVALID_ARG;
+    k_lookup<<<grid_for(s.max_blocks, kThreads, 1 << 30), kThreads, 0, st>>>(p);
+  }
   k_probe_out<<<rgrid, 256, 0, st>>>(p, out, status);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
