@@ -214,7 +214,8 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.pos_key = cv.take<uint64_t>(B);
   t.pos_req = cv.take<uint32_t>(B);
   t.seg_req = cv.take<uint32_t>((size_t)d.max_segments);
-  t.seg_state = cv.take<uint64_t>((size_t)d.max_segments);
+  t.seg_cin = cv.take<uint64_t>((size_t)d.max_segments);
+  t.seg_tot = cv.take<uint64_t>((size_t)d.max_segments);
   t.pos_blk = cv.take<uint32_t>(B);
   t.pos_claim = cv.take<uint32_t>(B);
   t.pos_elig = cv.take<uint8_t>(B);

@@ -90,7 +90,6 @@ struct Ctl {
   uint32_t ticket;         // last-block-done counter for the radix passes and the split
   int32_t nlaunch;         // kernels launched by the step (conditional bodies run or not)
   int32_t wide_nrows;      // segments counted by the last first-digit pass
-  unsigned long long hash_ticket;  // next segment a hashing warp takes
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
 };
 
@@ -202,7 +201,8 @@ struct DevState {
   uint64_t* pos_key;       // chain partial, then the block key
   uint32_t* pos_req;       // request of the position
   uint32_t* seg_req;       // request of each hashing segment
-  uint64_t* seg_state;     // look-back word: value | kind << 61 (1 aggregate, 2 inclusive)
+  uint64_t* seg_cin;       // chain value entering the segment
+  uint64_t* seg_tot;       // local chain value at the segment's end
   uint32_t* pos_blk;       // resident block hit by lookup (or kNone)
   uint32_t* pos_claim;     // claim-map slot (or kNone)
   uint8_t* pos_elig;       // touch was promotion-eligible

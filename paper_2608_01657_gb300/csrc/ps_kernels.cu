@@ -117,15 +117,6 @@ __device__ __forceinline__ void agg_min_u32(uint32_t* base, uint32_t i, uint32_t
   const uint32_t m = __reduce_min_sync(peers, v);
   if (lane_id() == __ffs(peers) - 1) atomicMin(base + i, m);
 }
-// Relaxed device-scope accesses of one 64-bit word (polled across warps).
-__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p) {
-  uint64_t v;
-  asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
-  return v;
-}
-__device__ __forceinline__ void st_relaxed_u64(uint64_t* p, uint64_t v) {
-  asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
-}
 __device__ __forceinline__ uint64_t ldcg_u64(const uint64_t* p) { return __ldcg(reinterpret_cast<const unsigned long long*>(p)); }
 __device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
 
@@ -354,10 +345,7 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
     if (i < R) {
       s.rq_pbase[i] = carry + ex;
       s.rq_sbase[i] = scarry + sex;
-      for (int j = 0; j < nseg; ++j) {
-        s.seg_req[scarry + sex + j] = (uint32_t)i;
-        s.seg_state[scarry + sex + j] = 0;  // nothing published yet
-      }
+      for (int j = 0; j < nseg; ++j) s.seg_req[scarry + sex + j] = (uint32_t)i;
     }
     carry += tot;
     scarry += stot;
@@ -367,7 +355,6 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
     c->T = T;
     c->nblocks = carry;
     c->nsegs = scarry;
-    c->hash_ticket = 0;
     if (!probe) {
       c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
       c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
@@ -395,9 +382,7 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
 // routed to lane = block.  The chain C_m = Kc C_{m-1} + D_m (mod 2^61-1) is a
 // composition of affine maps, so a warp scan gives every block its chain
 // value relative to the segment start (B_m, with the value before the segment
-// taken as 0).  A decoupled look-back over the request's earlier segments
-// gives the value entering the segment, and the warp finishes its blocks'
-// keys; k_lookup probes the table for them.
+// taken as 0); k_keys_lookup then folds in the true value entering it.
 template <int PPB>
 struct HashCfg {
   static constexpr int BS = 2 * PPB;
@@ -418,14 +403,10 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
   using Cfg = HashCfg<PPB>;
   constexpr int BS = Cfg::BS;
   constexpr int G32 = 32 / PPB;
-  Ctl* c = s.ctl;
+  const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int warp = threadIdx.x >> 5, lane = lane_id();
-  // segments are handed out in ticket order, so every segment a warp waits
-  // for below belongs to a warp that is already running
-  unsigned long long tk = 0;
-  if (lane == 0) tk = atomicAdd(&c->hash_ticket, 1ull);
-  const int64_t seg = (int64_t)__shfl_sync(kFull, tk, 0);
+  const int64_t seg = (int64_t)blockIdx.x * Cfg::kWarps + warp;
   if (seg >= c->nsegs) return;
   int32_t* buf = smem_tokens + warp * Cfg::kWindow;
   uint64_t* mbar = reinterpret_cast<uint64_t*>(smem_tokens + Cfg::kWarps * Cfg::kWindow) + warp;
@@ -469,10 +450,7 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
       return __all_sync(kFull, done != 0);
     };
     if (!wait_copy(1 << 22)) {
-      if (lane == 0) {
-        s.ctl->internal_error = 1;
-        st_relaxed_u64(s.seg_state + seg, 2ull << 61);  // later segments must not wait for it
-      }
+      if (lane == 0) s.ctl->internal_error = 1;
       wait_copy(1 << 22);
       return;
     }
@@ -493,13 +471,7 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
   for (int j = 0; j < 5; ++j) kp[j] = s.kc_pow[1 << j];
   const uint64_t kpl = s.kc_pow[lane + 1];
   uint64_t carry = 0;  // local chain value at the block before the chunk
-  constexpr int kChunks = kSegBlocks / 32;
-  uint64_t Bv[kChunks];  // lane's block of each chunk: chain value relative to the segment start
-#pragma unroll
-  for (int cc = 0; cc < kChunks; ++cc) {
-    const int c0 = m0 + cc * 32;
-    Bv[cc] = 0;
-    if (c0 >= m1) continue;  // warp-uniform
+  for (int c0 = m0; c0 < m1; c0 += 32) {
     const int nb = tmin(32, m1 - c0);
     const int32_t* cb = buf + shift_tok + (c0 - m0) * BS;
     uint64_t d1 = 0, d2 = 0;
@@ -562,64 +534,21 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
       if (lane >= (1 << j)) bb = add61(bb, mul61(kp[j], t));
     }
     const uint64_t B = add61(mul61(kpl, carry), bb);
-    Bv[cc] = B;
+    if (lane < nb) {
+      s.pos_key[pbase + c0 + lane] = B;
+      s.pos_req[pbase + c0 + lane] = i;
+    }
     carry = __shfl_sync(kFull, B, nb - 1);
   }
-  // The chain value entering the segment (decoupled look-back over the
-  // request's earlier segments).  The segment maps x -> Kc^nb x + carry; a
-  // request's first segment starts from the group's seed.  Each segment
-  // publishes its map's constant at once (kind 1), then its outgoing chain
-  // value (kind 2); a later segment composes the constants it meets until it
-  // reaches an outgoing value.  Waits are bounded.
-  const uint32_t g = (uint32_t)s.in_group[i];
-  const int js = m0 / kSegBlocks;
-  uint64_t cin = 0;
-  if (lane == 0) {
-    uint64_t* st = s.seg_state + seg;
-    const uint64_t A = s.kc_pow[m1 - m0];
-    if (js == 0) {
-      cin = red61(chain_seed(s.hash_seed, g));
-    } else {
-      st_relaxed_u64(st, carry | (1ull << 61));
-      const uint64_t Kfull = s.kc_pow[kSegBlocks];  // every earlier segment is full
-      uint64_t accA = 1, accT = 0;                   // maps of the segments walked so far
-      for (int64_t p = seg - 1;; --p) {
-        uint64_t w = 0;
-        int spins = 0;
-        while (((w = ld_relaxed_u64(s.seg_state + p)) >> 61) == 0 && ++spins < (1 << 22)) __nanosleep(32);
-        const uint64_t kind = w >> 61, v = w & kP61;
-        if (kind == 2) {
-          cin = add61(mul61(accA, v), accT);
-          break;
-        }
-        if (kind != 1 || p <= seg - js) {  // timed out, or a first segment without its value
-          c->internal_error = 1;
-          break;
-        }
-        accT = add61(mul61(accA, v), accT);
-        accA = mul61(accA, Kfull);
-      }
-    }
-    st_relaxed_u64(st, add61(mul61(A, cin), carry) | (2ull << 61));
-  }
-  cin = __shfl_sync(kFull, cin, 0);
-  // the blocks' keys: key_m = mix(C_m ^ (m+1) c), C_m = Kc^(k+1) C_in + B_m
-#pragma unroll
-  for (int cc = 0; cc < kChunks; ++cc) {
-    const int k = cc * 32 + lane;
-    const int m = m0 + k;
-    if (m < m1) {
-      const uint64_t C = add61(mul61(s.kc_pow[k + 1], cin), Bv[cc]);
-      s.pos_key[pbase + m] = fix_reserved(mix64(C ^ ((uint64_t)(m + 1) * 0xD1B54A32D192ED03ull)));
-      s.pos_req[pbase + m] = i;
-    }
-  }
+  if (lane == 0) s.seg_tot[seg] = carry;
 }
 
-// Stage 2: the longest cached prefix (n_cached of Alg. 1), thread per
-// position: a table probe; a miss lowers the request's h_i to its position
-// (one atomic per request per warp).
-__global__ void __launch_bounds__(kThreads) k_lookup(DevState s) {
+// Stage 2: block keys and the longest cached prefix (n_cached of Alg. 1),
+// thread per position: C_in = the chain value entering the position's
+// segment (C = Kc^256 C + B_end over the request's earlier segments),
+// key_m = mix(C_m ^ (m+1) c) with C_m = Kc^(k+1) C_in + B_m, then a table
+// probe; a miss lowers the request's h_i to its position.
+__global__ void __launch_bounds__(kThreads) k_keys_lookup(DevState s) {
   s = with_args(s);
   const Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
@@ -628,10 +557,19 @@ __global__ void __launch_bounds__(kThreads) k_lookup(DevState s) {
   const bool valid = pos_ref(s, pos, &r);
   bool miss = false;
   if (valid) {
-    const uint32_t blk = table_find(s, s.pos_key[pos], (uint32_t)s.in_group[r.i]);
+    // chain value entering this position's segment: fold the earlier segments
+    const int64_t sb = s.rq_sbase[r.i];
+    const int js = r.m / kSegBlocks;
+    uint64_t cin = red61(chain_seed(s.hash_seed, s.in_group[r.i]));
+    for (int j = 0; j < js; ++j) cin = add61(mul61(s.kc_pow[kSegBlocks], cin), s.seg_tot[sb + j]);
+    const uint64_t C = add61(mul61(s.kc_pow[r.m % kSegBlocks + 1], cin), s.pos_key[pos]);
+    const uint64_t key = fix_reserved(mix64(C ^ ((uint64_t)(r.m + 1) * 0xD1B54A32D192ED03ull)));
+    s.pos_key[pos] = key;
+    const uint32_t blk = table_find(s, key, (uint32_t)s.in_group[r.i]);
     s.pos_blk[pos] = blk;
     miss = blk == kNone;
   }
+  // h_i = the first miss: one atomic per request per warp
   agg_min_u32(reinterpret_cast<uint32_t*>(s.rq_h), valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, miss);
 }
 
@@ -2295,7 +2233,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(1);
   if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
   ++launches;
-  PS_LAUNCH(k_lookup<<<pgrid, kThreads, 0, st>>>(s));
+  PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
   mark(2);
   PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
@@ -2400,12 +2338,13 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
 
 int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* status) {
   const int rgrid = grid_for(s.R, 256, 1 << 20);
+  const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
   DevState p = s;
   p.args = nullptr;  // the probe's kernels take every argument by value
   k_validate<<<1, 1024, 0, st>>>(p, 1);
   if (s.R > 0) {
     if (launch_hash(p, st) != PS_OK) return PS_ERR_INVALID_ARG;
-    k_lookup<<<grid_for(s.max_blocks, kThreads, 1 << 30), kThreads, 0, st>>>(p);
+    k_keys_lookup<<<pgrid, kThreads, 0, st>>>(p);
   }
   k_probe_out<<<rgrid, 256, 0, st>>>(p, out, status);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;

@@ -29,7 +29,7 @@ constexpr size_t kOffCtl = 0;
 constexpr size_t kOffRq = align256(kOffCtl + sizeof(Ctl));
 constexpr size_t kRqArrays = 6;  // n, h, s, fu, pbase, sbase
 constexpr size_t kOffSeg = align256(kOffRq + kRqArrays * align256(4 * kNaMaxRequests));
-constexpr size_t kOffPos = align256(kOffSeg + align256(4 * kNaMaxSegments) + align256(8 * kNaMaxSegments));
+constexpr size_t kOffPos = align256(kOffSeg + align256(4 * kNaMaxSegments) + 2 * align256(8 * kNaMaxSegments));
 constexpr size_t kScratchBytes = align256(kOffPos + align256(8 * kNaMaxBlocks) + 2 * align256(4 * kNaMaxBlocks));
 
 // The scratch itself (about 2.3 MB).  In host code 'g_probe_scratch' names a
@@ -92,7 +92,8 @@ extern "C" int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_
   s.rq_pbase = reinterpret_cast<int32_t*>(base + kOffRq + 4 * rq);
   s.rq_sbase = reinterpret_cast<int32_t*>(base + kOffRq + 5 * rq);
   s.seg_req = reinterpret_cast<uint32_t*>(base + kOffSeg);
-  s.seg_state = reinterpret_cast<uint64_t*>(base + kOffSeg + align256(4 * kNaMaxSegments));
+  s.seg_cin = reinterpret_cast<uint64_t*>(base + kOffSeg + align256(4 * kNaMaxSegments));
+  s.seg_tot = reinterpret_cast<uint64_t*>(base + kOffSeg + align256(4 * kNaMaxSegments) + align256(8 * kNaMaxSegments));
   s.pos_key = reinterpret_cast<uint64_t*>(base + kOffPos);
   s.pos_req = reinterpret_cast<uint32_t*>(base + kOffPos + align256(8 * kNaMaxBlocks));
   s.pos_blk = reinterpret_cast<uint32_t*>(base + kOffPos + align256(8 * kNaMaxBlocks) + align256(4 * kNaMaxBlocks));
