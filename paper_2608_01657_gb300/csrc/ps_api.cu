@@ -229,6 +229,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.grp_delta = cv.take<int64_t>(G);
   t.grp_x = cv.take<int64_t>(G);
   t.grp_pinned = cv.take<int64_t>(G);
+  t.grp_full = cv.take<uint8_t>(G);
   t.sel = cv.take<SelSeg>(G);
   t.cls = cv.take<ClsRange>(G * kClasses);
   t.hist_bins = cv.take<uint32_t>(G * kRadixBins);

@@ -216,6 +216,7 @@ struct DevState {
   int64_t* grp_delta;      // Eq. 8 decrement
   int64_t* grp_x;          // victims taken from the group in the debt phase (StaticQuota: its overflow)
   int64_t* grp_pinned;     // blocks pinned this step, per group (StaticQuota grants)
+  uint8_t* grp_full;       // the debt phase takes all of the group's candidates
   SelSeg* sel;             // [G] segments
   ClsRange* cls;           // [G * kClasses] candidates per (segment, class)
   uint32_t* hist_bins;     // [G][256] radix histogram

@@ -1261,7 +1261,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   const bool seg = !(s.flags & PS_FLAG_NO_SEGMENTATION);
   const int64_t m = (c->status == PS_OK) ? c->mvict : 0;
   if (m == 0) {
-    for (int g = threadIdx.x; g < G; g += blockDim.x) { s.sel[g].active = 0; s.grp_x[g] = 0; }
+    for (int g = threadIdx.x; g < G; g += blockDim.x) { s.sel[g].active = 0; s.grp_x[g] = 0; s.grp_full[g] = 0; }
     if (threadIdx.x == 0) c->m_fb = 0;
     return;
   }
@@ -1293,12 +1293,16 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   if (pm) atomicMax(reinterpret_cast<unsigned long long*>(&s_pmax), (unsigned long long)pm);
   __syncthreads();
   if (E <= m) {
+    // a group that gives all its candidates needs no select: the split takes
+    // them whole
     for (int g = threadIdx.x; g < G; g += blockDim.x) {
       const int64_t x = items_gt(g, eps);
+      const bool full = x > 0 && x == sQ[g];
       s.grp_x[g] = x;
+      s.grp_full[g] = full ? 1 : 0;
       SelSeg z = s.sel[g];
-      z.rank = x;
-      z.active = x > 0;
+      z.rank = full ? 0 : x;
+      z.active = x > 0 && !full;
       z.incl = 1;
       sel_start_group(s, g, z, seg);
       s.sel[g] = z;
@@ -1376,6 +1380,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
     sel_start_group(s, g, z, seg);
     s.sel[g] = z;
     s.grp_x[g] = xa + (tied ? 1 : 0);
+    s.grp_full[g] = 0;
   }
   above = block_sum(above);
   ntie = block_sum(ntie);
@@ -1704,15 +1709,16 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
         w[k] = make_uint4(0, 0, 0, 0);
     }
   }
-  // the segments' state, once per CTA
+  // the segments' state, once per CTA (s_act: 1 selecting, 2 taken whole)
   __shared__ uint64_t s_pre[PS_MAX_GROUPS], s_msk[PS_MAX_GROUPS];
   __shared__ uint8_t s_act[PS_MAX_GROUPS];
   const int nseg = single ? 1 : s.G;
+  const bool whole = !single && s.policy == PS_PREFIXSHIELD;
   for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
     const SelSeg ss = s.sel[g];
     s_pre[g] = ss.prefix;
     s_msk[g] = ss.mask;
-    s_act[g] = ss.active ? 1 : 0;
+    s_act[g] = (whole && s.grp_full[g]) ? 2 : (ss.active ? 1 : 0);
   }
   __syncthreads();
   int marked = 0;
@@ -1726,7 +1732,9 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
       const int grp = single ? 0 : s.blk_group[b];
       if (key != ~0ull && !(fallback && ((s.bm_victim[b >> 5] >> (b & 31)) & 1))) {
         seg = grp;
-        if (s_act[seg]) {
+        if (s_act[seg] == 2) {
+          v = true;
+        } else if (s_act[seg]) {
           const uint64_t k = key & s_msk[seg];
           v = k < s_pre[seg];
           to_list = k == s_pre[seg];
