@@ -38,7 +38,7 @@ WORKLOAD = ("scale: 64 groups (8 victim, 8 attacker, 48 benign chat), pool 1,048
             "block_size 16, 4096 requests/step")
 CONFIG_INDEX = 4
 STAGES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
-          "freetake_evict", "id_lists", "insert", "commit")
+          "take_lists", "evict", "insert", "commit")
 
 
 def parse_args():

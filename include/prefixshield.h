@@ -239,8 +239,8 @@ int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_t num_reque
 /* Profiling hook.  When enabled, ps_step() records a CUDA event on its
  * stream before each of its PS_NUM_STAGES stages and after the last one:
  *   0 validate, 1 hash + lookup, 2 claims + orphans, 3 grant + in-step hits,
- *   4 metering, 5 touch + gate, 6 victim selection, 7 free-take + eviction,
- *   8 id lists, 9 insertion, 10 commit.
+ *   4 metering, 5 touch + gate, 6 victim selection, 7 free-take + id lists,
+ *   8 eviction, 9 insertion, 10 commit.
  * Creating the events is the only work; no device memory is allocated. */
 #define PS_NUM_STAGES 11
 int32_t ps_set_stage_timing(ps_handle_t* h, int32_t enable);

@@ -35,7 +35,7 @@ EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_st
             "ps_cached_prefix_noalloc", "ps_uses_graph", "ps_set_graph")
 PS_NUM_STAGES = 11
 STAGE_NAMES = ("validate", "hash_lookup", "claims", "grant_instep", "meter", "touch_gate", "select",
-               "freetake_evict", "id_lists", "insert", "commit")
+               "take_lists", "evict", "insert", "commit")
 
 
 class PsParams(C.Structure):

@@ -221,7 +221,6 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.pos_elig = cv.take<uint8_t>(B);
   t.claims = cv.take<ClaimEntry>((size_t)kClaimWays << d.cl_log2);
   t.bm_victim = cv.take<uint32_t>((size_t)d.nwords);
-  t.bm_alloc = cv.take<uint32_t>((size_t)d.nwords);
   t.bm_inval = cv.take<uint32_t>((size_t)d.nwords);
   t.csk = cv.take<uint64_t>(N);
   t.grp_qsize = cv.take<int64_t>(G);
@@ -243,7 +242,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.lst_key = cv.take<uint64_t>(N);
   t.lst_blk = cv.take<uint32_t>(N);
   t.lst_seg = cv.take<uint16_t>(N);
-  t.bm_chunk_cnt = cv.take<int32_t>(3 * (((size_t)d.nwords + kBmChunk - 1) / kBmChunk));
+  t.bm_chunk_cnt = cv.take<int32_t>(3 * (((size_t)d.nwords + kBmChunk - 1) / kBmChunk));  // free, evicted, invalidated
   StepArgs* step_args = cv.take<StepArgs>(1);
   // staging for ps_step_host
   int32_t* st_group = cv.take<int32_t>(R);

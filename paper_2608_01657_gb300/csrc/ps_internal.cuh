@@ -208,7 +208,6 @@ struct DevState {
   uint8_t* pos_elig;       // touch was promotion-eligible
   ClaimEntry* claims;
   uint32_t* bm_victim;     // per-step bitmaps over block ids
-  uint32_t* bm_alloc;
   uint32_t* bm_inval;
   uint64_t* csk;           // candidate sort keys (~0 = not a candidate)
   int64_t* grp_qsize;      // candidates per group

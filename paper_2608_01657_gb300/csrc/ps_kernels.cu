@@ -1177,9 +1177,8 @@ __device__ __forceinline__ void sel_start_group(const DevState& s, int g, SelSeg
 // the debt phase of prefixshield left, in (class, stamp) order (Eq. 9).  The
 // debt phase took group g's x_g smallest keys, so of class k it took
 // clamp(x_g - (members of lower classes), 0, members of class k).
-__global__ void __launch_bounds__(32) k_sel_single(DevState s, int fallback) {
-  s = with_args(s);
-  Ctl* c = s.ctl;
+// One warp: the segment-0 state of a global select (lru, or the fallback).
+__device__ void start_global_select(const DevState& s, Ctl* c, int fallback) {
   const int lane = lane_id();
   int64_t m = 0;
   if (c->status == PS_OK) m = fallback ? c->m_fb : c->mvict;
@@ -1221,6 +1220,10 @@ __global__ void __launch_bounds__(32) k_sel_single(DevState s, int fallback) {
   sel_start_cls(z, cnt, lo, hi, segmented);
   s.sel[0] = z;
   c->lst_n = 0;
+}
+__global__ void __launch_bounds__(32) k_sel_single(DevState s, int fallback) {
+  s = with_args(s);
+  start_global_select(s, s.ctl, fallback);
 }
 
 // StaticQuota: each group reclaims its overflow m_g from its own blocks, in
@@ -1811,11 +1814,17 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, in
   __shared__ int s_nrows;
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
+  // the debt phase's last launch also starts the fallback's select (the
+  // groups' final take counts are known here)
+  const bool start_fb = !single && !long_list && s.policy == PS_PREFIXSHIELD;
   if (single && !s.sel[0].active) return;
   const int nseg = single ? 1 : s.G;
   const int64_t n = c->lst_n;
   const bool small = n <= kFinCap;
-  if (small == (long_list != 0)) return;  // the other launch's list
+  if (small == (long_list != 0)) {  // the other launch's list
+    if (start_fb && (threadIdx.x >> 5) == 0) start_global_select(s, c, 1);
+    return;
+  }
   const int warp = threadIdx.x >> 5, lane = lane_id();
   for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
     const SelSeg v = list_view(s.sel[g]);
@@ -1925,6 +1934,10 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, in
       s.sel[g] = v;
     }
   }
+  if (start_fb) {
+    __syncthreads();  // every reader of segment 0's state is done
+    if ((threadIdx.x >> 5) == 0) start_global_select(s, c, 1);
+  }
 }
 
 // Mark a long list's victims (multi-CTA): keys below (or at, if incl) their
@@ -1946,93 +1959,89 @@ __global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
   }
 }
 
-// TakeTrueFree (Alg. 2): the ftake smallest free block ids (one CTA,
-// contiguous word ranges per thread).  With the victims they form the
-// allocated set; the id-list compaction takes their union.
-__global__ void __launch_bounds__(1024) k_freetake(DevState s) {
-  s = with_args(s);
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK || c->ftake == 0) return;
-  const int64_t ftake = c->ftake;
-  const int64_t nw = s.nwords;
-  const int64_t per = (nw + blockDim.x - 1) / blockDim.x;
-  const int64_t w0 = tmin<int64_t>(nw, threadIdx.x * per), w1 = tmin<int64_t>(nw, w0 + per);
-  auto free_word = [&](int64_t w) -> uint32_t {
-    uint32_t f = ~s.res_bits[w];
-    const int64_t hi = (w + 1) * 32;
-    if (hi > s.N) f &= (1u << (uint32_t)(32 - (hi - s.N))) - 1u;
-    return f;
-  };
-  int64_t cnt = 0;
-  if (ftake > 0)
-    for (int64_t w = w0; w < w1; ++w) cnt += __popc(free_word(w));
-  int64_t tot;
-  int64_t before = block_excl_scan(cnt, &tot);
-  for (int64_t w = w0; w < w1; ++w) {
-    uint32_t take = 0;
-    if (ftake > 0 && before < ftake) {
-      uint32_t f = free_word(w);
-      while (f && before < ftake) {
-        const uint32_t lsb = f & (0u - f);
-        take |= lsb;
-        f ^= lsb;
-        ++before;
-      }
-    }
-    s.bm_alloc[w] = take;
-  }
+// TakeTrueFree (Alg. 2) and the step's id lists (allocated, evicted,
+// invalidated), all ascending, from the bitmaps.  Each CTA owns kBmChunk
+// bitmap words.  Pass 1 counts each chunk's free, evicted and invalidated
+// ids.  Pass 2: the ftake smallest free ids are taken greedily from low ids,
+// so a chunk takes min(ftake, free before it + its own) - min(ftake, free
+// before it) of its free ids, its lowest ones; with the victims they form the
+// allocated set, whose ids become resident.
+__device__ __forceinline__ uint32_t free_word(const DevState& s, int64_t w) {
+  uint32_t f = ~s.res_bits[w];
+  const int64_t hi = (w + 1) * 32;
+  if (hi > s.N) f &= (1u << (uint32_t)(32 - (hi - s.N))) - 1u;
+  return f;
 }
-
-// Bitmaps -> ascending id lists (allocated, evicted, invalidated).  Each CTA
-// owns kBmChunk bitmap words; pass 1 counts, pass 2 scans the counts and writes.
 __global__ void __launch_bounds__(kBmChunk) k_bm_count(DevState s) {
   s = with_args(s);
-  if (s.ctl->status != PS_OK) return;
+  const Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
   const int64_t w = (int64_t)blockIdx.x * kBmChunk + threadIdx.x;
-  const uint32_t* bms[3] = {s.bm_alloc, s.bm_victim, s.bm_inval};
   const int nchunks = gridDim.x;
-  for (int k = 0; k < 3; ++k) {
-    uint32_t bits = w < s.nwords ? bms[k][w] : 0u;
-    if (k == 0 && w < s.nwords) {
-      bits |= s.bm_victim[w];
-      s.res_bits[w] |= bits;  // every allocated id is resident after the step
-    }
-    const int v = __popc(bits);
-    const int t = block_sum(v);
-    if (threadIdx.x == 0) s.bm_chunk_cnt[k * nchunks + blockIdx.x] = t;
+  const bool in = w < s.nwords;
+  const int nv = in ? __popc(s.bm_victim[w]) : 0;
+  const int ni = in ? __popc(s.bm_inval[w]) : 0;
+  const int nf = (in && c->ftake > 0) ? __popc(free_word(s, w)) : 0;
+  const int tv = block_sum(nv), ti = block_sum(ni), tf = block_sum(nf);
+  if (threadIdx.x == 0) {
+    s.bm_chunk_cnt[0 * nchunks + blockIdx.x] = tf;
+    s.bm_chunk_cnt[1 * nchunks + blockIdx.x] = tv;
+    s.bm_chunk_cnt[2 * nchunks + blockIdx.x] = ti;
   }
 }
 __global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
   s = with_args(s);
-  if (s.ctl->status != PS_OK) return;
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
   const int64_t w = (int64_t)blockIdx.x * kBmChunk + threadIdx.x;
-  uint32_t* bms[3] = {s.bm_alloc, s.bm_victim, s.bm_inval};
-  int32_t* outs[3] = {s.out.admitted_ids, s.out.evicted_ids, s.out.invalidated_ids};
   const int nchunks = gridDim.x;
+  const bool in = w < s.nwords;
+  const int64_t ftake = c->ftake;
+  // earlier chunks: free, evicted and invalidated ids
+  int64_t fb = 0, vb = 0, ib = 0;
+  for (int j = threadIdx.x; j < (int)blockIdx.x; j += blockDim.x) {
+    fb += s.bm_chunk_cnt[0 * nchunks + j];
+    vb += s.bm_chunk_cnt[1 * nchunks + j];
+    ib += s.bm_chunk_cnt[2 * nchunks + j];
+  }
+  fb = block_sum(fb);
+  vb = block_sum(vb);
+  ib = block_sum(ib);
+  const int64_t take_here = tmin(ftake, fb + s.bm_chunk_cnt[blockIdx.x]) - tmin(ftake, fb);
+  // this word's taken free ids: the chunk's lowest take_here free ids
+  uint32_t f = (in && take_here > 0) ? free_word(s, w) : 0u;
+  int64_t ftot;
+  int64_t fl = block_excl_scan<int64_t>(__popc(f), &ftot);
+  uint32_t taken = 0;
+  while (f && fl < take_here) {
+    const uint32_t lsb = f & (0u - f);
+    taken |= lsb;
+    f ^= lsb;
+    ++fl;
+  }
+  const uint32_t vic = in ? s.bm_victim[w] : 0u, inv = in ? s.bm_inval[w] : 0u;
+  const uint32_t alloc = taken | vic;
+  if (in) s.res_bits[w] |= alloc;  // every allocated id is resident after the step
+  const uint32_t bitsk[3] = {alloc, vic, inv};
+  const int64_t basek[3] = {vb + tmin(ftake, fb), vb, ib};
+  int32_t* outs[3] = {s.out.admitted_ids, s.out.evicted_ids, s.out.invalidated_ids};
+#pragma unroll
   for (int k = 0; k < 3; ++k) {
-    int base = 0;
-    for (int j = threadIdx.x; j < blockIdx.x; j += blockDim.x) base += s.bm_chunk_cnt[k * nchunks + j];
-    base = block_sum(base);
-    uint32_t bits = w < s.nwords ? bms[k][w] : 0u;
-    if (k == 0 && w < s.nwords) {
-      bits |= s.bm_victim[w];
-      s.res_bits[w] |= bits;  // every allocated id is resident after the step
-    }
-    int tot;
-    const int ex = block_excl_scan(__popc(bits), &tot);
-    int o = base + ex;
-    uint32_t b = bits;
-    while (b) {
-      const int j = __ffs(b) - 1;
-      b &= b - 1;
-      if (o < s.max_blocks) outs[k][o] = (int32_t)(w * 32 + j);
+    int64_t tot;
+    const int64_t ex = block_excl_scan<int64_t>(__popc(bitsk[k]), &tot);
+    int64_t o = basek[k] + ex;
+    for (uint32_t b = bitsk[k]; b; b &= b - 1) {
+      if (o < s.max_blocks) outs[k][o] = (int32_t)(w * 32 + __ffs(b) - 1);
       ++o;
     }
-    if (w < s.nwords) bms[k][w] = 0;
     if (blockIdx.x == nchunks - 1 && threadIdx.x == 0) {
-      if (k == 0) s.ctl->n_alloc = base + tot;
-      if (k == 1) s.ctl->n_evicted = base + tot;
+      if (k == 0) c->n_alloc = basek[0] + tot;
+      if (k == 1) c->n_evicted = basek[1] + tot;
     }
+  }
+  if (in) {
+    s.bm_victim[w] = 0;
+    s.bm_inval[w] = 0;
   }
 }
 
@@ -2311,8 +2320,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
         return PS_ERR_CUDA;
       f = cap->aux;
     }
-    PS_LAUNCH(k_sel_single<<<1, 32, 0, f>>>(s, 1));
-    select(f, 1, 1, conds, h_fb_long, conds ? cap->aux2 : f);
+    select(f, 1, 1, conds, h_fb_long, conds ? cap->aux2 : f);  // started by the debt phase's finish
     if (!cond_ok) return PS_ERR_CUDA;
     if (conds && !cond_close(cap->aux)) return PS_ERR_CUDA;
   } else if (s.policy == PS_STATICQUOTA) {
@@ -2327,11 +2335,10 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
     PS_LAUNCH(launch_s3_evict(s, st));
   }
   mark(7);
-  PS_LAUNCH(k_freetake<<<1, 1024, 0, st>>>(s));
-  mark(8);
   const int nchunks = (int)((s.nwords + kBmChunk - 1) / kBmChunk);
   PS_LAUNCH(k_bm_count<<<nchunks, kBmChunk, 0, st>>>(s));
   PS_LAUNCH(k_bm_write<<<nchunks, kBmChunk, 0, st>>>(s));
+  mark(8);
   PS_LAUNCH(k_evict<<<pgrid, kThreads, 0, st>>>(s));
   mark(9);
   PS_LAUNCH(k_insert<<<pgrid, kThreads, 0, st>>>(s));
