@@ -144,8 +144,10 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   // native table: 8-way buckets at load <= 1/2
   d.tb_log2 = log2_pow2_at_least((uint64_t)((N + 3) / 4 > 1 ? (N + 3) / 4 : 1));
   if (d.tb_log2 < 1) d.tb_log2 = 1;
-  // claim map: 4-way buckets, capacity >= 2 x blocks of a step
-  d.cl_log2 = log2_pow2_at_least((uint64_t)(d.max_blocks / 2 > 1 ? d.max_blocks / 2 : 1));
+  // claim map: 4-way buckets, at least one slot per block of a step (load <=
+  // 1 even if every block of a full step is new; about a quarter of that in
+  // typical steps)
+  d.cl_log2 = log2_pow2_at_least((uint64_t)(d.max_blocks / 4 > 1 ? d.max_blocks / 4 : 1));
   if (d.cl_log2 < 1) d.cl_log2 = 1;
   d.hist_log2 = log2_pow2_at_least((uint64_t)(2 * (P->history_capacity + max_requests)));
   if (d.hist_log2 < 1) d.hist_log2 = 1;
