@@ -199,13 +199,20 @@ __device__ uint32_t table_insert(const DevState& s, uint64_t key, uint32_t g, ui
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
   uint32_t b = table_home(key, g, s.tb_nbuckets_log2);
   for (uint32_t it = 0; it <= mask; ++it) {
-    for (int w = 0; w < kTableWays; ++w) {
-      TableEntry* e = s.table + (size_t)b * kTableWays + w;
-      if (ldcg_u32(&e->blk) == kNone && atomicCAS(&e->blk, kNone, blk) == kNone) {
-        e->key = key;
-        e->grp = g;
+    // the bucket's occupancy in one round of loads; then CAS the first free
+    // way (a lost race marks that way taken and moves on)
+    TableEntry* e = s.table + (size_t)b * kTableWays;
+    uint32_t occ = 0;
+#pragma unroll
+    for (int w = 0; w < kTableWays; ++w) occ |= (ldcg_u32(&e[w].blk) != kNone ? 1u : 0u) << w;
+    while (occ != (1u << kTableWays) - 1) {
+      const int w = __ffs(~occ) - 1;
+      if (atomicCAS(&e[w].blk, kNone, blk) == kNone) {
+        e[w].key = key;
+        e[w].grp = g;
         return (b * kTableWays + w) | (it ? kDisplaced : 0u);
       }
+      occ |= 1u << w;
     }
     atomicAdd(s.table_ovf + b, 1u);
     b = (b + 1) & mask;
@@ -232,19 +239,25 @@ __device__ uint32_t claim_insert(const DevState& s, uint64_t key, uint32_t req) 
   const uint32_t mask = (1u << s.cl_nbuckets_log2) - 1;
   uint32_t b = claim_home(key, s.cl_nbuckets_log2);
   for (uint32_t it = 0; it <= mask; ++it) {
+    // the bucket's keys in one round of loads.  Keys only arrive during a
+    // step, each in the first free way, so walking the ways in order with a
+    // CAS on each free one meets the key wherever another thread put it.
+    ClaimEntry* e = s.claims + (size_t)b * kClaimWays;
+    uint64_t cur[kClaimWays];
+#pragma unroll
+    for (int w = 0; w < kClaimWays; ++w) cur[w] = ldcg_u64(&e[w].key);
+#pragma unroll
     for (int w = 0; w < kClaimWays; ++w) {
-      ClaimEntry* e = s.claims + (size_t)b * kClaimWays + w;
-      uint64_t cur = ldcg_u64(&e->key);
-      if (cur == 0)
-        cur = atomicCAS(reinterpret_cast<unsigned long long*>(&e->key), 0ull, (unsigned long long)key);
-      if (cur == 0 || cur == key) {
-        atomicMin(&e->minreq, req);
+      uint64_t v = cur[w];
+      if (v == 0) v = atomicCAS(reinterpret_cast<unsigned long long*>(&e[w].key), 0ull, (unsigned long long)key);
+      if (v == 0 || v == key) {
+        atomicMin(&e[w].minreq, req);
         return b * kClaimWays + w;
       }
     }
     b = (b + 1) & mask;
   }
-  return kNone;  // unreachable: the map is sized for twice the blocks of a step
+  return kNone;  // unreachable: the map has a slot for every block of a step
 }
 
 // ---- block state changes -----------------------------------------------------
