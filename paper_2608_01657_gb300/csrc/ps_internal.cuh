@@ -279,20 +279,29 @@ struct CaptureCtx {
   cudaStream_t aux2;  // bodies of conditional nodes inside those
 };
 
-// Copy the call's arguments from device memory into the kernel's DevState.
+// Copy the call's arguments from device memory into the kernel's DevState,
+// then wait for the preceding kernel of the step.  Step kernels are launched
+// with programmatic stream serialization, so a kernel's CTAs may already be
+// resident while its predecessor runs: every kernel passes this wait before it
+// reads or writes any state, and then lets its own successor be scheduled.
+// The argument block itself is written only by the host before the step.
+// Without that launch attribute both instructions are no-ops.
 __device__ __forceinline__ DevState with_args(DevState s) {
   const StepArgs* a = s.args;
-  if (a == nullptr) return s;  // launched directly with its arguments by value
-  if (blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(&s.ctl->nlaunch, 1);
-  s.now = a->now;
-  s.R = a->R;
-  s.tokens_aligned16 = a->tokens_aligned16;
-  s.in_group = a->in_group;
-  s.in_offsets = a->in_offsets;
-  s.in_tokens = a->in_tokens;
-  s.in_contract = a->in_contract;
-  s.in_prefix = a->in_prefix;
-  s.out = a->out;
+  if (a != nullptr) {
+    s.now = a->now;
+    s.R = a->R;
+    s.tokens_aligned16 = a->tokens_aligned16;
+    s.in_group = a->in_group;
+    s.in_offsets = a->in_offsets;
+    s.in_tokens = a->in_tokens;
+    s.in_contract = a->in_contract;
+    s.in_prefix = a->in_prefix;
+    s.out = a->out;
+  }
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  if (a != nullptr && blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(&s.ctl->nlaunch, 1);
   return s;
 }
 // The host-side argument block of a DevState.

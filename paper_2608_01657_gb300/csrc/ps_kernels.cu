@@ -2206,6 +2206,24 @@ void configure_kernels(const DevState& s) {
   cudaFuncSetAttribute(k_hash<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<32>::kSmem);
 }
 
+// Launch with programmatic stream serialization: the kernel may be scheduled
+// while its predecessor finishes (its CTAs wait in with_args until the
+// predecessor's writes are visible), hiding the gap between dependent kernels.
+template <typename... KArgs, typename... Args>
+static void launch_k(void (*kernel)(KArgs...), int grid, int block, size_t smem, cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3((unsigned)block);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // Under stream capture: append an 'if' conditional node to the graph being
 // captured on st, and start capturing its body on aux.  Returns false (and
 // the capture then fails as a whole) if any step is refused.
@@ -2259,27 +2277,27 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
   mark(0);
-  PS_LAUNCH(k_validate<<<1, 1024, 0, st>>>(s, 0));
+  PS_LAUNCH(launch_k(k_validate, 1, 1024, 0, st, s, 0));
   mark(1);
   if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
   ++launches;
   PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
   mark(2);
-  PS_LAUNCH(k_claims<<<pgrid, kThreads, 0, st>>>(s));
+  PS_LAUNCH(launch_k(k_claims, pgrid, kThreads, 0, st, s));
   mark(3);
-  if (s.policy == PS_STATICQUOTA) PS_LAUNCH(k_grant_quota<<<s.G, 1024, 0, st>>>(s));
-  PS_LAUNCH(k_grant<<<1, 1024, 0, st>>>(s));
-  PS_LAUNCH(k_instep<<<pgrid, kThreads, 0, st>>>(s));
-  PS_LAUNCH(k_instep_fin<<<rgrid, 256, 0, st>>>(s));
+  if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
+  PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
+  PS_LAUNCH(launch_k(k_instep, pgrid, kThreads, 0, st, s));
+  PS_LAUNCH(launch_k(k_instep_fin, rgrid, 256, 0, st, s));
   mark(4);
-  PS_LAUNCH(k_meter<<<s.G, 512, 0, st>>>(s));
+  PS_LAUNCH(launch_k(k_meter, s.G, 512, 0, st, s));
   mark(5);
-  PS_LAUNCH(k_touch<<<pgrid, kThreads, 0, st>>>(s));
-  PS_LAUNCH(k_touch2<<<pgrid, kThreads, 0, st>>>(s));
+  PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, st, s));
+  PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, st, s));
   mark(6);
   const int cand_smem = (s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA ? s.G : 1) * kClasses * 5 * 4;
-  if (s.policy != PS_S3FIFO) PS_LAUNCH(k_cand<<<grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, st>>>(s));
+  if (s.policy != PS_S3FIFO) PS_LAUNCH(launch_k(k_cand, grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, st, s));
   // Under capture, phases that many steps skip become conditional bodies:
   // the long-list passes of a select, and the global fallback of Alg. 2.
   cudaGraphConditionalHandle h_fb = 0, h_long = 0;
@@ -2304,22 +2322,22 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   // on the auxiliary stream outside a capture would run)
   auto select = [&](cudaStream_t q, int single, int fallback, bool cond, cudaGraphConditionalHandle hl,
                     cudaStream_t body) {
-    PS_LAUNCH(k_wide_pass<<<cgrid, 256, 0, q>>>(s, single, fallback));
-    PS_LAUNCH(k_wide_resolve<<<single ? 1 : s.G, 32, 0, q>>>(s, single));
-    PS_LAUNCH(k_split<<<cgrid, 256, 0, q>>>(s, single, fallback, hl, cond ? 1 : 0));
+    PS_LAUNCH(launch_k(k_wide_pass, cgrid, 256, 0, q, s, single, fallback));
+    PS_LAUNCH(launch_k(k_wide_resolve, single ? 1 : s.G, 32, 0, q, s, single));
+    PS_LAUNCH(launch_k(k_split, cgrid, 256, 0, q, s, single, fallback, hl, cond ? 1 : 0));
     cudaStream_t b = q;
     if (cond) {
       if (!cond_open(q, body, hl)) { cond_ok = false; return; }
       b = body;
     }
-    for (int d = 0; d < 7; ++d) PS_LAUNCH(k_digit_pass<<<lgrid, 256, radix_smem, b>>>(s, single, fallback, 1));
-    PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, b>>>(s, single, 1));
-    PS_LAUNCH(k_mark_list<<<lgrid, 256, 0, b>>>(s, single));
+    for (int d = 0; d < 7; ++d) PS_LAUNCH(launch_k(k_digit_pass, lgrid, 256, radix_smem, b, s, single, fallback, 1));
+    PS_LAUNCH(launch_k(k_list_finish, 1, 1024, kFinSmem, b, s, single, 1));
+    PS_LAUNCH(launch_k(k_mark_list, lgrid, 256, 0, b, s, single));
     if (cond && !cond_close(body)) { cond_ok = false; return; }
-    PS_LAUNCH(k_list_finish<<<1, 1024, kFinSmem, q>>>(s, single, 0));
+    PS_LAUNCH(launch_k(k_list_finish, 1, 1024, kFinSmem, q, s, single, 0));
   };
   if (s.policy == PS_PREFIXSHIELD) {
-    PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s, h_fb, conds ? 1 : 0));
+    PS_LAUNCH(launch_k(k_waterfill, 1, 1024, 0, st, s, h_fb, conds ? 1 : 0));
     select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
     cudaStream_t f = st;
@@ -2337,11 +2355,11 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
     if (!cond_ok) return PS_ERR_CUDA;
     if (conds && !cond_close(cap->aux)) return PS_ERR_CUDA;
   } else if (s.policy == PS_STATICQUOTA) {
-    PS_LAUNCH(k_quota_sel<<<1, 1024, 0, st>>>(s));
+    PS_LAUNCH(launch_k(k_quota_sel, 1, 1024, 0, st, s));
     select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
   } else if (s.policy == PS_LRU) {
-    PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));
+    PS_LAUNCH(launch_k(k_sel_single, 1, 32, 0, st, s, 0));
     select(st, 1, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
   } else {
@@ -2349,15 +2367,15 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   }
   mark(7);
   const int nchunks = (int)((s.nwords + kBmChunk - 1) / kBmChunk);
-  PS_LAUNCH(k_bm_count<<<nchunks, kBmChunk, 0, st>>>(s));
-  PS_LAUNCH(k_bm_write<<<nchunks, kBmChunk, 0, st>>>(s));
+  PS_LAUNCH(launch_k(k_bm_count, nchunks, kBmChunk, 0, st, s));
+  PS_LAUNCH(launch_k(k_bm_write, nchunks, kBmChunk, 0, st, s));
   mark(8);
-  PS_LAUNCH(k_evict<<<pgrid, kThreads, 0, st>>>(s));
+  PS_LAUNCH(launch_k(k_evict, pgrid, kThreads, 0, st, s));
   mark(9);
-  PS_LAUNCH(k_insert<<<pgrid, kThreads, 0, st>>>(s));
+  PS_LAUNCH(launch_k(k_insert, pgrid, kThreads, 0, st, s));
   if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));
   mark(10);
-  PS_LAUNCH(k_finalize<<<1, 32, 0, st>>>(s));
+  PS_LAUNCH(launch_k(k_finalize, 1, 32, 0, st, s));
   mark(11);
 #undef PS_LAUNCH
   if (tr) tr->launches = launches;
