@@ -22,7 +22,7 @@ from typing import Dict, Iterator, List, Optional, Sequence
 import numpy as np
 
 VOCAB = 32000
-_TAGS = {"labels": 1, "hot": 2, "fresh": 3, "atk": 4, "sys": 5, "conv": 6, "emit": 7, "pick": 8, "fuzz": 9}
+_TAGS = {"labels": 1, "hot": 2, "fresh": 3, "atk": 4, "sys": 5, "conv": 6, "emit": 7, "pick": 8, "fuzz": 9, "burst": 10}
 
 
 def _rng(seed: int, tag: str, *ids: int) -> np.random.Generator:
@@ -290,6 +290,57 @@ class LowAndSlow(Workload):
         return _pack(s, groups, pieces)
 
 
+class DelayedReplay(Workload):
+    """Delayed replay (the debt-gate ablation of Sec. V-D), one group per
+    contract of Sec. V-A: victim (group 0, critical 64/256), attacker
+    (group 1, best-effort 16/128), neutral (group 2, standard 40/192).
+
+    * steps 0-2: the victim admits three 1536-token hot prefixes (96 blocks
+      each); steps 3-5 replay them, so they are proven and promoted;
+    * step 6 (tick 7): the attacker bursts two fresh 1536-token prompts,
+      192 blocks against a 128-block bucket: 64 blocks of debt, cleared by
+      refill at tick 7 + ceil(64 / 16) = 11;
+    * ``wait`` empty steps, then the attacker replays both prompts (tick
+      8 + wait): every one of the 192 blocks is replay-eligible, gated while
+      debt is outstanding (wait 0 or 1, the half-clearance point), promoted
+      from wait 3 on (the designed clearance time);
+    * ``pressure`` steps of neutral pressure: the neutral group sends one
+      fresh 1536-token prompt, then the victim sends hot prefix k % 3.
+    The pool holds 511 blocks, so the attack fits without eviction and the
+    pressure steps reclaim."""
+
+    VICTIM, ATTACKER, NEUTRAL = 0, 1, 2
+    HOT, LEN = 3, 1536
+    BURST_STEP = 6
+
+    def __init__(self, spec, seed, wait=0, pressure=4):
+        super().__init__(spec, seed)
+        self.hot = [_tokens(_rng(seed, "hot", 0, j), self.LEN) for j in range(self.HOT)]
+        self.atk = [_tokens(_rng(seed, "burst", 1, j), self.LEN) for j in range(2)]
+        self.wait, self.pressure = int(wait), int(pressure)
+        self.replay_step = self.BURST_STEP + 1 + self.wait
+
+    @property
+    def num_steps(self) -> int:
+        return self.replay_step + 1 + self.pressure
+
+    def steps(self, count: Optional[int] = None) -> Iterator[Step]:
+        n = self.num_steps if count is None else min(count, self.num_steps)
+        for s in range(n):
+            yield self.make_step(s)
+
+    def make_step(self, s: int) -> Step:
+        if s < 2 * self.HOT:
+            return _pack(s, [self.VICTIM], [[self.hot[s % self.HOT]]])
+        if s == self.BURST_STEP or s == self.replay_step:
+            return _pack(s, [self.ATTACKER] * 2, [[a] for a in self.atk])
+        if s < self.replay_step:
+            return _pack(s, [], [])
+        k = s - self.replay_step - 1
+        fresh = _Fresh(self.seed, s, self.LEN)
+        return _pack(s, [self.NEUTRAL, self.VICTIM], [[fresh.take(self.LEN)], [self.hot[k % self.HOT]]])
+
+
 def _lognormal_2048(r):
     return _lognormal_len(r, np.log(2048.0), 0.5, 256, 8192)
 
@@ -311,13 +362,20 @@ CONFIGS = {
                     contract_of_group=(0, 1),
                     description="victim: 4 hot 1536-token prefixes in rotation + 32 fresh, one a step; "
                                 "attacker: one fresh 1536-token prompt every third step; 511 usable blocks"),
+    6: WorkloadSpec("delayed replay", 3, 511, 16, 2, 18, rho=(64, 40, 16), beta=(256, 192, 128),
+                    contract_of_group=(0, 2, 1),
+                    description="victim admits and replays 3 hot 1536-token prefixes; attacker bursts 192 "
+                                "blocks into 64 blocks of debt, waits, replays them; then 4 steps of neutral "
+                                "pressure (one fresh 1536-token prompt) with victim re-requests; 511 blocks"),
 }
 
 
 def make_workload(config: int, seed: int = 1, requests_per_step: Optional[int] = None,
-                  total_requests: Optional[int] = None) -> Workload:
-    """The seeded trace of one configuration (0..5).  ``requests_per_step``
-    overrides the batch size (e.g. the discriminative 8-request variants)."""
+                  total_requests: Optional[int] = None, wait: int = 0) -> Workload:
+    """The seeded trace of one configuration (0..6).  ``requests_per_step``
+    overrides the batch size (e.g. the discriminative 8-request variants);
+    ``wait`` is the delayed-replay trace's number of empty steps between the
+    attacker's burst and its replay."""
     spec = CONFIGS[config]
     if requests_per_step is not None or total_requests is not None:
         spec = dataclasses.replace(
@@ -339,6 +397,8 @@ def make_workload(config: int, seed: int = 1, requests_per_step: Optional[int] =
         return Scale(spec, seed)
     if config == 5:
         return LowAndSlow(spec, seed)
+    if config == 6:
+        return DelayedReplay(spec, seed, wait=wait)
     raise KeyError(config)
 
 

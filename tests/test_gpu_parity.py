@@ -115,6 +115,21 @@ def test_parity_configs(policy, cfg, nsteps, rps):
     _run(gpu, orc, steps, state_every=10, label=f"cfg{cfg}/{policy}")
 
 
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+@pytest.mark.parametrize("wait,flags", [(0, 0), (0, O.FLAG_NO_DEBT_GATE), (1, 0), (3, 0), (3, O.FLAG_NO_DEBT_GATE),
+                                        (0, O.FLAG_NO_SEGMENTATION)])
+def test_parity_delayed_replay(policy, wait, flags):
+    """The delayed-replay trace with three contracts (critical, standard,
+    best-effort): burst into debt, gated or ungated replay, neutral pressure."""
+    wl = W.make_workload(6, seed=4, wait=wait)
+    sp = wl.spec
+    steps = list(wl.steps())
+    kw = dict(rho=sp.rho, beta=sp.beta, contract_of_group=list(sp.contract_of_group), flags=flags)
+    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, kw,
+                     max_requests=sp.requests_per_step, max_tokens=2 * 1536)
+    _run(gpu, orc, steps, label=f"cfg6/w{wait}/f{flags}/{policy}")
+
+
 def test_parity_alg2_ties():
     """Groups with equal debt and equal decrements force Eq. 7's tie rule."""
     G = 6
