@@ -12,113 +12,14 @@
 
 #include <vector>
 
-#include "ps_internal.cuh"
+#include "ps_device.cuh"
+#include "ps_launch.cuh"
 
 namespace ps {
 
-constexpr unsigned kFull = 0xFFFFFFFFu;
-constexpr int kThreads = 256;     // position-parallel kernels
 constexpr int kRadixSmemRows = 48;  // radix rows counted in shared memory (48 KB)
 constexpr int kFinCap = 8192;  // split lists up to this size are finished by one CTA in shared memory
 constexpr int kFinRows = 32;   // rows k_list_finish counts at once (32 KB)
-
-// ---------------------------------------------------------------------------
-// small device helpers
-__device__ __forceinline__ int lane_id() { return threadIdx.x & 31; }
-template <typename T>
-__device__ __forceinline__ T tmin(T a, T b) { return a < b ? a : b; }
-template <typename T>
-__device__ __forceinline__ T tmax(T a, T b) { return a < b ? b : a; }
-
-template <typename T>
-__device__ __forceinline__ T warp_incl_scan(T v) {
-  const int lane = lane_id();
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    T n = __shfl_up_sync(kFull, v, o);
-    if (lane >= o) v += n;
-  }
-  return v;
-}
-template <typename T>
-__device__ __forceinline__ T warp_sum(T v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
-  return v;
-}
-
-// Exclusive scan across the CTA (blockDim a multiple of 32).  Returns the
-// thread's exclusive prefix and writes the CTA total to *total.
-template <typename T>
-__device__ T block_excl_scan(T v, T* total) {
-  __shared__ T wsum[32];
-  const int lane = lane_id(), warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  T incl = warp_incl_scan(v);
-  if (lane == 31) wsum[warp] = incl;
-  __syncthreads();
-  if (warp == 0) {
-    T w = lane < nw ? wsum[lane] : T(0);
-    T wi = warp_incl_scan(w);
-    __syncwarp();
-    wsum[lane] = wi;
-  }
-  __syncthreads();
-  T base = warp ? wsum[warp - 1] : T(0);
-  *total = wsum[nw - 1];
-  __syncthreads();
-  return base + incl - v;
-}
-template <typename T>
-__device__ T block_sum(T v) {
-  T tot;
-  block_excl_scan(v, &tot);
-  return tot;
-}
-
-__device__ __forceinline__ void atomic_add_i64(int64_t* p, int64_t v) {
-  atomicAdd(reinterpret_cast<unsigned long long*>(p), static_cast<unsigned long long>(v));
-}
-__device__ __forceinline__ int64_t* stat_ptr(const DevState& s, int g, int k) {
-  return s.stats + (int64_t)g * PS_NUM_STATS + k;
-}
-// Add v to stat k of group g, combining lanes of the warp with equal g.
-__device__ __forceinline__ void agg_stat(const DevState& s, uint32_t g, int k, int64_t v, bool active) {
-  const bool on = active && v != 0;
-  const unsigned act = __ballot_sync(kFull, on);
-  if (!on) return;
-  const unsigned peers = __match_any_sync(act, g);
-  int64_t sum = 0;
-  for (unsigned m = peers; m; m &= m - 1) sum += __shfl_sync(peers, v, __ffs(m) - 1);
-  if (lane_id() == __ffs(peers) - 1) atomic_add_i64(stat_ptr(s, (int)g, k), sum);
-}
-// Warp-aggregated increment of bins[idx] for the lanes with 'active'.
-__device__ __forceinline__ void agg_inc(uint32_t* bins, uint32_t idx, bool active) {
-  const unsigned act = __ballot_sync(kFull, active);
-  if (!active) return;
-  const unsigned peers = __match_any_sync(act, idx);
-  if (lane_id() == __ffs(peers) - 1) atomicAdd(bins + idx, (uint32_t)__popc(peers));
-}
-// base[i] += v, lanes of the warp with equal i combined first (every lane of
-// the warp must call it).
-__device__ __forceinline__ void agg_add_i64(int64_t* base, uint32_t i, int64_t v, bool active) {
-  const unsigned act = __ballot_sync(kFull, active);
-  if (!active) return;
-  const unsigned peers = __match_any_sync(act, i);
-  int64_t sum = 0;
-  for (unsigned m = peers; m; m &= m - 1) sum += __shfl_sync(peers, v, __ffs(m) - 1);
-  if (lane_id() == __ffs(peers) - 1) atomicAdd(reinterpret_cast<unsigned long long*>(base + i), (unsigned long long)sum);
-}
-// atomicMin of v into base[i], lanes of the warp with equal i combined first
-// (every lane of the warp must call it).
-__device__ __forceinline__ void agg_min_u32(uint32_t* base, uint32_t i, uint32_t v, bool active) {
-  const unsigned act = __ballot_sync(kFull, active);
-  if (!active) return;
-  const unsigned peers = __match_any_sync(act, i);
-  const uint32_t m = __reduce_min_sync(peers, v);
-  if (lane_id() == __ffs(peers) - 1) atomicMin(base + i, m);
-}
-__device__ __forceinline__ uint64_t ldcg_u64(const uint64_t* p) { return __ldcg(reinterpret_cast<const unsigned long long*>(p)); }
-__device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
 
 // 128-bit compare-and-swap (sm_90+): installs the (p, group) identity of a
 // history entry atomically, so two requests of one (group, prefix) that race
@@ -2204,55 +2105,6 @@ void configure_kernels(const DevState& s) {
   cudaFuncSetAttribute(k_hash<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<8>::kSmem);
   cudaFuncSetAttribute(k_hash<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<16>::kSmem);
   cudaFuncSetAttribute(k_hash<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<32>::kSmem);
-}
-
-// Launch with programmatic stream serialization: the kernel may be scheduled
-// while its predecessor finishes (its CTAs wait in with_args until the
-// predecessor's writes are visible), hiding the gap between dependent kernels.
-template <typename... KArgs, typename... Args>
-static void launch_k(void (*kernel)(KArgs...), int grid, int block, size_t smem, cudaStream_t st, Args... args) {
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3((unsigned)block);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
-}
-
-// Under stream capture: append an 'if' conditional node to the graph being
-// captured on st, and start capturing its body on aux.  Returns false (and
-// the capture then fails as a whole) if any step is refused.
-static bool cond_open(cudaStream_t st, cudaStream_t aux, cudaGraphConditionalHandle h, cudaGraph_t* body_out = nullptr) {
-  cudaStreamCaptureStatus cs;
-  cudaGraph_t g = nullptr;
-  const cudaGraphNode_t* deps = nullptr;
-  size_t nd = 0;
-  if (cudaStreamGetCaptureInfo(st, &cs, nullptr, &g, &deps, nullptr, &nd) != cudaSuccess ||
-      cs != cudaStreamCaptureStatusActive)
-    return false;
-  std::vector<cudaGraphNode_t> dv(deps, deps + nd);
-  cudaGraphNodeParams p{};
-  p.type = cudaGraphNodeTypeConditional;
-  p.conditional.handle = h;
-  p.conditional.type = cudaGraphCondTypeIf;
-  p.conditional.size = 1;
-  cudaGraphNode_t node;
-  const bool ok = cudaGraphAddNode(&node, g, dv.data(), nullptr, nd, &p) == cudaSuccess &&
-                  cudaStreamUpdateCaptureDependencies(st, &node, nullptr, 1, cudaStreamSetCaptureDependencies) ==
-                      cudaSuccess &&
-                  cudaStreamBeginCaptureToGraph(aux, p.conditional.phGraph_out[0], nullptr, nullptr, 0,
-                                                cudaStreamCaptureModeThreadLocal) == cudaSuccess;
-  if (ok && body_out) *body_out = p.conditional.phGraph_out[0];
-  return ok;
-}
-static bool cond_close(cudaStream_t aux) {
-  cudaGraph_t body = nullptr;
-  return cudaStreamEndCapture(aux, &body) == cudaSuccess;
 }
 
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const CaptureCtx* cap) {
