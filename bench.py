@@ -55,6 +55,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch the step kernel by kernel (profilers cannot see inside its graph)")
+    ap.add_argument("--queues", action="store_true",
+                    help="select victims from the indexed per-(group, class) queues instead of candidate scans")
     return ap.parse_args()
 
 
@@ -257,7 +259,8 @@ def run_own(args, ws, rank, local):
     for st in steps:
         dsteps.append((st.now, torch.from_numpy(st.groups).to(dev), torch.from_numpy(st.offsets).to(dev),
                        torch.from_numpy(st.tokens).to(dev)))
-    params = B.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20)
+    params = B.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20,
+                      flags=B.PS_FLAG_INDEXED_QUEUES if args.queues else 0)
     cache = B.Cache(spec.capacity_blocks, spec.block_size, spec.num_groups, args.policy, params,
                     max_requests=R, max_tokens=maxT)
     cache.set_stage_timing(True)
@@ -347,7 +350,8 @@ def run_own(args, ws, rank, local):
                    "requests_per_step": R, "block_size": spec.block_size, "capacity_blocks": spec.capacity_blocks,
                    "groups": spec.num_groups, "l2": "flushed (256 MiB write) between timed steps",
                    "parallelism": f"replicas x{ws}",
-                   "launch": "cuda graph" if cache.uses_graph() else "kernel by kernel"},
+                   "launch": "cuda graph" if cache.uses_graph() else "kernel by kernel",
+                   "select": "indexed queues" if args.queues else "candidate scan"},
         "kv_blocks_per_s": blk_all / total_max,
         "step_roofline": {"bound": "hbm", "achieved": step_gbs, "peak": peak, "unit": "GB/s",
                           "frac": step_gbs / peak, "algorithmic_bytes_per_step": alg / args.steps,

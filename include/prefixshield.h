@@ -70,6 +70,13 @@ enum {
 
 #define PS_FLAG_NO_SEGMENTATION 1u /* ablation: victims inside a group by recency only */
 #define PS_FLAG_NO_DEBT_GATE 2u    /* ablation: promote regardless of debt (Eq. 4 off) */
+/* Victim selection from indexed per-(group, class) queues (the indexed
+ * per-group, per-segment queues Sec. VIII proposes) instead of a scan of
+ * every candidate.  Same victims, same results; lru, prefixshield and
+ * staticquota (ignored for s3fifo, which keeps its own queues).  The
+ * workspace grows by two buffers of 8 x (N + max_tokens / block_size)
+ * entries of 12 bytes each, plus per-step scratch. */
+#define PS_FLAG_INDEXED_QUEUES 4u
 
 /* Per-group statistics, int64 each, row-major [num_groups][PS_NUM_STATS]. */
 enum {

@@ -28,6 +28,8 @@ STAT_NAMES = (
 POLICIES = {"lru": 0, "s3fifo": 1, "prefixshield": 2, "staticquota": 3}
 OK, ERR_INVALID_ARG, ERR_CAPACITY, ERR_CLOCK = 0, -1, -2, -3
 FLAG_NO_SEGMENTATION, FLAG_NO_DEBT_GATE = 1, 2
+# the CUDA library's indexed-queue victim selection: same victims, ignored here
+FLAG_INDEXED_QUEUES = 4
 
 
 class OrcParams(C.Structure):

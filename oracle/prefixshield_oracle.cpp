@@ -13,7 +13,8 @@
 //   S0 lazy token-bucket refill            Eq. 1 (evaluated at the step's clock)
 //   S1 chained full-block hashing          Sec. III (native content-hash key)
 //   S2 longest cached prefix lookup        Alg. 1 (n_cached), Sec. II-C namespaces
-//   S3 grant of new blocks against the pool  (batch reading)
+//   S3 grant of new blocks against the pool  (the batch reading of Alg. 1:
+//                                          one Alg. 2 batch per step)
 //   S4 per request, in request order:
 //        OnRequest                          Alg. 1
 //        OnTouch (debt-gated promotion)     Alg. 1, Eq. 4
@@ -24,8 +25,10 @@
 //                                          partitions (staticquota)
 //   S6 eviction, id assignment, insertion
 //
-// Parity status of each function is listed in the design doc; every function below
-// is pinned by a CPU test (tests/test_oracle_*.py).
+// Every function below is pinned by a CPU test (tests/test_oracle_*.py).
+//
+// Flag bit 4 (indexed queues) selects the CUDA library's victim data
+// structure; the victims are the same, so this oracle ignores it.
 
 #include <algorithm>
 #include <cstdint>

@@ -132,6 +132,10 @@ struct Dims {
   uint32_t gh_log2;
   int32_t bs, G, C, max_requests;
   uint32_t tb_log2, cl_log2, hist_log2;
+  // indexed queues
+  bool lg;
+  int32_t lg_L;
+  int64_t lg_P, lg_max_chunks, lg_app_chunks;
 };
 
 Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t max_requests, int64_t max_tokens) {
@@ -158,6 +162,15 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   d.gh_log2 = log2_pow2_at_least((uint64_t)((d.s3_ghost_cap + 3) / 4 > 1 ? (d.s3_ghost_cap + 3) / 4 : 1));
   if (d.gh_log2 < 1) d.gh_log2 = 1;
   d.ghost_ring_cap = 1ull << log2_pow2_at_least((uint64_t)(2 * d.s3_ghost_cap + 64));
+  // indexed queues: at most two live entries a block (its group's log and its
+  // class's global log) and two a position of a step; each buffer holds four
+  // times that, so a compaction leaves at least three quarters free
+  d.lg = (P->flags & PS_FLAG_INDEXED_QUEUES) != 0;
+  d.lg_L = G * kClasses + kClasses;
+  d.lg_P = 2 * 4 * (N + d.max_blocks);
+  d.lg_max_chunks = d.lg_P / kLogChunk + d.lg_L + 2;
+  d.lg_app_chunks = (d.max_blocks + kAppChunk - 1) / kAppChunk;
+  if (d.lg_app_chunks < 1) d.lg_app_chunks = 1;
   return d;
 }
 
@@ -245,6 +258,27 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.lst_blk = cv.take<uint32_t>(N);
   t.lst_seg = cv.take<uint16_t>(N);
   t.bm_chunk_cnt = cv.take<int32_t>(3 * (((size_t)d.nwords + kBmChunk - 1) / kBmChunk));  // free, evicted, invalidated
+  if (d.lg) {
+    const size_t L = (size_t)d.lg_L;
+    t.lg_L = d.lg_L;
+    t.lg_P = d.lg_P;
+    t.lg_max_chunks = d.lg_max_chunks;
+    t.lg_app_chunks = d.lg_app_chunks;
+    t.lg_blk = cv.take<uint32_t>(2 * (size_t)d.lg_P);
+    t.lg_st = cv.take<uint64_t>(2 * (size_t)d.lg_P);
+    t.lg_desc = cv.take<LogDesc>(L);
+    t.lg_new = cv.take<LogDesc>(L);
+    t.lg_live = cv.take<int64_t>(L);
+    t.lg_add = cv.take<int64_t>(L);
+    t.lg_pin = cv.take<int64_t>(L);
+    t.lg_slot = cv.take<uint32_t>(B);
+    t.lg_app = cv.take<uint32_t>(L * (size_t)d.lg_app_chunks);
+    t.lg_tk = cv.take<LogTake>(L);
+    t.lg_c0 = cv.take<int32_t>(L + 1);
+    t.lg_ck = cv.take<uint32_t>((size_t)d.lg_max_chunks);
+    t.lg_ck_out = cv.take<int64_t>((size_t)d.lg_max_chunks);
+    t.lg_tie = cv.take<TieItem>(G);
+  }
   StepArgs* step_args = cv.take<StepArgs>(1);
   // staging for ps_step_host
   int32_t* st_group = cv.take<int32_t>(R);
@@ -373,6 +407,7 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   carve(d, static_cast<char*>(d_workspace), &s, h);
   s.N = capacity_blocks; s.bs = block_size; s.G = num_groups; s.C = params->num_contracts; s.policy = policy;
   s.flags = params->flags; s.fp_shift = params->fp_shift; s.eps = params->epsilon_fp; s.hash_seed = params->hash_seed;
+  s.lg_on = d.lg && policy != PS_S3FIFO;
   s.rho_min = params->rho_fp[0];
   for (int c = 0; c < PS_MAX_CONTRACTS; ++c) {
     s.rho[c] = c < s.C ? params->rho_fp[c] : 1;

@@ -107,4 +107,17 @@ __device__ __forceinline__ void agg_min_u32(uint32_t* base, uint32_t i, uint32_t
 __device__ __forceinline__ uint64_t ldcg_u64(const uint64_t* p) { return __ldcg(reinterpret_cast<const unsigned long long*>(p)); }
 __device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
 
+// ---- indexed queues: which logs hold a block ---------------------------------
+__device__ __forceinline__ bool lg_segmented(const DevState& s) {
+  return s.policy == PS_PREFIXSHIELD && !(s.flags & PS_FLAG_NO_SEGMENTATION);
+}
+// The per-group log (A) and the global log (B) of a block of group g and
+// class k; -1 where the policy keeps no such log.
+__device__ __forceinline__ int32_t lg_log_a(const DevState& s, uint32_t g, uint32_t k) {
+  return s.policy == PS_LRU ? -1 : (int32_t)(g * kClasses + (lg_segmented(s) ? k : 0u));
+}
+__device__ __forceinline__ int32_t lg_log_b(const DevState& s, uint32_t k) {
+  return s.policy == PS_STATICQUOTA ? -1 : (int32_t)((uint32_t)s.G * kClasses + (lg_segmented(s) ? k : 0u));
+}
+
 }  // namespace ps

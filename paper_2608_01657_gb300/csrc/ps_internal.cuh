@@ -91,6 +91,13 @@ struct Ctl {
   int32_t nlaunch;         // kernels launched by the step (conditional bodies run or not)
   int32_t wide_nrows;      // segments counted by the last first-digit pass
   int32_t internal_error;  // an invariant of the step failed (reported, never expected)
+  // indexed queues (PS_FLAG_INDEXED_QUEUES)
+  int32_t lg_buf;          // entry buffer holding the logs (0 or 1)
+  int32_t lg_ntk;          // takes of the select phase in progress
+  int32_t lg_nchunks;      // chunks of the scan in progress
+  int32_t lg_more;         // a take's window ended short of its last victim: another round
+  int32_t lg_cmp;          // a log lacks room for this step's appends: compact first
+  uint32_t lg_ticket;      // last-CTA-done counter of the append and compaction writes
 };
 
 // Per-segment state of the segmented radix select.
@@ -108,6 +115,37 @@ struct __align__(16) SelSeg {
 // of their stamps' top and bottom 32 bits.
 struct ClsRange {
   uint32_t cnt, hmin, hmax, lmin, lmax;
+};
+
+// ---- indexed queues (the per-group, per-segment queues of Sec. VIII) -------
+// Each queue is a log of (block, stamp) entries in stamp order: a block is
+// appended at the end of every step that restamps or admits it, and an entry
+// is live while the block is resident with that stamp.  Logs 3g + k hold
+// group g's blocks of class k; logs 3G + k hold every group's blocks of
+// class k (class 0 only, for all classes, when the policy ignores classes).
+constexpr int kLogChunk = 1024;  // log entries per chunk of a scan
+constexpr int kAppChunk = 256;   // stamps per chunk of the end-of-step append
+constexpr int kMaxLogs = PS_MAX_GROUPS * 3 + 3;
+struct LogDesc {
+  int64_t start, head, tail, end;  // positions in the current entry buffer
+};
+// One log's share of a select phase: consume its first 'want' live entries.
+struct LogTake {
+  int64_t want;      // live entries to consume (with 'tie', the last one is recorded, not taken)
+  int64_t got;       // consumed in earlier rounds
+  int64_t cur;       // where this round's window starts
+  int64_t wend;      // where it ends
+  int64_t cut_rank;  // entries to consume in the cut chunk
+  int32_t log;
+  int32_t tie;       // the last entry is the group's tie candidate (Eq. 7)
+  int32_t cut;       // chunk holding the last entry in this round, or -1
+  int32_t done;      // the last entry was found (this round or earlier)
+};
+struct TieItem {
+  uint64_t key;  // (class, stamp) order key of the tied group's next candidate
+  int64_t pos;   // its position in the log
+  uint32_t blk;
+  int32_t log;
 };
 constexpr int kClasses = 3;
 // The first digit of a select is 16 bits wide while at most kWideRows
@@ -226,6 +264,26 @@ struct DevState {
   uint32_t* lst_blk;
   uint16_t* lst_seg;
   int32_t* bm_chunk_cnt;   // [3][chunks] bitmap compaction counts
+  // indexed queues (allocated only with PS_FLAG_INDEXED_QUEUES)
+  int32_t lg_on;           // victims come from the queues instead of a candidate scan
+  int32_t lg_L;            // logs: 3G + 3
+  int64_t lg_P;            // entries per buffer
+  int64_t lg_max_chunks;   // chunks a scan can span
+  int64_t lg_app_chunks;   // append chunks of the largest step
+  uint32_t* lg_blk;        // [2][P] entries: block
+  uint64_t* lg_st;         // [2][P]          stamp when appended
+  LogDesc* lg_desc;        // [L]
+  LogDesc* lg_new;         // [L] layout after a compaction
+  int64_t* lg_live;        // [L] live entries (candidates)
+  int64_t* lg_add;         // [L] entries this step appends
+  int64_t* lg_pin;         // [L] entries this step's pins take out (applied once the step goes ahead)
+  uint32_t* lg_slot;       // [max_blocks] block holding each stamp of this step
+  uint32_t* lg_app;        // [L][app_chunks] append counts per chunk, then offsets
+  LogTake* lg_tk;          // [L] takes of a select phase
+  int32_t* lg_c0;          // [L + 1] first chunk of each take (or log)
+  uint32_t* lg_ck;         // [max_chunks] live entries per chunk
+  int64_t* lg_ck_out;      // [max_chunks] where a chunk's live entries go (compaction)
+  TieItem* lg_tie;         // [G]
   StepArgs* args;          // this call's arguments (device memory)
   // current step inputs / outputs (kernels refresh them from *args)
   int64_t now;
@@ -317,6 +375,13 @@ inline StepArgs args_of(const DevState& s) {
 void configure_kernels(const DevState& s);
 void launch_init(const DevState& s, cudaStream_t st);
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const CaptureCtx* cap = nullptr);
+// Indexed queues (ps_queues.cu).  The select phases are 0 Alg. 2's debt
+// phase, 1 its global fallback, 2 lru, 3 StaticQuota.
+void launch_queue_init(const DevState& s, cudaStream_t st);
+int32_t launch_queue_cand(const DevState& s, cudaStream_t st, int* launches);
+int32_t launch_queue_select(const DevState& s, cudaStream_t st, const CaptureCtx* cap, int phase, int depth,
+                            int* launches);
+int32_t launch_queue_append(const DevState& s, cudaStream_t st, const CaptureCtx* cap, int* launches);
 // S3-FIFO (ps_s3fifo.cu)
 void launch_s3_evict(const DevState& s, cudaStream_t st);
 void launch_s3_insert(const DevState& s, cudaStream_t st);

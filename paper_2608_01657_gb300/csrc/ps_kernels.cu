@@ -500,7 +500,7 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
   const int64_t nb = c->nblocks;
   const uint32_t step32 = (uint32_t)c->step;
   bool newpin = false;
-  uint32_t pin_group = 0;
+  uint32_t pin_group = 0, pin_klass = 0;
   if (t < nb) {
     PosRef r;
     pos_ref(s, t, &r);
@@ -508,6 +508,7 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
       const uint32_t b = s.pos_blk[t];
       newpin = atomicExch(s.blk_pin + b, step32) != step32;
       pin_group = (uint32_t)s.in_group[r.i];  // the owner: hits are namespaced by group
+      if (newpin && s.lg_on) pin_klass = s.blk_klass[b];
       if (newpin && s.policy == PS_S3FIFO) atomic_add_i64(&c->s3_pinned[(s.blk_flags[b] >> 1) & 1], 1);
       s.pos_claim[t] = kNone;
     } else {
@@ -546,6 +547,11 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
   const int np = __popc(__ballot_sync(kFull, newpin));
   if (lane_id() == 0 && np) atomic_add_i64(&c->pinned, np);
   if (s.policy == PS_STATICQUOTA) agg_add_i64(s.grp_pinned, pin_group, 1, newpin);
+  if (s.lg_on) {  // a pinned block is no candidate: it leaves its queues' live counts (applied in k_lg_cand)
+    const int32_t A = lg_log_a(s, pin_group, pin_klass), B = lg_log_b(s, pin_klass);
+    agg_add_i64(s.lg_pin, (uint32_t)A, 1, newpin && A >= 0);
+    agg_add_i64(s.lg_pin, (uint32_t)B, 1, newpin && B >= 0);
+  }
 }
 
 // Stage 2 (cont.): the first own claim s_i of each request, and orphans.  A
@@ -562,7 +568,7 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   const uint32_t step32 = (uint32_t)c->step;
   bool inv = false;
-  uint32_t ginv = 0;
+  uint32_t ginv = 0, kinv = 0;
   PosRef r;
   bool own = false;
   const bool valid = pos_ref(s, pos, &r);
@@ -573,6 +579,7 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
       const uint32_t b = s.pos_blk[pos];
       if (b != kNone && ldcg_u32(s.blk_pin + b) != step32 && atomicExch(s.blk_inval + b, step32) != step32) {
         ginv = drop_block(s, b);
+        if (s.lg_on) kinv = s.blk_klass[b];
         atomicOr(s.bm_inval + (b >> 5), 1u << (b & 31));
         if (s.policy == PS_S3FIFO) s.s3_inval[atomicAdd(reinterpret_cast<unsigned long long*>(&c->s3_ninval), 1ull)] = b;
         inv = true;
@@ -581,6 +588,11 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
   }
   // s_i = the first own claim: one atomic per request per warp
   agg_min_u32(reinterpret_cast<uint32_t*>(s.rq_s), valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, own);
+  if (s.lg_on) {  // an invalidated block leaves its queues
+    const int32_t A = lg_log_a(s, ginv, kinv), B = lg_log_b(s, kinv);
+    agg_add_i64(s.lg_live, (uint32_t)A, -1, inv && A >= 0);
+    agg_add_i64(s.lg_live, (uint32_t)B, -1, inv && B >= 0);
+  }
   agg_stat(s, ginv, PS_STAT_INVALIDATED_BLOCKS, 1, inv);
   agg_stat(s, ginv, PS_STAT_RESIDENT_BLOCKS, -1, inv);
   const int ni = __popc(__ballot_sync(kFull, inv));
@@ -901,6 +913,7 @@ __global__ void __launch_bounds__(kThreads) k_touch(DevState s) {
     const uint32_t b = s.pos_blk[pos];
     atomicMax(reinterpret_cast<unsigned long long*>(s.blk_stamp + b),
               (unsigned long long)make_stamp(c->stamp_base, s.rq_pbase[i], s.rq_n[i], m));
+    if (s.lg_on) s.lg_slot[s.rq_pbase[i] + (s.rq_n[i] - 1 - m)] = b;  // the queues' append reads it back
     atomicAdd(s.blk_acc + b, 1u);
     atomicAdd(s.blk_freq + b, 1u);
     elig = proven && s.blk_contract[b] == cid && s.blk_prefix[b] == p && s.blk_klass[b] != kReuse;
@@ -2017,6 +2030,7 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
         s.blk_klass[b] = e.promo != kNone ? (uint8_t)kReuse : s.rq_knew[i];
         const uint32_t toucher = e.last ? e.last - 1 : i;  // the last request that touched it
         s.blk_stamp[b] = make_stamp(c->stamp_base, s.rq_pbase[toucher], s.rq_n[toucher], r.m);
+        if (s.lg_on) s.lg_slot[s.rq_pbase[toucher] + (s.rq_n[toucher] - 1 - r.m)] = b;
         s.blk_acc[b] = e.tcnt;
         s.blk_freq[b] = e.tcnt;
         s.blk_flags[b] = 1;
@@ -2074,6 +2088,7 @@ static int grid_for(int64_t items, int threads, int max_ctas) {
 void launch_init(const DevState& s, cudaStream_t st) {
   k_init_blocks<<<grid_for((int64_t)kClaimWays << s.cl_nbuckets_log2, 256, 152 * 8), 256, 0, st>>>(s);
   k_init_ctl<<<1, 1024, 0, st>>>(s);
+  launch_queue_init(s, st);
 }
 
 template <int PPB>
@@ -2149,7 +2164,27 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, st, s));
   mark(6);
   const int cand_smem = (s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA ? s.G : 1) * kClasses * 5 * 4;
-  if (s.policy != PS_S3FIFO) PS_LAUNCH(launch_k(k_cand, grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, st, s));
+  if (s.lg_on) {
+    // indexed queues: the same victims, taken from the queues' heads
+    if (launch_queue_cand(s, st, &launches) != PS_OK) return PS_ERR_CUDA;
+    cudaGraphConditionalHandle hq_fb = 0;
+    if (s.policy == PS_PREFIXSHIELD) {
+      if (cap && !cond_handle(st, &hq_fb)) return PS_ERR_CUDA;
+      PS_LAUNCH(launch_k(k_waterfill, 1, 1024, 0, st, s, hq_fb, cap ? 1 : 0));
+      if (launch_queue_select(s, st, cap, 0, 0, &launches) != PS_OK) return PS_ERR_CUDA;
+      cudaStream_t f = st;
+      if (cap) {
+        if (!cond_open(st, cap->aux, hq_fb)) return PS_ERR_CUDA;
+        f = cap->aux;
+      }
+      if (launch_queue_select(s, f, cap, 1, 1, &launches) != PS_OK) return PS_ERR_CUDA;
+      if (cap && !cond_close(cap->aux)) return PS_ERR_CUDA;
+    } else if (launch_queue_select(s, st, cap, s.policy == PS_LRU ? 2 : 3, 0, &launches) != PS_OK) {
+      return PS_ERR_CUDA;
+    }
+  }
+  if (s.policy != PS_S3FIFO && !s.lg_on)
+    PS_LAUNCH(launch_k(k_cand, grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, st, s));
   // Under capture, phases that many steps skip become conditional bodies:
   // the long-list passes of a select, and the global fallback of Alg. 2.
   cudaGraphConditionalHandle h_fb = 0, h_long = 0;
@@ -2159,7 +2194,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
     cudaGraph_t g = nullptr;
     // a handle that no conditional node uses can make instantiation fail:
     // create only the ones this policy's sequence uses
-    conds = s.policy != PS_S3FIFO;
+    conds = s.policy != PS_S3FIFO && !s.lg_on;
     if (conds &&
         !(cudaStreamGetCaptureInfo(st, &cs, nullptr, &g) == cudaSuccess && cs == cudaStreamCaptureStatusActive &&
           cudaGraphConditionalHandleCreate(&h_long, g, 0, cudaGraphCondAssignDefault) == cudaSuccess &&
@@ -2188,7 +2223,9 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
     if (cond && !cond_close(body)) { cond_ok = false; return; }
     PS_LAUNCH(launch_k(k_list_finish, 1, 1024, kFinSmem, q, s, single, 0));
   };
-  if (s.policy == PS_PREFIXSHIELD) {
+  if (s.lg_on) {
+    // selected above
+  } else if (s.policy == PS_PREFIXSHIELD) {
     PS_LAUNCH(launch_k(k_waterfill, 1, 1024, 0, st, s, h_fb, conds ? 1 : 0));
     select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
@@ -2226,6 +2263,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(9);
   PS_LAUNCH(launch_k(k_insert, pgrid, kThreads, 0, st, s));
   if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));
+  if (s.lg_on && launch_queue_append(s, st, cap, &launches) != PS_OK) return PS_ERR_CUDA;
   mark(10);
   PS_LAUNCH(launch_k(k_finalize, 1, 32, 0, st, s));
   mark(11);

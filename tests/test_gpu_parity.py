@@ -26,8 +26,9 @@ def _pair(N, bs, G, policy, params_kw, max_requests, max_tokens):
     return gpu, orc
 
 
-def _run(gpu, orc, steps, state_every=1, s3=False, label=""):
+def _run(gpu, orc, steps, state_every=1, s3=False, label="", graph=True):
     dev = torch.device("cuda")
+    gpu.set_graph(graph)
     for k, st in enumerate(steps):
         g = torch.from_numpy(st.groups).to(dev)
         o = torch.from_numpy(st.offsets).to(dev)
@@ -36,7 +37,7 @@ def _run(gpu, orc, steps, state_every=1, s3=False, label=""):
         p = None if st.prefixes is None else torch.from_numpy(st.prefixes.view(np.int64)).to(dev)
         rc = gpu.step(st.now, g, o, t, c, p)
         assert rc == 0, f"{label} step {k}: launch rc {rc}"
-        assert gpu.uses_graph(), f"{label} step {k}: the step is not replayed as a graph"
+        assert gpu.uses_graph() == graph, f"{label} step {k}: graph replay is {gpu.uses_graph()}"
         got = gpu.fetch(st.num_requests)
         want = orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts, st.prefixes)
         compare_outputs(got, want, f"{label} step {k}")
@@ -128,6 +129,66 @@ def test_parity_delayed_replay(policy, wait, flags):
     gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, kw,
                      max_requests=sp.requests_per_step, max_tokens=2 * 1536)
     _run(gpu, orc, steps, label=f"cfg6/w{wait}/f{flags}/{policy}")
+
+
+QUEUE_POLICIES = ["lru", "prefixshield", "staticquota"]
+IQ = O.FLAG_INDEXED_QUEUES
+
+
+@pytest.mark.parametrize("policy", QUEUE_POLICIES)
+@pytest.mark.parametrize("seed,N,G,R,contracts,prefixes,flags", [
+    (1, 24, 2, 3, 0, False, 0),
+    (2, 40, 3, 6, 0, False, 0),
+    (3, 64, 4, 8, 3, True, 0),
+    (4, 12, 1, 2, 0, False, 0),
+    (5, 30, 3, 5, 3, True, 1),
+    (6, 30, 3, 5, 3, True, 2),
+    (11, 20, 2, 4, 2, False, 0),
+])
+def test_parity_queues_fuzz(policy, seed, N, G, R, contracts, prefixes, flags):
+    """Victims from the indexed queues over long fuzz traces.  The token
+    bound is the trace's own, so the logs' buffers are small and every log is
+    compacted many times."""
+    steps = W.fuzz_steps(seed, G, R, 240, docs_per_group=3, doc_blocks=7, fresh_max_blocks=2,
+                         with_contracts=contracts, with_prefixes=prefixes, now_stride=2, empty_every=9)
+    kw = dict(rho=(2.0, 1.5, 1.0), beta=(6.0, 5.0, 4.0), flags=flags | IQ, contract_of_group=[g % 3 for g in range(G)])
+    gpu, orc = _pair(N, 16, G, policy, kw, max_requests=R, max_tokens=max(16, max(st.num_tokens for st in steps)))
+    _run(gpu, orc, steps, state_every=7, label=f"queues/fuzz{seed}/{policy}")
+
+
+@pytest.mark.parametrize("policy", QUEUE_POLICIES)
+def test_parity_queues_direct_launches(policy):
+    """The indexed queues launched kernel by kernel (their second scan round
+    and the compaction then run as kernels that find nothing to do)."""
+    steps = W.fuzz_steps(12, 3, 5, 120, docs_per_group=3, doc_blocks=7, fresh_max_blocks=3, empty_every=7)
+    kw = dict(rho=(2.0,), beta=(6.0,), flags=IQ)
+    gpu, orc = _pair(30, 16, 3, policy, kw, max_requests=5, max_tokens=max(st.num_tokens for st in steps))
+    _run(gpu, orc, steps, state_every=5, label=f"queues/direct/{policy}", graph=False)
+
+
+@pytest.mark.parametrize("policy", QUEUE_POLICIES)
+@pytest.mark.parametrize("cfg,nsteps,rps,wait,flags", [(1, 60, 8, 0, 0), (3, 30, None, 0, 0), (5, 120, None, 0, 0),
+                                                       (6, None, None, 0, 0), (6, None, None, 1, 2)])
+def test_parity_queues_configs(policy, cfg, nsteps, rps, wait, flags):
+    wl = W.make_workload(cfg, seed=2, requests_per_step=rps, wait=wait)
+    sp = wl.spec
+    steps = list(wl.steps(nsteps))
+    kw = dict(rho=sp.rho, beta=sp.beta, flags=flags | IQ)
+    if sp.contract_of_group is not None:
+        kw["contract_of_group"] = list(sp.contract_of_group)
+    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, kw,
+                     max_requests=sp.requests_per_step, max_tokens=max(st.num_tokens for st in steps))
+    _run(gpu, orc, steps, state_every=10, label=f"queues/cfg{cfg}/{policy}")
+
+
+def test_parity_queues_alg2_ties():
+    """Eq. 7's tie rule with the tie candidates read from the queues."""
+    G = 6
+    steps = W.fuzz_steps(31, G, 6, 120, docs_per_group=2, doc_blocks=6, fresh_max_blocks=3)
+    for flags in (0, 1):
+        kw = dict(rho=(1.0,), beta=(2.0,), flags=flags | IQ)
+        gpu, orc = _pair(36, 16, G, "prefixshield", kw, max_requests=6, max_tokens=4096)
+        _run(gpu, orc, steps, label=f"queues/ties/f{flags}")
 
 
 def test_parity_alg2_ties():
@@ -223,6 +284,19 @@ def test_parity_scale_full_size(policy):
                      max_requests=spec.requests_per_step, max_tokens=maxT)
     _run(gpu, orc, steps, state_every=4, label=f"scale/{policy}")
     assert orc.stats()[:, O.STAT_NAMES.index("evicted_blocks")].sum() > 0  # reclamation was exercised
+
+
+@pytest.mark.parametrize("policy", ["lru", "prefixshield"])
+def test_parity_queues_scale_full_size(policy):
+    """The benchmarked configuration with victims from the indexed queues:
+    every output of every step and the final state equal the oracle's."""
+    spec, steps = _scale_steps(9)
+    maxT = max(s.num_tokens for s in steps)
+    gpu, orc = _pair(spec.capacity_blocks, spec.block_size, spec.num_groups, policy,
+                     dict(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20, flags=IQ),
+                     max_requests=spec.requests_per_step, max_tokens=maxT)
+    _run(gpu, orc, steps, state_every=4, label=f"queues/scale/{policy}")
+    assert orc.stats()[:, O.STAT_NAMES.index("evicted_blocks")].sum() > 0
 
 
 @pytest.mark.parametrize("policy", GPU_POLICIES)

@@ -2,8 +2,8 @@
 
 * LRU: hand-traced golden trace, and reduction to textbook LRU
   (collections.OrderedDict) when every step carries one single-block request.
-* S3-FIFO: hand-traced golden trace of the published algorithm with the
-  readings listed in the design doc.
+* S3-FIFO: hand-traced golden trace of the published algorithm under the
+  readings of its batch form stated in the trace file's header.
 * PrefixShield: a hand-derived Alg. 2 example where debt directs reclamation
   to the indebted group even though its blocks are newer (Eq. 6-8).
 * Chain release order: a request releases its blocks tail first.
