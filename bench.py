@@ -22,6 +22,7 @@ path).
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import gc
 import json
 import os
@@ -55,6 +56,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-graph", action="store_true",
                     help="launch the step kernel by kernel (profilers cannot see inside its graph)")
+    ap.add_argument("--capacity-blocks", type=int, default=0,
+                    help="pool size override for a scaling measurement (the headline workload's is 1,048,576); "
+                         "give --prefill enough steps to fill it")
     ap.add_argument("--queues", action="store_true",
                     help="select victims from the indexed per-(group, class) queues instead of candidate scans")
     return ap.parse_args()
@@ -253,6 +257,8 @@ def run_own(args, ws, rank, local):
     stream = torch.cuda.current_stream()
     n_total = args.prefill + args.warmup + args.steps
     spec, steps = make_steps(args.seed + rank, n_total)
+    if args.capacity_blocks:
+        spec = dataclasses.replace(spec, capacity_blocks=args.capacity_blocks)
     maxT = max(s.num_tokens for s in steps)
     R = spec.requests_per_step
     dsteps = []
@@ -346,7 +352,9 @@ def run_own(args, ws, rank, local):
         "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": 1e3 * total_max / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "policy": args.policy, "prefill_steps": args.prefill,
+        "config": {"workload": WORKLOAD if not args.capacity_blocks else
+                   WORKLOAD.replace("pool 1,048,576 blocks", f"pool {spec.capacity_blocks:,} blocks"),
+                   "policy": args.policy, "prefill_steps": args.prefill,
                    "requests_per_step": R, "block_size": spec.block_size, "capacity_blocks": spec.capacity_blocks,
                    "groups": spec.num_groups, "l2": "flushed (256 MiB write) between timed steps",
                    "parallelism": f"replicas x{ws}",

@@ -74,7 +74,7 @@ enum {
  * per-group, per-segment queues Sec. VIII proposes) instead of a scan of
  * every candidate.  Same victims, same results; lru, prefixshield and
  * staticquota (ignored for s3fifo, which keeps its own queues).  The
- * workspace grows by two buffers of 8 x (N + max_tokens / block_size)
+ * workspace grows by two buffers of 16 x (N + max_tokens / block_size)
  * entries of 12 bytes each, plus per-step scratch. */
 #define PS_FLAG_INDEXED_QUEUES 4u
 

@@ -163,11 +163,11 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   if (d.gh_log2 < 1) d.gh_log2 = 1;
   d.ghost_ring_cap = 1ull << log2_pow2_at_least((uint64_t)(2 * d.s3_ghost_cap + 64));
   // indexed queues: at most two live entries a block (its group's log and its
-  // class's global log) and two a position of a step; each buffer holds four
-  // times that, so a compaction leaves at least three quarters free
+  // class's global log) and two a position of a step; each buffer holds eight
+  // times that, so a compaction leaves at least seven eighths free
   d.lg = (P->flags & PS_FLAG_INDEXED_QUEUES) != 0;
   d.lg_L = G * kClasses + kClasses;
-  d.lg_P = 2 * 4 * (N + d.max_blocks);
+  d.lg_P = 2 * 8 * (N + d.max_blocks);
   d.lg_max_chunks = d.lg_P / kLogChunk + d.lg_L + 2;
   d.lg_app_chunks = (d.max_blocks + kAppChunk - 1) / kAppChunk;
   if (d.lg_app_chunks < 1) d.lg_app_chunks = 1;

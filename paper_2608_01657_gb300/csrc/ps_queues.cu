@@ -426,25 +426,38 @@ __global__ void __launch_bounds__(kAppChunk) k_lg_app_count(DevState s) {
   for (int l = threadIdx.x; l < s.lg_L; l += blockDim.x) s.lg_app[(int64_t)l * s.lg_app_chunks + q] = hist[l];
 }
 
-// Per log (a warp each): chunk offsets of the appends, their total, and
-// whether the log has room for them.
-__global__ void __launch_bounds__(1024) k_lg_app_scan(DevState s, cudaGraphConditionalHandle hc, int has_cond) {
+// Per log (a CTA each): chunk offsets of the appends, their total, and
+// whether the log has room for them.  Each thread scans a run of
+// consecutive chunks, so the loads of a log's row are all in flight at once.
+constexpr int kScanRun = 16;  // chunk counts a thread holds (up to 4096 x 16 chunks per pass)
+__global__ void __launch_bounds__(256) k_lg_app_scan(DevState s, cudaGraphConditionalHandle hc, int has_cond) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   const int nch = (int)((c->nblocks + kAppChunk - 1) / kAppChunk);
-  const int l = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = lane_id();
-  if (l >= s.lg_L) return;
+  const int l = blockIdx.x;
   uint32_t* row = s.lg_app + (int64_t)l * s.lg_app_chunks;
   uint32_t before = 0;
-  for (int q0 = 0; q0 < nch; q0 += 32) {
-    const int q = q0 + lane;
-    const uint32_t v = q < nch ? row[q] : 0u;
-    const uint32_t incl = warp_incl_scan(v);
-    if (q < nch) row[q] = before + incl - v;
-    before += __shfl_sync(kFull, incl, 31);
+  for (int base = 0; base < nch; base += (int)blockDim.x * kScanRun) {
+    const int q0 = base + threadIdx.x * kScanRun;
+    uint32_t v[kScanRun];
+    uint32_t sum = 0;
+#pragma unroll
+    for (int u = 0; u < kScanRun; ++u) {
+      v[u] = q0 + u < nch ? row[q0 + u] : 0u;
+      sum += v[u];
+    }
+    uint32_t tot;
+    uint32_t run = before + block_excl_scan(sum, &tot);
+#pragma unroll
+    for (int u = 0; u < kScanRun; ++u)
+      if (q0 + u < nch) {
+        row[q0 + u] = run;
+        run += v[u];
+      }
+    before += tot;
   }
-  if (lane == 0) {
+  if (threadIdx.x == 0) {
     s.lg_add[l] = before;
     const LogDesc d = s.lg_desc[l];
     if (d.tail + (int64_t)before > d.end) {
@@ -509,28 +522,46 @@ __global__ void __launch_bounds__(kScanThreads) k_lg_cmp_count(DevState s) {
   }
 }
 
+// Per log (a CTA each): its live entries, and each chunk's offset inside it.
+__global__ void __launch_bounds__(256) k_lg_cmp_live(DevState s) {
+  s = with_args(s);
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK || !c->lg_cmp) return;
+  const int l = blockIdx.x;
+  const int q0 = s.lg_c0[l], q1 = s.lg_c0[l + 1];
+  int64_t before = 0;
+  for (int base = q0; base < q1; base += (int)blockDim.x * kScanRun) {
+    const int qa = base + threadIdx.x * kScanRun;
+    uint32_t v[kScanRun];
+    int64_t sum = 0;
+#pragma unroll
+    for (int u = 0; u < kScanRun; ++u) {
+      v[u] = qa + u < q1 ? s.lg_ck[qa + u] : 0u;
+      sum += v[u];
+    }
+    int64_t tot;
+    int64_t run = before + block_excl_scan(sum, &tot);
+#pragma unroll
+    for (int u = 0; u < kScanRun; ++u)
+      if (qa + u < q1) {
+        s.lg_ck_out[qa + u] = run;
+        run += v[u];
+      }
+    before += tot;
+  }
+  if (threadIdx.x == 0) {
+    if (before != s.lg_live[l]) c->internal_error = 1;  // the live count drifted
+    s.lg_new[l].tail = before;  // live count, for k_lg_cmp_layout
+  }
+}
+
 // The new layout: each log gets its live entries, this step's appends, and a
 // share of the free room in proportion to its appends (plus one).
-__global__ void __launch_bounds__(1024) k_lg_cmp_plan2(DevState s) {
+__global__ void __launch_bounds__(1024) k_lg_cmp_layout(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK || !c->lg_cmp) return;
   const int L = s.lg_L;
-  const int w = threadIdx.x >> 5, lane = lane_id(), nw = blockDim.x >> 5;
-  // live entries per log, and each chunk's offset inside its log
-  for (int l = w; l < L; l += nw) {
-    const int q0 = s.lg_c0[l], q1 = s.lg_c0[l + 1];
-    int64_t before = 0;
-    for (int qb = q0; qb < q1; qb += 32) {
-      const int q = qb + lane;
-      const int64_t v = q < q1 ? (int64_t)s.lg_ck[q] : 0;
-      const int64_t incl = warp_incl_scan(v);
-      if (q < q1) s.lg_ck_out[q] = before + incl - v;
-      before += __shfl_sync(kFull, incl, 31);
-    }
-    if (lane == 0) s.lg_new[l].tail = before;  // live count, for now
-  }
-  __syncthreads();
   const int per = (L + (int)blockDim.x - 1) / (int)blockDim.x;
   const int l0 = threadIdx.x * per, l1 = l0 + per < L ? l0 + per : L;
   int64_t need = 0, wsum = 0;
@@ -543,21 +574,14 @@ __global__ void __launch_bounds__(1024) k_lg_cmp_plan2(DevState s) {
   if (room < 0 && threadIdx.x == 0) c->internal_error = 1;  // sized so that this cannot happen
   const int64_t free_room = room > 0 ? room : 0;
   int64_t caps = 0;
-  for (int l = l0; l < l1; ++l)
-    caps += s.lg_new[l].tail + s.lg_add[l] + free_room * (s.lg_add[l] + 1) / tot_w;
+  for (int l = l0; l < l1; ++l) caps += s.lg_new[l].tail + s.lg_add[l] + free_room * (s.lg_add[l] + 1) / tot_w;
   int64_t tot_cap;
   int64_t start = block_excl_scan(caps, &tot_cap);
   for (int l = l0; l < l1; ++l) {
     const int64_t live = s.lg_new[l].tail;
     const int64_t cap = live + s.lg_add[l] + free_room * (s.lg_add[l] + 1) / tot_w;
-    if (live != s.lg_live[l]) c->internal_error = 1;  // the live count drifted
     s.lg_new[l] = LogDesc{start, start, start + live, start + cap};
     start += cap;
-  }
-  __syncthreads();
-  for (int l = w; l < L; l += nw) {
-    const int64_t st0 = s.lg_new[l].start;
-    for (int q = s.lg_c0[l] + lane; q < s.lg_c0[l + 1]; q += 32) s.lg_ck_out[q] += st0;
   }
 }
 
@@ -595,7 +619,7 @@ __global__ void __launch_bounds__(kScanThreads) k_lg_cmp_write(DevState s) {
       n += live[u];
     }
     int tot;
-    int64_t o = s.lg_ck_out[q] + block_excl_scan(n, &tot);
+    int64_t o = s.lg_new[l].start + s.lg_ck_out[q] + block_excl_scan(n, &tot);
 #pragma unroll
     for (int u = 0; u < 4; ++u)
       if (live[u]) {
@@ -715,11 +739,10 @@ int32_t launch_queue_select(const DevState& s, cudaStream_t st, const CaptureCtx
 
 int32_t launch_queue_append(const DevState& s, cudaStream_t st, const CaptureCtx* cap, int* launches) {
   const int ach = (int)s.lg_app_chunks;
-  const int sgrid = (s.lg_L * 32 + 1023) / 1024;
   cudaGraphConditionalHandle hc = 0;
   if (cap && !cond_handle(st, &hc)) return PS_ERR_CUDA;
   launch_k(k_lg_app_count, ach, kAppChunk, 0, st, s);
-  launch_k(k_lg_app_scan, sgrid, 1024, 0, st, s, hc, cap ? 1 : 0);
+  launch_k(k_lg_app_scan, s.lg_L, 256, 0, st, s, hc, cap ? 1 : 0);
   *launches += 2;
   cudaStream_t b = st;
   if (cap) {
@@ -728,9 +751,10 @@ int32_t launch_queue_append(const DevState& s, cudaStream_t st, const CaptureCtx
   }
   launch_k(k_lg_cmp_plan, 1, 1024, 0, b, s);
   launch_k(k_lg_cmp_count, kScanGrid, kScanThreads, 0, b, s);
-  launch_k(k_lg_cmp_plan2, 1, 1024, 0, b, s);
+  launch_k(k_lg_cmp_live, s.lg_L, 256, 0, b, s);
+  launch_k(k_lg_cmp_layout, 1, 1024, 0, b, s);
   launch_k(k_lg_cmp_write, kScanGrid, kScanThreads, 0, b, s);
-  *launches += 4;
+  *launches += 5;
   if (cap && !cond_close(cap->aux)) return PS_ERR_CUDA;
   launch_k(k_lg_app_write, ach, kAppChunk, 0, st, s);
   ++*launches;
