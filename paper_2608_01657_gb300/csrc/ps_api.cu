@@ -31,6 +31,8 @@ struct ps_handle {
   cudaStream_t cap_stream = nullptr;
   cudaStream_t cap_aux = nullptr;   // conditional bodies are captured here
   cudaStream_t cap_aux2 = nullptr;  // and bodies nested in them here
+  cudaStream_t cap_side = nullptr;  // a parallel branch of the step graph
+  cudaEvent_t cap_fork = nullptr, cap_join = nullptr;
   cudaGraph_t graph = nullptr;
   cudaGraphExec_t exec = nullptr;
   bool exec_timing = false;
@@ -342,9 +344,10 @@ void capture_step(ps_handle* h) {
   tmpl.R = 0;
   bool ok = cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
   if (ok) {
-    const CaptureCtx ctx{h->cap_aux, h->cap_aux2};
+    const CaptureCtx ctx{h->cap_aux, h->cap_aux2, h->cap_side, h->cap_fork, h->cap_join};
     const int32_t rc = launch_step(tmpl, h->cap_stream, &h->trace, &ctx);
     // a body whose capture did not close leaves an auxiliary stream capturing
+    // (the side stream joined the main capture: it ends with it)
     for (cudaStream_t a : {h->cap_aux2, h->cap_aux}) {
       cudaStreamCaptureStatus aux_cs = cudaStreamCaptureStatusNone;
       if (cudaStreamIsCapturing(a, &aux_cs) == cudaSuccess && aux_cs != cudaStreamCaptureStatusNone) {
@@ -434,7 +437,10 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   if (rc == PS_OK) rc = upload_constants(h, st);
   if (rc == PS_OK && (cudaStreamCreateWithFlags(&h->cap_stream, cudaStreamNonBlocking) != cudaSuccess ||
                       cudaStreamCreateWithFlags(&h->cap_aux, cudaStreamNonBlocking) != cudaSuccess ||
-                      cudaStreamCreateWithFlags(&h->cap_aux2, cudaStreamNonBlocking) != cudaSuccess))
+                      cudaStreamCreateWithFlags(&h->cap_aux2, cudaStreamNonBlocking) != cudaSuccess ||
+                      cudaStreamCreateWithFlags(&h->cap_side, cudaStreamNonBlocking) != cudaSuccess ||
+                      cudaEventCreateWithFlags(&h->cap_fork, cudaEventDisableTiming) != cudaSuccess ||
+                      cudaEventCreateWithFlags(&h->cap_join, cudaEventDisableTiming) != cudaSuccess))
     rc = PS_ERR_CUDA;
   if (rc != PS_OK) {
     delete h;
@@ -559,6 +565,9 @@ void ps_destroy(ps_handle_t* h) {
   if (h->cap_stream) cudaStreamDestroy(h->cap_stream);
   if (h->cap_aux) cudaStreamDestroy(h->cap_aux);
   if (h->cap_aux2) cudaStreamDestroy(h->cap_aux2);
+  if (h->cap_side) cudaStreamDestroy(h->cap_side);
+  if (h->cap_fork) cudaEventDestroy(h->cap_fork);
+  if (h->cap_join) cudaEventDestroy(h->cap_join);
   if (h->trace.timing)
     for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
   delete h;

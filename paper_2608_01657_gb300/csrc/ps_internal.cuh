@@ -335,6 +335,8 @@ struct StepTrace {
 struct CaptureCtx {
   cudaStream_t aux;   // bodies of top-level conditional nodes
   cudaStream_t aux2;  // bodies of conditional nodes inside those
+  cudaStream_t side;  // a parallel branch of the step graph (the candidate scan)
+  cudaEvent_t fork, join;
 };
 
 // Copy the call's arguments from device memory into the kernel's DevState,
@@ -380,7 +382,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
 void launch_queue_init(const DevState& s, cudaStream_t st);
 int32_t launch_queue_cand(const DevState& s, cudaStream_t st, int* launches);
 int32_t launch_queue_select(const DevState& s, cudaStream_t st, const CaptureCtx* cap, int phase, int depth,
-                            int* launches);
+                            bool plain_first, int* launches);
 int32_t launch_queue_append(const DevState& s, cudaStream_t st, const CaptureCtx* cap, int* launches);
 // S3-FIFO (ps_s3fifo.cu)
 void launch_s3_evict(const DevState& s, cudaStream_t st);

@@ -280,6 +280,11 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
   }
   if (!probe && s.policy == PS_STATICQUOTA)
     for (int g = threadIdx.x; g < s.G; g += blockDim.x) s.grp_pinned[g] = 0;
+  if (!probe)  // the candidate counts (k_cand accumulates them beside S3-S4)
+    for (int r = threadIdx.x; r < s.G * kClasses; r += blockDim.x) {
+      if (r < s.G) s.grp_qsize[r] = 0;
+      s.cls[r] = ClsRange{0, ~0u, 0, ~0u, 0};
+    }
 }
 
 // ===========================================================================
@@ -874,14 +879,12 @@ __global__ void __launch_bounds__(512) k_meter(DevState s0) {
     s.out.debt_norm[g] = norm;
     s.grp_P[g] = norm;
     s.grp_delta[g] = rmax ? muldiv(unit, s.rho_min, rmax) : 0;  // 1/W_g of Eq. 8
-    s.grp_qsize[g] = 0;
     SelSeg z{};
     z.kmin = ~0ull;
     z.kmax = 0;
     z.qmin = ~0ull;
     z.qmax = 0;
     s.sel[g] = z;
-    for (int k = 0; k < kClasses; ++k) s.cls[g * kClasses + k] = ClsRange{0, ~0u, 0, ~0u, 0};
   }
 }
 
@@ -970,7 +973,7 @@ __global__ void __launch_bounds__(1024) k_cand(DevState s) {
   s = with_args(s);
   extern __shared__ uint32_t cand_smem[];  // 5 arrays of nseg * kClasses
   Ctl* c = s.ctl;
-  if (c->status != PS_OK || c->mvict == 0) return;
+  if (c->status != PS_OK) return;  // runs beside S3-S4: the victim count is not known yet
   const uint32_t step32 = (uint32_t)c->step;
   // segments: groups for prefixshield and staticquota, one for lru; retention
   // classes only for prefixshield
@@ -2153,6 +2156,23 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(2);
   PS_LAUNCH(launch_k(k_claims, pgrid, kThreads, 0, st, s));
   mark(3);
+  // The candidates read pins and residency (final from here on) and the class
+  // and stamp of unpinned blocks, which S3-S4 leave alone: under capture
+  // they are counted on a side branch that runs beside S3-S4.
+  const bool fork = cap && s.policy != PS_S3FIFO;
+  cudaStream_t cs = st;
+  if (fork) {
+    if (cudaEventRecord(cap->fork, st) != cudaSuccess || cudaStreamWaitEvent(cap->side, cap->fork, 0) != cudaSuccess)
+      return PS_ERR_CUDA;
+    cs = cap->side;
+  }
+  const int cand_smem = (s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA ? s.G : 1) * kClasses * 5 * 4;
+  if (s.lg_on) {
+    if (launch_queue_cand(s, cs, &launches) != PS_OK) return PS_ERR_CUDA;
+  } else if (s.policy != PS_S3FIFO) {
+    PS_LAUNCH(k_cand<<<grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, cs>>>(s));
+  }
+  if (fork && cudaEventRecord(cap->join, cs) != cudaSuccess) return PS_ERR_CUDA;
   if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
   PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
   PS_LAUNCH(launch_k(k_instep, pgrid, kThreads, 0, st, s));
@@ -2163,28 +2183,27 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, st, s));
   PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, st, s));
   mark(6);
-  const int cand_smem = (s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA ? s.G : 1) * kClasses * 5 * 4;
+  if (fork && cudaStreamWaitEvent(st, cap->join, 0) != cudaSuccess) return PS_ERR_CUDA;
   if (s.lg_on) {
     // indexed queues: the same victims, taken from the queues' heads
-    if (launch_queue_cand(s, st, &launches) != PS_OK) return PS_ERR_CUDA;
     cudaGraphConditionalHandle hq_fb = 0;
     if (s.policy == PS_PREFIXSHIELD) {
       if (cap && !cond_handle(st, &hq_fb)) return PS_ERR_CUDA;
-      PS_LAUNCH(launch_k(k_waterfill, 1, 1024, 0, st, s, hq_fb, cap ? 1 : 0));
-      if (launch_queue_select(s, st, cap, 0, 0, &launches) != PS_OK) return PS_ERR_CUDA;
+      // the first kernel after the side branch's join depends on two nodes:
+      // a plain launch (a programmatic edge takes a single kernel predecessor)
+      PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s, hq_fb, cap ? 1 : 0));
+      if (launch_queue_select(s, st, cap, 0, 0, false, &launches) != PS_OK) return PS_ERR_CUDA;
       cudaStream_t f = st;
       if (cap) {
         if (!cond_open(st, cap->aux, hq_fb)) return PS_ERR_CUDA;
         f = cap->aux;
       }
-      if (launch_queue_select(s, f, cap, 1, 1, &launches) != PS_OK) return PS_ERR_CUDA;
+      if (launch_queue_select(s, f, cap, 1, 1, false, &launches) != PS_OK) return PS_ERR_CUDA;
       if (cap && !cond_close(cap->aux)) return PS_ERR_CUDA;
-    } else if (launch_queue_select(s, st, cap, s.policy == PS_LRU ? 2 : 3, 0, &launches) != PS_OK) {
+    } else if (launch_queue_select(s, st, cap, s.policy == PS_LRU ? 2 : 3, 0, fork, &launches) != PS_OK) {
       return PS_ERR_CUDA;
     }
   }
-  if (s.policy != PS_S3FIFO && !s.lg_on)
-    PS_LAUNCH(launch_k(k_cand, grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, st, s));
   // Under capture, phases that many steps skip become conditional bodies:
   // the long-list passes of a select, and the global fallback of Alg. 2.
   cudaGraphConditionalHandle h_fb = 0, h_long = 0;
@@ -2226,7 +2245,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   if (s.lg_on) {
     // selected above
   } else if (s.policy == PS_PREFIXSHIELD) {
-    PS_LAUNCH(launch_k(k_waterfill, 1, 1024, 0, st, s, h_fb, conds ? 1 : 0));
+    PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s, h_fb, conds ? 1 : 0));  // after the join: plain
     select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
     cudaStream_t f = st;
@@ -2244,11 +2263,11 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
     if (!cond_ok) return PS_ERR_CUDA;
     if (conds && !cond_close(cap->aux)) return PS_ERR_CUDA;
   } else if (s.policy == PS_STATICQUOTA) {
-    PS_LAUNCH(launch_k(k_quota_sel, 1, 1024, 0, st, s));
+    PS_LAUNCH(k_quota_sel<<<1, 1024, 0, st>>>(s));  // after the join: plain
     select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
   } else if (s.policy == PS_LRU) {
-    PS_LAUNCH(launch_k(k_sel_single, 1, 32, 0, st, s, 0));
+    PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));  // after the join: plain
     select(st, 1, 0, conds, h_long, conds ? cap->aux : st);
     if (!cond_ok) return PS_ERR_CUDA;
   } else {

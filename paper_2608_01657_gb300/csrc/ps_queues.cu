@@ -116,7 +116,7 @@ __global__ void __launch_bounds__(1024) k_lg_cand(DevState s) {
     }
   }
   __syncthreads();
-  if (!ok || c->mvict == 0 || s.policy == PS_LRU) return;
+  if (!ok || s.policy == PS_LRU) return;
   for (int g = threadIdx.x; g < s.G; g += blockDim.x) {
     int64_t q = 0;
     for (int k = 0; k < kClasses; ++k) {
@@ -702,18 +702,19 @@ void launch_queue_init(const DevState& s, cudaStream_t st) {
 }
 
 int32_t launch_queue_cand(const DevState& s, cudaStream_t st, int* launches) {
-  launch_k(k_lg_cand, 1, 1024, 0, st, s);
+  k_lg_cand<<<1, 1024, 0, st>>>(s);  // may start a side branch: a plain launch
   ++*launches;
   return PS_OK;
 }
 
 int32_t launch_queue_select(const DevState& s, cudaStream_t st, const CaptureCtx* cap, int phase, int depth,
-                            int* launches) {
+                            bool plain_first, int* launches) {
   cudaGraphConditionalHandle h1 = 0;
   if (cap && !cond_handle(st, &h1)) return PS_ERR_CUDA;
   const int rgrid = (s.lg_L * 32 + 1023) / 1024;
   auto round = [&](cudaStream_t q, int r) {
-    launch_k(k_lg_plan, 1, 1024, 0, q, s, phase, r);
+    if (plain_first && r == 0) k_lg_plan<<<1, 1024, 0, q>>>(s, phase, r);  // its predecessor is a join
+    else launch_k(k_lg_plan, 1, 1024, 0, q, s, phase, r);
     launch_k(k_lg_count, kScanGrid, kScanThreads, 0, q, s, phase);
     launch_k(k_lg_resolve, rgrid, 1024, 0, q, s, h1, (cap && r == 0) ? 1 : 0);
     launch_k(k_lg_mark, kScanGrid, kScanThreads, 0, q, s, phase);
