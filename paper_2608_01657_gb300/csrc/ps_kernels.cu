@@ -2156,9 +2156,11 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(2);
   PS_LAUNCH(launch_k(k_claims, pgrid, kThreads, 0, st, s));
   mark(3);
+  if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
+  PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
   // The candidates read pins and residency (final from here on) and the class
   // and stamp of unpinned blocks, which S3-S4 leave alone: under capture
-  // they are counted on a side branch that runs beside S3-S4.
+  // they are counted on a side branch that runs beside the rest of S3-S4.
   const bool fork = cap && s.policy != PS_S3FIFO;
   cudaStream_t cs = st;
   if (fork) {
@@ -2170,11 +2172,10 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   if (s.lg_on) {
     if (launch_queue_cand(s, cs, &launches) != PS_OK) return PS_ERR_CUDA;
   } else if (s.policy != PS_S3FIFO) {
-    PS_LAUNCH(k_cand<<<grid_for(s.N, 1024 * 4, 152), 1024, cand_smem, cs>>>(s));
+    // one 512-thread CTA per SM: the main branch keeps room on every SM
+    PS_LAUNCH(k_cand<<<fork ? 152 : grid_for(s.N, 1024 * 4, 152), fork ? 512 : 1024, cand_smem, cs>>>(s));
   }
   if (fork && cudaEventRecord(cap->join, cs) != cudaSuccess) return PS_ERR_CUDA;
-  if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
-  PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
   PS_LAUNCH(launch_k(k_instep, pgrid, kThreads, 0, st, s));
   PS_LAUNCH(launch_k(k_instep_fin, rgrid, 256, 0, st, s));
   mark(4);
