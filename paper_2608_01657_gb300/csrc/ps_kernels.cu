@@ -213,6 +213,7 @@ __global__ void k_init_ctl(DevState s) {
 // ===========================================================================
 // Stage 0: validation of the step's inputs; n_i, block positions, hashing
 // segments.  One CTA.  'probe' skips the clock and step checks.
+
 __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
   s = with_args(s);
   Ctl* c = s.ctl;
@@ -611,6 +612,10 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
 // Stage 3: grant new blocks against the pool.  avail = free + unpinned
 // resident = N - pinned; claims are ranked in (request, position) order; the
 // first avail ranks are materialized.  One CTA.
+// k_grant takes kReqPer consecutive requests a thread, so that one CTA scan
+// covers 1024 x kReqPer requests.
+constexpr int kReqPer = 4;
+
 __global__ void __launch_bounds__(1024) k_grant(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
@@ -618,28 +623,45 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
   const int R = s.R;
   const bool quota = s.policy == PS_STATICQUOTA;  // a_i already granted per group
   const int64_t avail = s.N - c->pinned;
-  int64_t carry_c = 0, carry_a = 0;
-  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
-    const int i = t0 + threadIdx.x;
-    int32_t cl = 0;
-    if (i < R) cl = s.rq_n[i] - s.rq_s[i];
-    int32_t tot_c;
-    const int32_t ex_c = block_excl_scan(cl, &tot_c);
-    int32_t a = 0;
-    if (i < R) a = quota ? s.rq_a[i] : (int32_t)tmin<int64_t>(cl, tmax<int64_t>(0, avail - (carry_c + ex_c)));
-    int32_t tot_a;
-    const int32_t ex_a = block_excl_scan(a, &tot_a);
-    if (i < R) {
-      // granted keys are paired with the allocated ids in (request, position)
-      // order: request i's first granted key is the (carry_a + ex_a)-th
-      s.rq_cbase[i] = (int32_t)(carry_a + ex_a);
-      s.rq_a[i] = a;
-      s.out.admitted_blocks[i] = a;
-      s.out.admitted_offsets[i] = (int32_t)(carry_a + ex_a);
+  const int tile = (int)blockDim.x * kReqPer;
+  // Granted ranks are the first avail in (request, position) order, so the
+  // grants before request i number min(avail, base_i), base_i the claims
+  // before it, and a_i = min(avail, base_i + c_i) - min(avail, base_i).  One
+  // packed scan a tile: claims in the high half, StaticQuota grants in the low.
+  uint64_t carry = 0;
+  for (int t0 = 0; t0 < R; t0 += tile) {
+    const int i0 = t0 + (int)threadIdx.x * kReqPer;
+    int32_t cl[kReqPer], aq[kReqPer];
+    uint64_t sum = 0;
+#pragma unroll
+    for (int u = 0; u < kReqPer; ++u) {
+      const bool in = i0 + u < R;
+      cl[u] = in ? s.rq_n[i0 + u] - s.rq_s[i0 + u] : 0;
+      aq[u] = in && quota ? s.rq_a[i0 + u] : 0;
+      sum += (uint64_t)cl[u] << 32 | (uint64_t)aq[u];
     }
-    carry_c += tot_c;
-    carry_a += tot_a;
+    uint64_t tot;
+    uint64_t ex = carry + block_excl_scan(sum, &tot);
+#pragma unroll
+    for (int u = 0; u < kReqPer; ++u) {
+      const int i = i0 + u;
+      if (i < R) {
+        const int64_t base_c = (int64_t)(ex >> 32);
+        const int64_t lo = quota ? (int64_t)(uint32_t)ex : tmin(avail, base_c);
+        const int32_t a = quota ? aq[u] : (int32_t)(tmin(avail, base_c + cl[u]) - lo);
+        // granted keys are paired with the allocated ids in (request,
+        // position) order: request i's first granted key is the lo-th
+        s.rq_cbase[i] = (int32_t)lo;
+        s.rq_a[i] = a;
+        s.out.admitted_blocks[i] = a;
+        s.out.admitted_offsets[i] = (int32_t)lo;
+      }
+      ex += (uint64_t)cl[u] << 32 | (uint64_t)aq[u];
+    }
+    carry += tot;
   }
+  const int64_t carry_c = (int64_t)(carry >> 32);
+  const int64_t carry_a = quota ? (int64_t)(uint32_t)carry : tmin(avail, carry_c);
   int64_t qv = 0;  // StaticQuota: the groups' overflows are the victims
   if (quota)
     for (int g = threadIdx.x; g < s.G; g += blockDim.x) qv += s.grp_x[g];
