@@ -170,6 +170,26 @@ int32_t ps_step_host(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t nu
                      const int32_t* h_group_ids, const int64_t* h_token_offsets, const int32_t* h_tokens,
                      const int32_t* h_contract_ids, const uint64_t* h_prefix_ids, const ps_host_out_t* h_out);
 
+/* Pipelined form of ps_step_host(): enqueue one step from host buffers and
+ * return at once, so that the next step's input copy overlaps this step's
+ * work.  Two steps may be in flight, on staging slots 0 and 1 (use them in
+ * turn; a slot is reused only after ps_step_host_wait() on it).  The inputs
+ * are copied on the handle's own copy stream into the slot's staging area
+ * (pinned host memory keeps that asynchronous; the buffers must stay
+ * unchanged until the wait).  The step itself runs on 'stream', in order with
+ * the caller's other work there.  The outputs are written by a kernel
+ * directly into h_out, whose non-null arrays must be page-locked host memory
+ * (device-accessible; else PS_ERR_INVALID_ARG); the id lists receive only
+ * their counts' worth.  Returns PS_OK or a launch error; the step's own
+ * status comes from ps_step_host_wait(). */
+int32_t ps_step_host_async(ps_handle_t* h, void* stream, int32_t slot, int64_t now_ticks, int32_t num_requests,
+                           const int32_t* h_group_ids, const int64_t* h_token_offsets, const int32_t* h_tokens,
+                           const int32_t* h_contract_ids, const uint64_t* h_prefix_ids, const ps_host_out_t* h_out);
+
+/* Block until the step enqueued on 'slot' by ps_step_host_async() has
+ * written its outputs; returns that step's status (h_out counts[3]). */
+int32_t ps_step_host_wait(ps_handle_t* h, int32_t slot);
+
 /* Copy the per-group statistics into h_stats [num_groups][PS_NUM_STATS];
  * synchronizes 'stream'.  Returns the sticky status (PS_OK or PS_ERR_CAPACITY). */
 int32_t ps_stats(ps_handle_t* h, void* stream, int64_t* h_stats);

@@ -29,7 +29,8 @@ POLICIES = {"lru": 0, "s3fifo": 1, "prefixshield": 2, "staticquota": 3}
 PS_OK, PS_ERR_INVALID_ARG, PS_ERR_CAPACITY, PS_ERR_CLOCK, PS_ERR_CUDA = 0, -1, -2, -3, -4
 PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE, PS_FLAG_INDEXED_QUEUES = 1, 2, 4
 
-EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_stats", "ps_clear_status",
+EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_step_host_async",
+            "ps_step_host_wait", "ps_stats", "ps_clear_status",
             "ps_reset", "ps_destroy", "ps_status_string", "ps_export_state", "ps_export_history",
             "ps_export_ghost", "ps_set_stage_timing", "ps_get_stage_times", "ps_cached_prefix",
             "ps_cached_prefix_noalloc", "ps_uses_graph", "ps_set_graph")
@@ -90,6 +91,10 @@ def load():
     L.ps_step.argtypes = [vp, vp, i64, i32, vp, vp, vp, vp, vp, C.POINTER(PsStepOut)]
     L.ps_step_host.restype = i32
     L.ps_step_host.argtypes = [vp, vp, i64, i32, vp, vp, vp, vp, vp, C.POINTER(PsStepOut)]
+    L.ps_step_host_async.restype = i32
+    L.ps_step_host_async.argtypes = [vp, vp, i32, i64, i32, vp, vp, vp, vp, vp, C.POINTER(PsStepOut)]
+    L.ps_step_host_wait.restype = i32
+    L.ps_step_host_wait.argtypes = [vp, i32]
     L.ps_stats.restype = i32
     L.ps_stats.argtypes = [vp, vp, vp]
     L.ps_clear_status.restype = i32
@@ -266,6 +271,22 @@ class Cache:
                                  _ptr(tokens), _ptr(contracts), _ptr(prefixes), C.byref(o))
         out["rc"] = rc
         return out
+
+    def step_host_async(self, slot: int, now: int, groups, offsets, tokens, out: dict, contracts=None,
+                        prefixes=None, stream=None) -> int:
+        """Pipelined end-to-end call: enqueue a step from host buffers on
+        staging slot 0 or 1 and return at once.  ``out`` must come from
+        ``host_outputs(..., pinned=True)``; inputs and ``out`` must stay
+        alive and unchanged until ``step_host_wait(slot)``."""
+        R = int(len(groups))
+        o = PsStepOut(**{k: _ptr(out[k]) for k, _ in PsStepOut._fields_})
+        out["_keep"] = (o, groups, offsets, tokens, contracts, prefixes)
+        return load().ps_step_host_async(self._h, _stream_ptr(stream), int(slot), int(now), R, _ptr(groups),
+                                         _ptr(offsets), _ptr(tokens), _ptr(contracts), _ptr(prefixes), C.byref(o))
+
+    def step_host_wait(self, slot: int) -> int:
+        """Wait for the step on ``slot``; returns its status."""
+        return load().ps_step_host_wait(self._h, int(slot))
 
     def fetch(self, R: int, stream=None) -> dict:
         """Copy the last step's outputs to host numpy arrays (synchronizes)."""

@@ -17,13 +17,18 @@ struct ps_handle {
   void* workspace;
   size_t workspace_bytes;
   int device;
-  // staging area for ps_step_host()
-  int32_t* st_group;
-  int64_t* st_offsets;
-  int32_t* st_tokens;
-  int32_t* st_contract;
-  uint64_t* st_prefix;
+  // staging areas for ps_step_host() (slot 0) and ps_step_host_async() (slots 0, 1)
+  struct Staging {
+    int32_t* group;
+    int64_t* offsets;
+    int32_t* tokens;
+    int32_t* contract;
+    uint64_t* prefix;
+  } stg[2];
   ps_step_out_t st_out;
+  cudaStream_t copy_stream = nullptr;  // the pipelined inputs' copies
+  cudaEvent_t in_ready[2] = {nullptr, nullptr}, slot_free[2] = {nullptr, nullptr}, done[2] = {nullptr, nullptr};
+  const ps_host_out_t* pending[2] = {nullptr, nullptr};
   StepTrace trace;
   std::vector<int32_t> contract_of_group;
   // the step as one CUDA graph, captured on a private stream at first use
@@ -283,11 +288,14 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   }
   StepArgs* step_args = cv.take<StepArgs>(1);
   // staging for ps_step_host
-  int32_t* st_group = cv.take<int32_t>(R);
-  int64_t* st_offsets = cv.take<int64_t>(R + 1);
-  int32_t* st_tokens = cv.take<int32_t>((size_t)d.max_tokens);
-  int32_t* st_contract = cv.take<int32_t>(R);
-  uint64_t* st_prefix = cv.take<uint64_t>(R);
+  ps_handle::Staging stg[2];
+  for (auto& x : stg) {
+    x.group = cv.take<int32_t>(R);
+    x.offsets = cv.take<int64_t>(R + 1);
+    x.tokens = cv.take<int32_t>((size_t)d.max_tokens);
+    x.contract = cv.take<int32_t>(R);
+    x.prefix = cv.take<uint64_t>(R);
+  }
   ps_step_out_t so{};
   so.hit_blocks = cv.take<int32_t>(R);
   so.admitted_blocks = cv.take<int32_t>(R);
@@ -301,8 +309,9 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   const size_t total = align_up(cv.off, 256);
   if (base) {
     *s = t;
-    h->st_group = st_group; h->st_offsets = st_offsets; h->st_tokens = st_tokens;
-    h->st_contract = st_contract; h->st_prefix = st_prefix; h->st_out = so;
+    h->stg[0] = stg[0];
+    h->stg[1] = stg[1];
+    h->st_out = so;
     h->step_args = step_args;
   }
   (void)zero_end;
@@ -440,7 +449,13 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
                       cudaStreamCreateWithFlags(&h->cap_aux2, cudaStreamNonBlocking) != cudaSuccess ||
                       cudaStreamCreateWithFlags(&h->cap_side, cudaStreamNonBlocking) != cudaSuccess ||
                       cudaEventCreateWithFlags(&h->cap_fork, cudaEventDisableTiming) != cudaSuccess ||
-                      cudaEventCreateWithFlags(&h->cap_join, cudaEventDisableTiming) != cudaSuccess))
+                      cudaEventCreateWithFlags(&h->cap_join, cudaEventDisableTiming) != cudaSuccess ||
+                      cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking) != cudaSuccess))
+    rc = PS_ERR_CUDA;
+  for (int k = 0; k < 2 && rc == PS_OK; ++k)
+    if (cudaEventCreateWithFlags(&h->in_ready[k], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->slot_free[k], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->done[k], cudaEventDisableTiming) != cudaSuccess)
     rc = PS_ERR_CUDA;
   if (rc != PS_OK) {
     delete h;
@@ -491,13 +506,13 @@ int32_t ps_step_host(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t nu
   auto h2d = [&](void* d, const void* src, size_t bytes) {
     return bytes == 0 || cudaMemcpyAsync(d, src, bytes, cudaMemcpyHostToDevice, st) == cudaSuccess;
   };
-  if (!h2d(h->st_offsets, h_token_offsets, (R + 1) * 8) || !h2d(h->st_group, h_group_ids, R * 4) ||
-      !h2d(h->st_tokens, h_tokens, (size_t)T * 4) ||
-      (h_contract_ids && !h2d(h->st_contract, h_contract_ids, R * 4)) ||
-      (h_prefix_ids && !h2d(h->st_prefix, h_prefix_ids, R * 8)))
+  const ps_handle::Staging& sg = h->stg[0];
+  if (!h2d(sg.offsets, h_token_offsets, (R + 1) * 8) || !h2d(sg.group, h_group_ids, R * 4) ||
+      !h2d(sg.tokens, h_tokens, (size_t)T * 4) || (h_contract_ids && !h2d(sg.contract, h_contract_ids, R * 4)) ||
+      (h_prefix_ids && !h2d(sg.prefix, h_prefix_ids, R * 8)))
     return PS_ERR_CUDA;
-  int32_t rc = ps_step(h, stream, now_ticks, num_requests, h->st_group, h->st_offsets, h->st_tokens,
-                       h_contract_ids ? h->st_contract : nullptr, h_prefix_ids ? h->st_prefix : nullptr, &h->st_out);
+  int32_t rc = ps_step(h, stream, now_ticks, num_requests, sg.group, sg.offsets, sg.tokens,
+                       h_contract_ids ? sg.contract : nullptr, h_prefix_ids ? sg.prefix : nullptr, &h->st_out);
   if (rc != PS_OK) return rc;
   const ps_step_out_t& o = h->st_out;
   auto d2h = [&](void* dst, const void* d, size_t bytes) {
@@ -516,6 +531,64 @@ int32_t ps_step_host(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t nu
       cudaStreamSynchronize(st) != cudaSuccess)
     return PS_ERR_CUDA;
   return PS_OK;
+}
+
+namespace {
+// A host array a kernel may write: page-locked (or otherwise device-mapped).
+bool device_writable(const void* p) {
+  if (!p) return true;
+  cudaPointerAttributes a{};
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeHost || a.type == cudaMemoryTypeManaged;
+}
+}  // namespace
+
+int32_t ps_step_host_async(ps_handle_t* h, void* stream, int32_t slot, int64_t now_ticks, int32_t num_requests,
+                           const int32_t* h_group_ids, const int64_t* h_token_offsets, const int32_t* h_tokens,
+                           const int32_t* h_contract_ids, const uint64_t* h_prefix_ids, const ps_host_out_t* h_out) {
+  if (!h || !h_out || slot < 0 || slot > 1 || h->pending[slot] || num_requests < 0 ||
+      num_requests > h->base.max_requests || !h_token_offsets || !h_out->counts)
+    return PS_ERR_INVALID_ARG;
+  const int64_t T = num_requests > 0 ? h_token_offsets[num_requests] : 0;
+  if (T < 0 || T > h->base.max_tokens || (num_requests > 0 && (!h_group_ids || (T > 0 && !h_tokens))))
+    return PS_ERR_INVALID_ARG;
+  for (const void* p : {(const void*)h_out->hit_blocks, (const void*)h_out->admitted_blocks,
+                        (const void*)h_out->admitted_offsets, (const void*)h_out->admitted_ids,
+                        (const void*)h_out->evicted_ids, (const void*)h_out->invalidated_ids,
+                        (const void*)h_out->counts, (const void*)h_out->debt_raw, (const void*)h_out->debt_norm})
+    if (!device_writable(p)) return PS_ERR_INVALID_ARG;
+  cudaStream_t st = as_stream(stream), cs = h->copy_stream;
+  const size_t R = (size_t)num_requests;
+  const ps_handle::Staging& sg = h->stg[slot];
+  auto h2d = [&](void* d, const void* src, size_t bytes) {
+    return bytes == 0 || cudaMemcpyAsync(d, src, bytes, cudaMemcpyHostToDevice, cs) == cudaSuccess;
+  };
+  // the slot's staging is free once the step that last read it has run
+  if (cudaStreamWaitEvent(cs, h->slot_free[slot], 0) != cudaSuccess) return PS_ERR_CUDA;
+  if (!h2d(sg.offsets, h_token_offsets, (R + 1) * 8) || !h2d(sg.group, h_group_ids, R * 4) ||
+      !h2d(sg.tokens, h_tokens, (size_t)T * 4) || (h_contract_ids && !h2d(sg.contract, h_contract_ids, R * 4)) ||
+      (h_prefix_ids && !h2d(sg.prefix, h_prefix_ids, R * 8)) ||
+      cudaEventRecord(h->in_ready[slot], cs) != cudaSuccess || cudaStreamWaitEvent(st, h->in_ready[slot], 0) != cudaSuccess)
+    return PS_ERR_CUDA;
+  const int32_t rc = ps_step(h, stream, now_ticks, num_requests, sg.group, sg.offsets, sg.tokens,
+                             h_contract_ids ? sg.contract : nullptr, h_prefix_ids ? sg.prefix : nullptr, &h->st_out);
+  if (rc != PS_OK) return rc;
+  if (cudaEventRecord(h->slot_free[slot], st) != cudaSuccess) return PS_ERR_CUDA;
+  launch_host_out(h->st_out, *h_out, num_requests, h->base.G, st);
+  if (cudaGetLastError() != cudaSuccess || cudaEventRecord(h->done[slot], st) != cudaSuccess) return PS_ERR_CUDA;
+  h->pending[slot] = h_out;
+  return PS_OK;
+}
+
+int32_t ps_step_host_wait(ps_handle_t* h, int32_t slot) {
+  if (!h || slot < 0 || slot > 1 || !h->pending[slot]) return PS_ERR_INVALID_ARG;
+  const ps_host_out_t* o = h->pending[slot];
+  h->pending[slot] = nullptr;
+  if (cudaEventSynchronize(h->done[slot]) != cudaSuccess) return PS_ERR_CUDA;
+  return o->counts[3];
 }
 
 int32_t ps_stats(ps_handle_t* h, void* stream, int64_t* h_stats) {
@@ -568,6 +641,10 @@ void ps_destroy(ps_handle_t* h) {
   if (h->cap_side) cudaStreamDestroy(h->cap_side);
   if (h->cap_fork) cudaEventDestroy(h->cap_fork);
   if (h->cap_join) cudaEventDestroy(h->cap_join);
+  if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
+  for (int k = 0; k < 2; ++k)
+    for (cudaEvent_t e : {h->in_ready[k], h->slot_free[k], h->done[k]})
+      if (e) cudaEventDestroy(e);
   if (h->trace.timing)
     for (cudaEvent_t e : h->trace.ev) cudaEventDestroy(e);
   delete h;

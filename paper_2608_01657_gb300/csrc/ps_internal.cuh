@@ -387,6 +387,9 @@ int32_t launch_queue_append(const DevState& s, cudaStream_t st, const CaptureCtx
 // S3-FIFO (ps_s3fifo.cu)
 void launch_s3_evict(const DevState& s, cudaStream_t st);
 void launch_s3_insert(const DevState& s, cudaStream_t st);
+// A step's outputs (device) written into page-locked host buffers, the id
+// lists by their device-side counts (ps_step_host_async).
+void launch_host_out(const ps_step_out_t& dev, const ps_step_out_t& host, int32_t R, int32_t G, cudaStream_t st);
 // Read-only cached-prefix probe; 'out' receives h_i per request, 'status' the outcome.
 int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* status);
 

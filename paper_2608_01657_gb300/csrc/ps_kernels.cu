@@ -2314,6 +2314,35 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
+// The step's outputs into the caller's page-locked host buffers (one pass,
+// grid-stride; the id lists by the counts the step wrote).
+__global__ void __launch_bounds__(256) k_host_out(ps_step_out_t d, ps_step_out_t h, int32_t R, int32_t G) {
+  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x, nt = (int64_t)gridDim.x * blockDim.x;
+  const bool ok = d.counts[3] == PS_OK;
+  const int64_t n0 = ok ? d.counts[0] : 0, n1 = ok ? d.counts[1] : 0, n2 = ok ? d.counts[2] : 0;
+  if (h.counts && t < 4) h.counts[t] = d.counts[t];
+  for (int64_t i = t; i < R; i += nt) {
+    if (h.hit_blocks) h.hit_blocks[i] = d.hit_blocks[i];
+    if (h.admitted_blocks) h.admitted_blocks[i] = d.admitted_blocks[i];
+  }
+  if (h.admitted_offsets)
+    for (int64_t i = t; i <= R; i += nt) h.admitted_offsets[i] = d.admitted_offsets[i];
+  for (int64_t i = t; i < G; i += nt) {
+    if (h.debt_raw) h.debt_raw[i] = d.debt_raw[i];
+    if (h.debt_norm) h.debt_norm[i] = d.debt_norm[i];
+  }
+  if (h.admitted_ids)
+    for (int64_t i = t; i < n0; i += nt) h.admitted_ids[i] = d.admitted_ids[i];
+  if (h.evicted_ids)
+    for (int64_t i = t; i < n1; i += nt) h.evicted_ids[i] = d.evicted_ids[i];
+  if (h.invalidated_ids)
+    for (int64_t i = t; i < n2; i += nt) h.invalidated_ids[i] = d.invalidated_ids[i];
+}
+
+void launch_host_out(const ps_step_out_t& dev, const ps_step_out_t& host, int32_t R, int32_t G, cudaStream_t st) {
+  k_host_out<<<152 * 2, 256, 0, st>>>(dev, host, R, G);
+}
+
 int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* status) {
   const int rgrid = grid_for(s.R, 256, 1 << 20);
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);

@@ -261,6 +261,48 @@ def test_step_host_matches_step(N):
         compare_outputs(got, orc.step(st.now, st.groups, st.offsets, st.tokens), f"step {st.index}")
 
 
+@pytest.mark.parametrize("policy", ["lru", "prefixshield"])
+def test_parity_host_pipelined(policy):
+    """ps_step_host_async on alternating slots, two steps in flight: every
+    output equals the oracle's; unpinned output buffers are refused."""
+    from paper_2608_01657_gb300 import binding as B
+    steps = W.fuzz_steps(43, 3, 5, 40, docs_per_group=3, doc_blocks=6, with_contracts=3, empty_every=7)
+    kw = dict(rho=(2.0, 1.5, 1.0), beta=(6.0, 5.0, 4.0), contract_of_group=[0, 1, 2])
+    a = B.Cache(40, 16, 3, policy, B.Params(**kw), max_requests=5, max_tokens=2048)
+    orc = O.OracleCache(40, 16, 3, policy, O.Params(**kw))
+    outs = [B.host_outputs(5, a.max_blocks, 3, pinned=True) for _ in range(2)]
+
+    def pinned(x):
+        return torch.from_numpy(np.ascontiguousarray(x)).pin_memory().numpy()
+
+    host = [(st, pinned(st.groups), pinned(st.offsets), pinned(st.tokens if st.num_tokens else np.zeros(4, np.int32)),
+             pinned(st.contracts)) for st in steps]
+
+    def check(j):
+        st = host[j][0]
+        assert a.step_host_wait(j % 2) == 0
+        out = outs[j % 2]
+        cnt = out["counts"]
+        got = {"status": int(cnt[3]), "hit_blocks": out["hit_blocks"][:st.num_requests],
+               "admitted_blocks": out["admitted_blocks"][:st.num_requests],
+               "admitted_offsets": out["admitted_offsets"][:st.num_requests + 1],
+               "admitted_ids": out["admitted_ids"][:cnt[0]], "evicted_ids": out["evicted_ids"][:cnt[1]],
+               "invalidated_ids": out["invalidated_ids"][:cnt[2]], "debt_raw": out["debt_raw"],
+               "debt_norm": out["debt_norm"]}
+        compare_outputs(got, orc.step(st.now, st.groups, st.offsets, st.tokens, st.contracts), f"step {st.index}")
+
+    for k, (st, g, o, t, c) in enumerate(host):
+        assert a.step_host_async(k % 2, st.now, g, o, t, outs[k % 2], contracts=c) == 0
+        if k >= 1:
+            check(k - 1)
+    check(len(host) - 1)
+    assert np.array_equal(a.stats(), orc.stats())
+    # output buffers a kernel cannot write are refused before anything is enqueued
+    st = steps[0]
+    plain = B.host_outputs(5, a.max_blocks, 3, pinned=False)
+    assert a.step_host_async(0, st.now + 1000, host[0][1], host[0][2], host[0][3], plain) == B.PS_ERR_INVALID_ARG
+
+
 _SCALE = {}
 
 
