@@ -77,6 +77,10 @@ enum {
  * workspace grows by two buffers of 16 x (N + max_tokens / block_size)
  * entries of 12 bytes each, plus per-step scratch. */
 #define PS_FLAG_INDEXED_QUEUES 4u
+/* With PS_FLAG_INDEXED_QUEUES: the first scan round of a take covers a single
+ * 1024-entry chunk, so a take that needs more finishes in the second round.
+ * Same results, slower; it exercises the second round on small pools. */
+#define PS_FLAG_QUEUE_SHORT_WINDOWS 8u
 
 /* Per-group statistics, int64 each, row-major [num_groups][PS_NUM_STATS]. */
 enum {

@@ -30,6 +30,7 @@ OK, ERR_INVALID_ARG, ERR_CAPACITY, ERR_CLOCK = 0, -1, -2, -3
 FLAG_NO_SEGMENTATION, FLAG_NO_DEBT_GATE = 1, 2
 # the CUDA library's indexed-queue victim selection: same victims, ignored here
 FLAG_INDEXED_QUEUES = 4
+FLAG_QUEUE_SHORT_WINDOWS = 8
 
 
 class OrcParams(C.Structure):

@@ -27,8 +27,9 @@
 //
 // Every function below is pinned by a CPU test (tests/test_oracle_*.py).
 //
-// Flag bit 4 (indexed queues) selects the CUDA library's victim data
-// structure; the victims are the same, so this oracle ignores it.
+// Flag bits 4 and 8 (indexed queues, and their short first scan windows)
+// select the CUDA library's victim data structure; the victims are the same,
+// so this oracle ignores them.
 
 #include <algorithm>
 #include <cstdint>

@@ -196,7 +196,8 @@ __global__ void __launch_bounds__(1024) k_lg_plan(DevState s, int phase, int rou
         if (round > 0) k.cur = k.wend;  // the last window held too few live entries
         const int64_t avail = s.lg_desc[k.log].tail - k.cur;
         const int64_t rem = k.want - k.got;
-        const int64_t wl = round == 0 ? tmin<int64_t>(avail, rem + rem / 4 + kLogChunk) : avail;
+        const int64_t first = (s.flags & PS_FLAG_QUEUE_SHORT_WINDOWS) ? kLogChunk : rem + rem / 4 + kLogChunk;
+        const int64_t wl = round == 0 ? tmin<int64_t>(avail, first) : avail;
         k.wend = k.cur + wl;
         k.cut = -1;
         nch = (int)((wl + kLogChunk - 1) / kLogChunk);

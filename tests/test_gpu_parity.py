@@ -181,6 +181,21 @@ def test_parity_queues_configs(policy, cfg, nsteps, rps, wait, flags):
     _run(gpu, orc, steps, state_every=10, label=f"queues/cfg{cfg}/{policy}")
 
 
+@pytest.mark.parametrize("policy", QUEUE_POLICIES)
+@pytest.mark.parametrize("cfg,nsteps,rps", [(1, 60, None), (3, 30, None)])
+def test_parity_queues_second_round(policy, cfg, nsteps, rps):
+    """First scan rounds of one chunk: every take longer than 1024 live
+    entries, or behind dead ones, finishes in the second round."""
+    wl = W.make_workload(cfg, seed=3, requests_per_step=rps)
+    sp = wl.spec
+    steps = list(wl.steps(nsteps))
+    kw = dict(rho=sp.rho, beta=sp.beta, flags=IQ | O.FLAG_QUEUE_SHORT_WINDOWS)
+    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, kw,
+                     max_requests=sp.requests_per_step, max_tokens=max(st.num_tokens for st in steps))
+    _run(gpu, orc, steps, state_every=10, label=f"queues/short/cfg{cfg}/{policy}")
+    assert orc.stats()[:, O.STAT_NAMES.index("evicted_blocks")].sum() > 1024
+
+
 def test_parity_queues_alg2_ties():
     """Eq. 7's tie rule with the tie candidates read from the queues."""
     G = 6
