@@ -55,6 +55,37 @@ __device__ T block_excl_scan(T v, T* total) {
   __syncthreads();
   return base + incl - v;
 }
+// Four exclusive scans in one pass: thread t holds the elements
+// u * blockDim.x + t (u = 0..3) of a 4 * blockDim.x tile, so its loads stay
+// coalesced; ex[u] receives the exclusive prefix of its element u in tile
+// order, *total the tile's sum.  Two barriers for the whole tile.
+template <typename T>
+__device__ void block_excl_scan4(const T (&v)[4], T (&ex)[4], T* total) {
+  __shared__ T wsum[4][32];
+  const int lane = lane_id(), warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  T incl[4];
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    incl[u] = warp_incl_scan(v[u]);
+    if (lane == 31) wsum[u][warp] = incl[u];
+  }
+  __syncthreads();
+  if (warp < 4) {  // warp u scans row u of the warp totals
+    T w = lane < nw ? wsum[warp][lane] : T(0);
+    T wi = warp_incl_scan(w);
+    __syncwarp();
+    wsum[warp][lane] = wi;
+  }
+  __syncthreads();
+  T carry = T(0);
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    ex[u] = carry + (warp ? wsum[u][warp - 1] : T(0)) + incl[u] - v[u];
+    carry += wsum[u][nw - 1];
+  }
+  *total = carry;
+  __syncthreads();
+}
 template <typename T>
 __device__ T block_sum(T v) {
   T tot;

@@ -217,19 +217,17 @@ __global__ void k_init_ctl(DevState s) {
 __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
   s = with_args(s);
   Ctl* c = s.ctl;
-  __shared__ int s_bad;
-  if (threadIdx.x == 0) s_bad = 0;
-  __syncthreads();
   const int R = s.R;
+  bool bad = false;
+#pragma unroll 4
   for (int i = threadIdx.x; i < R; i += blockDim.x) {
     const int64_t o0 = s.in_offsets[i], o1 = s.in_offsets[i + 1];
     const int g = s.in_group[i];
-    bool bad = o1 < o0 || g < 0 || g >= s.G || (o1 - o0) / s.bs > (int64_t)kMaxPos;
+    bad |= o1 < o0 || g < 0 || g >= s.G || (o1 - o0) / s.bs > (int64_t)kMaxPos;
     if (s.in_contract) bad |= s.in_contract[i] < 0 || s.in_contract[i] >= s.C;
     if (s.in_prefix) bad |= s.in_prefix[i] == 0;
-    if (bad) atomicOr(&s_bad, 1);
   }
-  __syncthreads();
+  const int s_bad = __syncthreads_or(bad);
   int32_t st = PS_OK;
   const int64_t T = R > 0 ? s.in_offsets[R] : 0;
   if (!probe && c->sticky != PS_OK) st = c->sticky;
@@ -241,35 +239,50 @@ __global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
     if (threadIdx.x == 0) { c->status = st; c->nblocks = 0; c->nsegs = 0; }
     return;
   }
-  int32_t carry = 0, scarry = 0;
-  for (int t0 = 0; t0 < R; t0 += blockDim.x) {
-    const int i = t0 + threadIdx.x;
-    int32_t n = 0, nseg = 0;
-    if (i < R) {
-      n = (int32_t)((s.in_offsets[i + 1] - s.in_offsets[i]) / s.bs);
-      nseg = (n + kSegBlocks - 1) / kSegBlocks;
-      s.rq_n[i] = n;
-      s.rq_h[i] = n;
-      s.rq_s[i] = n;
-      s.rq_fu[i] = kNone;
-      if (!probe) s.rq_cid[i] = s.in_contract ? s.in_contract[i] : s.contract_of_group[s.in_group[i]];
+  // blocks and hashing segments per request (blocks in the high half, segments
+  // in the low half of one scanned word), four 1024-request sub-tiles a pass
+  uint64_t carry = 0;
+  const int tile = 4 * (int)blockDim.x;
+  for (int t0 = 0; t0 < R; t0 += tile) {
+    uint64_t v[4], ex[4];
+    int32_t n[4], ns[4], cid[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = t0 + u * (int)blockDim.x + (int)threadIdx.x;
+      n[u] = 0;
+      cid[u] = 0;
+      if (i < R) {
+        n[u] = (int32_t)((s.in_offsets[i + 1] - s.in_offsets[i]) / s.bs);
+        if (!probe) cid[u] = s.in_contract ? s.in_contract[i] : s.contract_of_group[s.in_group[i]];
+      }
+      ns[u] = (n[u] + kSegBlocks - 1) / kSegBlocks;
+      v[u] = (uint64_t)n[u] << 32 | (uint64_t)ns[u];
     }
-    int32_t tot, stot;
-    const int32_t ex = block_excl_scan(n, &tot);
-    const int32_t sex = block_excl_scan(nseg, &stot);
-    if (i < R) {
-      s.rq_pbase[i] = carry + ex;
-      s.rq_sbase[i] = scarry + sex;
-      for (int j = 0; j < nseg; ++j) s.seg_req[scarry + sex + j] = (uint32_t)i;
+    uint64_t tot;
+    block_excl_scan4(v, ex, &tot);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = t0 + u * (int)blockDim.x + (int)threadIdx.x;
+      if (i < R) {
+        const uint64_t e = carry + ex[u];
+        s.rq_n[i] = n[u];
+        s.rq_h[i] = n[u];
+        s.rq_s[i] = n[u];
+        s.rq_fu[i] = kNone;
+        if (!probe) s.rq_cid[i] = cid[u];
+        s.rq_pbase[i] = (int32_t)(e >> 32);
+        s.rq_sbase[i] = (int32_t)(uint32_t)e;
+        for (int j = 0; j < ns[u]; ++j) s.seg_req[(uint32_t)e + j] = (uint32_t)i;
+      }
     }
     carry += tot;
-    scarry += stot;
   }
+  const int32_t nblocks = (int32_t)(carry >> 32), nsegs = (int32_t)(uint32_t)carry;
   if (threadIdx.x == 0) {
     c->status = PS_OK;
     c->T = T;
-    c->nblocks = carry;
-    c->nsegs = scarry;
+    c->nblocks = nblocks;
+    c->nsegs = nsegs;
     if (!probe) {
       c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
       c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
@@ -612,10 +625,6 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
 // Stage 3: grant new blocks against the pool.  avail = free + unpinned
 // resident = N - pinned; claims are ranked in (request, position) order; the
 // first avail ranks are materialized.  One CTA.
-// k_grant takes kReqPer consecutive requests a thread, so that one CTA scan
-// covers 1024 x kReqPer requests.
-constexpr int kReqPer = 4;
-
 __global__ void __launch_bounds__(1024) k_grant(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
@@ -623,31 +632,33 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
   const int R = s.R;
   const bool quota = s.policy == PS_STATICQUOTA;  // a_i already granted per group
   const int64_t avail = s.N - c->pinned;
-  const int tile = (int)blockDim.x * kReqPer;
   // Granted ranks are the first avail in (request, position) order, so the
   // grants before request i number min(avail, base_i), base_i the claims
   // before it, and a_i = min(avail, base_i + c_i) - min(avail, base_i).  One
-  // packed scan a tile: claims in the high half, StaticQuota grants in the low.
+  // scanned word per request: claims in the high half, StaticQuota grants in
+  // the low; four 1024-request sub-tiles a pass.
   uint64_t carry = 0;
+  const int tile = 4 * (int)blockDim.x;
   for (int t0 = 0; t0 < R; t0 += tile) {
-    const int i0 = t0 + (int)threadIdx.x * kReqPer;
-    int32_t cl[kReqPer], aq[kReqPer];
-    uint64_t sum = 0;
+    uint64_t v[4], ex[4];
+    int32_t cl[4], aq[4];
 #pragma unroll
-    for (int u = 0; u < kReqPer; ++u) {
-      const bool in = i0 + u < R;
-      cl[u] = in ? s.rq_n[i0 + u] - s.rq_s[i0 + u] : 0;
-      aq[u] = in && quota ? s.rq_a[i0 + u] : 0;
-      sum += (uint64_t)cl[u] << 32 | (uint64_t)aq[u];
+    for (int u = 0; u < 4; ++u) {
+      const int i = t0 + u * (int)blockDim.x + (int)threadIdx.x;
+      const bool in = i < R;
+      cl[u] = in ? s.rq_n[i] - s.rq_s[i] : 0;
+      aq[u] = in && quota ? s.rq_a[i] : 0;
+      v[u] = (uint64_t)cl[u] << 32 | (uint64_t)aq[u];
     }
     uint64_t tot;
-    uint64_t ex = carry + block_excl_scan(sum, &tot);
+    block_excl_scan4(v, ex, &tot);
 #pragma unroll
-    for (int u = 0; u < kReqPer; ++u) {
-      const int i = i0 + u;
+    for (int u = 0; u < 4; ++u) {
+      const int i = t0 + u * (int)blockDim.x + (int)threadIdx.x;
       if (i < R) {
-        const int64_t base_c = (int64_t)(ex >> 32);
-        const int64_t lo = quota ? (int64_t)(uint32_t)ex : tmin(avail, base_c);
+        const uint64_t e = carry + ex[u];
+        const int64_t base_c = (int64_t)(e >> 32);
+        const int64_t lo = quota ? (int64_t)(uint32_t)e : tmin(avail, base_c);
         const int32_t a = quota ? aq[u] : (int32_t)(tmin(avail, base_c + cl[u]) - lo);
         // granted keys are paired with the allocated ids in (request,
         // position) order: request i's first granted key is the lo-th
@@ -656,7 +667,6 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
         s.out.admitted_blocks[i] = a;
         s.out.admitted_offsets[i] = (int32_t)lo;
       }
-      ex += (uint64_t)cl[u] << 32 | (uint64_t)aq[u];
     }
     carry += tot;
   }
