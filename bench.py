@@ -269,7 +269,6 @@ def run_own(args, ws, rank, local):
                       flags=B.PS_FLAG_INDEXED_QUEUES if args.queues else 0)
     cache = B.Cache(spec.capacity_blocks, spec.block_size, spec.num_groups, args.policy, params,
                     max_requests=R, max_tokens=maxT)
-    cache.set_stage_timing(True)
     cache.set_graph(not args.no_graph)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
 
@@ -279,15 +278,20 @@ def run_own(args, ws, rank, local):
         if rc != 0:
             raise RuntimeError(f"ps_step rc={rc}")
 
-    for k in range(args.prefill + args.warmup):
-        run(k)
-    torch.cuda.synchronize()
-    if int(cache.out["counts"][3].item()) != 0:
-        raise RuntimeError("step status error during warmup")
+    def fill():
+        cache.reset()
+        for k in range(args.prefill + args.warmup):
+            run(k)
+        torch.cuda.synchronize()
+        if int(cache.out["counts"][3].item()) != 0:
+            raise RuntimeError("step status error during warmup")
+
+    # Pass A, the headline: the step as a user runs it (no stage events in the
+    # graph), one CUDA event pair around each step, the L2 flushed before it.
+    cache.set_stage_timing(False)
+    fill()
     s0 = cache.stats()
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    stage_ms = np.zeros(len(STAGES))
-    launches = 0
     barrier(ws)
     torch.cuda.synchronize()
     gc.collect()
@@ -299,18 +303,32 @@ def run_own(args, ws, rank, local):
             e0.record(stream)
             run(args.prefill + args.warmup + j)
             e1.record(stream)
-            ms, nl = cache.stage_times()
-            stage_ms[: len(ms)] += ms
-            launches += nl
         torch.cuda.synchronize()
     gc.enable()
     barrier(ws)
     step_ms = [e0.elapsed_time(e1) for e0, e1 in evs]
-    total_s = sum(step_ms) / 1e3
+    s1 = cache.stats()
     status = int(cache.out["counts"][3].item())
     if status != 0:
         raise RuntimeError(f"step status {status}")
-    s1 = cache.stats()
+    # Pass B, the breakdown: the same steps from the same state with an event
+    # between the stages (the events add about 4 us each to a step, so they
+    # stay out of the headline).  The kernels are the same ones: their
+    # device-side count per step is the launches of pass A.
+    cache.set_stage_timing(True)
+    fill()
+    stage_ms = np.zeros(len(STAGES))
+    launches = 0
+    torch.cuda.synchronize()
+    for j in range(args.steps):
+        flush.zero_()
+        run(args.prefill + args.warmup + j)
+        ms, nl = cache.stage_times()
+        stage_ms[: len(ms)] += ms
+        launches += nl
+    torch.cuda.synchronize()
+    cache.set_stage_timing(False)
+    total_s = sum(step_ms) / 1e3
     d = s1 - s0
     col = {n: i for i, n in enumerate(B.STAT_NAMES)}
     timed = steps[args.prefill + args.warmup:]
