@@ -21,9 +21,10 @@
 // pinned, invalidated, taken and appended, so no step scans the pool.
 //
 // A select phase turns victim counts into "takes" (log, number of live
-// entries to consume from its head), scans a window past each head in
-// 1024-entry chunks (count, locate the chunk of the last victim, mark), and
-// repeats once over the rest of a log when dead entries made a window short.
+// entries to consume from its head) and scans a window past each head in
+// 1024-entry chunks, one pass that counts, finds each chunk's place in its
+// take by a decoupled look-back and marks; it repeats once over the rest of
+// a log when dead entries made a window short.
 // Logs live in one of two entry buffers; when a log lacks room for a step's
 // appends, every log's live entries are compacted into the other buffer, in
 // order, each log given room in proportion to its recent appends.
@@ -201,6 +202,7 @@ __global__ void __launch_bounds__(1024) k_lg_plan(DevState s, int phase, int rou
         k.wend = k.cur + wl;
         k.cut = -1;
         nch = (int)((wl + kLogChunk - 1) / kLogChunk);
+        if (nch == 0) c->internal_error = 1;  // victims owed by a log with nothing left to scan
         s.lg_tk[t] = k;
       }
     }
@@ -212,103 +214,49 @@ __global__ void __launch_bounds__(1024) k_lg_plan(DevState s, int phase, int rou
   if (threadIdx.x == 0) {
     s.lg_c0[ntk] = chunk_base;
     c->lg_nchunks = chunk_base;
+    c->lg_ticket = 0;
   }
+  for (int q = threadIdx.x; q < chunk_base; q += blockDim.x) s.lg_ck_out[q] = 0;  // k_lg_take's status words
 }
 
-// Live entries per chunk of the round's windows.
-__global__ void __launch_bounds__(kScanThreads) k_lg_count(DevState s, int phase) {
+// One take round in one pass (a decoupled look-back over the chunks of each
+// take).  CTAs draw chunks in order from a ticket; each counts its chunk's
+// live entries and publishes the count at once, then adds up the published
+// counts of the take's earlier chunks (their inclusive prefix where already
+// known) to learn how many of the take's live entries lie before it, and
+// consumes the ones that fall within the take: victims marked in log order,
+// live counts, the head.  A tied group's last entry is recorded for the tie
+// rule instead.  The take's last chunk, if the window ended short, leaves
+// the count for a second round.  Status words: 0 unpublished, kAgg | count,
+// kIncl | inclusive prefix.  The wait for a predecessor is bounded.
+constexpr uint64_t kAgg = 1ull << 62, kIncl = 2ull << 62, kValMask = (1ull << 62) - 1;
+constexpr int kLookbackSpins = 1 << 22;
+
+__global__ void __launch_bounds__(kScanThreads) k_lg_take(DevState s, int phase, cudaGraphConditionalHandle next,
+                                                          int has_next) {
   s = with_args(s);
   __shared__ int32_t sc0[kMaxLogs + 1];
-  const Ctl* c = s.ctl;
-  const int nch = c->lg_nchunks;
-  if (nch == 0) return;
-  const int ntk = c->lg_ntk;
-  for (int t = threadIdx.x; t <= ntk; t += blockDim.x) sc0[t] = s.lg_c0[t];
-  __syncthreads();
-  const uint32_t* eb = ent_blk(s, c->lg_buf);
-  const uint64_t* es = ent_st(s, c->lg_buf);
-  for (int q = blockIdx.x; q < nch; q += gridDim.x) {
-    const int t = range_of(sc0, ntk, q);
-    const int64_t cur = s.lg_tk[t].cur, wend = s.lg_tk[t].wend;
-    const int64_t e0 = cur + (int64_t)(q - sc0[t]) * kLogChunk + threadIdx.x * 4;
-    int n = 0;
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int64_t e = e0 + u;
-      if (e < wend && live_entry(s, eb[e], es[e], phase == 1)) ++n;
-    }
-    const int tot = block_sum(n);
-    if (threadIdx.x == 0) s.lg_ck[q] = (uint32_t)tot;
-  }
-}
-
-// Per take (a warp each): the chunk holding its last entry, or, when the
-// window falls short, another round over the rest of the log.
-__global__ void __launch_bounds__(1024) k_lg_resolve(DevState s, cudaGraphConditionalHandle next, int has_next) {
-  s = with_args(s);
-  Ctl* c = s.ctl;
-  if (c->lg_nchunks == 0) return;
-  const int ntk = c->lg_ntk;
-  const int w = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = lane_id();
-  if (w >= ntk) return;
-  LogTake k = s.lg_tk[w];
-  if (k.done) return;
-  const int q0 = s.lg_c0[w], q1 = s.lg_c0[w + 1];
-  const int64_t rem = k.want - k.got;
-  int64_t before = 0, cut_rank = 0;
-  int cut = -1;
-  for (int qb = q0; qb < q1; qb += 32) {
-    const int q = qb + lane;
-    const int64_t v = q < q1 ? (int64_t)s.lg_ck[q] : 0;
-    const int64_t incl = warp_incl_scan(v);
-    const unsigned hit = __ballot_sync(kFull, q < q1 && before + incl >= rem);
-    if (hit) {
-      const int l = __ffs(hit) - 1;
-      const int64_t il = __shfl_sync(kFull, incl, l), vl = __shfl_sync(kFull, v, l);
-      cut = qb + l;
-      cut_rank = rem - (before + il - vl);
-      break;
-    }
-    before += __shfl_sync(kFull, incl, 31);
-  }
-  if (lane != 0) return;
-  if (cut >= 0) {
-    k.cut = cut;
-    k.cut_rank = cut_rank;
-    k.done = 1;
-  } else {
-    k.got += before;  // the window's live entries are all taken this round
-    if (k.wend >= s.lg_desc[k.log].tail) {
-      c->internal_error = 1;  // the log holds fewer live entries than counted
-    } else {
-      c->lg_more = 1;
-      if (has_next) cudaGraphSetConditional(next, 1);
-    }
-  }
-  s.lg_tk[w] = k;
-}
-
-// Consume each take's entries up to its last one: mark the victims, take
-// them off their logs' live counts, move the heads.  A tied group's last
-// entry is recorded for the tie rule instead.
-__global__ void __launch_bounds__(kScanThreads) k_lg_mark(DevState s, int phase) {
-  s = with_args(s);
-  __shared__ int32_t sc0[kMaxLogs + 1];
+  __shared__ int s_q;
+  __shared__ int64_t s_before;
   Ctl* c = s.ctl;
   const int nch = c->lg_nchunks;
   if (nch == 0) return;
   const int ntk = c->lg_ntk;
   for (int t = threadIdx.x; t <= ntk; t += blockDim.x) sc0[t] = s.lg_c0[t];
-  __syncthreads();
   const uint32_t* eb = ent_blk(s, c->lg_buf);
   const uint64_t* es = ent_st(s, c->lg_buf);
+  unsigned long long* status = reinterpret_cast<unsigned long long*>(s.lg_ck_out);
   const int32_t gk = s.G * kClasses;
-  for (int q = blockIdx.x; q < nch; q += gridDim.x) {
+  for (;;) {
+    __syncthreads();  // sc0 loaded; s_q, s_before of the last chunk consumed
+    if (threadIdx.x == 0) s_q = (int)atomicAdd(&c->lg_ticket, 1u);
+    __syncthreads();
+    const int q = s_q;
+    if (q >= nch) break;
     const int t = range_of(sc0, ntk, q);
     const LogTake k = s.lg_tk[t];
-    if (k.cut >= 0 && q > k.cut) continue;
-    const int64_t lim = (k.cut >= 0 && q == k.cut) ? k.cut_rank : LLONG_MAX;
-    const int64_t e0 = k.cur + (int64_t)(q - sc0[t]) * kLogChunk + threadIdx.x * 4;
+    const int qf = sc0[t], ql = sc0[t + 1] - 1;
+    const int64_t e0 = k.cur + (int64_t)(q - qf) * kLogChunk + threadIdx.x * 4;
     uint32_t b[4];
     uint64_t st[4];
     bool live[4];
@@ -326,15 +274,45 @@ __global__ void __launch_bounds__(kScanThreads) k_lg_mark(DevState s, int phase)
     }
     int tot;
     int64_t r = block_excl_scan(n, &tot);
+    if (threadIdx.x == 0) {
+      int64_t before = 0;
+      if (q == qf) {
+        atomicExch(status + q, kIncl | (uint64_t)tot);
+      } else {
+        atomicExch(status + q, kAgg | (uint64_t)tot);
+        int j = q - 1, spins = 0;
+        for (;;) {
+          const uint64_t w = *reinterpret_cast<volatile unsigned long long*>(status + j);
+          if (w & kIncl) {
+            before += (int64_t)(w & kValMask);
+            break;
+          }
+          if (w & kAgg) {
+            before += (int64_t)(w & kValMask);
+            --j;  // the take's first chunk publishes an inclusive prefix: j stays >= qf
+            continue;
+          }
+          if (++spins > kLookbackSpins) {
+            c->internal_error = 1;  // never expected: reported as a step status
+            break;
+          }
+          __nanosleep(64);
+        }
+        atomicExch(status + q, kIncl | (uint64_t)(before + tot));
+      }
+      s_before = before;
+    }
+    __syncthreads();
+    const int64_t rem = k.want - (k.got + s_before);  // the take's entries still to consume here
     int taken = 0;
     int32_t other[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       other[u] = -1;
       if (!live[u]) continue;
-      if (r < lim) {
+      if (r < rem) {
         const int64_t e = e0 + u;
-        const bool last = k.cut >= 0 && q == k.cut && r == lim - 1;
+        const bool last = r == rem - 1;
         if (last && k.tie) {
           const uint64_t key = lg_segmented(s) ? (st[u] | (uint64_t)s.blk_klass[b[u]] << 62) : st[u];
           s.lg_tie[k.log / kClasses] = TieItem{key, e, b[u], k.log};
@@ -353,13 +331,28 @@ __global__ void __launch_bounds__(kScanThreads) k_lg_mark(DevState s, int phase)
 #pragma unroll
     for (int u = 0; u < 4; ++u) agg_add_i64(s.lg_live, (uint32_t)other[u], -1, other[u] >= 0);
     const int sum = block_sum(taken);
-    if (threadIdx.x == 0 && sum) {
-      atomic_add_i64(s.lg_live + k.log, -sum);
-      if (phase == 0) {
-        const int32_t B = lg_log_b(s, (uint32_t)(k.log % kClasses));
-        if (B >= 0) atomic_add_i64(s.lg_live + B, -sum);
+    if (threadIdx.x == 0) {
+      if (sum) {
+        atomic_add_i64(s.lg_live + k.log, -sum);
+        if (phase == 0) {
+          const int32_t B = lg_log_b(s, (uint32_t)(k.log % kClasses));
+          if (B >= 0) atomic_add_i64(s.lg_live + B, -sum);
+        }
+        atomic_add_i64(&c->n_victims_marked, sum);
       }
-      atomic_add_i64(&c->n_victims_marked, sum);
+      if (rem > 0 && rem <= tot) {
+        s.lg_tk[t].done = 1;
+      } else if (q == ql && rem > tot) {
+        // the window ended short: every live entry in it is taken, and a
+        // second round continues from its end
+        s.lg_tk[t].got = k.got + s_before + tot;
+        if (k.wend >= s.lg_desc[k.log].tail) {
+          c->internal_error = 1;  // the log holds fewer live entries than counted
+        } else {
+          c->lg_more = 1;
+          if (has_next) cudaGraphSetConditional(next, 1);
+        }
+      }
     }
   }
 }
@@ -411,7 +404,10 @@ __global__ void __launch_bounds__(kAppChunk) k_lg_app_count(DevState s) {
   s = with_args(s);
   __shared__ uint32_t hist[kMaxLogs];
   Ctl* c = s.ctl;
-  if (blockIdx.x == 0 && threadIdx.x == 0) c->lg_cmp = 0;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    c->lg_cmp = 0;
+    c->lg_ticket = 0;  // k_lg_take left its chunk count there
+  }
   if (c->status != PS_OK) return;
   const int64_t nb = c->nblocks;
   const int q = blockIdx.x;
@@ -712,14 +708,11 @@ int32_t launch_queue_select(const DevState& s, cudaStream_t st, const CaptureCtx
                             bool plain_first, int* launches) {
   cudaGraphConditionalHandle h1 = 0;
   if (cap && !cond_handle(st, &h1)) return PS_ERR_CUDA;
-  const int rgrid = (s.lg_L * 32 + 1023) / 1024;
   auto round = [&](cudaStream_t q, int r) {
     if (plain_first && r == 0) k_lg_plan<<<1, 1024, 0, q>>>(s, phase, r);  // its predecessor is a join
     else launch_k(k_lg_plan, 1, 1024, 0, q, s, phase, r);
-    launch_k(k_lg_count, kScanGrid, kScanThreads, 0, q, s, phase);
-    launch_k(k_lg_resolve, rgrid, 1024, 0, q, s, h1, (cap && r == 0) ? 1 : 0);
-    launch_k(k_lg_mark, kScanGrid, kScanThreads, 0, q, s, phase);
-    *launches += 4;
+    launch_k(k_lg_take, kScanGrid, kScanThreads, 0, q, s, phase, h1, (cap && r == 0) ? 1 : 0);
+    *launches += 2;
   };
   round(st, 0);
   if (cap) {
