@@ -52,3 +52,28 @@ def test_workspace_size_is_host_computable(lib):
     assert n > 0 and n % 256 == 0
     assert L.ps_workspace_bytes(1 << 20, 15, 64, ctypes.byref(p), 4096, 12_000_000) == 0  # odd block size
     assert L.ps_workspace_bytes(0, 16, 64, ctypes.byref(p), 4096, 12_000_000) == 0
+
+
+def test_queue_flags_grow_the_workspace_by_the_log_buffers(lib):
+    """PS_FLAG_INDEXED_QUEUES adds two buffers of 16 (N + max_tokens / bs)
+    entries of 12 bytes (block id, stamp) plus per-step scratch."""
+    from paper_2608_01657_gb300 import binding as B
+    L = B.load()
+    N, bs, G, R, T = 1 << 16, 16, 8, 256, 1 << 20
+    base = B.Params(rho=(2.0,), beta=(6.0,)).to_c(G)
+    q = B.Params(rho=(2.0,), beta=(6.0,), flags=B.PS_FLAG_INDEXED_QUEUES).to_c(G)
+    n0 = L.ps_workspace_bytes(N, bs, G, ctypes.byref(base), R, T)
+    n1 = L.ps_workspace_bytes(N, bs, G, ctypes.byref(q), R, T)
+    P = 16 * (N + T // bs)
+    assert n1 - n0 >= 2 * 12 * P
+    assert n1 - n0 < 2 * 12 * P + (16 << 20)
+
+
+def test_host_calls_refuse_bad_arguments_before_any_device_work(lib):
+    """Null handles and out-of-range slots return PS_ERR_INVALID_ARG."""
+    from paper_2608_01657_gb300 import binding as B
+    L = B.load()
+    assert L.ps_step_host_wait(None, 0) == B.PS_ERR_INVALID_ARG
+    assert L.ps_step_host_async(None, None, 0, 1, 0, None, None, None, None, None, None) == B.PS_ERR_INVALID_ARG
+    assert L.ps_step_host(None, None, 1, 0, None, None, None, None, None, None) == B.PS_ERR_INVALID_ARG
+    assert L.ps_step(None, None, 1, 0, None, None, None, None, None, None) == B.PS_ERR_INVALID_ARG
