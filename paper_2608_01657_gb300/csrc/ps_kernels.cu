@@ -320,8 +320,10 @@ template <int PPB>
 struct HashCfg {
   static constexpr int BS = 2 * PPB;
   static constexpr int kWindow = kSegBlocks * BS + 8;  // tokens staged per warp (+ alignment slack)
-  static constexpr int kWarps = (64 * 1024) / (kWindow * 4) < 1 ? 1
-                                : ((64 * 1024) / (kWindow * 4) > 8 ? 8 : (64 * 1024) / (kWindow * 4));
+  // staging windows of up to 66 KB a CTA: three CTAs fit an SM's shared
+  // memory (and, at 80 registers a thread, its register file)
+  static constexpr int kWarps = (66 * 1024) / (kWindow * 4) < 1 ? 1
+                                : ((66 * 1024) / (kWindow * 4) > 8 ? 8 : (66 * 1024) / (kWindow * 4));
   static constexpr size_t kSmem = (size_t)kWarps * kWindow * 4 + (size_t)kWarps * 8;
 };
 
