@@ -382,7 +382,7 @@ def run_own(args, ws, rank, local):
         "step_roofline": {"bound": "hbm", "achieved": step_gbs, "peak": peak, "unit": "GB/s",
                           "frac": step_gbs / peak, "algorithmic_bytes_per_step": alg / args.steps,
                           "peak_kind": peak_kind},
-        "roofline": {"bound": "hbm", "kernel": "hash_lookup stage: k_hash + k_keys_lookup + k_pin_claim", "achieved": hl_gbs, "peak": peak, "unit": "GB/s",
+        "roofline": {"bound": "hbm", "kernel": "hash_lookup stage: k_hash_lane + k_keys_lookup + k_pin_claim", "achieved": hl_gbs, "peak": peak, "unit": "GB/s",
                      "frac": hl_gbs / peak, "traffic": hash_lookup_traffic(), "bytes_per_launch": hl_bytes,
                      "ms_per_launch": hl_ms, "peak_kind": peak_kind},
         "stages_ms_per_step": {n: round(float(v) / args.steps, 4) for n, v in zip(STAGES, stage_ms)},

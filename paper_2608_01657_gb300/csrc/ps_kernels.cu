@@ -478,6 +478,109 @@ __global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) 
   if (lane == 0) s.seg_tot[seg] = carry;
 }
 
+// Stage 1, one lane per block (block sizes 4, 8 and 16): each lane reads its
+// block's tokens straight from global memory and forms both NH sums itself,
+// so no staging window limits the resident warps and no shuffle network
+// combines partial sums.  A segment belongs to one request, whose blocks all
+// start at the same word offset r = (o_i + m bs) mod 4: each lane loads the
+// 16-byte words covering its block (bs / 4 + 1 of them) and takes its tokens
+// at the warp-uniform offset r.  A block whose words would run past the
+// step's last token, or a token buffer that is not 16-byte aligned, is read
+// token by token.  The chain scan and its outputs are those of k_hash.
+template <int PPB>
+__global__ void __launch_bounds__(256) k_hash_lane(DevState s) {
+  s = with_args(s);
+  constexpr int BS = 2 * PPB;
+  constexpr int NW = BS / 4 + 1;  // 16-byte words covering a block at any word offset
+  static_assert(BS % 4 == 0, "whole-block lanes need bs a multiple of 4");
+  __shared__ uint32_t sk[BS + 2];  // the NH key words (read by every lane alike)
+  const Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  if (threadIdx.x < BS + 2) sk[threadIdx.x] = s.key_words[threadIdx.x];
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = lane_id();
+  const int64_t seg = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
+  if (seg >= c->nsegs) return;
+  const uint32_t i = s.seg_req[seg];
+  const int n = s.rq_n[i];
+  const int m0 = (int)(seg - s.rq_sbase[i]) * kSegBlocks;
+  const int m1 = tmin(n, m0 + kSegBlocks);
+  const int64_t o0 = s.in_offsets[i];
+  const int pbase = s.rq_pbase[i];
+  const int64_t T = c->T;
+  const int r = (int)(o0 & 3);  // the same for every block of the request
+  const bool vec = s.tokens_aligned16;
+  const uint64_t Kd = s.digest_mul;
+  uint64_t kp[5];
+#pragma unroll
+  for (int j = 0; j < 5; ++j) kp[j] = s.kc_pow[1 << j];
+  const uint64_t kpl = s.kc_pow[lane + 1];
+  uint64_t carry = 0;  // local chain value at the block before the chunk
+  for (int c0 = m0; c0 < m1; c0 += 32) {
+    const int nb = tmin(32, m1 - c0);
+    uint64_t d1 = 0, d2 = 0;
+    if (lane < nb) {
+      const int64_t g0 = o0 + (int64_t)(c0 + lane) * BS;  // the block's first token
+      const int64_t a0 = g0 - r;                            // 16-byte aligned when vec
+      uint32_t tok[BS];
+      if (vec && a0 + 4 * NW <= T) {
+        uint32_t w[4 * NW];
+        const uint4* src = reinterpret_cast<const uint4*>(s.in_tokens + a0);
+#pragma unroll
+        for (int q = 0; q < NW; ++q) {
+          const uint4 v = __ldg(src + q);
+          w[4 * q] = v.x;
+          w[4 * q + 1] = v.y;
+          w[4 * q + 2] = v.z;
+          w[4 * q + 3] = v.w;
+        }
+        // r is warp-uniform: four statically indexed forms
+        switch (r) {
+          case 0:
+#pragma unroll
+            for (int j = 0; j < BS; ++j) tok[j] = w[j];
+            break;
+          case 1:
+#pragma unroll
+            for (int j = 0; j < BS; ++j) tok[j] = w[j + 1];
+            break;
+          case 2:
+#pragma unroll
+            for (int j = 0; j < BS; ++j) tok[j] = w[j + 2];
+            break;
+          default:
+#pragma unroll
+            for (int j = 0; j < BS; ++j) tok[j] = w[j + 3];
+            break;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < BS; ++j) tok[j] = (uint32_t)s.in_tokens[g0 + j];
+      }
+#pragma unroll
+      for (int k = 0; k < PPB; ++k) {
+        const uint32_t tx = tok[2 * k], ty = tok[2 * k + 1];
+        d1 += (uint64_t)(tx + sk[2 * k]) * (uint64_t)(ty + sk[2 * k + 1]);
+        d2 += (uint64_t)(tx + sk[2 * k + 2]) * (uint64_t)(ty + sk[2 * k + 3]);
+      }
+    }
+    // D_m, then the inclusive scan of the affine maps x -> Kc x + D
+    uint64_t bb = lane < nb ? add61(red61(d1), mul61(Kd, red61(d2))) : 0;
+#pragma unroll
+    for (int j = 0; j < 5; ++j) {
+      const uint64_t t = __shfl_up_sync(kFull, bb, 1 << j);
+      if (lane >= (1 << j)) bb = add61(bb, mul61(kp[j], t));
+    }
+    const uint64_t B = add61(mul61(kpl, carry), bb);
+    if (lane < nb) {
+      s.pos_key[pbase + c0 + lane] = B;
+      s.pos_req[pbase + c0 + lane] = i;
+    }
+    carry = __shfl_sync(kFull, B, nb - 1);
+  }
+  if (lane == 0) s.seg_tot[seg] = carry;
+}
+
 // Stage 2: block keys and the longest cached prefix (n_cached of Alg. 1),
 // thread per position: C_in = the chain value entering the position's
 // segment (C = Kc^256 C + B_end over the request's earlier segments),
@@ -2133,12 +2236,16 @@ static void launch_hash_t(const DevState& s, cudaStream_t st) {
   using Cfg = HashCfg<PPB>;
   k_hash<PPB><<<(int)((s.max_segments + Cfg::kWarps - 1) / Cfg::kWarps), Cfg::kWarps * 32, Cfg::kSmem, st>>>(s);
 }
+template <int PPB>
+static void launch_hash_lane(const DevState& s, cudaStream_t st) {
+  k_hash_lane<PPB><<<(int)((s.max_segments + 7) / 8), 256, 0, st>>>(s);
+}
 static int32_t launch_hash(const DevState& s, cudaStream_t st) {
   switch (s.bs / 2) {
     case 1: launch_hash_t<1>(s, st); break;
-    case 2: launch_hash_t<2>(s, st); break;
-    case 4: launch_hash_t<4>(s, st); break;
-    case 8: launch_hash_t<8>(s, st); break;
+    case 2: launch_hash_lane<2>(s, st); break;
+    case 4: launch_hash_lane<4>(s, st); break;
+    case 8: launch_hash_lane<8>(s, st); break;
     case 16: launch_hash_t<16>(s, st); break;
     case 32: launch_hash_t<32>(s, st); break;
     default: return PS_ERR_INVALID_ARG;
