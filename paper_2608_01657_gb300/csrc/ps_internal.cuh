@@ -131,15 +131,14 @@ struct LogDesc {
 };
 // One log's share of a select phase: consume its first 'want' live entries.
 struct LogTake {
-  int64_t want;      // live entries to consume (with 'tie', the last one is recorded, not taken)
-  int64_t got;       // consumed in earlier rounds
-  int64_t cur;       // where this round's window starts
-  int64_t wend;      // where it ends
-  int64_t cut_rank;  // entries to consume in the cut chunk
+  int64_t want;  // live entries to consume (with 'tie', the last one is recorded, not taken)
+  int64_t got;   // consumed in earlier rounds
+  int64_t cur;   // where this round's window starts
+  int64_t wend;  // where it ends
   int32_t log;
-  int32_t tie;       // the last entry is the group's tie candidate (Eq. 7)
-  int32_t cut;       // chunk holding the last entry in this round, or -1
-  int32_t done;      // the last entry was found (this round or earlier)
+  int32_t tie;   // the last entry is the group's tie candidate (Eq. 7)
+  int32_t done;  // the last entry was found (this round or earlier)
+  int32_t pad;
 };
 struct TieItem {
   uint64_t key;  // (class, stamp) order key of the tied group's next candidate
@@ -281,8 +280,9 @@ struct DevState {
   uint32_t* lg_app;        // [L][app_chunks] append counts per chunk, then offsets
   LogTake* lg_tk;          // [L] takes of a select phase
   int32_t* lg_c0;          // [L + 1] first chunk of each take (or log)
-  uint32_t* lg_ck;         // [max_chunks] live entries per chunk
-  int64_t* lg_ck_out;      // [max_chunks] where a chunk's live entries go (compaction)
+  uint32_t* lg_ck;         // [max_chunks] live entries per chunk (compaction)
+  int64_t* lg_ck_out;      // [max_chunks] a take round's look-back status words; in a
+                           // compaction, where each chunk's live entries go
   TieItem* lg_tie;         // [G]
   StepArgs* args;          // this call's arguments (device memory)
   // current step inputs / outputs (kernels refresh them from *args)

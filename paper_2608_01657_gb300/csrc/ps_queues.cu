@@ -169,7 +169,6 @@ __global__ void __launch_bounds__(1024) k_lg_plan(DevState s, int phase, int rou
             t.want = w;
             t.log = l;
             t.tie = tie && x == 0;
-            t.cut = -1;
             t.cur = s.lg_desc[l].head;
             tk[nt++] = t;
           }
@@ -200,7 +199,6 @@ __global__ void __launch_bounds__(1024) k_lg_plan(DevState s, int phase, int rou
         const int64_t first = (s.flags & PS_FLAG_QUEUE_SHORT_WINDOWS) ? kLogChunk : rem + rem / 4 + kLogChunk;
         const int64_t wl = round == 0 ? tmin<int64_t>(avail, first) : avail;
         k.wend = k.cur + wl;
-        k.cut = -1;
         nch = (int)((wl + kLogChunk - 1) / kLogChunk);
         if (nch == 0) c->internal_error = 1;  // victims owed by a log with nothing left to scan
         s.lg_tk[t] = k;
