@@ -157,6 +157,19 @@ def test_parity_queues_fuzz(policy, seed, N, G, R, contracts, prefixes, flags):
 
 
 @pytest.mark.parametrize("policy", QUEUE_POLICIES)
+@pytest.mark.parametrize("flags", [0, 1, 2])
+def test_parity_queues_many_groups(policy, flags):
+    """37 groups (114 logs), three contracts, ragged requests: many logs
+    share each scan, layout and compaction."""
+    G = 37
+    steps = W.fuzz_steps(17, G, 12, 120, docs_per_group=2, doc_blocks=6, fresh_max_blocks=3,
+                         with_contracts=3, now_stride=2, empty_every=13)
+    kw = dict(rho=(2.0, 1.5, 1.0), beta=(6.0, 5.0, 4.0), flags=flags | IQ, contract_of_group=[g % 3 for g in range(G)])
+    gpu, orc = _pair(180, 16, G, policy, kw, max_requests=12, max_tokens=max(st.num_tokens for st in steps))
+    _run(gpu, orc, steps, state_every=9, label=f"queues/groups{G}/f{flags}/{policy}")
+
+
+@pytest.mark.parametrize("policy", QUEUE_POLICIES)
 def test_parity_queues_direct_launches(policy):
     """The indexed queues launched kernel by kernel (their second scan round
     and the compaction then run as kernels that find nothing to do)."""
