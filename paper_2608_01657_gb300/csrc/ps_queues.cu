@@ -129,9 +129,10 @@ __global__ void __launch_bounds__(1024) k_lg_cand(DevState s) {
   }
 }
 
-// Round 0 lists the phase's takes; every round sizes the window of each take
-// still open (round 0: a quarter more than the entries it still needs plus a
-// chunk; round 1: the rest of the log) and numbers the chunks.
+// The first scan round lists the phase's takes; every round sizes the window
+// of each take still open (the first: a quarter more than the entries it
+// still needs plus a chunk; the second: the rest of the log) and numbers the
+// chunks.
 __global__ void __launch_bounds__(1024) k_lg_plan(DevState s, int phase, int round) {
   s = with_args(s);
   Ctl* c = s.ctl;
