@@ -151,3 +151,34 @@ def test_no_segmentation_flag_uses_recency_inside_the_group():
         # segmented: Prob first -> the older Prob block Y (id 1); unsegmented:
         # plain recency -> X (id 0, stamped at t=2 before Y and Z)
         assert list(r["evicted_ids"]) == ([1] if want == "new" else [0])
+
+
+def test_normalized_debt_and_decrements_with_three_contracts():
+    """Eq. 5 and Eq. 8 with the paper's three contract tiers (rho 64, 40, 16
+    blocks a tick, beta 256, 192, 128), hand-derived in fixed point.
+
+    Tick 1: group A (contract rho 40) admits 217 blocks: B = 192 - 217 = -25;
+    group B (contract rho 16 = rho_min) admits 134: B = -6.  Eq. 5:
+      D~_A = floor(25 * 2^20 * 16 / 40) = 10 * 2^20,   D~_B = 6 * 2^20.
+    Eq. 8 (rho_max over the indebted contracts of each group):
+      delta_A = floor(2^20 * 16 / 40) = 419430,        delta_B = 2^20.
+    The pool (351 blocks) is then full.  Still at tick 1 (no refill), group C
+    (contract rho 64, no debt) admits 20 fresh blocks: 20 victims.  Alg. 2
+    takes the larger projected score each time: A while 10485760 - k*419430
+    exceeds 6291456 (k = 0..10: 11 victims, the last at 6291460), then B,
+    A, A, B, A, A, A (4194310 > 4194304), B, A: 17 from A and 3 from B.
+    Raw instead of normalized debt, or the ratio inverted, changes the split.
+    """
+    prm = O.Params(rho=(64.0, 40.0, 16.0), beta=(256.0, 192.0, 128.0), contract_of_group=[1, 2, 0])
+    oc = O.OracleCache(351, 16, 3, "prefixshield", prm)
+    g, o, t, _ = make_step([obj_tokens("A", blocks=217), obj_tokens("B", blocks=134)], [0, 1])
+    r = oc.step(1, g, o, t)
+    assert r["status"] == 0 and list(r["admitted_blocks"]) == [217, 134]
+    assert [int(x) for x in r["debt_raw"]] == [25 << 20, 6 << 20, 0]
+    assert [int(x) for x in r["debt_norm"]] == [10 << 20, 6 << 20, 0]
+    before = oc.export()
+    g, o, t, _ = make_step([obj_tokens("C", blocks=20)], [2])
+    r = oc.step(1, g, o, t)
+    assert r["status"] == 0 and int(r["admitted_blocks"][0]) == 20
+    owners = before["group"][r["evicted_ids"]]
+    assert (int((owners == 0).sum()), int((owners == 1).sum()), int((owners == 2).sum())) == (17, 3, 0)
