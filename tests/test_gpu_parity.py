@@ -219,6 +219,24 @@ def test_parity_queues_alg2_ties():
         _run(gpu, orc, steps, label=f"queues/ties/f{flags}")
 
 
+@pytest.mark.parametrize("flags", [0, O.FLAG_INDEXED_QUEUES])
+def test_parity_three_contract_tiers(flags):
+    """The paper's contract tiers with debts whose fixed-point decrements are
+    not whole blocks (Eq. 5, Eq. 8): the hand-derived scenario of the oracle
+    pins, then fuzz steps on the same pool."""
+    from _util import make_step, obj_tokens
+    kw = dict(rho=(64.0, 40.0, 16.0), beta=(256.0, 192.0, 128.0), contract_of_group=[1, 2, 0], flags=flags)
+    gpu, orc = _pair(351, 16, 3, "prefixshield", kw, max_requests=4, max_tokens=217 * 16 + 134 * 16)
+    seq = []
+    g, o, t, _ = make_step([obj_tokens("A", blocks=217), obj_tokens("B", blocks=134)], [0, 1])
+    seq.append(W.Step(index=0, now=1, groups=g, offsets=o, tokens=t))
+    g, o, t, _ = make_step([obj_tokens("C", blocks=20)], [2])
+    seq.append(W.Step(index=1, now=1, groups=g, offsets=o, tokens=t))
+    for k, st in enumerate(W.fuzz_steps(23, 3, 4, 40, docs_per_group=3, doc_blocks=40, fresh_max_blocks=30)):
+        seq.append(W.Step(index=2 + k, now=2 + k, groups=st.groups, offsets=st.offsets, tokens=st.tokens))
+    _run(gpu, orc, seq, state_every=5, label=f"tiers/f{flags}")
+
+
 def test_parity_alg2_ties():
     """Groups with equal debt and equal decrements force Eq. 7's tie rule."""
     G = 6
