@@ -356,7 +356,12 @@ def run_own(args, ws, rank, local):
 
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, cache, steps, dsteps, flush, R)
+        e2e = run_e2e(args, cache, steps, dsteps, flush, R, ws)
+        # the whole job: every rank's requests over the slowest rank's time
+        reqs_all = sum_over_ranks(ws, e2e.pop("_requests"))
+        t_e2e = max_over_ranks(ws, e2e.pop("_seconds"))
+        e2e["value"] = reqs_all / t_e2e
+        e2e["ms_per_step"] = 1e3 * t_e2e / args.steps
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         n_cpu = args.prefill + args.cpu_steps
@@ -395,7 +400,7 @@ def run_own(args, ws, rank, local):
     print(json.dumps(line), flush=True)
 
 
-def run_e2e(args, cache, steps, dsteps, flush, R):
+def run_e2e(args, cache, steps, dsteps, flush, R, ws=1):
     """Same steps through ps_step_host_async: pinned host inputs copied in,
     outputs written back to pinned host memory, inside the timed region."""
     import numpy as np
@@ -434,6 +439,7 @@ def run_e2e(args, cache, steps, dsteps, flush, R):
     gc.collect()
     gc.disable()  # no collector pauses inside the timed host loop
     torch.cuda.synchronize()
+    barrier(ws)
     t0 = time.perf_counter()
     for k, (now, g, o, t) in enumerate(host):
         flush.zero_()
@@ -448,9 +454,11 @@ def run_e2e(args, cache, steps, dsteps, flush, R):
     gc.enable()
     n = len(host)
     per = [b - a for a, b in zip([t0] + done_at[:-1], done_at)]
-    return {"value": sum(len(h[1]) for h in host) / t_sum, "unit": "requests/s",
+    nreq = sum(len(h[1]) for h in host)
+    return {"value": nreq / t_sum, "unit": "requests/s",
             "h2d_bytes_per_step": h2d // n, "d2h_bytes_per_step": d2h // n,
             "ms_per_step": 1e3 * t_sum / n, "api": "ps_step_host_async (two slots in flight)",
+            "_requests": nreq, "_seconds": t_sum,
             "step_ms": {"min": 1e3 * min(per), "median": 1e3 * statistics.median(per), "max": 1e3 * max(per)}}
 
 
