@@ -182,3 +182,27 @@ def test_normalized_debt_and_decrements_with_three_contracts():
     assert r["status"] == 0 and int(r["admitted_blocks"][0]) == 20
     owners = before["group"][r["evicted_ids"]]
     assert (int((owners == 0).sum()), int((owners == 1).sum()), int((owners == 2).sum())) == (17, 3, 0)
+
+
+def test_gate_reads_debt_before_the_request_charge_class_after():
+    """Reading A14 (OnRequest, OnTouch, OnCacheFullBlocks in that order),
+    derived by hand.  beta = 4, rho = 1, all at tick 1 (no refill):
+      step 1: P (2 blocks) admitted: B = 2, class Prob (first admission);
+      step 2: P + X (X = 3 new blocks): P is proven (q = 1, admitted) and the
+        gate reads D before this request's charge (0): both P blocks are
+        promoted.  Then the charge: B = 2 - 3 = -1, so X's blocks are Prob
+        (B < -eps) and the raw debt is 1 block.
+    A gate that read the debt after the charge would hold P back; a class
+    taken from the balance before the charge would make X Normal."""
+    oc = O.OracleCache(64, 16, 1, "prefixshield", O.Params(rho=(1.0,), beta=(4.0,)))
+    P, X = obj_tokens("P", blocks=2), obj_tokens("X", blocks=3)
+    r = oc.step(1, *make_step([P])[:3])
+    assert r["admitted_ids"].tolist() == [0, 1]
+    r = oc.step(1, *make_step([np.concatenate([P, X])])[:3])
+    assert r["hit_blocks"].tolist() == [2] and r["admitted_blocks"].tolist() == [3]
+    s = oc.stats()[0]
+    assert (int(s[O.STAT_NAMES.index("promotions")]), int(s[O.STAT_NAMES.index("gated_reuses")])) == (2, 0)
+    e = oc.export()
+    assert e["klass"][:2].tolist() == [2, 2]      # P: Reuse
+    assert e["klass"][2:5].tolist() == [0, 0, 0]  # X: Probationary
+    assert int(r["debt_raw"][0]) == 1 << 20
