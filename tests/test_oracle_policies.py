@@ -206,3 +206,20 @@ def test_gate_reads_debt_before_the_request_charge_class_after():
     assert e["klass"][:2].tolist() == [2, 2]      # P: Reuse
     assert e["klass"][2:5].tolist() == [0, 0, 0]  # X: Probationary
     assert int(r["debt_raw"][0]) == 1 << 20
+
+
+def test_history_includes_earlier_requests_of_the_same_step():
+    """Reading A13, derived by hand: one step, r0 = P (2 new blocks, first
+    admission: Prob, B = 4 - 2 = 2), then r1 = P: its two keys are r0's
+    granted claims (in-step hits).  r1's q counts r0's request (q = 1) and
+    P counts as admitted by r0, so r1's touch is proven; the gate reads
+    D = 0 and both new blocks are promoted: they enter the pool as Reuse."""
+    oc = O.OracleCache(64, 16, 1, "prefixshield", O.Params(rho=(1.0,), beta=(4.0,)))
+    P = obj_tokens("P", blocks=2)
+    r = oc.step(1, *make_step([P, P])[:3])
+    assert r["hit_blocks"].tolist() == [0, 2] and r["admitted_blocks"].tolist() == [2, 0]
+    s = oc.stats()[0]
+    assert int(s[O.STAT_NAMES.index("instep_hit_blocks")]) == 2
+    assert (int(s[O.STAT_NAMES.index("promotions")]), int(s[O.STAT_NAMES.index("gated_reuses")])) == (2, 0)
+    assert oc.export()["klass"][:2].tolist() == [2, 2]
+    assert int(r["debt_raw"][0]) == 0
