@@ -237,6 +237,29 @@ def test_parity_three_contract_tiers(flags):
     _run(gpu, orc, seq, state_every=5, label=f"tiers/f{flags}")
 
 
+@pytest.mark.parametrize("flags", [0, O.FLAG_INDEXED_QUEUES])
+def test_parity_hand_derived_corners(flags):
+    """The hand-derived oracle pins of the grant rule, the hook order inside a
+    request and history within a step, replayed through the GPU step."""
+    from _util import make_step, obj_tokens
+    P, Q, S, T, X = (obj_tokens(n, blocks=b) for n, b in (("P", 3), ("Q", 1), ("S", 3), ("T", 1), ("X", 3)))
+    P2 = obj_tokens("P2", blocks=2)
+    cases = [
+        (5, 100.0, [[P, np.concatenate([P, Q]), S], [S]]),       # ranks past avail
+        (4, 100.0, [[P, S, np.concatenate([S, T])]]),            # a run stopped by an ungranted key
+        (64, 4.0, [[P2], [np.concatenate([P2, X])]]),            # gate before the charge, class after
+        (64, 4.0, [[P2, P2]]),                                   # history within a step
+    ]
+    for ci, (N, beta, steps) in enumerate(cases):
+        kw = dict(rho=(1.0,) if beta == 4.0 else (100.0,), beta=(beta,), flags=flags)
+        gpu, orc = _pair(N, 16, 1, "prefixshield", kw, max_requests=3, max_tokens=2048)
+        seq = []
+        for k, prompts in enumerate(steps):
+            g, o, t, _ = make_step(prompts)
+            seq.append(W.Step(index=k, now=1, groups=g, offsets=o, tokens=t))
+        _run(gpu, orc, seq, label=f"corner{ci}/f{flags}")
+
+
 def test_parity_alg2_ties():
     """Groups with equal debt and equal decrements force Eq. 7's tie rule."""
     G = 6
