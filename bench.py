@@ -59,6 +59,11 @@ def parse_args():
     ap.add_argument("--capacity-blocks", type=int, default=0,
                     help="pool size override for a scaling measurement (the headline workload's is 1,048,576); "
                          "give --prefill enough steps to fill it")
+    ap.add_argument("--flags", type=int, default=0,
+                    help="ablation bits: 1 no retention segmentation, 2 no debt gate")
+    ap.add_argument("--tiers", action="store_true",
+                    help="the paper's three contract tiers (rho 64:40:16, beta 256:192:128, scaled to the "
+                         "workload's refill): victims critical, benign standard, attackers best-effort")
     ap.add_argument("--queues", action="store_true",
                     help="select victims from the indexed per-(group, class) queues instead of candidate scans")
     return ap.parse_args()
@@ -165,7 +170,8 @@ def run_oracle_steps(spec, steps, timed_from):
     """Oracle over steps; returns (seconds over steps[timed_from:], requests timed)."""
     import oracle as O
     oc = O.OracleCache(spec.capacity_blocks, spec.block_size, spec.num_groups, "prefixshield",
-                       O.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20))
+                       O.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20,
+                                contract_of_group=list(spec.contract_of_group) if spec.contract_of_group else None))
     t_sum, reqs = 0.0, 0
     for k, st in enumerate(steps):
         t0 = time.perf_counter()
@@ -259,6 +265,13 @@ def run_own(args, ws, rank, local):
     spec, steps = make_steps(args.seed + rank, n_total)
     if args.capacity_blocks:
         spec = dataclasses.replace(spec, capacity_blocks=args.capacity_blocks)
+    if args.tiers:
+        # rho and beta of the critical tier are the workload's own; the
+        # standard and best-effort tiers keep the paper's ratios to it
+        r0, b0 = spec.rho[0], spec.beta[0]
+        tier = [0] * 8 + [2] * 8 + [1] * (spec.num_groups - 16)  # victims, attackers, benign
+        spec = dataclasses.replace(spec, rho=(r0, r0 * 40 / 64, r0 * 16 / 64), beta=(b0, b0 * 192 / 256, b0 * 128 / 256),
+                                   contract_of_group=tier)
     maxT = max(s.num_tokens for s in steps)
     R = spec.requests_per_step
     dsteps = []
@@ -266,7 +279,8 @@ def run_own(args, ws, rank, local):
         dsteps.append((st.now, torch.from_numpy(st.groups).to(dev), torch.from_numpy(st.offsets).to(dev),
                        torch.from_numpy(st.tokens).to(dev)))
     params = B.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20,
-                      flags=B.PS_FLAG_INDEXED_QUEUES if args.queues else 0)
+                      contract_of_group=list(spec.contract_of_group) if spec.contract_of_group else None,
+                      flags=(B.PS_FLAG_INDEXED_QUEUES if args.queues else 0) | args.flags)
     cache = B.Cache(spec.capacity_blocks, spec.block_size, spec.num_groups, args.policy, params,
                     max_requests=R, max_tokens=maxT)
     cache.set_graph(not args.no_graph)
@@ -382,7 +396,8 @@ def run_own(args, ws, rank, local):
                    "groups": spec.num_groups, "l2": "flushed (256 MiB write) between timed steps",
                    "parallelism": f"replicas x{ws}",
                    "launch": "cuda graph" if cache.uses_graph() else "kernel by kernel",
-                   "select": "indexed queues" if args.queues else "candidate scan"},
+                   "select": "indexed queues" if args.queues else "candidate scan",
+                   "flags": args.flags, "contracts": "paper tiers" if args.tiers else "one"},
         "kv_blocks_per_s": blk_all / total_max,
         "step_roofline": {"bound": "hbm", "achieved": step_gbs, "peak": peak, "unit": "GB/s",
                           "frac": step_gbs / peak, "algorithmic_bytes_per_step": alg / args.steps,
