@@ -27,8 +27,10 @@
  *    any work is enqueued.  Errors only the device can see (bad offsets or
  *    group ids, a clock that goes backwards) make that step a no-op that
  *    leaves all state unchanged and report the code in out->counts[3].
- *    Running out of prefix-history capacity is sticky: every later step is a
- *    no-op reporting PS_ERR_CAPACITY until ps_reset().
+ *    Running out of prefix-history capacity (a step that would hold more
+ *    than history_capacity distinct (group, prefix id) entries) also leaves
+ *    all state unchanged, and is sticky: every later step is a no-op
+ *    reporting PS_ERR_CAPACITY until ps_clear_status() or ps_reset().
  *  - A handle is not thread-safe; steps on one handle must be issued in
  *    order on one stream (or with equivalent ordering).
  */
@@ -120,7 +122,13 @@ typedef struct {
 } ps_params_t;
 
 /* Outputs of one step, all device pointers, caller-owned.  R = num_requests,
- * B = max_tokens / block_size (the handle's per-step block capacity). */
+ * B = max_tokens / block_size (the handle's per-step block capacity).  A step
+ * can write up to B ids into each id list (the lists' lengths are known only
+ * on the device), so each must hold B: ids_capacity (elements in each of the
+ * three id arrays) below B, or req_capacity (elements in hit_blocks and
+ * admitted_blocks; admitted_offsets holds one more) below R, is refused with
+ * PS_ERR_INVALID_ARG before anything is enqueued.  The arrays' real sizes
+ * are the caller's to state truthfully: the library cannot check pointers. */
 typedef struct {
   int32_t* hit_blocks;        /* [R]   cached prefix + in-step hits of each request */
   int32_t* admitted_blocks;   /* [R]   newly materialized (charged) blocks n_r */
@@ -131,6 +139,9 @@ typedef struct {
   int32_t* counts;            /* [4]   n_admitted, n_evicted, n_invalidated, step status */
   int64_t* debt_raw;          /* [G]   D_g after the step (Eq. 3) */
   int64_t* debt_norm;         /* [G]   normalized debt after the step (Eq. 5) */
+  int64_t ids_capacity;       /* elements in each of admitted_ids, evicted_ids, invalidated_ids (>= B) */
+  int32_t req_capacity;       /* elements in hit_blocks and admitted_blocks (>= R) */
+  int32_t pad;
 } ps_step_out_t;
 
 /* Host-side copy of a step's outputs for ps_step_host(); same layout. */
@@ -198,7 +209,10 @@ int32_t ps_step_host_wait(ps_handle_t* h, int32_t slot);
  * synchronizes 'stream'.  Returns the sticky status (PS_OK or PS_ERR_CAPACITY). */
 int32_t ps_stats(ps_handle_t* h, void* stream, int64_t* h_stats);
 
-/* Clear a sticky capacity error without resetting the pool (enqueued). */
+/* Clear a sticky capacity error without resetting the pool (enqueued).  The
+ * failed step left no trace, so the next step continues from the state before
+ * it; a step that again needs more history entries than the capacity fails
+ * again (and is sticky again). */
 int32_t ps_clear_status(ps_handle_t* h, void* stream);
 
 /* Return the pool to its state right after ps_create() (enqueued). */
@@ -249,20 +263,24 @@ int32_t ps_cached_prefix(ps_handle_t* h, void* stream, int32_t num_requests, con
 
 /* ps_cached_prefix() for callers that cannot allocate device memory.  The
  * paper has no counterpart: this is a deployment convenience.  Some callers
- * may not call cudaMalloc or touch a workspace they do not own -- code inside
- * a CUDA graph capture region, code under a framework whose allocator owns
- * every device allocation, or a thread that only queries a cache another
- * thread steps.  This variant computes the same counts as ps_cached_prefix()
- * with its scratch in one fixed array compiled into the library (about
- * 2.3 MB, held on every GPU that loads the library until the process exits).
- * It allocates nothing; the caller passes inputs and outputs as for
- * ps_cached_prefix().  Limits of one call: 4096 requests (more returns
- * PS_ERR_CAPACITY at once) and 131072 full blocks (more tokens than
- * 131072 * block_size make d_status PS_ERR_INVALID_ARG).  The first call on
- * a device looks up the array's device address for that device; make that
- * first call before any stream capture.  Every call on a device shares the
- * one array: calls that overlap on the GPU (other streams, other handles,
- * other threads) race and must be serialized by the caller. */
+ * may not call cudaMalloc or write into a workspace they do not own -- code
+ * inside a CUDA graph capture region, or code under a framework whose
+ * allocator owns every device allocation.  This variant computes the same
+ * counts as ps_cached_prefix() with its scratch in one fixed array compiled
+ * into the library (about 2.3 MB, held on every GPU that loads the library
+ * until the process exits).  It allocates nothing; the caller passes inputs
+ * and outputs as for ps_cached_prefix().  Only the scratch leaves the
+ * workspace: the probe reads the pool's table, which every ps_step() of the
+ * handle rewrites, so it must be ordered on the GPU (same stream, or events)
+ * against every ps_step() of that handle.  Limits of one call: the handle's
+ * max_requests (more returns PS_ERR_INVALID_ARG, as ps_cached_prefix()
+ * does), 4096 requests (more returns PS_ERR_CAPACITY at once), and 131072
+ * full blocks (more tokens than 131072 * block_size make d_status
+ * PS_ERR_INVALID_ARG).  The first call on a device looks up the array's
+ * device address for that device; make that first call before any stream
+ * capture.  Every call on a device shares the one array: calls that overlap
+ * on the GPU (other streams, other handles, other threads) race and must be
+ * serialized by the caller. */
 int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_t num_requests, const int32_t* d_group_ids,
                                  const int64_t* d_token_offsets, const int32_t* d_tokens, int32_t* d_cached_blocks,
                                  int32_t* d_status);

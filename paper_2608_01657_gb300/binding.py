@@ -58,10 +58,25 @@ class PsParams(C.Structure):
     ]
 
 
+OUT_ARRAYS = ("hit_blocks", "admitted_blocks", "admitted_offsets", "admitted_ids", "evicted_ids",
+              "invalidated_ids", "counts", "debt_raw", "debt_norm")
+
+
 class PsStepOut(C.Structure):
-    _fields_ = [(n, C.c_void_p) for n in (
-        "hit_blocks", "admitted_blocks", "admitted_offsets", "admitted_ids", "evicted_ids",
-        "invalidated_ids", "counts", "debt_raw", "debt_norm")]
+    _fields_ = [(n, C.c_void_p) for n in OUT_ARRAYS] + [
+        ("ids_capacity", C.c_int64), ("req_capacity", C.c_int32), ("pad", C.c_int32)]
+
+
+def step_out(arrays: dict) -> PsStepOut:
+    """The C output descriptor of a dict of arrays (device tensors or host
+    numpy arrays): pointers, and the id lists' and per-request arrays' sizes."""
+    def n(k):
+        a = arrays.get(k)
+        return 0 if a is None else int(a.shape[0])
+    o = PsStepOut(**{k: _ptr(arrays.get(k)) for k in OUT_ARRAYS})
+    o.ids_capacity = min(n("admitted_ids"), n("evicted_ids"), n("invalidated_ids"))
+    o.req_capacity = min(n("hit_blocks"), n("admitted_blocks"), max(0, n("admitted_offsets") - 1))
+    return o
 
 
 class PsStateView(C.Structure):
@@ -212,7 +227,7 @@ class Cache:
             "debt_raw": torch.empty(G, dtype=torch.int64, device=dev),
             "debt_norm": torch.empty(G, dtype=torch.int64, device=dev),
         }
-        self._out = PsStepOut(**{k: _ptr(v) for k, v in self.out.items()})
+        self._out = step_out(self.out)
         h = C.c_void_p()
         rc = L.ps_create(C.byref(h), self.N, self.bs, self.G, POLICIES[policy], C.byref(self._p),
                          _ptr(self.workspace), nbytes, self.max_requests, self.max_tokens, _stream_ptr(stream))
@@ -266,7 +281,7 @@ class Cache:
         R = int(len(groups))
         if out is None:
             out = host_outputs(R, self.max_blocks, self.G)
-        o = PsStepOut(**{k: _ptr(out[k]) for k, _ in PsStepOut._fields_})
+        o = step_out(out)
         rc = load().ps_step_host(self._h, _stream_ptr(stream), int(now), R, _ptr(groups), _ptr(offsets),
                                  _ptr(tokens), _ptr(contracts), _ptr(prefixes), C.byref(o))
         out["rc"] = rc
@@ -279,7 +294,7 @@ class Cache:
         ``host_outputs(..., pinned=True)``; inputs and ``out`` must stay
         alive and unchanged until ``step_host_wait(slot)``."""
         R = int(len(groups))
-        o = PsStepOut(**{k: _ptr(out[k]) for k, _ in PsStepOut._fields_})
+        o = step_out(out)
         out["_keep"] = (o, groups, offsets, tokens, contracts, prefixes)
         return load().ps_step_host_async(self._h, _stream_ptr(stream), int(slot), int(now), R, _ptr(groups),
                                          _ptr(offsets), _ptr(tokens), _ptr(contracts), _ptr(prefixes), C.byref(o))

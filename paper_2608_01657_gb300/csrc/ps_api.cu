@@ -306,6 +306,8 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   so.counts = cv.take<int32_t>(4);
   so.debt_raw = cv.take<int64_t>(G);
   so.debt_norm = cv.take<int64_t>(G);
+  so.ids_capacity = (int64_t)B;
+  so.req_capacity = (int32_t)R;
   const size_t total = align_up(cv.off, 256);
   if (base) {
     *s = t;
@@ -335,6 +337,15 @@ int32_t init_state(ps_handle* h, cudaStream_t st) {
 }
 
 inline cudaStream_t as_stream(void* p) { return reinterpret_cast<cudaStream_t>(p); }
+
+// The stated sizes of a step's output arrays against what a step may write:
+// B ids in each id list, R entries per request array.  Arrays left null (the
+// host calls allow that) need no size.
+bool capacities_ok(const ps_step_out_t& o, int64_t B, int32_t R) {
+  const bool ids = o.admitted_ids || o.evicted_ids || o.invalidated_ids;
+  const bool reqs = o.hit_blocks || o.admitted_blocks || o.admitted_offsets;
+  return (!ids || o.ids_capacity >= B) && (!reqs || o.req_capacity >= R);
+}
 
 void drop_graph(ps_handle* h) {
   if (h->exec) cudaGraphExecDestroy(h->exec);
@@ -471,7 +482,8 @@ int32_t ps_step(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t num_req
   if (!h || !out || num_requests < 0 || num_requests > h->base.max_requests || !d_token_offsets) return PS_ERR_INVALID_ARG;
   if (num_requests > 0 && (!d_group_ids || !d_tokens)) return PS_ERR_INVALID_ARG;
   if (!out->hit_blocks || !out->admitted_blocks || !out->admitted_offsets || !out->admitted_ids || !out->evicted_ids ||
-      !out->invalidated_ids || !out->counts || !out->debt_raw || !out->debt_norm)
+      !out->invalidated_ids || !out->counts || !out->debt_raw || !out->debt_norm ||
+      !capacities_ok(*out, h->base.max_blocks, num_requests))
     return PS_ERR_INVALID_ARG;
   DevState s = h->base;
   s.now = now_ticks;
@@ -499,7 +511,8 @@ int32_t ps_step_host(ps_handle_t* h, void* stream, int64_t now_ticks, int32_t nu
   if (!h || !h_out || num_requests < 0 || num_requests > h->base.max_requests || !h_token_offsets)
     return PS_ERR_INVALID_ARG;
   const int64_t T = num_requests > 0 ? h_token_offsets[num_requests] : 0;
-  if (T < 0 || T > h->base.max_tokens || (num_requests > 0 && (!h_group_ids || (T > 0 && !h_tokens))))
+  if (T < 0 || T > h->base.max_tokens || (num_requests > 0 && (!h_group_ids || (T > 0 && !h_tokens))) ||
+      !capacities_ok(*h_out, h->base.max_blocks, num_requests))
     return PS_ERR_INVALID_ARG;
   cudaStream_t st = as_stream(stream);
   const size_t R = (size_t)num_requests;
@@ -553,7 +566,8 @@ int32_t ps_step_host_async(ps_handle_t* h, void* stream, int32_t slot, int64_t n
       num_requests > h->base.max_requests || !h_token_offsets || !h_out->counts)
     return PS_ERR_INVALID_ARG;
   const int64_t T = num_requests > 0 ? h_token_offsets[num_requests] : 0;
-  if (T < 0 || T > h->base.max_tokens || (num_requests > 0 && (!h_group_ids || (T > 0 && !h_tokens))))
+  if (T < 0 || T > h->base.max_tokens || (num_requests > 0 && (!h_group_ids || (T > 0 && !h_tokens))) ||
+      !capacities_ok(*h_out, h->base.max_blocks, num_requests))
     return PS_ERR_INVALID_ARG;
   for (const void* p : {(const void*)h_out->hit_blocks, (const void*)h_out->admitted_blocks,
                         (const void*)h_out->admitted_offsets, (const void*)h_out->admitted_ids,
@@ -755,10 +769,9 @@ int64_t ps_export_history(ps_handle_t* h, void* stream, int32_t* h_group, uint64
     return PS_ERR_CUDA;
   int64_t k = 0;
   for (const HistEntry& x : e) {
-    if (x.g1 == 0) continue;
+    if (x.g1 == 0) continue;  // every installed entry, so a failed step's leftovers would show
     const uint32_t rc = x.refadm & 0x7FFFFFFFu;
     const bool adm = x.refadm >> 31;
-    if (rc == 0 && !adm) continue;
     if (h_group && k < cap) {
       h_group[k] = (int32_t)x.g1 - 1;
       h_prefix[k] = x.p;

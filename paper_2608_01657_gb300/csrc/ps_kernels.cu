@@ -678,15 +678,57 @@ __global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
   }
 }
 
+// A step whose new (group, prefix) entries would overflow the history map
+// fails as a whole, leaving the pool as it was (Alg. 1's hooks change state
+// only for a request that goes ahead).  k_pin_claim has written three things
+// by then, undone here thread by thread over the same positions and requests:
+//  - pin tags of the cached prefix: set to a tag no step compares against
+//    (the previous step's), so the retried step pins them afresh;
+//  - claim-map entries: cleared (the map holds only this step's keys);
+//  - history entries: an entry with no committed reference was installed by
+//    this step and is removed (entries are never removed otherwise, so no
+//    probe sequence ran through it); every other touched entry loses the
+//    step's first-reference tag.
+// The error itself is raised by k_grant, after every thread here is done.
+__device__ __forceinline__ bool history_overflows(const DevState& s, const Ctl* c) {
+  return c->hist_live + c->hist_new > s.history_capacity;
+}
+__device__ void undo_pin_claim(const DevState& s, const Ctl* c, int64_t t) {
+  const int64_t nb = c->nblocks;
+  const uint32_t step32 = (uint32_t)c->step;
+  if (t < nb) {
+    PosRef r;
+    pos_ref(s, t, &r);
+    if (r.m < s.rq_h[r.i]) {
+      s.blk_pin[s.pos_blk[t]] = step32 - 1u;
+    } else {
+      const uint32_t slot = s.pos_claim[t];
+      if (slot != kNone) {
+        ClaimEntry z{};
+        z.key = 0; z.minreq = kNone; z.last = 0; z.tcnt = 0; z.promo = kNone; z.pad0 = 0; z.pad1 = 0;
+        s.claims[slot] = z;
+      }
+    }
+  } else if (t < nb + s.R) {
+    const uint32_t hs = s.rq_hs[t - nb];
+    if (hs != kNone) {
+      HistEntry* e = s.hist + hs;
+      if (ldcg_u32(&e->refadm) == 0) *e = HistEntry{};
+      else e->ftag = 0;
+    }
+  }
+}
+
 // Stage 2 (cont.): the first own claim s_i of each request, and orphans.  A
 // resident block past a request's first miss cannot be reached by lookup; it
-// is dropped (invalidated) unless some request pinned it.
+// is dropped (invalidated) unless some request pinned it.  Threads past the
+// positions take the requests (used only to undo a failing step).
 __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
-  if (c->hist_live + c->hist_new > s.history_capacity) {  // history capacity is sticky
-    if (blockIdx.x == 0 && threadIdx.x == 0) { c->status = PS_ERR_CAPACITY; c->sticky = PS_ERR_CAPACITY; }
+  if (history_overflows(s, c)) {
+    undo_pin_claim(s, c, blockIdx.x * (int64_t)blockDim.x + threadIdx.x);
     return;
   }
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
@@ -734,6 +776,10 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
+  if (history_overflows(s, c)) {  // undone by k_claims; the error is sticky
+    if (threadIdx.x == 0) { c->status = PS_ERR_CAPACITY; c->sticky = PS_ERR_CAPACITY; }
+    return;
+  }
   const int R = s.R;
   const bool quota = s.policy == PS_STATICQUOTA;  // a_i already granted per group
   const int64_t avail = s.N - c->pinned;
@@ -2295,7 +2341,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
   PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
   mark(2);
-  PS_LAUNCH(launch_k(k_claims, pgrid, kThreads, 0, st, s));
+  PS_LAUNCH(launch_k(k_claims, prgrid, kThreads, 0, st, s));
   mark(3);
   if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
   PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));

@@ -4,12 +4,14 @@
 // ps_cached_prefix() keeps its per-call scratch (block offsets, hashing
 // segments, per-position chain values, keys and lookup results) in the
 // handle's workspace.  Some callers may not call cudaMalloc at all, or may not
-// touch a workspace they do not own: code running inside a CUDA graph capture
-// region, inside a framework whose allocator owns every device allocation, or
-// a second thread that only asks the cache questions while another thread
-// owns and steps it.  This entry point gives them the same answer with its
-// scratch in one fixed, file-scope device array that the library holds for
-// as long as it is loaded, on every GPU that loads it.
+// write into a workspace they do not own: code running inside a CUDA graph
+// capture region, or inside a framework whose allocator owns every device
+// allocation.  This entry point gives them the same answer with its scratch
+// in one fixed, file-scope device array that the library holds for as long
+// as it is loaded, on every GPU that loads it.  Only the scratch moves out of
+// the workspace: the probe still reads the pool's table, which every ps_step()
+// of the handle rewrites, so a probe must be stream-ordered against the
+// handle's steps (an unordered probe could read a half-updated table).
 #include <mutex>
 
 #include "ps_internal.cuh"
@@ -68,6 +70,9 @@ extern "C" int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_
                                             const int32_t* d_group_ids, const int64_t* d_token_offsets,
                                             const int32_t* d_tokens, int32_t* d_cached_blocks, int32_t* d_status) {
   if (!h || num_requests < 0 || !d_token_offsets || !d_status) return PS_ERR_INVALID_ARG;
+  // more requests than the handle takes: refused as by ps_cached_prefix();
+  // more than the scratch array holds: a capacity error
+  if (num_requests > handle_state(h)->max_requests) return PS_ERR_INVALID_ARG;
   if (num_requests > kNaMaxRequests) return PS_ERR_CAPACITY;
   if (num_requests > 0 && (!d_group_ids || !d_tokens || !d_cached_blocks)) return PS_ERR_INVALID_ARG;
   unsigned char* base = nullptr;
@@ -76,7 +81,6 @@ extern "C" int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_
   DevState s = *handle_state(h);
   // bounds of one call: the smaller of the handle's and the scratch's
   s.max_requests = s.max_requests < kNaMaxRequests ? s.max_requests : (int32_t)kNaMaxRequests;
-  if (num_requests > s.max_requests) return PS_ERR_CAPACITY;
   if (s.max_blocks > kNaMaxBlocks) {
     s.max_blocks = kNaMaxBlocks;
     s.max_tokens = kNaMaxBlocks * s.bs;

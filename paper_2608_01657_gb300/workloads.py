@@ -371,12 +371,18 @@ CONFIGS = {
 
 
 def make_workload(config: int, seed: int = 1, requests_per_step: Optional[int] = None,
-                  total_requests: Optional[int] = None, wait: int = 0) -> Workload:
+                  total_requests: Optional[int] = None, wait: int = 0,
+                  attacker_prompts: Optional[int] = None) -> Workload:
     """The seeded trace of one configuration (0..6).  ``requests_per_step``
     overrides the batch size (e.g. the discriminative 8-request variants);
     ``wait`` is the delayed-replay trace's number of empty steps between the
-    attacker's burst and its replay."""
+    attacker's burst and its replay; ``attacker_prompts`` shortens the
+    two-pass replay trace (config 2) to that many fresh attacker prompts
+    replayed once, with as many victim requests (the same 1:1 mix), so its
+    second pass starts within a short run."""
     spec = CONFIGS[config]
+    if config == 2 and attacker_prompts is not None:
+        total_requests = 4 * int(attacker_prompts)
     if requests_per_step is not None or total_requests is not None:
         spec = dataclasses.replace(
             spec,
@@ -389,8 +395,9 @@ def make_workload(config: int, seed: int = 1, requests_per_step: Optional[int] =
         return OneTouch(spec, seed, hot_len=2048, n_hot=8, zipf_s=1.0, victim_suffix=128,
                         atk_len=_lognormal_2048, n_victim=10000, n_attacker=10000)
     if config == 2:
+        half = spec.total_requests // 2
         return OneTouch(spec, seed, hot_len=2048, n_hot=8, zipf_s=1.0, victim_suffix=128,
-                        atk_len=_lognormal_2048, n_victim=20000, n_attacker=20000, replay=True)
+                        atk_len=_lognormal_2048, n_victim=half, n_attacker=half, replay=True)
     if config == 3:
         return BenignChat(spec, seed)
     if config == 4:

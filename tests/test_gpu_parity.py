@@ -102,7 +102,8 @@ def test_parity_tiny_one_touch(policy):
 
 
 @pytest.mark.parametrize("policy", GPU_POLICIES)
-@pytest.mark.parametrize("cfg,nsteps,rps", [(1, 40, None), (1, 60, 8), (2, 40, 8), (3, 30, None), (5, 120, None)])
+@pytest.mark.parametrize("cfg,nsteps,rps", [(1, 40, None), (1, 60, 8), (2, 40, None), (2, 40, 8), (3, 30, None),
+                                           (5, 120, None)])
 def test_parity_configs(policy, cfg, nsteps, rps):
     wl = W.make_workload(cfg, seed=2, requests_per_step=rps)
     sp = wl.spec
@@ -114,6 +115,41 @@ def test_parity_configs(policy, cfg, nsteps, rps):
     gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy, kw,
                      max_requests=sp.requests_per_step, max_tokens=maxT)
     _run(gpu, orc, steps, state_every=10, label=f"cfg{cfg}/{policy}")
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+@pytest.mark.parametrize("flags", [0, O.FLAG_INDEXED_QUEUES])
+def test_parity_two_pass_replay(policy, flags):
+    """The two-pass replay trace (Sec. V-B) shortened to 24 fresh attacker
+    prompts replayed once, 8 requests a step, so the second pass runs: every
+    step of both passes equals the oracle, and the oracle's replayed attacker
+    prompts hit the cache (except under StaticQuota, whose cap on the
+    attacker's partition leaves nothing to replay)."""
+    if flags and policy == "s3fifo":
+        pytest.skip("s3fifo keeps its own queues")
+    wl = W.make_workload(2, seed=2, requests_per_step=8, attacker_prompts=24)
+    sp = wl.spec
+    steps = list(wl.steps())
+    gpu, orc = _pair(sp.capacity_blocks, sp.block_size, sp.num_groups, policy,
+                     dict(rho=sp.rho, beta=sp.beta, flags=flags), max_requests=sp.requests_per_step,
+                     max_tokens=max(s.num_tokens for s in steps))
+    dev = torch.device("cuda")
+    seen = replay_hits = 0
+    for k, st in enumerate(steps):
+        rc = gpu.step(st.now, torch.from_numpy(st.groups).to(dev), torch.from_numpy(st.offsets).to(dev),
+                      torch.from_numpy(st.tokens).to(dev))
+        assert rc == 0
+        want = orc.step(st.now, st.groups, st.offsets, st.tokens)
+        compare_outputs(gpu.fetch(st.num_requests), want, f"replay/{policy} step {k}")
+        for i, g in enumerate(st.groups):
+            if g == 1:
+                seen += 1
+                if seen > 24:
+                    replay_hits += int(want["hit_blocks"][i])
+    compare_state(gpu.export(), orc.export(), f"replay/{policy}", s3=policy == "s3fifo")
+    assert np.array_equal(gpu.stats(), orc.stats())
+    assert seen == 48
+    assert (replay_hits == 0) if policy == "staticquota" else (replay_hits > 0)
 
 
 @pytest.mark.parametrize("policy", GPU_POLICIES)
@@ -258,6 +294,28 @@ def test_parity_hand_derived_corners(flags):
             g, o, t, _ = make_step(prompts)
             seq.append(W.Step(index=k, now=1, groups=g, offsets=o, tokens=t))
         _run(gpu, orc, seq, label=f"corner{ci}/f{flags}")
+
+
+@pytest.mark.parametrize("policy", GPU_POLICIES)
+@pytest.mark.parametrize("flags", [0, O.FLAG_INDEXED_QUEUES])
+def test_parity_orphan_scenario(policy, flags):
+    """The hand-derived orphan scenario of the oracle pins (a chain with two
+    holes, a chain with no first block, a later request holding an orphan
+    again), replayed through the GPU step with its explicit prefix ids."""
+    from _util import make_step, obj_tokens
+    if flags and policy == "s3fifo":
+        pytest.skip("s3fifo keeps its own queues")
+    X, V, Y = obj_tokens("X", blocks=6), obj_tokens("V", blocks=2), obj_tokens("Y", blocks=6)
+    plan = [[(X, 3, 0, 1), (V, 1, 0, 21)], [(X, 4, 0, 2), (V, 2, 0, 22)], [(X, 5, 0, 3)], [(X, 6, 0, 4)],
+            [(X, 4, 0, 2), (V, 2, 0, 22)], [(X, 6, 0, 4)], [(Y, 6, 1, 31)],
+            [(X, 6, 0, 4), (V, 2, 0, 22), (X, 4, 0, 4)]]
+    seq = []
+    for k, reqs in enumerate(plan):
+        g, o, t, _ = make_step([tk[: 16 * nb] for tk, nb, _, _ in reqs], [grp for _, _, grp, _ in reqs])
+        seq.append(W.Step(k, k + 1, g, o, t, None, np.array([pid for _, _, _, pid in reqs], np.uint64)))
+    gpu, orc = _pair(11, 16, 2, policy, dict(rho=(1000.0,), beta=(1000.0,), flags=flags), max_requests=3,
+                     max_tokens=12 * 16)
+    _run(gpu, orc, seq, label=f"orphans/{policy}/f{flags}")
 
 
 def test_parity_alg2_ties():
