@@ -75,9 +75,13 @@ KeySchedule key_schedule(uint64_t seed, int32_t bs) {
   k.kd = splitmix_next(&st) % kP61;
   if (k.kc == 0) k.kc = 1;
   if (k.kd == 0) k.kd = 1;
-  k.kc_pow.resize(kSegBlocks + 1);
+  // Kc^j for j = 0..kSegBlocks, then Kc^(kSegBlocks t) for t = 0..32
+  k.kc_pow.resize(2 * (kSegBlocks + 1));
   k.kc_pow[0] = 1;
   for (int j = 1; j <= kSegBlocks; ++j) k.kc_pow[j] = host_mul61(k.kc_pow[j - 1], k.kc);
+  k.kc_pow[kSegBlocks + 1] = 1;
+  for (int t = 1; t <= kSegBlocks; ++t)
+    k.kc_pow[kSegBlocks + 1 + t] = host_mul61(k.kc_pow[kSegBlocks + t], k.kc_pow[kSegBlocks]);
   return k;
 }
 
@@ -153,7 +157,9 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   d.max_segments = d.max_blocks / kSegBlocks + max_requests + 1;
   d.nwords = (N + 31) / 32;
   // native table: 8-way buckets at load <= 1/2
-  d.tb_log2 = log2_pow2_at_least((uint64_t)((N + 3) / 4 > 1 ? (N + 3) / 4 : 1));
+  // 8-way buckets for 4N entries: at most a quarter full, so a probe rarely
+  // continues past its home bucket
+  d.tb_log2 = log2_pow2_at_least((uint64_t)((N + 1) / 2 > 1 ? (N + 1) / 2 : 1));
   if (d.tb_log2 < 1) d.tb_log2 = 1;
   // claim map: 4-way buckets, at least one slot per block of a step (load <=
   // 1 even if every block of a full step is new; about a quarter of that in
@@ -216,7 +222,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.ledger = cv.take<int64_t>(G * d.C);
   t.contract_of_group = cv.take<int32_t>(G);
   t.key_words = cv.take<uint32_t>((size_t)d.bs + 2);
-  t.kc_pow = cv.take<uint64_t>((size_t)kSegBlocks + 1);
+  t.kc_pow = cv.take<uint64_t>(2 * ((size_t)kSegBlocks + 1));
   t.stats = cv.take<int64_t>(G * PS_NUM_STATS);
   t.hist = cv.take<HistEntry>((size_t)1 << d.hist_log2);
   t.rq_n = cv.take<int32_t>(R);
@@ -226,7 +232,6 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.rq_cbase = cv.take<int32_t>(R);
   t.rq_a = cv.take<int32_t>(R);
   t.rq_e = cv.take<int32_t>(R);
-  t.rq_sbase = cv.take<int32_t>(R);
   t.rq_fu = cv.take<uint32_t>(R);
   t.rq_cid = cv.take<int32_t>(R);
   t.rq_hs = cv.take<uint32_t>(R);
@@ -235,9 +240,9 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.rq_knew = cv.take<uint8_t>(R);
   t.pos_key = cv.take<uint64_t>(B);
   t.pos_req = cv.take<uint32_t>(B);
-  t.seg_req = cv.take<uint32_t>((size_t)d.max_segments);
-  t.seg_cin = cv.take<uint64_t>((size_t)d.max_segments);
-  t.seg_tot = cv.take<uint64_t>((size_t)d.max_segments);
+  t.chunks = cv.take<ChunkDesc>((size_t)d.max_segments);
+  t.val_tile = cv.take<uint64_t>(R / 256 + 1);
+  t.seg_word = cv.take<uint64_t>((size_t)d.max_segments);
   t.pos_blk = cv.take<uint32_t>(B);
   t.pos_claim = cv.take<uint32_t>(B);
   t.pos_elig = cv.take<uint8_t>(B);

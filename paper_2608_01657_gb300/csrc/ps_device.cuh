@@ -138,6 +138,30 @@ __device__ __forceinline__ void agg_min_u32(uint32_t* base, uint32_t i, uint32_t
 __device__ __forceinline__ uint64_t ldcg_u64(const uint64_t* p) { return __ldcg(reinterpret_cast<const unsigned long long*>(p)); }
 __device__ __forceinline__ uint32_t ldcg_u32(const uint32_t* p) { return __ldcg(p); }
 
+// ---- published words: a value and its flags in one aligned 64-bit word -----
+// One relaxed 64-bit store publishes both, and one relaxed 64-bit load reads
+// both, so no fence is needed to order them.
+constexpr int kSpinLimit = 1 << 20;
+
+__device__ __forceinline__ void st_relaxed_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.relaxed.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
+}
+__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return v;
+}
+// Wait (bounded) until every bit of 'need' is set in *w; the word, or 0 if
+// the wait ran out.
+__device__ __forceinline__ uint64_t wait_word(const uint64_t* w, uint64_t need) {
+  for (int it = 0; it < kSpinLimit; ++it) {
+    const uint64_t v = ld_relaxed_u64(w);
+    if ((v & need) == need) return v;
+    __nanosleep(32);
+  }
+  return 0;
+}
+
 // ---- indexed queues: which logs hold a block ---------------------------------
 __device__ __forceinline__ bool lg_segmented(const DevState& s) {
   return s.policy == PS_PREFIXSHIELD && !(s.flags & PS_FLAG_NO_SEGMENTATION);

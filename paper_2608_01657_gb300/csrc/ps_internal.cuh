@@ -24,7 +24,7 @@ constexpr int kTableWays = 8;    // native prefix table: 8 x 16 B entries per 12
 constexpr int kClaimWays = 4;    // per-step claim map: 4 x 32 B entries per bucket
 constexpr int kRadixBits = 8;
 constexpr int kRadixBins = 1 << kRadixBits;
-constexpr int kSegBlocks = 128;  // blocks of one prompt hashed by one warp
+constexpr int kSegBlocks = 32;   // blocks of one prompt hashed by one warp (a chunk)
 constexpr int kBmChunk = 256;    // bitmap words per CTA of the id-list compaction
 constexpr uint64_t kP61 = (1ull << 61) - 1;  // chain modulus, a Mersenne prime
 
@@ -98,6 +98,21 @@ struct Ctl {
   int32_t lg_more;         // a take's window ended short of its last victim: another round
   int32_t lg_cmp;          // a log lacks room for this step's appends: compact first
   uint32_t lg_ticket;      // last-CTA-done counter of the append and compaction writes
+  uint32_t hash_ticket;    // chunks handed out to k_hash_lookup's CTAs, in order
+  uint32_t v_ticket;       // k_validate: CTAs done (the last one finishes the call)
+  uint32_t v_bad;          // k_validate: bit 0 an invalid request, bit 1 a look-back ran out
+  uint64_t v_sum;          // k_validate: blocks (high half) and chunks (low half) of the call
+};
+
+// One hashing chunk: up to kSegBlocks consecutive blocks of one request.
+struct __align__(16) ChunkDesc {
+  int64_t o0;      // the request's first token
+  uint32_t req;    // request index
+  int32_t n;       // the request's full blocks
+  int32_t pbase;   // position of the request's block 0
+  int32_t k;       // this chunk's index within the request
+  uint32_t group;  // the request's group
+  int32_t sb;      // the request's first chunk
 };
 
 // Per-segment state of the segmented radix select.
@@ -217,7 +232,7 @@ struct DevState {
   int64_t* ledger;         // B_{g,c}, fixed point
   int32_t* contract_of_group;
   uint32_t* key_words;     // NH key schedule, bs + 2 words
-  uint64_t* kc_pow;        // Kc^k mod p, k = 0..kSegBlocks
+  uint64_t* kc_pow;        // Kc^k mod p, k = 0..kSegBlocks, then Kc^(kSegBlocks t), t = 0..32
   int64_t* stats;          // [G][PS_NUM_STATS]
   HistEntry* hist;
   // per-step scratch
@@ -228,7 +243,6 @@ struct DevState {
   int32_t* rq_cbase;       // exclusive scan of claims
   int32_t* rq_a;           // granted (admitted) blocks
   int32_t* rq_e;           // in-step hits
-  int32_t* rq_sbase;       // first hashing segment of the request
   uint32_t* rq_fu;         // first ungranted in-step position
   int32_t* rq_cid;         // contract
   uint32_t* rq_hs;         // history slot
@@ -237,9 +251,9 @@ struct DevState {
   uint8_t* rq_knew;        // class of newly admitted blocks
   uint64_t* pos_key;       // chain partial, then the block key
   uint32_t* pos_req;       // request of the position
-  uint32_t* seg_req;       // request of each hashing segment
-  uint64_t* seg_cin;       // chain value entering the segment
-  uint64_t* seg_tot;       // local chain value at the segment's end
+  ChunkDesc* chunks;       // hashing chunks of the call, in request order
+  uint64_t* val_tile;      // k_validate's published per-tile totals (zero between calls)
+  uint64_t* seg_word;      // the chunk's published chain total and miss bit (k_hash_lookup)
   uint32_t* pos_blk;       // resident block hit by lookup (or kNone)
   uint32_t* pos_claim;     // claim-map slot (or kNone)
   uint8_t* pos_elig;       // touch was promotion-eligible

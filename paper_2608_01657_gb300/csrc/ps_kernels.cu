@@ -76,18 +76,24 @@ __device__ __forceinline__ uint64_t mul61(uint64_t a, uint64_t b) {  // a, b < p
 // ---- native prefix table ---------------------------------------------------
 // Lookup by one thread: the 128-byte home bucket (8 entries), then following
 // buckets while the overflow count says some key probed past.
+// All eight ways and the overflow count are loaded before any is compared,
+// so a bucket costs one round trip (a return inside the loads would keep the
+// compiler from issuing a later way's load before an earlier way's compare).
 __device__ uint32_t table_find(const DevState& s, uint64_t key, uint32_t g) {
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
   uint32_t b = table_home(key, g, s.tb_nbuckets_log2);
   for (uint32_t it = 0; it <= mask; ++it) {
     const uint4* e = reinterpret_cast<const uint4*>(s.table + (size_t)b * kTableWays);
-    const uint32_t ovf = __ldg(s.table_ovf + b);  // issued with the bucket: a miss needs no second trip
+    uint4 raw[kTableWays];
 #pragma unroll
-    for (int w = 0; w < kTableWays; ++w) {
-      const uint4 raw = __ldg(e + w);
-      if (raw.z != kNone && raw.x == (uint32_t)key && raw.y == (uint32_t)(key >> 32) && raw.w == g) return raw.z;
-    }
-    if (ovf == 0) return kNone;
+    for (int w = 0; w < kTableWays; ++w) raw[w] = __ldg(e + w);
+    const uint32_t ovf = __ldg(s.table_ovf + b);  // issued with the bucket: a miss needs no second trip
+    uint32_t hit = kNone;
+#pragma unroll
+    for (int w = 0; w < kTableWays; ++w)
+      if (raw[w].z != kNone && raw[w].x == (uint32_t)key && raw[w].y == (uint32_t)(key >> 32) && raw[w].w == g)
+        hit = raw[w].z;
+    if (hit != kNone || ovf == 0) return hit;
     b = (b + 1) & mask;
   }
   return kNone;
@@ -136,6 +142,9 @@ __device__ void table_delete(const DevState& s, uint32_t blk) {
 }
 
 // ---- per-step claim map ------------------------------------------------------
+// The bucket's keys are loaded first, so the many requests that claim one
+// popular key in a step mostly find it with a plain load and swap nothing
+// (a swap first would serialize them on one address).
 __device__ uint32_t claim_insert(const DevState& s, uint64_t key, uint32_t req) {
   const uint32_t mask = (1u << s.cl_nbuckets_log2) - 1;
   uint32_t b = claim_home(key, s.cl_nbuckets_log2);
@@ -211,318 +220,237 @@ __global__ void k_init_ctl(DevState s) {
 }
 
 // ===========================================================================
-// Stage 0: validation of the step's inputs; n_i, block positions, hashing
-// segments.  One CTA.  'probe' skips the clock and step checks.
+// Stage 0: validation of the step's inputs; n_i, block positions and the
+// chunk descriptors of the hashing stage.  One CTA per kValTile requests;
+// the exclusive scans of blocks and chunks over the requests take each
+// tile's base from its predecessors' published totals (a decoupled look-back
+// without inclusive prefixes: a tile sums every earlier tile's total, and no
+// total waits on anything).  The last CTA to finish sets the call's status
+// and per-step scalars, and clears the tile words for the next call.
+// 'probe' skips the clock and step checks.  Every write is bounds-checked, so
+// inputs that turn out invalid write nothing outside the scratch arrays.
+constexpr int kValTile = 256;
+constexpr uint64_t kTileFlag = 1ull << 63;
 
-__global__ void __launch_bounds__(1024) k_validate(DevState s, int probe) {
+__global__ void __launch_bounds__(kValTile) k_validate(DevState s, int probe) {
   s = with_args(s);
+  __shared__ uint64_t s_base;
+  __shared__ bool s_last;
   Ctl* c = s.ctl;
   const int R = s.R;
+  const int tile = blockIdx.x;
+  const int i = tile * kValTile + (int)threadIdx.x;
+  const bool in = i < R;
   bool bad = false;
-#pragma unroll 4
-  for (int i = threadIdx.x; i < R; i += blockDim.x) {
-    const int64_t o0 = s.in_offsets[i], o1 = s.in_offsets[i + 1];
-    const int g = s.in_group[i];
-    bad |= o1 < o0 || g < 0 || g >= s.G || (o1 - o0) / s.bs > (int64_t)kMaxPos;
-    if (s.in_contract) bad |= s.in_contract[i] < 0 || s.in_contract[i] >= s.C;
+  int32_t n = 0, ns = 0, cid = 0, g = 0;
+  int64_t o0 = 0;
+  if (in) {
+    o0 = s.in_offsets[i];
+    const int64_t o1 = s.in_offsets[i + 1];
+    g = s.in_group[i];
+    const int64_t nb = (o1 - o0) / s.bs;
+    bad = o1 < o0 || g < 0 || g >= s.G || nb > (int64_t)kMaxPos;
+    if (s.in_contract) {
+      cid = s.in_contract[i];
+      bad |= cid < 0 || cid >= s.C;
+    } else if (!probe && !bad) {
+      cid = s.contract_of_group[g];
+    }
     if (s.in_prefix) bad |= s.in_prefix[i] == 0;
+    n = bad ? 0 : (int32_t)nb;
   }
-  const int s_bad = __syncthreads_or(bad);
-  int32_t st = PS_OK;
-  const int64_t T = R > 0 ? s.in_offsets[R] : 0;
-  if (!probe && c->sticky != PS_OK) st = c->sticky;
-  else if (!probe && s.now < c->t_prev) st = PS_ERR_CLOCK;
-  else if (!probe && c->step > kMaxStep) st = PS_ERR_CAPACITY;
-  else if (s_bad || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens) st = PS_ERR_INVALID_ARG;
-  if (st != PS_OK) {
-    __syncthreads();
-    if (threadIdx.x == 0) { c->status = st; c->nblocks = 0; c->nsegs = 0; }
-    return;
-  }
-  // blocks and hashing segments per request (blocks in the high half, segments
-  // in the low half of one scanned word), four 1024-request sub-tiles a pass
-  uint64_t carry = 0;
-  const int tile = 4 * (int)blockDim.x;
-  for (int t0 = 0; t0 < R; t0 += tile) {
-    uint64_t v[4], ex[4];
-    int32_t n[4], ns[4], cid[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int i = t0 + u * (int)blockDim.x + (int)threadIdx.x;
-      n[u] = 0;
-      cid[u] = 0;
-      if (i < R) {
-        n[u] = (int32_t)((s.in_offsets[i + 1] - s.in_offsets[i]) / s.bs);
-        if (!probe) cid[u] = s.in_contract ? s.in_contract[i] : s.contract_of_group[s.in_group[i]];
-      }
-      ns[u] = (n[u] + kSegBlocks - 1) / kSegBlocks;
-      v[u] = (uint64_t)n[u] << 32 | (uint64_t)ns[u];
-    }
-    uint64_t tot;
-    block_excl_scan4(v, ex, &tot);
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int i = t0 + u * (int)blockDim.x + (int)threadIdx.x;
-      if (i < R) {
-        const uint64_t e = carry + ex[u];
-        s.rq_n[i] = n[u];
-        s.rq_h[i] = n[u];
-        s.rq_s[i] = n[u];
-        s.rq_fu[i] = kNone;
-        if (!probe) s.rq_cid[i] = cid[u];
-        s.rq_pbase[i] = (int32_t)(e >> 32);
-        s.rq_sbase[i] = (int32_t)(uint32_t)e;
-        for (int j = 0; j < ns[u]; ++j) s.seg_req[(uint32_t)e + j] = (uint32_t)i;
+  ns = (n + kSegBlocks - 1) / kSegBlocks;
+  const int tile_bad = __syncthreads_or(bad);
+  // blocks in the high half, chunks in the low half of one scanned word
+  uint64_t tot;
+  const uint64_t ex = block_excl_scan<uint64_t>((uint64_t)n << 32 | (uint64_t)ns, &tot);
+  if (threadIdx.x == 0) st_relaxed_u64(s.val_tile + tile, tot | kTileFlag);
+  if (threadIdx.x < 32 && tile * kValTile < R) {  // the tile's base: every earlier tile's total
+    const int lane = threadIdx.x;
+    uint64_t sum = 0;
+    bool ok = true;
+    for (int t0 = 0; t0 < tile; t0 += 32) {
+      if (t0 + lane < tile) {
+        const uint64_t v = wait_word(s.val_tile + t0 + lane, kTileFlag);
+        ok = ok && v != 0;
+        sum += v & ~kTileFlag;
       }
     }
-    carry += tot;
+    sum = warp_sum(sum);
+    if (!__all_sync(kFull, ok) && lane == 0) atomicOr(&c->v_bad, 2u);  // never expected
+    if (lane == 0) s_base = sum;
+  } else if (threadIdx.x == 0) {
+    s_base = 0;  // a tile past the step's requests writes nothing
   }
-  const int32_t nblocks = (int32_t)(carry >> 32), nsegs = (int32_t)(uint32_t)carry;
-  if (threadIdx.x == 0) {
-    c->status = PS_OK;
-    c->T = T;
-    c->nblocks = nblocks;
-    c->nsegs = nsegs;
+  __syncthreads();
+  const uint64_t e = s_base + ex;
+  const int64_t pbase = (int64_t)(e >> 32), sbase = (int64_t)(uint32_t)e;
+  if (in && pbase + n <= s.max_blocks && sbase + ns <= s.max_segments) {
+    s.rq_n[i] = n;
+    s.rq_h[i] = n;
+    s.rq_s[i] = n;
+    s.rq_fu[i] = kNone;
+    s.rq_pbase[i] = (int32_t)pbase;
     if (!probe) {
-      c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
-      c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
-      c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
-      c->internal_error = 0;
-      c->nlaunch = 1;  // this kernel; every later kernel of the step adds itself
-      c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
+      s.rq_cid[i] = cid;
+      s.rq_hs[i] = kNone;  // a request with no full block has no history entry
+      s.rq_p[i] = 0;
     }
   }
-  if (!probe && s.policy == PS_STATICQUOTA)
-    for (int g = threadIdx.x; g < s.G; g += blockDim.x) s.grp_pinned[g] = 0;
-  if (!probe)  // the candidate counts (k_cand accumulates them beside S3-S4)
-    for (int r = threadIdx.x; r < s.G * kClasses; r += blockDim.x) {
+  // each request's chunk descriptors; the warp writes one request's chunks
+  // at a time, so the stores coalesce
+  const bool room = in && pbase + n <= s.max_blocks && sbase + ns <= s.max_segments;
+  for (unsigned todo = __ballot_sync(kFull, room && ns > 0); todo; todo &= todo - 1) {
+    const int src = __ffs(todo) - 1;
+    const int64_t ro0 = __shfl_sync(kFull, o0, src);
+    const int64_t rsb = __shfl_sync(kFull, sbase, src);
+    const int32_t rpb = (int32_t)__shfl_sync(kFull, pbase, src);
+    const int32_t rn = __shfl_sync(kFull, n, src), rns = __shfl_sync(kFull, ns, src);
+    const uint32_t ri = (uint32_t)__shfl_sync(kFull, i, src), rg = (uint32_t)__shfl_sync(kFull, g, src);
+    for (int k = lane_id(); k < rns; k += 32) {
+      ChunkDesc d;
+      d.o0 = ro0;
+      d.req = ri;
+      d.n = rn;
+      d.pbase = rpb;
+      d.k = k;
+      d.group = rg;
+      d.sb = (int32_t)rsb;
+      s.chunks[rsb + k] = d;
+      s.seg_word[rsb + k] = 0;
+    }
+  }
+  if (!probe && tile == 0) {  // per-step counts accumulated by later kernels
+    if (s.policy == PS_STATICQUOTA)
+      for (int gg = threadIdx.x; gg < s.G; gg += blockDim.x) s.grp_pinned[gg] = 0;
+    for (int r = threadIdx.x; r < s.G * kClasses; r += blockDim.x) {  // the candidate counts (k_cand)
       if (r < s.G) s.grp_qsize[r] = 0;
       s.cls[r] = ClsRange{0, ~0u, 0, ~0u, 0};
     }
+  }
+  // the last CTA to finish: status and per-call scalars
+  if (threadIdx.x == 0) {
+    if (tile_bad) atomicOr(&c->v_bad, 1u);
+    if (tot) atomicAdd(reinterpret_cast<unsigned long long*>(&c->v_sum), (unsigned long long)tot);
+    __threadfence();
+    s_last = atomicAdd(&c->v_ticket, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (int t = threadIdx.x; t < (int)gridDim.x; t += blockDim.x) s.val_tile[t] = 0;
+  if (threadIdx.x != 0) return;
+  const uint32_t vb = ldcg_u32(&c->v_bad);
+  const uint64_t all = ldcg_u64(&c->v_sum);  // blocks (high half) and chunks (low half) of the step
+  c->v_bad = 0;
+  c->v_ticket = 0;
+  c->v_sum = 0;
+  const int64_t T = R > 0 ? s.in_offsets[R] : 0;
+  int32_t st = PS_OK;
+  if (!probe && c->sticky != PS_OK) st = c->sticky;
+  else if (!probe && s.now < c->t_prev) st = PS_ERR_CLOCK;
+  else if (!probe && c->step > kMaxStep) st = PS_ERR_CAPACITY;
+  else if (vb || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens) st = PS_ERR_INVALID_ARG;
+  c->status = st;
+  c->T = T;
+  c->hash_ticket = 0;
+  if (st != PS_OK) {
+    c->nblocks = 0;
+    c->nsegs = 0;
+    return;
+  }
+  c->nblocks = (int64_t)(all >> 32);
+  c->nsegs = (int64_t)(uint32_t)all;
+  if (!probe) {
+    c->pinned = 0; c->n_inval = 0; c->total_claims = 0; c->avail = 0; c->need = 0;
+    c->nfree = 0; c->ftake = 0; c->mvict = 0; c->hist_new = 0; c->n_evicted = 0;
+    c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
+    c->internal_error = (vb & 2) ? 1 : 0;
+    c->nlaunch = 1;  // this kernel; every later kernel of the step adds itself
+    c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
+  }
 }
 
 // ===========================================================================
-// Stage 1: chained block hashing (Sec. III-B native content key), one warp
-// per segment of up to kSegBlocks blocks of one prompt.
+// Stages 1-2 in one kernel: chained block hashing (Sec. III-B native content
+// key), the longest cached prefix (n_cached of Alg. 1), the pins of the
+// cached prefix, the claims of every block past it, and each request's
+// history entry (OnRequest of Alg. 1).
 //
-// The segment's tokens arrive in shared memory with one TMA bulk copy
-// (cp.async.bulk, completion counted on an mbarrier) of the 16-byte aligned
-// window around them, so each warp has its whole segment in flight at once;
-// a window that would end past the token buffer, or an unaligned buffer, is
-// loaded with plain coalesced loads instead.  NH products are spread over the
-// warp: lane l takes pair (l % PPB) of block (l / PPB + (32 / PPB) r) in
-// round r, PPB = bs / 2; the pair sums are reduced with xor shuffles and
-// routed to lane = block.  The chain C_m = Kc C_{m-1} + D_m (mod 2^61-1) is a
-// composition of affine maps, so a warp scan gives every block its chain
-// value relative to the segment start (B_m, with the value before the segment
-// taken as 0); k_keys_lookup then folds in the true value entering it.
-template <int PPB>
-struct HashCfg {
-  static constexpr int BS = 2 * PPB;
-  static constexpr int kWindow = kSegBlocks * BS + 8;  // tokens staged per warp (+ alignment slack)
-  // staging windows of up to 66 KB a CTA: three CTAs fit an SM's shared
-  // memory (and, at 80 registers a thread, its register file)
-  static constexpr int kWarps = (66 * 1024) / (kWindow * 4) < 1 ? 1
-                                : ((66 * 1024) / (kWindow * 4) > 8 ? 8 : (66 * 1024) / (kWindow * 4));
-  static constexpr size_t kSmem = (size_t)kWarps * kWindow * 4 + (size_t)kWarps * 8;
-};
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p) {
-  return (uint32_t)__cvta_generic_to_shared(p);
+// A chunk is up to kSegBlocks = 32 consecutive blocks of one prompt; one warp
+// takes one chunk, one lane one block.  Chunks are numbered in request order
+// (a request's chunks are consecutive) and CTAs draw their chunks in that
+// order from a ticket, so every chunk's predecessors belong to warps that
+// have already started.  Each lane reads its block's tokens with 16-byte
+// loads and forms the block digest D_m itself.  The chain
+// C_m = Kc C_{m-1} + D_m (mod 2^61 - 1) composes affine maps, so a warp scan
+// gives each block its chain value B_m relative to the chunk's start (value 0
+// entering it), and the chunk's total (B at its last block) is published
+// under a flag.  The value entering chunk k of a request is then
+//   Kc^(32k) C_seed + sum_{l<k} Kc^(32(k-1-l)) total_l,
+// and no total waits on anything, so the warp folds its k predecessors'
+// totals directly, in windows of 32 (one lane each).  With C_m the lanes form
+// their keys and probe the table.  A block is in the cached prefix iff no
+// block before it in its request misses: the chunk's "some block missed" bit
+// is the second published flag, and the warp ORs its predecessors'.  The
+// cached prefix is pinned for the step; every block past it is claimed in the
+// claim map (lowest request index wins: one materialization, one charge, I1).
+// The warp of a request's first chunk installs the request's history entry.
+//
+// Each chunk publishes one 64-bit word (seg_word, zeroed per call by
+// k_validate): bits 0-60 its chain total (a value mod 2^61 - 1), bit 61 set
+// once the total is there, bit 62 once its miss bit (bit 63) is.  Value and
+// flags travel in one aligned 64-bit store, read with one relaxed 64-bit
+// load, so no fence orders them.  Every wait is bounded; a wait that runs
+// out reports an internal error.
+constexpr uint64_t kWordTotal = 1ull << 61, kWordMiss = 1ull << 62, kWordMissBit = 1ull << 63;
+// A chunk descriptor in two 16-byte loads.
+__device__ __forceinline__ ChunkDesc load_chunk(const ChunkDesc* p) {
+  const uint4 a = __ldg(reinterpret_cast<const uint4*>(p)), b = __ldg(reinterpret_cast<const uint4*>(p) + 1);
+  ChunkDesc d;
+  d.o0 = (int64_t)((uint64_t)a.y << 32 | a.x);
+  d.req = a.z;
+  d.n = (int32_t)a.w;
+  d.pbase = (int32_t)b.x;
+  d.k = (int32_t)b.y;
+  d.group = b.z;
+  d.sb = (int32_t)b.w;
+  return d;
 }
 
-template <int PPB>
-__global__ void __launch_bounds__(HashCfg<PPB>::kWarps * 32) k_hash(DevState s) {
-  s = with_args(s);
-  extern __shared__ __align__(16) int32_t smem_tokens[];
-  using Cfg = HashCfg<PPB>;
-  constexpr int BS = Cfg::BS;
-  constexpr int G32 = 32 / PPB;
-  const Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int64_t seg = (int64_t)blockIdx.x * Cfg::kWarps + warp;
-  if (seg >= c->nsegs) return;
-  int32_t* buf = smem_tokens + warp * Cfg::kWindow;
-  uint64_t* mbar = reinterpret_cast<uint64_t*>(smem_tokens + Cfg::kWarps * Cfg::kWindow) + warp;
-  const uint32_t i = s.seg_req[seg];
-  const int n = s.rq_n[i];
-  const int m0 = (int)(seg - s.rq_sbase[i]) * kSegBlocks;
-  const int m1 = tmin(n, m0 + kSegBlocks);
-  const int64_t o0 = s.in_offsets[i];
-  const int pbase = s.rq_pbase[i];
-  const int64_t T = c->T;
-  // the segment's tokens [cs, ce) and their 16-byte aligned window [ws, we)
-  const int64_t cs = o0 + (int64_t)m0 * BS, ce = o0 + (int64_t)m1 * BS;
-  const int64_t ws = cs & ~3ll, we = (ce + 3) & ~3ll;
-  const int off = (int)(cs - ws);
-  bool staged = false;
-  if (s.tokens_aligned16 && we <= T) {
-    const uint32_t bytes = (uint32_t)((we - ws) * 4);
-    if (lane == 0) {
-      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_addr(mbar)) : "memory");
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(mbar)), "r"(bytes)
-                   : "memory");
-      asm volatile(
-          "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-              smem_addr(buf)),
-          "l"(s.in_tokens + ws), "r"(bytes), "r"(smem_addr(mbar))
-          : "memory");
-    }
-    __syncwarp();
-    // bounded wait for the copy (phase 0); a copy that does not land in time
-    // is reported, and waited for once more (again bounded) before the warp
-    // leaves, so it never writes into released shared memory
-    auto wait_copy = [&](int limit) -> bool {
-      uint32_t done = 0;
-      for (int it = 0; it < limit && !done; ++it)
-        asm volatile(
-            "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n\tselp.u32 %0, 1, 0, p;\n\t}"
-            : "=r"(done)
-            : "r"(smem_addr(mbar))
-            : "memory");
-      return __all_sync(kFull, done != 0);
-    };
-    if (!wait_copy(1 << 22)) {
-      if (lane == 0) s.ctl->internal_error = 1;
-      wait_copy(1 << 22);
-      return;
-    }
-    staged = true;
+// NH sums over a piece of PIECE tokens held in w[] from word OFF on (OFF the
+// warp-uniform word offset, a compile-time constant in each of four forms),
+// with key words from pair index kk0 on.  Summing straight from w[] keeps
+// no second, re-indexed copy of the tokens live.
+template <int OFF, int PIECE, int NWORDS>
+__device__ __forceinline__ void nh_piece(const uint32_t (&w)[NWORDS], const uint32_t* sk, int kk0, uint64_t* a1,
+                                         uint64_t* a2) {
+#pragma unroll
+  for (int k = 0; k < PIECE / 2; ++k) {
+    const int kk = kk0 + k;
+    const uint32_t tx = w[OFF + 2 * k], ty = w[OFF + 2 * k + 1];
+    *a1 += (uint64_t)(tx + sk[2 * kk]) * (uint64_t)(ty + sk[2 * kk + 1]);
+    *a2 += (uint64_t)(tx + sk[2 * kk + 2]) * (uint64_t)(ty + sk[2 * kk + 3]);
   }
-  const int64_t base_tok = staged ? ws : cs;
-  if (!staged) {
-    for (int64_t t = cs + lane; t < ce; t += 32) buf[t - cs] = s.in_tokens[t];
-    __syncwarp();
-  }
-  const int shift_tok = (int)(cs - base_tok);  // 0..3 when staged, 0 otherwise
-  const int k = lane % PPB;
-  const uint32_t K0 = s.key_words[2 * k], K1 = s.key_words[2 * k + 1];
-  const uint32_t K2 = s.key_words[2 * k + 2], K3 = s.key_words[2 * k + 3];
-  const uint64_t Kd = s.digest_mul;
-  uint64_t kp[5];
-#pragma unroll
-  for (int j = 0; j < 5; ++j) kp[j] = s.kc_pow[1 << j];
-  const uint64_t kpl = s.kc_pow[lane + 1];
-  uint64_t carry = 0;  // local chain value at the block before the chunk
-  for (int c0 = m0; c0 < m1; c0 += 32) {
-    const int nb = tmin(32, m1 - c0);
-    const int32_t* cb = buf + shift_tok + (c0 - m0) * BS;
-    uint64_t d1 = 0, d2 = 0;
-    if constexpr (PPB <= 8) {
-      // Round r: the PPB lanes of group q = lane / PPB each take one token
-      // pair of block q + G32 r.  Every lane keeps its PPB partial products;
-      // a reduce-scatter over the group's lanes (recursive halving) leaves
-      // lane k of the group with round k's full sums, and one shuffle moves
-      // block b's sums to lane b.
-      uint64_t a1[PPB], a2[PPB];
-#pragma unroll
-      for (int r = 0; r < PPB; ++r) {
-        const int b = lane / PPB + G32 * r;
-        a1[r] = a2[r] = 0;
-        if (b < nb) {
-          const int32_t tx = cb[b * BS + 2 * k], ty = cb[b * BS + 2 * k + 1];
-          a1[r] = (uint64_t)((uint32_t)tx + K0) * (uint64_t)((uint32_t)ty + K1);
-          a2[r] = (uint64_t)((uint32_t)tx + K2) * (uint64_t)((uint32_t)ty + K3);
-        }
-      }
-#pragma unroll
-      for (int d = PPB / 2; d >= 1; d >>= 1) {
-        const bool up = (k & d) != 0;
-#pragma unroll
-        for (int j = 0; j < d; ++j) {
-          const uint64_t s1 = up ? a1[j] : a1[j + d], s2 = up ? a2[j] : a2[j + d];
-          const uint64_t k1 = up ? a1[j + d] : a1[j], k2 = up ? a2[j + d] : a2[j];
-          a1[j] = k1 + __shfl_xor_sync(kFull, s1, d);
-          a2[j] = k2 + __shfl_xor_sync(kFull, s2, d);
-        }
-      }
-      const int src = (lane % G32) * PPB + lane / G32;  // holder of block `lane`
-      d1 = __shfl_sync(kFull, a1[0], src);
-      d2 = __shfl_sync(kFull, a2[0], src);
-    } else {
-#pragma unroll
-      for (int r = 0; r < PPB; ++r) {
-        const int b = lane / PPB + G32 * r;
-        uint64_t p1 = 0, p2 = 0;
-        if (b < nb) {
-          const int32_t tx = cb[b * BS + 2 * k], ty = cb[b * BS + 2 * k + 1];
-          p1 = (uint64_t)((uint32_t)tx + K0) * (uint64_t)((uint32_t)ty + K1);
-          p2 = (uint64_t)((uint32_t)tx + K2) * (uint64_t)((uint32_t)ty + K3);
-        }
-#pragma unroll
-        for (int o = 1; o < PPB; o <<= 1) {
-          p1 += __shfl_xor_sync(kFull, p1, o);
-          p2 += __shfl_xor_sync(kFull, p2, o);
-        }
-        const int src = (lane % G32) * PPB;
-        const uint64_t q1 = __shfl_sync(kFull, p1, src), q2 = __shfl_sync(kFull, p2, src);
-        if (lane / G32 == r) { d1 = q1; d2 = q2; }
-      }
-    }
-    // D_m, then the inclusive scan of the affine maps x -> Kc x + D
-    uint64_t bb = lane < nb ? add61(red61(d1), mul61(Kd, red61(d2))) : 0;
-#pragma unroll
-    for (int j = 0; j < 5; ++j) {
-      const uint64_t t = __shfl_up_sync(kFull, bb, 1 << j);
-      if (lane >= (1 << j)) bb = add61(bb, mul61(kp[j], t));
-    }
-    const uint64_t B = add61(mul61(kpl, carry), bb);
-    if (lane < nb) {
-      s.pos_key[pbase + c0 + lane] = B;
-      s.pos_req[pbase + c0 + lane] = i;
-    }
-    carry = __shfl_sync(kFull, B, nb - 1);
-  }
-  if (lane == 0) s.seg_tot[seg] = carry;
 }
 
-// Stage 1, one lane per block (block sizes 4, 8 and 16): each lane reads its
-// block's tokens straight from global memory and forms both NH sums itself,
-// so no staging window limits the resident warps and no shuffle network
-// combines partial sums.  A segment belongs to one request, whose blocks all
-// start at the same word offset r = (o_i + m bs) mod 4: each lane loads the
-// 16-byte words covering its block (bs / 4 + 1 of them) and takes its tokens
-// at the warp-uniform offset r.  A block whose words would run past the
-// step's last token, or a token buffer that is not 16-byte aligned, is read
-// token by token.  The chain scan and its outputs are those of k_hash.
-template <int PPB>
-__global__ void __launch_bounds__(256) k_hash_lane(DevState s) {
-  s = with_args(s);
-  constexpr int BS = 2 * PPB;
-  constexpr int NW = BS / 4 + 1;  // 16-byte words covering a block at any word offset
-  static_assert(BS % 4 == 0, "whole-block lanes need bs a multiple of 4");
-  __shared__ uint32_t sk[BS + 2];  // the NH key words (read by every lane alike)
-  const Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  if (threadIdx.x < BS + 2) sk[threadIdx.x] = s.key_words[threadIdx.x];
-  __syncthreads();
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  const int64_t seg = (int64_t)blockIdx.x * (blockDim.x >> 5) + warp;
-  if (seg >= c->nsegs) return;
-  const uint32_t i = s.seg_req[seg];
-  const int n = s.rq_n[i];
-  const int m0 = (int)(seg - s.rq_sbase[i]) * kSegBlocks;
-  const int m1 = tmin(n, m0 + kSegBlocks);
-  const int64_t o0 = s.in_offsets[i];
-  const int pbase = s.rq_pbase[i];
-  const int64_t T = c->T;
-  const int r = (int)(o0 & 3);  // the same for every block of the request
-  const bool vec = s.tokens_aligned16;
-  const uint64_t Kd = s.digest_mul;
-  uint64_t kp[5];
+// The two NH sums of one block (bs tokens from token index g0).  r is the
+// request's word offset (g0 mod 4, the same for all its blocks); with a
+// 16-byte aligned token buffer the block's tokens are read as the 16-byte
+// words that cover them, 16 tokens at a time, otherwise token by token (as
+// they are near the step's last token, where the covering words could pass
+// it).
+template <int BS>
+__device__ __forceinline__ void block_nh(const DevState& s, const uint32_t* sk, int64_t g0, int r, bool vec, int64_t T,
+                                         uint64_t* d1, uint64_t* d2) {
+  constexpr int PIECE = BS < 16 ? BS : 16;  // tokens per piece
+  uint64_t a1 = 0, a2 = 0;
 #pragma unroll
-  for (int j = 0; j < 5; ++j) kp[j] = s.kc_pow[1 << j];
-  const uint64_t kpl = s.kc_pow[lane + 1];
-  uint64_t carry = 0;  // local chain value at the block before the chunk
-  for (int c0 = m0; c0 < m1; c0 += 32) {
-    const int nb = tmin(32, m1 - c0);
-    uint64_t d1 = 0, d2 = 0;
-    if (lane < nb) {
-      const int64_t g0 = o0 + (int64_t)(c0 + lane) * BS;  // the block's first token
-      const int64_t a0 = g0 - r;                            // 16-byte aligned when vec
-      uint32_t tok[BS];
+  for (int q0 = 0; q0 < BS; q0 += PIECE) {
+    const int64_t a0 = g0 + q0 - r;
+    bool done = false;
+    if constexpr (PIECE % 4 == 0) {
+      constexpr int NW = PIECE / 4 + 1;  // 16-byte words covering a piece at any word offset
       if (vec && a0 + 4 * NW <= T) {
         uint32_t w[4 * NW];
         const uint4* src = reinterpret_cast<const uint4*>(s.in_tokens + a0);
@@ -534,149 +462,185 @@ __global__ void __launch_bounds__(256) k_hash_lane(DevState s) {
           w[4 * q + 2] = v.z;
           w[4 * q + 3] = v.w;
         }
-        // r is warp-uniform: four statically indexed forms
-        switch (r) {
-          case 0:
-#pragma unroll
-            for (int j = 0; j < BS; ++j) tok[j] = w[j];
-            break;
-          case 1:
-#pragma unroll
-            for (int j = 0; j < BS; ++j) tok[j] = w[j + 1];
-            break;
-          case 2:
-#pragma unroll
-            for (int j = 0; j < BS; ++j) tok[j] = w[j + 2];
-            break;
-          default:
-#pragma unroll
-            for (int j = 0; j < BS; ++j) tok[j] = w[j + 3];
-            break;
+        switch (r) {  // warp-uniform
+          case 0: nh_piece<0, PIECE>(w, sk, q0 / 2, &a1, &a2); break;
+          case 1: nh_piece<1, PIECE>(w, sk, q0 / 2, &a1, &a2); break;
+          case 2: nh_piece<2, PIECE>(w, sk, q0 / 2, &a1, &a2); break;
+          default: nh_piece<3, PIECE>(w, sk, q0 / 2, &a1, &a2); break;
         }
-      } else {
-#pragma unroll
-        for (int j = 0; j < BS; ++j) tok[j] = (uint32_t)s.in_tokens[g0 + j];
-      }
-#pragma unroll
-      for (int k = 0; k < PPB; ++k) {
-        const uint32_t tx = tok[2 * k], ty = tok[2 * k + 1];
-        d1 += (uint64_t)(tx + sk[2 * k]) * (uint64_t)(ty + sk[2 * k + 1]);
-        d2 += (uint64_t)(tx + sk[2 * k + 2]) * (uint64_t)(ty + sk[2 * k + 3]);
+        done = true;
       }
     }
-    // D_m, then the inclusive scan of the affine maps x -> Kc x + D
-    uint64_t bb = lane < nb ? add61(red61(d1), mul61(Kd, red61(d2))) : 0;
+    if (!done) {
+      uint32_t w[PIECE];
 #pragma unroll
-    for (int j = 0; j < 5; ++j) {
-      const uint64_t t = __shfl_up_sync(kFull, bb, 1 << j);
-      if (lane >= (1 << j)) bb = add61(bb, mul61(kp[j], t));
+      for (int j = 0; j < PIECE; ++j) w[j] = (uint32_t)s.in_tokens[g0 + q0 + j];
+      nh_piece<0, PIECE>(w, sk, q0 / 2, &a1, &a2);
     }
-    const uint64_t B = add61(mul61(kpl, carry), bb);
-    if (lane < nb) {
-      s.pos_key[pbase + c0 + lane] = B;
-      s.pos_req[pbase + c0 + lane] = i;
-    }
-    carry = __shfl_sync(kFull, B, nb - 1);
   }
-  if (lane == 0) s.seg_tot[seg] = carry;
+  *d1 = a1;
+  *d2 = a2;
 }
 
-// Stage 2: block keys and the longest cached prefix (n_cached of Alg. 1),
-// thread per position: C_in = the chain value entering the position's
-// segment (C = Kc^256 C + B_end over the request's earlier segments),
-// key_m = mix(C_m ^ (m+1) c) with C_m = Kc^(k+1) C_in + B_m, then a table
-// probe; a miss lowers the request's h_i to its position.
-__global__ void __launch_bounds__(kThreads) k_keys_lookup(DevState s) {
-  s = with_args(s);
-  const Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  PosRef r;
-  const bool valid = pos_ref(s, pos, &r);
-  bool miss = false;
-  if (valid) {
-    // chain value entering this position's segment: fold the earlier segments
-    const int64_t sb = s.rq_sbase[r.i];
-    const int js = r.m / kSegBlocks;
-    uint64_t cin = red61(chain_seed(s.hash_seed, s.in_group[r.i]));
-    for (int j = 0; j < js; ++j) cin = add61(mul61(s.kc_pow[kSegBlocks], cin), s.seg_tot[sb + j]);
-    const uint64_t C = add61(mul61(s.kc_pow[r.m % kSegBlocks + 1], cin), s.pos_key[pos]);
-    const uint64_t key = fix_reserved(mix64(C ^ ((uint64_t)(r.m + 1) * 0xD1B54A32D192ED03ull)));
-    s.pos_key[pos] = key;
-    const uint32_t blk = table_find(s, key, (uint32_t)s.in_group[r.i]);
-    s.pos_blk[pos] = blk;
-    miss = blk == kNone;
+// One chunk (j) of k_hash_lookup, by one warp.  Returns false if a wait for
+// a predecessor ran out (never expected).
+template <int BS>
+__device__ __forceinline__ bool hash_lookup_chunk(const DevState& s, Ctl* c, const uint32_t* sk, const uint64_t* kc,
+                                                  int64_t j, int probe) {
+  const int lane = lane_id();
+  const ChunkDesc d = load_chunk(s.chunks + j);
+  const uint32_t i = d.req;
+  const int n = d.n;
+  const int64_t sb = d.sb;
+  const int k = d.k;  // chunk index within the request
+  const int m0 = k * kSegBlocks;
+  const int nb = tmin(kSegBlocks, n - m0);
+  const int64_t o0 = d.o0;
+  const int pbase = d.pbase;
+  const uint32_t g = d.group;
+  const int64_t T = c->T;
+  const int m = m0 + lane;
+  // D_m, then the inclusive scan of the affine maps x -> Kc x + D
+  uint64_t bb = 0;
+  if (lane < nb) {
+    uint64_t d1, d2;
+    block_nh<BS>(s, sk, o0 + (int64_t)m * BS, (int)(o0 & 3), s.tokens_aligned16 != 0, T, &d1, &d2);
+    bb = add61(red61(d1), mul61(s.digest_mul, red61(d2)));
   }
-  // h_i = the first miss: one atomic per request per warp
-  agg_min_u32(reinterpret_cast<uint32_t*>(s.rq_h), valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, miss);
-}
-
-// Stage 2 (cont.): blocks of the cached prefix are pinned for the step;
-// every position at or past the first miss is claimed in the step's claim
-// map (lowest request index wins: one materialization, one charge, I1).
-// Threads past the positions record each request's history entry
-// (OnRequest of Alg. 1) under its prefix id.
-__global__ void __launch_bounds__(kThreads) k_pin_claim(DevState s) {
-  s = with_args(s);
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int64_t t = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  const int64_t nb = c->nblocks;
+#pragma unroll
+  for (int q = 0; q < 5; ++q) {
+    const uint64_t t = __shfl_up_sync(kFull, bb, 1 << q);
+    if (lane >= (1 << q)) bb = add61(bb, mul61(kc[1 << q], t));
+  }
+  const uint64_t total = __shfl_sync(kFull, bb, nb - 1);
+  if (lane == 0) st_relaxed_u64(s.seg_word + j, total | kWordTotal);
+  // the chain value entering the chunk
+  bool ok = true;
+  uint64_t cin = red61(chain_seed(s.hash_seed, (int32_t)g));
+  for (int l0 = 0; l0 < k; l0 += 32) {
+    const int w = tmin(32, k - l0);
+    uint64_t term = 0;
+    if (lane < w) {
+      const uint64_t v = wait_word(s.seg_word + sb + l0 + lane, kWordTotal);
+      ok = ok && v != 0;
+      term = mul61(kc[(kSegBlocks + 1) + (w - 1 - lane)], v & kP61);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) term = add61(term, __shfl_xor_sync(kFull, term, o));
+    cin = add61(mul61(kc[(kSegBlocks + 1) + w], cin), term);
+  }
+  // the lane's key and its table probe
+  uint64_t key = 0;
+  uint32_t blk = kNone;
+  if (lane < nb) {
+    const uint64_t C = add61(mul61(kc[lane + 1], cin), bb);
+    key = fix_reserved(mix64(C ^ ((uint64_t)(m + 1) * 0xD1B54A32D192ED03ull)));
+    blk = table_find(s, key, g);
+  }
+  const unsigned missmask = __ballot_sync(kFull, lane < nb && blk == kNone);
+  if (lane == 0) st_relaxed_u64(s.seg_word + j, total | kWordTotal | kWordMiss | (missmask ? kWordMissBit : 0));
+  // did any earlier block of the request miss?
+  bool missbefore = false;
+  for (int l0 = 0; l0 < k && !missbefore; l0 += 32) {
+    const int w = tmin(32, k - l0);
+    bool mb = false;
+    if (lane < w) {
+      const uint64_t v = wait_word(s.seg_word + sb + l0 + lane, kWordMiss);
+      ok = ok && v != 0;
+      mb = (v & kWordMissBit) != 0;
+    }
+    missbefore = __any_sync(kFull, mb);
+  }
+  if (!__all_sync(kFull, ok)) return false;  // a predecessor never published
+  const int first = missmask ? __ffs(missmask) - 1 : kSegBlocks;  // first miss in this chunk
+  if (!missbefore && missmask && lane == 0) s.rq_h[i] = m0 + first;  // h_i: its only writer
+  if (probe) return true;
+  const bool in_prefix = lane < nb && !missbefore && lane < first;
   const uint32_t step32 = (uint32_t)c->step;
   bool newpin = false;
-  uint32_t pin_group = 0, pin_klass = 0;
-  if (t < nb) {
-    PosRef r;
-    pos_ref(s, t, &r);
-    if (r.m < s.rq_h[r.i]) {
-      const uint32_t b = s.pos_blk[t];
-      newpin = atomicExch(s.blk_pin + b, step32) != step32;
-      pin_group = (uint32_t)s.in_group[r.i];  // the owner: hits are namespaced by group
-      if (newpin && s.lg_on) pin_klass = s.blk_klass[b];
-      if (newpin && s.policy == PS_S3FIFO) atomic_add_i64(&c->s3_pinned[(s.blk_flags[b] >> 1) & 1], 1);
-      s.pos_claim[t] = kNone;
+  uint32_t pin_klass = 0;
+  if (lane < nb) {
+    const int64_t p = pbase + m;
+    s.pos_key[p] = key;
+    s.pos_req[p] = i;
+    s.pos_blk[p] = blk;
+    if (in_prefix) {
+      newpin = atomicExch(s.blk_pin + blk, step32) != step32;
+      if (newpin && s.lg_on) pin_klass = s.blk_klass[blk];
+      if (newpin && s.policy == PS_S3FIFO) atomic_add_i64(&c->s3_pinned[(s.blk_flags[blk] >> 1) & 1], 1);
+      s.pos_claim[p] = kNone;
     } else {
-      s.pos_claim[t] = claim_insert(s, s.pos_key[t], r.i);
+      s.pos_claim[p] = claim_insert(s, key, i);
     }
-  } else if (t < nb + s.R) {
-    const int i = (int)(t - nb);
-    const int n = s.rq_n[i];
-    const uint32_t g = (uint32_t)s.in_group[i];
-    uint32_t hs = kNone;
-    uint64_t p = 0;
-    if (n > 0) {
-      p = s.in_prefix ? s.in_prefix[i] : s.pos_key[s.rq_pbase[i]];
-      const uint32_t hmask = (1u << s.hist_cap_log2) - 1;
-      uint32_t x = hist_home(p, g, s.hist_cap_log2);
-      for (uint32_t it = 0; it <= hmask; ++it, x = (x + 1) & hmask) {
-        uint64_t olo, ohi;
-        cas128(s.hist + x, 0ull, 0ull, p, (uint64_t)(g + 1), &olo, &ohi);
-        if (olo == 0 && ohi == 0) {
-          atomic_add_i64(&c->hist_new, 1);
-          hs = x;
-          break;
-        }
-        if (olo == p && (uint32_t)ohi == g + 1) {
-          hs = x;
-          break;
-        }
-      }
-      if (hs != kNone)
-        atomicMax(reinterpret_cast<unsigned long long*>(&s.hist[hs].ftag),
-                  (unsigned long long)step_tag(c->step, (uint32_t)i));
-    }
-    s.rq_hs[i] = hs;
-    s.rq_p[i] = p;
   }
   const int np = __popc(__ballot_sync(kFull, newpin));
-  if (lane_id() == 0 && np) atomic_add_i64(&c->pinned, np);
-  if (s.policy == PS_STATICQUOTA) agg_add_i64(s.grp_pinned, pin_group, 1, newpin);
+  if (lane == 0 && np) atomic_add_i64(&c->pinned, np);
+  // hits are namespaced by group: every block the warp pins is group g's
+  if (s.policy == PS_STATICQUOTA && lane == 0 && np) atomic_add_i64(s.grp_pinned + g, np);
   if (s.lg_on) {  // a pinned block is no candidate: it leaves its queues' live counts (applied in k_lg_cand)
-    const int32_t A = lg_log_a(s, pin_group, pin_klass), B = lg_log_b(s, pin_klass);
+    const int32_t A = lg_log_a(s, g, pin_klass), B = lg_log_b(s, pin_klass);
     agg_add_i64(s.lg_pin, (uint32_t)A, 1, newpin && A >= 0);
     agg_add_i64(s.lg_pin, (uint32_t)B, 1, newpin && B >= 0);
   }
+  // OnRequest of Alg. 1: the request's (group, prefix) history entry
+  if (k == 0 && lane == 0) {
+    const uint64_t pid = s.in_prefix ? s.in_prefix[i] : key;  // default: block 0's key
+    uint32_t hs = kNone;
+    const uint32_t hmask = (1u << s.hist_cap_log2) - 1;
+    uint32_t x = hist_home(pid, g, s.hist_cap_log2);
+    for (uint32_t it = 0; it <= hmask; ++it, x = (x + 1) & hmask) {
+      uint64_t olo, ohi;
+      cas128(s.hist + x, 0ull, 0ull, pid, (uint64_t)(g + 1), &olo, &ohi);
+      if (olo == 0 && ohi == 0) {
+        atomic_add_i64(&c->hist_new, 1);
+        hs = x;
+        break;
+      }
+      if (olo == pid && (uint32_t)ohi == g + 1) {
+        hs = x;
+        break;
+      }
+    }
+    if (hs != kNone)
+      atomicMax(reinterpret_cast<unsigned long long*>(&s.hist[hs].ftag), (unsigned long long)step_tag(c->step, i));
+    s.rq_hs[i] = hs;
+    s.rq_p[i] = pid;
+  }
+  return true;
 }
+
+// The kernel: persistent warps.  Each warp takes chunk tickets one at a time,
+// each only once it is free to start the chunk, so a chunk's predecessors
+// (lower tickets) have always started hashing before it, and their totals
+// arrive about when its own does.  A chunk waits only on chunks of lower
+// tickets, each held by a running warp: the waits always make progress.
+// probe = 1: the read-only probe (ps_cached_prefix): h_i only, no pins,
+// claims, history or per-position records.
+constexpr int kHashCtasPerSm = 6;
+template <int BS>
+__global__ void __launch_bounds__(256, kHashCtasPerSm) k_hash_lookup(DevState s, int probe) {
+  s = with_args(s);
+  __shared__ uint32_t sk[BS + 2];                // the NH key words (read by every lane alike)
+  __shared__ uint64_t kc[2 * (kSegBlocks + 1)];  // Kc^j, then Kc^(32 t)
+  Ctl* c = s.ctl;
+  if (c->status != PS_OK) return;
+  if (threadIdx.x < BS + 2) sk[threadIdx.x] = s.key_words[threadIdx.x];
+  if (threadIdx.x < 2 * (kSegBlocks + 1)) kc[threadIdx.x] = s.kc_pow[threadIdx.x];
+  __syncthreads();
+  const int lane = lane_id();
+  const int64_t nsegs = c->nsegs;
+  for (;;) {
+    uint32_t t = 0;
+    if (lane == 0) t = atomicAdd(&c->hash_ticket, 1u);
+    t = __shfl_sync(kFull, t, 0);
+    if ((int64_t)t >= nsegs) return;
+    if (!hash_lookup_chunk<BS>(s, c, sk, kc, (int64_t)t, probe)) {
+      if (lane == 0) c->internal_error = 1;
+      return;
+    }
+  }
+}
+
 
 // A step whose new (group, prefix) entries would overflow the history map
 // fails as a whole, leaving the pool as it was (Alg. 1's hooks change state
@@ -2277,23 +2241,23 @@ void launch_init(const DevState& s, cudaStream_t st) {
   launch_queue_init(s, st);
 }
 
-template <int PPB>
-static void launch_hash_t(const DevState& s, cudaStream_t st) {
-  using Cfg = HashCfg<PPB>;
-  k_hash<PPB><<<(int)((s.max_segments + Cfg::kWarps - 1) / Cfg::kWarps), Cfg::kWarps * 32, Cfg::kSmem, st>>>(s);
+template <int BS>
+static void launch_hash_lookup_t(const DevState& s, cudaStream_t st, int probe) {
+  // persistent: the CTAs that fit at once (more only queue behind them)
+  int dev = 0, nsm = 152;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (s.max_segments + 7) / 8;
+  const int grid = (int)(want < (int64_t)nsm * kHashCtasPerSm ? want : (int64_t)nsm * kHashCtasPerSm);
+  k_hash_lookup<BS><<<grid > 0 ? grid : 1, 256, 0, st>>>(s, probe);
 }
-template <int PPB>
-static void launch_hash_lane(const DevState& s, cudaStream_t st) {
-  k_hash_lane<PPB><<<(int)((s.max_segments + 7) / 8), 256, 0, st>>>(s);
-}
-static int32_t launch_hash(const DevState& s, cudaStream_t st) {
-  switch (s.bs / 2) {
-    case 1: launch_hash_t<1>(s, st); break;
-    case 2: launch_hash_lane<2>(s, st); break;
-    case 4: launch_hash_lane<4>(s, st); break;
-    case 8: launch_hash_lane<8>(s, st); break;
-    case 16: launch_hash_t<16>(s, st); break;
-    case 32: launch_hash_t<32>(s, st); break;
+static int32_t launch_hash_lookup(const DevState& s, cudaStream_t st, int probe) {
+  switch (s.bs) {
+    case 2: launch_hash_lookup_t<2>(s, st, probe); break;
+    case 4: launch_hash_lookup_t<4>(s, st, probe); break;
+    case 8: launch_hash_lookup_t<8>(s, st, probe); break;
+    case 16: launch_hash_lookup_t<16>(s, st, probe); break;
+    case 32: launch_hash_lookup_t<32>(s, st, probe); break;
+    case 64: launch_hash_lookup_t<64>(s, st, probe); break;
     default: return PS_ERR_INVALID_ARG;
   }
   return PS_OK;
@@ -2304,12 +2268,6 @@ void configure_kernels(const DevState& s) {
   cudaFuncSetAttribute(k_digit_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, kRadixSmemRows * kRadixBins * 4);
   cudaFuncSetAttribute(k_list_finish, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFinSmem);
   cudaFuncSetAttribute(k_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, PS_MAX_GROUPS * kClasses * 5 * 4);
-  cudaFuncSetAttribute(k_hash<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<1>::kSmem);
-  cudaFuncSetAttribute(k_hash<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<2>::kSmem);
-  cudaFuncSetAttribute(k_hash<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<4>::kSmem);
-  cudaFuncSetAttribute(k_hash<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<8>::kSmem);
-  cudaFuncSetAttribute(k_hash<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<16>::kSmem);
-  cudaFuncSetAttribute(k_hash<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)HashCfg<32>::kSmem);
 }
 
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const CaptureCtx* cap) {
@@ -2334,12 +2292,10 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   };
 #define PS_LAUNCH(...) do { __VA_ARGS__; ++launches; } while (0)
   mark(0);
-  PS_LAUNCH(launch_k(k_validate, 1, 1024, 0, st, s, 0));
+  PS_LAUNCH(launch_k(k_validate, grid_for(R, kValTile, 1 << 20), kValTile, 0, st, s, 0));
   mark(1);
-  if (launch_hash(s, st) != PS_OK) return PS_ERR_INVALID_ARG;
+  if (launch_hash_lookup(s, st, 0) != PS_OK) return PS_ERR_INVALID_ARG;
   ++launches;
-  PS_LAUNCH(k_keys_lookup<<<pgrid, kThreads, 0, st>>>(s));
-  PS_LAUNCH(k_pin_claim<<<prgrid, kThreads, 0, st>>>(s));
   mark(2);
   PS_LAUNCH(launch_k(k_claims, prgrid, kThreads, 0, st, s));
   mark(3);
@@ -2513,11 +2469,8 @@ int32_t launch_probe(const DevState& s, cudaStream_t st, int32_t* out, int32_t* 
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
   DevState p = s;
   p.args = nullptr;  // the probe's kernels take every argument by value
-  k_validate<<<1, 1024, 0, st>>>(p, 1);
-  if (s.R > 0) {
-    if (launch_hash(p, st) != PS_OK) return PS_ERR_INVALID_ARG;
-    k_keys_lookup<<<pgrid, kThreads, 0, st>>>(p);
-  }
+  k_validate<<<grid_for(p.max_requests, kValTile, 1 << 20), kValTile, 0, st>>>(p, 1);
+  if (s.R > 0 && launch_hash_lookup(p, st, 1) != PS_OK) return PS_ERR_INVALID_ARG;
   k_probe_out<<<rgrid, 256, 0, st>>>(p, out, status);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }

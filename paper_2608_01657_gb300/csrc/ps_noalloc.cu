@@ -29,9 +29,10 @@ constexpr int64_t kNaMaxSegments = kNaMaxBlocks / kSegBlocks + kNaMaxRequests + 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 constexpr size_t kOffCtl = 0;
 constexpr size_t kOffRq = align256(kOffCtl + sizeof(Ctl));
-constexpr size_t kRqArrays = 6;  // n, h, s, fu, pbase, sbase
-constexpr size_t kOffSeg = align256(kOffRq + kRqArrays * align256(4 * kNaMaxRequests));
-constexpr size_t kOffPos = align256(kOffSeg + align256(4 * kNaMaxSegments) + 2 * align256(8 * kNaMaxSegments));
+constexpr size_t kRqArrays = 5;  // n, h, s, fu, pbase
+constexpr size_t kOffTile = align256(kOffRq + kRqArrays * align256(4 * kNaMaxRequests));
+constexpr size_t kOffSeg = align256(kOffTile + 8 * (kNaMaxRequests / 256 + 1));
+constexpr size_t kOffPos = align256(kOffSeg + align256(sizeof(ChunkDesc) * kNaMaxSegments) + align256(8 * kNaMaxSegments));
 constexpr size_t kScratchBytes = align256(kOffPos + align256(8 * kNaMaxBlocks) + 2 * align256(4 * kNaMaxBlocks));
 
 // The scratch itself (about 2.3 MB).  In host code 'g_probe_scratch' names a
@@ -94,10 +95,9 @@ extern "C" int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_
   s.rq_s = reinterpret_cast<int32_t*>(base + kOffRq + 2 * rq);
   s.rq_fu = reinterpret_cast<uint32_t*>(base + kOffRq + 3 * rq);
   s.rq_pbase = reinterpret_cast<int32_t*>(base + kOffRq + 4 * rq);
-  s.rq_sbase = reinterpret_cast<int32_t*>(base + kOffRq + 5 * rq);
-  s.seg_req = reinterpret_cast<uint32_t*>(base + kOffSeg);
-  s.seg_cin = reinterpret_cast<uint64_t*>(base + kOffSeg + align256(4 * kNaMaxSegments));
-  s.seg_tot = reinterpret_cast<uint64_t*>(base + kOffSeg + align256(4 * kNaMaxSegments) + align256(8 * kNaMaxSegments));
+  s.val_tile = reinterpret_cast<uint64_t*>(base + kOffTile);
+  s.chunks = reinterpret_cast<ChunkDesc*>(base + kOffSeg);
+  s.seg_word = reinterpret_cast<uint64_t*>(base + kOffSeg + align256(sizeof(ChunkDesc) * kNaMaxSegments));
   s.pos_key = reinterpret_cast<uint64_t*>(base + kOffPos);
   s.pos_req = reinterpret_cast<uint32_t*>(base + kOffPos + align256(8 * kNaMaxBlocks));
   s.pos_blk = reinterpret_cast<uint32_t*>(base + kOffPos + align256(8 * kNaMaxBlocks) + align256(4 * kNaMaxBlocks));
@@ -108,7 +108,9 @@ extern "C" int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_
   s.in_contract = nullptr;
   s.in_prefix = nullptr;
   s.tokens_aligned16 = (reinterpret_cast<uintptr_t>(d_tokens) & 15) == 0;
-  // Every scratch word the probe reads it first writes in the same call
-  // (the control block's per-call fields included), so nothing is cleared.
+  // Every scratch word the probe reads it first writes in the same call (the
+  // control block's per-call fields included), except validation's tile
+  // totals and counters: those start at zero (a static array is zeroed at
+  // load) and every call leaves them at zero, so nothing is cleared here.
   return launch_probe(s, reinterpret_cast<cudaStream_t>(stream), d_cached_blocks, d_status);
 }
