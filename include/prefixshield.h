@@ -289,7 +289,8 @@ int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_t num_reque
  * stream before each of its PS_NUM_STAGES stages and after the last one:
  *   0 validate, 1 hash + lookup, 2 claims + orphans, 3 grant + in-step hits,
  *   4 metering, 5 touch + gate, 6 victim selection, 7 free-take + id lists,
- *   8 eviction, 9 insertion, 10 commit.
+ *   8 eviction (empty: each victim's old content is dropped by the insertion
+ *   that reuses its id), 9 eviction + insertion, 10 commit.
  * Creating the events is the only work; no device memory is allocated. */
 #define PS_NUM_STAGES 11
 int32_t ps_set_stage_timing(ps_handle_t* h, int32_t enable);

@@ -240,6 +240,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.rq_knew = cv.take<uint8_t>(R);
   t.pos_key = cv.take<uint64_t>(B);
   t.pos_req = cv.take<uint32_t>(B);
+  t.pos_m = cv.take<uint32_t>(B);
   t.chunks = cv.take<ChunkDesc>((size_t)d.max_segments);
   t.val_tile = cv.take<uint64_t>(R / 256 + 1);
   t.seg_word = cv.take<uint64_t>((size_t)d.max_segments);

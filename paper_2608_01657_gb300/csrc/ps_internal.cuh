@@ -46,11 +46,16 @@ struct __align__(16) TableEntry {   // native prefix table (group, key) -> block
 struct __align__(32) ClaimEntry {   // per-step: first request that needs a new key
   uint64_t key;     // 0 when empty
   uint32_t minreq;  // lowest request index containing the key (atomicMin)
-  uint32_t last;    // 1 + highest request index that hit it in-step (atomicMax)
   uint32_t tcnt;    // in-step touches
   uint32_t promo;   // lowest request index whose touch promotes it
-  uint32_t pad0, pad1;
+  uint32_t pad;
+  uint64_t stamp;   // recency stamp of the latest in-step touch (atomicMax; 0: none)
 };
+__host__ __device__ __forceinline__ ClaimEntry empty_claim() {
+  ClaimEntry e{};
+  e.key = 0; e.minreq = kNone; e.tcnt = 0; e.promo = kNone; e.pad = 0; e.stamp = 0;
+  return e;
+}
 
 struct __align__(32) HistEntry {    // (group, prefix id) -> reference history
   uint64_t p;       // 0 when empty
@@ -251,6 +256,7 @@ struct DevState {
   uint8_t* rq_knew;        // class of newly admitted blocks
   uint64_t* pos_key;       // chain partial, then the block key
   uint32_t* pos_req;       // request of the position
+  uint32_t* pos_m;         // the position's block index within its request
   ChunkDesc* chunks;       // hashing chunks of the call, in request order
   uint64_t* val_tile;      // k_validate's published per-tile totals (zero between calls)
   uint64_t* seg_word;      // the chunk's published chain total and miss bit (k_hash_lookup)

@@ -100,41 +100,40 @@ __device__ uint32_t table_find(const DevState& s, uint64_t key, uint32_t g) {
 }
 
 // Returns the slot, with kDisplaced set when it lies past the home bucket
-// (then a delete must repair the overflow counters on the way).
+// (then a delete must repair the overflow counters on the way).  The swap
+// starts at a way chosen by the key's own bits: at a quarter load that way
+// is usually free, so most inserts take one atomic and no load.  (No key is
+// inserted twice, so no swaps pile up on one way.)
 constexpr uint32_t kDisplaced = 0x80000000u;
 __device__ uint32_t table_insert(const DevState& s, uint64_t key, uint32_t g, uint32_t blk) {
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
   uint32_t b = table_home(key, g, s.tb_nbuckets_log2);
+  const uint32_t w0 = (uint32_t)(key >> 7) & (kTableWays - 1);
   for (uint32_t it = 0; it <= mask; ++it) {
-    // the bucket's occupancy in one round of loads; then CAS the first free
-    // way (a lost race marks that way taken and moves on)
     TableEntry* e = s.table + (size_t)b * kTableWays;
-    uint32_t occ = 0;
-#pragma unroll
-    for (int w = 0; w < kTableWays; ++w) occ |= (ldcg_u32(&e[w].blk) != kNone ? 1u : 0u) << w;
-    while (occ != (1u << kTableWays) - 1) {
-      const int w = __ffs(~occ) - 1;
+    for (int q = 0; q < kTableWays; ++q) {
+      const int w = (int)((w0 + (uint32_t)q) & (kTableWays - 1));
       if (atomicCAS(&e[w].blk, kNone, blk) == kNone) {
         e[w].key = key;
         e[w].grp = g;
         return (b * kTableWays + w) | (it ? kDisplaced : 0u);
       }
-      occ |= 1u << w;
     }
     atomicAdd(s.table_ovf + b, 1u);
     b = (b + 1) & mask;
   }
-  return kNone;  // unreachable: the table is at most half full
+  return kNone;  // unreachable: the table is at most a quarter full
 }
 
+// An entry is empty exactly when its block field is kNone (lookups test it
+// first), so a delete clears only that field: an insert that takes the slot
+// at once then writes its own key and group, and no late clearing store of
+// the delete can land on them.
 __device__ void table_delete(const DevState& s, uint32_t blk) {
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
   const uint32_t tagged = s.blk_slot[blk];
   const uint32_t slot = tagged & ~kDisplaced;
-  TableEntry* e = s.table + slot;
-  e->key = 0;
-  e->grp = 0;
-  e->blk = kNone;
+  s.table[slot].blk = kNone;
   if (!(tagged & kDisplaced)) return;  // in its home bucket: no counter passed
   const uint32_t bucket = slot / kTableWays;
   uint32_t x = table_home(s.blk_key[blk], s.blk_group[blk], s.tb_nbuckets_log2);
@@ -192,8 +191,8 @@ struct PosRef {
 };
 __device__ __forceinline__ bool pos_ref(const DevState& s, int64_t pos, PosRef* r) {
   if (pos >= s.ctl->nblocks) return false;
-  r->i = s.pos_req[pos];
-  r->m = (int)(pos - s.rq_pbase[r->i]);
+  r->i = s.pos_req[pos];  // both loads in one round trip
+  r->m = (int)s.pos_m[pos];
   return true;
 }
 
@@ -202,9 +201,7 @@ __device__ __forceinline__ bool pos_ref(const DevState& s, int64_t pos, PosRef* 
 __global__ void k_init_blocks(DevState s) {
   const int64_t nclaims = (int64_t)kClaimWays << s.cl_nbuckets_log2;
   for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < nclaims; c += (int64_t)gridDim.x * blockDim.x) {
-    ClaimEntry e{};
-    e.key = 0; e.minreq = kNone; e.last = 0; e.tcnt = 0; e.promo = kNone; e.pad0 = 0; e.pad1 = 0;
-    s.claims[c] = e;
+    s.claims[c] = empty_claim();
   }
 }
 __global__ void k_init_ctl(DevState s) {
@@ -563,6 +560,7 @@ __device__ __forceinline__ bool hash_lookup_chunk(const DevState& s, Ctl* c, con
     const int64_t p = pbase + m;
     s.pos_key[p] = key;
     s.pos_req[p] = i;
+    s.pos_m[p] = (uint32_t)m;
     s.pos_blk[p] = blk;
     if (in_prefix) {
       newpin = atomicExch(s.blk_pin + blk, step32) != step32;
@@ -667,11 +665,7 @@ __device__ void undo_pin_claim(const DevState& s, const Ctl* c, int64_t t) {
       s.blk_pin[s.pos_blk[t]] = step32 - 1u;
     } else {
       const uint32_t slot = s.pos_claim[t];
-      if (slot != kNone) {
-        ClaimEntry z{};
-        z.key = 0; z.minreq = kNone; z.last = 0; z.tcnt = 0; z.promo = kNone; z.pad0 = 0; z.pad1 = 0;
-        s.claims[slot] = z;
-      }
+      if (slot != kNone) s.claims[slot] = empty_claim();
     }
   } else if (t < nb + s.R) {
     const uint32_t hs = s.rq_hs[t - nb];
@@ -1072,7 +1066,9 @@ __global__ void __launch_bounds__(kThreads) k_touch(DevState s) {
   } else {
     ClaimEntry* e = s.claims + s.pos_claim[pos];
     const uint32_t j = e->minreq;
-    atomicMax(&e->last, i + 1);
+    // later requests give larger stamps: the maximum is the latest touch's
+    atomicMax(reinterpret_cast<unsigned long long*>(&e->stamp),
+              (unsigned long long)make_stamp(c->stamp_base, s.rq_pbase[i], s.rq_n[i], m));
     atomicAdd(&e->tcnt, 1u);
     elig = proven && s.rq_cid[j] == cid && s.rq_p[j] == p;  // new blocks are never Reuse yet
     if (elig && gate) atomicMin(&e->promo, i);
@@ -1417,32 +1413,34 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
     __syncthreads();
   }
   const int ng = s_ng;
-  int L = 1, logT = 10;  // blockDim.x == 1024 == T * L
-  while (L < ng && L < 32) { L <<= 1; --logT; }
-  const int T = 1 << logT;
   int64_t lo = eps + 1, hi = s_pmax;
-  const int jt = threadIdx.x / L, gl = threadIdx.x % L;
-  for (int r = 0; lo < hi; ++r) {
-    const int64_t span = hi - lo;  // >= 1
-    const int64_t stride = tmax<int64_t>(1, (span + T - 1) >> logT);
-    auto thr = [&](int jj) -> int64_t { return jj == T - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * jj); };
-    const int64_t t = thr(jt);
-    int64_t cnt = 0;
-    for (int k = gl; k < ng; k += L) cnt += items_gt(s_gid[k], t - 1);
-    for (int o = L / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
-    // J = the largest threshold still holding m items (counts fall as the
-    // threshold rises); slots rotate over three rounds, so one barrier a
-    // round separates every slot's reset, updates and reads
-    if (threadIdx.x == 0) s_J[(r + 1) % 3] = -1;
-    if (gl == 0 && cnt >= m) atomicMax(&s_J[r % 3], jt);
-    __syncthreads();
-    const int J = s_J[r % 3];
-    if (J < 0) {
-      hi = lo;
-    } else {
-      lo = thr(J);
-      hi = J + 1 < T ? thr(J + 1) - 1 : hi;
-      if (hi < lo) hi = lo;
+  {
+    int L = 1, logT = 10;  // blockDim.x == 1024 == T * L
+    while (L < ng && L < 32) { L <<= 1; --logT; }
+    const int T = 1 << logT;
+    const int jt = threadIdx.x / L, gl = threadIdx.x % L;
+    for (int r = 0; lo < hi; ++r) {
+      const int64_t span = hi - lo;  // >= 1
+      const int64_t stride = tmax<int64_t>(1, (span + T - 1) >> logT);
+      auto thr = [&](int jj) -> int64_t { return jj == T - 1 ? hi : tmin<int64_t>(hi, lo + 1 + stride * jj); };
+      const int64_t t = thr(jt);
+      int64_t cnt = 0;
+      for (int k = gl; k < ng; k += L) cnt += items_gt(s_gid[k], t - 1);
+      for (int o = L / 2; o > 0; o >>= 1) cnt += __shfl_xor_sync(kFull, cnt, o);
+      // J = the largest threshold still holding m items (counts fall as the
+      // threshold rises); slots rotate over three rounds, so one barrier a
+      // round separates every slot's reset, updates and reads
+      if (threadIdx.x == 0) s_J[(r + 1) % 3] = -1;
+      if (gl == 0 && cnt >= m) atomicMax(&s_J[r % 3], jt);
+      __syncthreads();
+      const int J = s_J[r % 3];
+      if (J < 0) {
+        hi = lo;
+      } else {
+        lo = thr(J);
+        hi = J + 1 < T ? thr(J + 1) - 1 : hi;
+        if (hi < lo) hi = lo;
+      }
     }
   }
   const int64_t tau = lo;
@@ -2122,28 +2120,16 @@ __global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
   }
 }
 
-// Evict the victims (thread per evicted id): drop table entries and metadata.
-__global__ void __launch_bounds__(kThreads) k_evict(DevState s) {
-  s = with_args(s);
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int64_t v = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-  const int64_t nv = c->n_evicted;
-  const bool act = v < nv && v < s.max_blocks;
-  uint32_t g = 0;
-  if (act) g = drop_block(s, (uint32_t)s.out.evicted_ids[v], false);
-  agg_stat(s, g, PS_STAT_EVICTED_BLOCKS, 1, act);
-  agg_stat(s, g, PS_STAT_RESIDENT_BLOCKS, -1, act);
-  const int k = __popc(__ballot_sync(kFull, act));
-  if (lane_id() == 0 && k) atomic_add_i64(&c->n_resident, -k);
-}
-
 // Stage 6: place granted claims (thread per position).  The allocated ids
 // (ascending) go to the granted keys in (request, position) order; each new
 // block carries the metadata OnCacheFullBlocks attached plus any in-step
-// touches.  Each claim's owning position then clears its claim-map slot (no
-// other thread reads it here), and each request's first position commits its
-// OnRequest / RecordSuccessfulAdmission history update.
+// touches.  An allocated id that is still resident is a victim (every victim
+// is allocated again in its step): its old content leaves the pool first, in
+// the same thread (Alg. 2 Evict: table entry and record), so no other thread
+// ever sees the block between its two contents.  Each claim's owning position
+// then clears its claim-map slot (no other thread reads it here), and each
+// request's first position commits its OnRequest / RecordSuccessfulAdmission
+// history update.
 __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
@@ -2151,8 +2137,8 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
   const int64_t pos = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
   if (pos == 0) c->hist_live += c->hist_new;
   PosRef r;
-  bool placed = false;
-  uint32_t g = 0;
+  bool placed = false, evicted = false;
+  uint32_t g = 0, gold = 0;
   if (pos_ref(s, pos, &r)) {
     const uint32_t i = r.i;
     const int si = s.rq_s[i], a = s.rq_a[i];
@@ -2171,16 +2157,22 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
       if (b >= (uint64_t)s.N) {
         c->internal_error = 1;  // the allocated set is short: never expected
       } else {
-        const ClaimEntry e = s.claims[s.pos_claim[pos]];
+        const ClaimEntry e = s.claims[slot];
         const uint64_t key = s.pos_key[pos];
+        if (s.blk_flags[b] & 1) {  // a victim: evict its old content
+          gold = drop_block(s, b, false);
+          evicted = true;
+        }
         s.blk_key[b] = key;
         s.blk_group[b] = (uint16_t)g;
         s.blk_contract[b] = (uint8_t)s.rq_cid[i];
         s.blk_prefix[b] = s.rq_p[i];
         s.blk_klass[b] = e.promo != kNone ? (uint8_t)kReuse : s.rq_knew[i];
-        const uint32_t toucher = e.last ? e.last - 1 : i;  // the last request that touched it
-        s.blk_stamp[b] = make_stamp(c->stamp_base, s.rq_pbase[toucher], s.rq_n[toucher], r.m);
-        if (s.lg_on) s.lg_slot[s.rq_pbase[toucher] + (s.rq_n[toucher] - 1 - r.m)] = b;
+        // the latest request that touched it: an in-step toucher's stamp, or
+        // the owner's own
+        const uint64_t st = tmax<uint64_t>(e.stamp, make_stamp(c->stamp_base, s.rq_pbase[i], s.rq_n[i], r.m));
+        s.blk_stamp[b] = st;
+        if (s.lg_on) s.lg_slot[st - c->stamp_base] = b;
         s.blk_acc[b] = e.tcnt;
         s.blk_freq[b] = e.tcnt;
         s.blk_flags[b] = 1;
@@ -2188,14 +2180,12 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
         placed = true;  // its resident bit was set with the allocated set
       }
     }
-    if (slot != kNone) {
-      ClaimEntry z{};
-      z.key = 0; z.minreq = kNone; z.last = 0; z.tcnt = 0; z.promo = kNone; z.pad0 = 0; z.pad1 = 0;
-      s.claims[slot] = z;
-    }
+    if (slot != kNone) s.claims[slot] = empty_claim();
   }
-  agg_stat(s, g, PS_STAT_RESIDENT_BLOCKS, placed ? 1 : 0, placed);
-  const int k = __popc(__ballot_sync(kFull, placed));
+  agg_stat(s, gold, PS_STAT_EVICTED_BLOCKS, 1, evicted);
+  agg_stat(s, gold, PS_STAT_RESIDENT_BLOCKS, -1, evicted);
+  agg_stat(s, g, PS_STAT_RESIDENT_BLOCKS, 1, placed);
+  const int k = __popc(__ballot_sync(kFull, placed)) - __popc(__ballot_sync(kFull, evicted));
   if (lane_id() == 0 && k) atomic_add_i64(&c->n_resident, k);
 }
 
@@ -2422,7 +2412,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(launch_k(k_bm_count, nchunks, kBmChunk, 0, st, s));
   PS_LAUNCH(launch_k(k_bm_write, nchunks, kBmChunk, 0, st, s));
   mark(8);
-  PS_LAUNCH(launch_k(k_evict, pgrid, kThreads, 0, st, s));
+  // (evictions happen in k_insert: every victim is allocated again in its step)
   mark(9);
   PS_LAUNCH(launch_k(k_insert, pgrid, kThreads, 0, st, s));
   if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));

@@ -56,11 +56,17 @@ __device__ uint32_t ghost_find(const DevState& s, uint64_t key, uint32_t g) {
   const uint32_t mask = (1u << s.gh_nbuckets_log2) - 1;
   uint32_t b = ghost_home(s, key, g);
   for (uint32_t it = 0; it <= mask; ++it) {
-    for (int w = 0; w < kTableWays; ++w) {
-      const TableEntry& e = s.ghost_map[(size_t)b * kTableWays + w];
-      if (e.blk != kNone && e.key == key && e.grp == g) return b * kTableWays + w;
-    }
-    if (s.ghost_ovf[b] == 0) return kNone;
+    // the bucket's ways and overflow count in one round of loads, then the
+    // compares (a return among the loads would serialize them)
+    TableEntry e[kTableWays];
+#pragma unroll
+    for (int w = 0; w < kTableWays; ++w) e[w] = s.ghost_map[(size_t)b * kTableWays + w];
+    const uint32_t ovf = s.ghost_ovf[b];
+    uint32_t hit = kNone;
+#pragma unroll
+    for (int w = kTableWays - 1; w >= 0; --w)
+      if (e[w].blk != kNone && e[w].key == key && e[w].grp == g) hit = b * kTableWays + w;
+    if (hit != kNone || ovf == 0) return hit;
     b = (b + 1) & mask;
   }
   return kNone;
