@@ -49,7 +49,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--prefill", type=int, default=6, help="untimed steps that fill the empty pool")
     ap.add_argument("--impl", choices=("own", "reference"), default="own")
-    ap.add_argument("--policy", choices=("prefixshield", "lru", "staticquota"), default="prefixshield")
+    ap.add_argument("--policy", choices=("prefixshield", "lru", "s3fifo", "staticquota"), default="prefixshield")
     ap.add_argument("--seed", type=int, default=1)
     ap.add_argument("--cpu-steps", type=int, default=3, help="timed oracle steps for cpu_baseline")
     ap.add_argument("--no-e2e", action="store_true")
@@ -166,10 +166,10 @@ def make_steps(seed, n):
     return wl.spec, list(wl.steps(n))
 
 
-def run_oracle_steps(spec, steps, timed_from):
+def run_oracle_steps(spec, steps, timed_from, policy="prefixshield"):
     """Oracle over steps; returns (seconds over steps[timed_from:], requests timed)."""
     import oracle as O
-    oc = O.OracleCache(spec.capacity_blocks, spec.block_size, spec.num_groups, "prefixshield",
+    oc = O.OracleCache(spec.capacity_blocks, spec.block_size, spec.num_groups, policy,
                        O.Params(rho=spec.rho, beta=spec.beta, history_capacity=1 << 20,
                                 contract_of_group=list(spec.contract_of_group) if spec.contract_of_group else None))
     t_sum, reqs = 0.0, 0
@@ -234,13 +234,13 @@ def run_reference(args, ws, rank):
         return
     n = args.prefill + args.warmup + args.steps
     spec, steps = make_steps(args.seed, n)
-    t, reqs = run_oracle_steps(spec, steps, args.prefill + args.warmup)
+    t, reqs = run_oracle_steps(spec, steps, args.prefill + args.warmup, args.policy)
     value = reqs / t
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / max(1, args.steps),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "policy": "prefixshield", "prefill_steps": args.prefill},
+        "config": {"workload": WORKLOAD, "policy": args.policy, "prefill_steps": args.prefill},
         "cpu_baseline": {"value": value, "unit": "requests/s", "cores": 1, "kind": "oracle",
                          "sample": f"{args.steps} steps of the scale trace after {args.prefill + args.warmup} "
                                    f"untimed ones ({reqs} requests)"},
@@ -370,16 +370,25 @@ def run_own(args, ws, rank, local):
 
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, cache, steps, dsteps, flush, R, ws)
+        # the API's own speed: no flush in the timed loop (every step streams
+        # its own inputs in and touches state far larger than the L2); then
+        # the same loop with the 256 MiB flush before each step, for comparison
+        e2e = run_e2e(args, cache, steps, dsteps, None, R, ws)
+        flushed = run_e2e(args, cache, steps, dsteps, flush, R, ws)
         # the whole job: every rank's requests over the slowest rank's time
         reqs_all = sum_over_ranks(ws, e2e.pop("_requests"))
         t_e2e = max_over_ranks(ws, e2e.pop("_seconds"))
         e2e["value"] = reqs_all / t_e2e
         e2e["ms_per_step"] = 1e3 * t_e2e / args.steps
+        t_fl = max_over_ranks(ws, flushed.pop("_seconds"))
+        e2e["l2_flushed"] = {"value": sum_over_ranks(ws, flushed.pop("_requests")) / t_fl,
+                             "ms_per_step": 1e3 * t_fl / args.steps,
+                             "note": "the same loop with a 256 MiB L2 flush enqueued before every step"}
+        e2e["l2"] = "not flushed in the timed loop (each step streams its inputs from the host)"
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         n_cpu = args.prefill + args.cpu_steps
-        t_cpu, r_cpu = run_oracle_steps(spec, steps[:n_cpu], args.prefill)
+        t_cpu, r_cpu = run_oracle_steps(spec, steps[:n_cpu], args.prefill, args.policy)
         cpu = {"value": r_cpu / t_cpu, "unit": "requests/s", "cores": 1, "kind": "oracle",
                "sample": f"{args.cpu_steps} steps of the scale trace ({r_cpu} requests) after {args.prefill} "
                          f"untimed fill steps, single-threaded C++ oracle"}
@@ -437,7 +446,8 @@ def run_e2e(args, cache, steps, dsteps, flush, R, ws=1):
     # ps_step_host_async on staging slots 0 and 1: step k+1's input copy (on
     # the library's copy stream) overlaps step k's work; each step's outputs
     # are written into page-locked host buffers and waited for before its
-    # slot is reused.  The L2 flush is enqueued before every step's work.
+    # slot is reused.  With 'flush', a 256 MiB L2 flush is enqueued before
+    # every step's work.
     outs = [B.host_outputs(R, cache.max_blocks, cache.G, pinned=True) for _ in range(2)]
     h2d = d2h = 0
     done_at = []
@@ -457,7 +467,8 @@ def run_e2e(args, cache, steps, dsteps, flush, R, ws=1):
     barrier(ws)
     t0 = time.perf_counter()
     for k, (now, g, o, t) in enumerate(host):
-        flush.zero_()
+        if flush is not None:
+            flush.zero_()
         rc = cache.step_host_async(k % 2, now, g, o, t, outs[k % 2])
         if rc != 0:
             raise RuntimeError(f"ps_step_host_async rc={rc}")

@@ -871,14 +871,18 @@ __global__ void k_instep_fin(DevState s) {
 
 // ===========================================================================
 // Stages 3-4: metering (Eq. 1-3, OnCacheFullBlocks of Alg. 1), in request
-// order, one CTA per group.  Block-wide exclusive scans give each request the
-// charges of the earlier requests of its group per contract, hence
+// order, one CTA per group.  The CTA compacts its group's requests of each
+// tile of kMeterTile requests into shared memory (in request order), then
+// works on the members only: block-wide exclusive scans give each member the
+// charges of the group's earlier requests per contract, hence
 //   D_g before the request (the gate of OnTouch, Eq. 4),
 //   B_{g,c} after the request's own charge (the class of its new blocks).
 // q_r >= 1 and "(g,p) was admitted" come from the history entry as it stood at
 // the start of the step and the first request of the step that referenced /
 // admitted it.  Also writes the group's statistics, balances and debts.
-__global__ void __launch_bounds__(512) k_meter(DevState s0) {
+constexpr int kMeterThreads = 512;
+constexpr int kMeterTile = 4 * kMeterThreads;  // requests compacted per pass
+__global__ void __launch_bounds__(kMeterThreads) k_meter(DevState s0) {
   // Contract arrays are read from the parameter block: indexing the per-step
   // copy by a run-time contract would move the whole copy to local memory.
   const DevState s = with_args(s0);
@@ -890,6 +894,7 @@ __global__ void __launch_bounds__(512) k_meter(DevState s0) {
   const uint64_t step = c->step;
   __shared__ int64_t B0[PS_MAX_CONTRACTS];
   __shared__ unsigned long long s_st[7];  // the group's request statistics
+  __shared__ int32_t s_mem[kMeterTile];   // this tile's members, in request order
   if (threadIdx.x < C) {
     const int cc = threadIdx.x;
     B0[cc] = refill(s.ledger[g * C + cc], s0.beta[cc], s0.rho[cc], s.now - c->t_prev);
@@ -901,85 +906,77 @@ __global__ void __launch_bounds__(512) k_meter(DevState s0) {
   for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) carry[cc] = 0;
   int64_t st_req = 0, st_ptok = 0, st_full = 0, st_hit = 0, st_inst = 0, st_adm = 0, st_ungr = 0;
   const int R = s.R;
-  // each thread takes kPer consecutive requests, so one block scan per
-  // contract places kPer * blockDim requests
-  constexpr int kPer = 4;
-  for (int base = 0; base < R; base += (int)blockDim.x * kPer) {
-    const int i0 = base + (int)threadIdx.x * kPer;
-    bool mem[kPer];
-    int n[kPer], a[kPer], cid[kPer];
+  for (int base = 0; base < R; base += kMeterTile) {
+    // members of this tile: four consecutive requests a thread, compacted by
+    // a block scan of their counts (the order is request order)
+    const int i0 = base + 4 * (int)threadIdx.x;
+    int32_t gg[4] = {-1, -1, -1, -1};
+    if (i0 + 3 < R && (reinterpret_cast<uintptr_t>(s.in_group + i0) & 15) == 0) {
+      const int4 v = *reinterpret_cast<const int4*>(s.in_group + i0);
+      gg[0] = v.x; gg[1] = v.y; gg[2] = v.z; gg[3] = v.w;
+    } else {
 #pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      mem[u] = i < R && s.in_group[i] == g;
-      n[u] = a[u] = cid[u] = 0;
-      if (mem[u]) { n[u] = s.rq_n[i]; a[u] = s.rq_a[i]; cid[u] = s.rq_cid[i]; }
+      for (int u = 0; u < 4; ++u)
+        if (i0 + u < R) gg[u] = s.in_group[i0 + u];
     }
-    // charges of this group's earlier requests, per contract: the thread's
-    // base from a block scan, then its own requests in order
-    int64_t S[PS_MAX_CONTRACTS];
+    int cnt = 0;
 #pragma unroll
-    for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
-      S[cc] = 0;
-      if (cc < C) {
-        int64_t mine = 0;
+    for (int u = 0; u < 4; ++u) cnt += gg[u] == g;
+    int nmem;
+    int at = block_excl_scan(cnt, &nmem);
 #pragma unroll
-        for (int u = 0; u < kPer; ++u) mine += (mem[u] && n[u] > 0 && cid[u] == cc) ? a[u] : 0;
-        int64_t tot;
-        const int64_t ex = block_excl_scan<int64_t>(mine, &tot);
-        S[cc] = carry[cc] + ex;
-        carry[cc] += tot;
+    for (int u = 0; u < 4; ++u)
+      if (gg[u] == g) s_mem[at++] = i0 + u;
+    __syncthreads();
+    for (int k0 = 0; k0 < nmem; k0 += kMeterThreads) {
+      const int k = k0 + (int)threadIdx.x;
+      const bool mem = k < nmem;
+      const int i = mem ? s_mem[k] : 0;
+      int n = 0, a = 0, cid = 0, rh = 0, re = 0, rs = 0;
+      uint32_t hs = kNone;
+      int64_t ptok = 0;
+      if (mem) {
+        n = s.rq_n[i]; a = s.rq_a[i]; cid = s.rq_cid[i]; hs = s.rq_hs[i];
+        rh = s.rq_h[i]; re = s.rq_e[i]; rs = s.rq_s[i];
+        ptok = s.in_offsets[i + 1] - s.in_offsets[i];
       }
-    }
-    // the requests' other inputs, loaded before any store below
-    HistEntry he[kPer];
-    int rh[kPer], re[kPer], rs[kPer];
-    int64_t ptok[kPer];
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      he[u] = HistEntry{};
-      rh[u] = re[u] = rs[u] = 0;
-      ptok[u] = 0;
-      if (mem[u]) {
-        const uint32_t hs = s.rq_hs[i];
-        if (n[u] > 0 && hs != kNone) he[u] = s.hist[hs];
-        rh[u] = s.rq_h[i];
-        re[u] = s.rq_e[i];
-        rs[u] = s.rq_s[i];
-        ptok[u] = s.in_offsets[i + 1] - s.in_offsets[i];
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kPer; ++u) {
-      const int i = i0 + u;
-      const bool pol = mem[u] && n[u] > 0;
-      // the raw debt before this request's charge (Eq. 3) and its balance after
-      int64_t d = 0, b_after = 0;
+      const bool pol = mem && n > 0;
+      HistEntry he{};
+      if (pol && hs != kNone) he = s.hist[hs];
+      // charges of this group's earlier requests, per contract
+      int64_t S[PS_MAX_CONTRACTS];
 #pragma unroll
       for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
+        S[cc] = 0;
         if (cc < C) {
-          d += tmax<int64_t>(0, -(B0[cc] - S[cc] * unit));
-          if (cid[u] == cc) b_after = B0[cc] - (S[cc] + a[u]) * unit;
+          int64_t tot;
+          const int64_t ex = block_excl_scan<int64_t>((pol && cid == cc) ? a : 0, &tot);
+          S[cc] = carry[cc] + ex;
+          carry[cc] += tot;
         }
       }
       if (pol) {
+        // the raw debt before this request's charge (Eq. 3) and its balance after
+        int64_t d = 0, b_after = 0;
+#pragma unroll
+        for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
+          if (cc < C) {
+            d += tmax<int64_t>(0, -(B0[cc] - S[cc] * unit));
+            if (cid == cc) b_after = B0[cc] - (S[cc] + a) * unit;
+          }
+        }
         const bool gate = (s.flags & PS_FLAG_NO_DEBT_GATE) || d <= s.eps;
-        const uint32_t refadm = he[u].refadm;
-        const bool q_ge1 = (refadm & 0x7FFFFFFFu) >= 1 || tag_req(he[u].ftag, step) < (uint32_t)i;
-        const bool adm_before = (refadm >> 31) || tag_req(he[u].atag, step) < (uint32_t)i;
+        const uint32_t refadm = he.refadm;
+        const bool q_ge1 = (refadm & 0x7FFFFFFFu) >= 1 || tag_req(he.ftag, step) < (uint32_t)i;
+        const bool adm_before = (refadm >> 31) || tag_req(he.atag, step) < (uint32_t)i;
         const bool proven = q_ge1 && adm_before;
         s.rq_flags[i] = (uint8_t)((proven ? 1 : 0) | (gate ? 2 : 0));
         s.rq_knew[i] = (uint8_t)((b_after < -s.eps || !adm_before) ? kProb : kNormal);
-        const int h = rh[u], e = re[u];
-        st_full += n[u]; st_hit += h + e; st_inst += e; st_adm += a[u]; st_ungr += (n[u] - rs[u]) - a[u];
-        // this request's own charge, for the requests after it in the thread
-#pragma unroll
-        for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc)
-          if (cc < C && cid[u] == cc) S[cc] += a[u];
+        st_full += n; st_hit += rh + re; st_inst += re; st_adm += a; st_ungr += (n - rs) - a;
       }
-      if (mem[u]) { st_req += 1; st_ptok += ptok[u]; }
+      if (mem) { st_req += 1; st_ptok += ptok; }
     }
+    __syncthreads();  // s_mem is rewritten by the next tile
   }
   {
     const int64_t v[7] = {st_req, st_ptok, st_full, st_hit, st_inst, st_adm, st_ungr};
@@ -2064,6 +2061,10 @@ __global__ void __launch_bounds__(kBmChunk) k_bm_count(DevState s) {
     s.bm_chunk_cnt[2 * nchunks + blockIdx.x] = ti;
   }
 }
+// Counts are packed into one 64-bit word (three 21-bit fields: a chunk holds
+// at most 8192 ids of each kind), so one block scan carries all three.
+__device__ __forceinline__ uint64_t pack3(uint64_t a, uint64_t b, uint64_t c) { return a | b << 21 | c << 42; }
+__device__ __forceinline__ int64_t field3(uint64_t v, int k) { return (int64_t)((v >> (21 * k)) & 0x1FFFFF); }
 __global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
@@ -2072,47 +2073,50 @@ __global__ void __launch_bounds__(kBmChunk) k_bm_write(DevState s) {
   const int nchunks = gridDim.x;
   const bool in = w < s.nwords;
   const int64_t ftake = c->ftake;
-  // earlier chunks: free, evicted and invalidated ids
+  // earlier chunks' free, evicted and invalidated ids (summed field by field)
   int64_t fb = 0, vb = 0, ib = 0;
   for (int j = threadIdx.x; j < (int)blockIdx.x; j += blockDim.x) {
     fb += s.bm_chunk_cnt[0 * nchunks + j];
     vb += s.bm_chunk_cnt[1 * nchunks + j];
     ib += s.bm_chunk_cnt[2 * nchunks + j];
   }
-  fb = block_sum(fb);
-  vb = block_sum(vb);
-  ib = block_sum(ib);
+  {
+    __shared__ int64_t s_before[3][kBmChunk / 32];
+    fb = warp_sum(fb); vb = warp_sum(vb); ib = warp_sum(ib);
+    if (lane_id() == 0) { s_before[0][threadIdx.x >> 5] = fb; s_before[1][threadIdx.x >> 5] = vb; s_before[2][threadIdx.x >> 5] = ib; }
+    __syncthreads();
+    fb = vb = ib = 0;
+#pragma unroll
+    for (int q = 0; q < kBmChunk / 32; ++q) { fb += s_before[0][q]; vb += s_before[1][q]; ib += s_before[2][q]; }
+  }
   const int64_t take_here = tmin(ftake, fb + s.bm_chunk_cnt[blockIdx.x]) - tmin(ftake, fb);
   // this word's taken free ids: the chunk's lowest take_here free ids
-  uint32_t f = (in && take_here > 0) ? free_word(s, w) : 0u;
-  int64_t ftot;
-  int64_t fl = block_excl_scan<int64_t>(__popc(f), &ftot);
-  uint32_t taken = 0;
-  while (f && fl < take_here) {
-    const uint32_t lsb = f & (0u - f);
-    taken |= lsb;
-    f ^= lsb;
-    ++fl;
-  }
+  const uint32_t f = (in && take_here > 0) ? free_word(s, w) : 0u;
   const uint32_t vic = in ? s.bm_victim[w] : 0u, inv = in ? s.bm_inval[w] : 0u;
+  uint64_t tot1;
+  const uint64_t ex1 = block_excl_scan<uint64_t>(pack3(__popc(f), __popc(vic), __popc(inv)), &tot1);
+  const int64_t fl = field3(ex1, 0);
+  const int64_t want = tmin<int64_t>(tmax<int64_t>(take_here - fl, 0), __popc(f));
+  // the lowest 'want' set bits of f: everything below the want-th set bit, and it
+  const uint32_t taken = want == 0 ? 0u : (want >= 32 ? f : (f & ((2u << __fns(f, 0, (int)want)) - 1u)));
   const uint32_t alloc = taken | vic;
   if (in) s.res_bits[w] |= alloc;  // every allocated id is resident after the step
+  uint64_t tot2;
+  const uint64_t ex2 = block_excl_scan<uint64_t>((uint64_t)__popc(alloc), &tot2);
   const uint32_t bitsk[3] = {alloc, vic, inv};
-  const int64_t basek[3] = {vb + tmin(ftake, fb), vb, ib};
+  const int64_t basek[3] = {vb + tmin(ftake, fb) + (int64_t)ex2, vb + field3(ex1, 1), ib + field3(ex1, 2)};
   int32_t* outs[3] = {s.out.admitted_ids, s.out.evicted_ids, s.out.invalidated_ids};
 #pragma unroll
   for (int k = 0; k < 3; ++k) {
-    int64_t tot;
-    const int64_t ex = block_excl_scan<int64_t>(__popc(bitsk[k]), &tot);
-    int64_t o = basek[k] + ex;
+    int64_t o = basek[k];
     for (uint32_t b = bitsk[k]; b; b &= b - 1) {
       if (o < s.max_blocks) outs[k][o] = (int32_t)(w * 32 + __ffs(b) - 1);
       ++o;
     }
-    if (blockIdx.x == nchunks - 1 && threadIdx.x == 0) {
-      if (k == 0) c->n_alloc = basek[0] + tot;
-      if (k == 1) c->n_evicted = basek[1] + tot;
-    }
+  }
+  if (blockIdx.x == nchunks - 1 && threadIdx.x == 0) {
+    c->n_alloc = vb + tmin(ftake, fb) + (int64_t)tot2;
+    c->n_evicted = vb + field3(tot1, 1);
   }
   if (in) {
     s.bm_victim[w] = 0;
