@@ -85,8 +85,8 @@ def algorithmic_bytes(T, R, H, A, E, Ag, V):
 
 
 def hash_lookup_traffic():
-    """DRAM bytes per launch of the hash_lookup stage from the committed ncu
-    capture, or None once its kernels' sources differ from the captured ones."""
+    """DRAM bytes per launch of k_hash_lookup from the committed ncu capture,
+    or None once the kernel's sources differ from the captured ones."""
     import hashlib
     try:
         with open(os.path.join(ROOT, "profiles", "hash_lookup_scale_traffic.json")) as f:
@@ -411,7 +411,8 @@ def run_own(args, ws, rank, local):
         "step_roofline": {"bound": "hbm", "achieved": step_gbs, "peak": peak, "unit": "GB/s",
                           "frac": step_gbs / peak, "algorithmic_bytes_per_step": alg / args.steps,
                           "peak_kind": peak_kind},
-        "roofline": {"bound": "hbm", "kernel": "hash_lookup stage: k_hash_lane + k_keys_lookup + k_pin_claim", "achieved": hl_gbs, "peak": peak, "unit": "GB/s",
+        "roofline": {"bound": "hbm", "kernel": "k_hash_lookup (hashing, lookup, pins and claims: one launch a step)",
+                     "achieved": hl_gbs, "peak": peak, "unit": "GB/s",
                      "frac": hl_gbs / peak, "traffic": hash_lookup_traffic(), "bytes_per_launch": hl_bytes,
                      "ms_per_launch": hl_ms, "peak_kind": peak_kind},
         "stages_ms_per_step": {n: round(float(v) / args.steps, 4) for n, v in zip(STAGES, stage_ms)},

@@ -642,7 +642,7 @@ __global__ void __launch_bounds__(256, kHashCtasPerSm) k_hash_lookup(DevState s,
 
 // A step whose new (group, prefix) entries would overflow the history map
 // fails as a whole, leaving the pool as it was (Alg. 1's hooks change state
-// only for a request that goes ahead).  k_pin_claim has written three things
+// only for a request that goes ahead).  k_hash_lookup has written three things
 // by then, undone here thread by thread over the same positions and requests:
 //  - pin tags of the cached prefix: set to a tag no step compares against
 //    (the previous step's), so the retried step pins them afresh;
