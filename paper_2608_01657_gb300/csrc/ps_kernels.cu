@@ -17,9 +17,9 @@
 
 namespace ps {
 
-constexpr int kRadixSmemRows = 48;  // radix rows counted in shared memory (48 KB)
 constexpr int kFinCap = 8192;  // split lists up to this size are finished by one CTA in shared memory
 constexpr int kFinRows = 32;   // rows k_list_finish counts at once (32 KB)
+constexpr int kFinCountCap = 512;  // split lists up to this size are ranked by counting
 
 // 128-bit compare-and-swap (sm_90+): installs the (p, group) identity of a
 // history entry atomically, so two requests of one (group, prefix) that race
@@ -1328,7 +1328,6 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   __shared__ int64_t sP[PS_MAX_GROUPS], sD[PS_MAX_GROUPS], sQ[PS_MAX_GROUPS];
   __shared__ uint64_t sRcp[PS_MAX_GROUPS];  // floor((2^64 - 1) / d) for the division below
   __shared__ int64_t s_pmax;
-  __shared__ int s_best;
   const int G = s.G;
   const int64_t eps = s.eps;
   const bool seg = !(s.flags & PS_FLAG_NO_SEGMENTATION);
@@ -1382,7 +1381,7 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
     }
     if (threadIdx.x == 0) {
       c->m_fb = m - E; c->sel_ntie = 0; c->sel_k = 0; c->lst_n = 0;
-      if (has_cond && m > E) cudaGraphSetConditional(fb_cond, 1);  // the fallback phase runs
+      if (has_cond && m > E) cudaGraphSetConditional(fb_cond, 1);  // the queues' fallback phase runs
     }
     return;
   }
@@ -1434,9 +1433,10 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
       if (J < 0) {
         hi = lo;
       } else {
-        lo = thr(J);
-        hi = J + 1 < T ? thr(J + 1) - 1 : hi;
-        if (hi < lo) hi = lo;
+        // both ends from this round's lo (thr reads lo and hi by reference)
+        const int64_t nlo = thr(J), nhi = J + 1 < T ? thr(J + 1) - 1 : hi;
+        lo = nlo;
+        hi = nhi < nlo ? nlo : nhi;
       }
     }
   }
@@ -1445,7 +1445,8 @@ __global__ void __launch_bounds__(1024) k_waterfill(DevState s, cudaGraphConditi
   for (int g = threadIdx.x; g < G; g += blockDim.x) {
     const int64_t P = sP[g], d = sD[g], q = sQ[g];
     const int64_t xa = items_gt(g, tau);
-    const bool tied = d > 0 && P >= tau && (P - tau) % d == 0 && (P - tau) / d < q;
+    const uint64_t qt = (d > 0 && P >= tau) ? div_d(g, (uint64_t)(P - tau)) : 0;
+    const bool tied = d > 0 && P >= tau && qt * (uint64_t)d == (uint64_t)(P - tau) && (int64_t)qt < q;
     above += xa;
     ntie += tied;
     SelSeg z = s.sel[g];
@@ -1652,124 +1653,10 @@ __global__ void __launch_bounds__(32) k_wide_resolve(DevState s, int single) {
   }
 }
 
-// One digit for every segment that still has one: over the whole candidate
-// array (from_list = 0) or over the split list (from_list = 1).
-__global__ void __launch_bounds__(256) k_digit_pass(DevState s, int single, int fallback, int from_list) {
-  s = with_args(s);
-  extern __shared__ uint32_t shist[];
-  __shared__ int16_t row_of[PS_MAX_GROUPS];
-  __shared__ int16_t seg_of_row[PS_MAX_GROUPS];
-  __shared__ int s_nrows;
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK || c->mvict == 0) return;
-  const int nseg = single ? 1 : s.G;
-  if (single && !s.sel[0].active) return;
-  if (from_list && c->lst_n <= kFinCap) return;  // k_list_finish takes short lists whole
-  // rows for the segments that still count (parallel flags, scanned)
-  {
-    int k = 0;
-    for (int base = 0; base < nseg; base += blockDim.x) {
-      const int g = base + threadIdx.x;
-      bool counts = false;
-      if (g < nseg) {
-        const SelSeg ss = from_list ? list_view(s.sel[g]) : s.sel[g];
-        counts = ss.active && next_shift(ss.mask) >= 0;
-      }
-      int tot;
-      const int ex = block_excl_scan((int)counts, &tot);
-      if (g < nseg) row_of[g] = counts ? (int16_t)(k + ex) : (int16_t)-1;
-      if (counts) seg_of_row[k + ex] = (int16_t)g;
-      k += tot;
-    }
-    if (threadIdx.x == 0) s_nrows = k;
-    __syncthreads();
-  }
-  const int nrows = s_nrows;
-  if (nrows == 0) return;  // uniform across CTAs: nothing counts, nothing to resolve
-  const bool use_smem = nrows <= kRadixSmemRows;
-  if (use_smem)
-    for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x) shist[k] = 0;
-  __syncthreads();
-  const int64_t n = from_list ? c->lst_n : s.N;
-  for (int64_t e0 = blockIdx.x * (int64_t)blockDim.x; e0 < n; e0 += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t e = e0 + threadIdx.x;
-    bool act = false;
-    uint32_t idx = 0;
-    if (e < n) {
-      uint64_t key;
-      int seg;
-      bool ok;
-      if (from_list) {
-        key = s.lst_key[e];
-        seg = s.lst_seg[e];
-        ok = true;
-      } else {
-        key = s.csk[e];
-        seg = single ? 0 : s.blk_group[e];  // issued with the key load
-        ok = key != ~0ull && !(fallback && ((s.bm_victim[e >> 5] >> (e & 31)) & 1));
-      }
-      if (ok) {
-        const int row = row_of[seg];
-        if (row >= 0) {
-          const SelSeg ss = from_list ? list_view(s.sel[seg]) : s.sel[seg];
-          if ((key & ss.mask) == ss.prefix) {
-            act = true;
-            const int sh = next_shift(ss.mask);
-            const uint32_t digit = (uint32_t)((key >> sh) & (kRadixBins - 1));
-            idx = use_smem ? (uint32_t)row * kRadixBins + digit : (uint32_t)seg * kRadixBins + digit;
-          }
-        }
-      }
-    }
-    agg_inc(use_smem ? shist : s.hist_bins, idx, act);
-  }
-  __syncthreads();
-  if (use_smem)
-    for (int k = threadIdx.x; k < nrows * kRadixBins; k += blockDim.x)
-      if (shist[k]) atomicAdd(s.hist_bins + (size_t)seg_of_row[k / kRadixBins] * kRadixBins + (k % kRadixBins), shist[k]);
-  __shared__ bool last;
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) last = atomicAdd(&c->ticket, 1u) == gridDim.x - 1;
-  __syncthreads();
-  if (!last) return;
-  __threadfence();
-  const int warp = threadIdx.x >> 5, lane = lane_id();
-  for (int r = warp; r < nrows; r += blockDim.x >> 5) {
-    const int seg = seg_of_row[r];
-    SelSeg ss = from_list ? list_view(s.sel[seg]) : s.sel[seg];
-    const int sh = next_shift(ss.mask);
-    uint32_t* row = s.hist_bins + (size_t)seg * kRadixBins;
-    uint32_t v[kRadixBins / 32];
-    uint32_t sum = 0;
-#pragma unroll
-    for (int j = 0; j < kRadixBins / 32; ++j) { v[j] = ldcg_u32(row + lane * (kRadixBins / 32) + j); sum += v[j]; }
-    const uint32_t incl = warp_incl_scan(sum);
-    const uint32_t excl = incl - sum;
-    const bool here = (uint64_t)excl < (uint64_t)ss.rank && (uint64_t)ss.rank <= (uint64_t)incl;
-    if (here) {
-      uint32_t run = excl;
-      int d = 0;
-      for (int j = 0; j < kRadixBins / 32; ++j) {
-        if ((uint64_t)ss.rank <= (uint64_t)(run + v[j])) { d = lane * (kRadixBins / 32) + j; break; }
-        run += v[j];
-      }
-      ss.prefix |= (uint64_t)d << sh;
-      ss.mask |= (uint64_t)(kRadixBins - 1) << sh;
-      ss.rank -= run;
-      s.sel[seg] = ss;
-    }
-#pragma unroll
-    for (int j = 0; j < kRadixBins / 32; ++j) row[lane * (kRadixBins / 32) + j] = 0;
-  }
-  if (threadIdx.x == 0) c->ticket = 0;
-}
-
 // Split: candidates below their segment's chosen bucket are victims; the
 // bucket's members go to the list for the remaining digits, with the list's
 // key range per segment.
-__global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallback, cudaGraphConditionalHandle long_cond,
-                                                int has_cond) {
+__global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallback) {
   s = with_args(s);
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
@@ -1845,27 +1732,16 @@ __global__ void __launch_bounds__(256) k_split(DevState s, int single, int fallb
     }
   }
   if (lane_id() == 0 && marked) atomic_add_i64(&c->n_victims_marked, marked);
-  if (!has_cond) return;
-  // the last CTA to finish knows the list's length: the multi-CTA list
-  // passes run only for a long list
-  __shared__ bool last;
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) last = atomicAdd(&c->ticket, 1u) == gridDim.x - 1;
-  __syncthreads();
-  if (last && threadIdx.x == 0) {
-    __threadfence();
-    c->ticket = 0;
-    if (ldcg_u64(reinterpret_cast<const uint64_t*>(&c->lst_n)) > (uint64_t)kFinCap) cudaGraphSetConditional(long_cond, 1);
-  }
 }
 
-// The rest of a select on one CTA.  A short split list (at most kFinCap
-// members; long_list = 0) is staged in shared memory with every segment's
-// state, and every remaining digit, Eq. 7's tie rule and the marking of the
-// list's victims run there.  A longer list (long_list = 1) has had all its
-// digits located by the multi-CTA list passes; here it gets only the tie
-// rule, and k_mark_list marks it.
+// The rest of a select on one CTA, with every segment's state in shared
+// memory.  A split list of at most kFinCap members is staged in shared memory
+// too; a longer one (rare: a boundary bucket of the first digit holding many
+// candidates) is read from global memory in each round.  The segments'
+// thresholds come from ranking by counting (lists of at most kFinCountCap
+// members) or from the remaining radix digits, one round per digit; then
+// Eq. 7's tie rule, then the list's victims.  One launch for every list
+// length keeps the step graph free of conditional nodes here.
 struct FinSeg {
   uint64_t prefix, mask;
   int64_t rank;
@@ -1874,7 +1750,7 @@ struct FinSeg {
 constexpr size_t kFinSmem = (size_t)kFinCap * 8 + (size_t)kFinCap * 2 + (size_t)kFinRows * kRadixBins * 4 +
                             (size_t)PS_MAX_GROUPS * sizeof(FinSeg);
 
-__global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, int long_list) {
+__global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single) {
   s = with_args(s);
   extern __shared__ __align__(16) unsigned char fin_smem[];
   FinSeg* sl = reinterpret_cast<FinSeg*>(fin_smem);
@@ -1886,17 +1762,13 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, in
   __shared__ int s_nrows;
   Ctl* c = s.ctl;
   if (c->status != PS_OK || c->mvict == 0) return;
-  // the debt phase's last launch also starts the fallback's select (the
-  // groups' final take counts are known here)
-  const bool start_fb = !single && !long_list && s.policy == PS_PREFIXSHIELD;
+  // the debt phase's launch also starts the fallback's select (the groups'
+  // final take counts are known here)
+  const bool start_fb = !single && s.policy == PS_PREFIXSHIELD;
   if (single && !s.sel[0].active) return;
   const int nseg = single ? 1 : s.G;
   const int64_t n = c->lst_n;
   const bool small = n <= kFinCap;
-  if (small == (long_list != 0)) {  // the other launch's list
-    if (start_fb && (threadIdx.x >> 5) == 0) start_global_select(s, c, 1);
-    return;
-  }
   const int warp = threadIdx.x >> 5, lane = lane_id();
   for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
     const SelSeg v = list_view(s.sel[g]);
@@ -1905,7 +1777,30 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, in
   if (small)
     for (int64_t e = threadIdx.x; e < n; e += blockDim.x) { lkey[e] = s.lst_key[e]; lseg[e] = s.lst_seg[e]; }
   __syncthreads();
-  for (int iter = 0; small && iter < 8; ++iter) {  // at most 8 digits in a 64-bit key
+  auto key_at = [&](int64_t e) -> uint64_t { return small ? lkey[e] : ldcg_u64(s.lst_key + e); };
+  auto seg_at = [&](int64_t e) -> int { return small ? (int)lseg[e] : (int)s.lst_seg[e]; };
+  // A short list (the usual case): a segment's threshold key is its member
+  // whose rank among the segment's list members (keys are unique) is its
+  // remaining rank - 1; each thread ranks one member by counting, so no
+  // digit rounds (and their barriers) are needed.
+  const bool by_count = small && n <= kFinCountCap;
+  if (by_count) {
+    for (int e = threadIdx.x; e < n; e += blockDim.x) {
+      const int g = lseg[e];
+      if (!sl[g].active) continue;
+      const uint64_t key = lkey[e];
+      int64_t below = 0;
+      for (int j = 0; j < n; ++j) below += (lseg[j] == g && lkey[j] < key) ? 1 : 0;
+      // one member per segment matches, and the loop reads only the
+      // segment's activity and rank, which nothing here writes
+      if (below == sl[g].rank - 1) {
+        sl[g].prefix = key;
+        sl[g].mask = ~0ull;
+      }
+    }
+    __syncthreads();
+  }
+  for (int iter = 0; !by_count && iter < 8; ++iter) {  // at most 8 digits in a 64-bit key
     {
       int k = 0;
       for (int base = 0; base < nseg; base += blockDim.x) {
@@ -1926,15 +1821,15 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, in
       const int rn = tmin(kFinRows, nrows - r0);
       for (int k = threadIdx.x; k < rn * kRadixBins; k += blockDim.x) fh[k] = 0;
       __syncthreads();
-      for (int e0 = 0; e0 < n; e0 += blockDim.x) {
-        const int e = e0 + threadIdx.x;
+      for (int64_t e0 = 0; e0 < n; e0 += blockDim.x) {
+        const int64_t e = e0 + threadIdx.x;
         bool act = false;
         uint32_t idx = 0;
         if (e < n) {
-          const int seg = lseg[e];
+          const int seg = seg_at(e);
           const int row = row_of[seg];
           if (row >= r0 && row < r0 + rn) {
-            const uint64_t key = lkey[e];
+            const uint64_t key = key_at(e);
             if ((key & sl[seg].mask) == sl[seg].prefix) {
               act = true;
               const int sh = next_shift(sl[seg].mask);
@@ -1987,47 +1882,18 @@ __global__ void __launch_bounds__(1024) k_list_finish(DevState s, int single, in
       if (sl[g].active && sl[g].incl == 2) sl[g].incl = (int32_t)fh[g];
     __syncthreads();
   }
-  if (small) {  // the list's victims: keys below (or at, if incl) the threshold
-    for (int e = threadIdx.x; e < n; e += blockDim.x) {
-      const uint64_t key = lkey[e];
-      const FinSeg& f = sl[lseg[e]];
-      if (f.active && (key < f.prefix || (f.incl && key == f.prefix))) {
-        const uint32_t b = s.lst_blk[e];
-        atomicOr(s.bm_victim + (b >> 5), 1u << (b & 31));
-      }
-    }
-  } else {  // k_mark_list marks a long list from the segments' final state
-    for (int g = threadIdx.x; g < nseg; g += blockDim.x) {
-      SelSeg v = s.sel[g];
-      v.prefix = sl[g].prefix;
-      v.mask = sl[g].mask;
-      v.rank = sl[g].rank;
-      v.incl = sl[g].incl;
-      s.sel[g] = v;
+  // the list's victims: keys below (or at, if incl) the threshold
+  for (int64_t e = threadIdx.x; e < n; e += blockDim.x) {
+    const uint64_t key = key_at(e);
+    const FinSeg& f = sl[seg_at(e)];
+    if (f.active && (key < f.prefix || (f.incl && key == f.prefix))) {
+      const uint32_t b = s.lst_blk[e];
+      atomicOr(s.bm_victim + (b >> 5), 1u << (b & 31));
     }
   }
   if (start_fb) {
     __syncthreads();  // every reader of segment 0's state is done
     if ((threadIdx.x >> 5) == 0) start_global_select(s, c, 1);
-  }
-}
-
-// Mark a long list's victims (multi-CTA): keys below (or at, if incl) their
-// segment's located threshold.
-__global__ void __launch_bounds__(256) k_mark_list(DevState s, int single) {
-  s = with_args(s);
-  Ctl* c = s.ctl;
-  if (c->status != PS_OK || c->mvict == 0) return;
-  if (single && !s.sel[0].active) return;
-  const int64_t n = c->lst_n;
-  if (n <= kFinCap) return;  // marked by k_list_finish
-  for (int64_t e = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
-    const uint64_t key = s.lst_key[e];
-    const SelSeg ss = list_view(s.sel[s.lst_seg[e]]);
-    if (ss.active && (key < ss.prefix || (ss.incl && key == ss.prefix))) {
-      const uint32_t b = s.lst_blk[e];
-      atomicOr(s.bm_victim + (b >> 5), 1u << (b & 31));
-    }
   }
 }
 
@@ -2259,7 +2125,6 @@ static int32_t launch_hash_lookup(const DevState& s, cudaStream_t st, int probe)
 
 void configure_kernels(const DevState& s) {
   (void)s;
-  cudaFuncSetAttribute(k_digit_pass, cudaFuncAttributeMaxDynamicSharedMemorySize, kRadixSmemRows * kRadixBins * 4);
   cudaFuncSetAttribute(k_list_finish, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFinSmem);
   cudaFuncSetAttribute(k_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, PS_MAX_GROUPS * kClasses * 5 * 4);
 }
@@ -2273,8 +2138,6 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   const int ngrid = grid_for(s.N, 256, 152 * 8);
   const int sgrid = grid_for(s.N, 256, 152 * 4);  // 48 KB histograms: 4 CTAs per SM
   const int cgrid = grid_for(s.N, 256, 152 * 8);
-  const int lgrid = 152;  // list passes: the split list is short
-  const int radix_smem = kRadixSmemRows * kRadixBins * 4;
   int launches = 0;
   auto mark = [&](int stage) {
     // under capture an external record becomes an event-record node of the
@@ -2293,26 +2156,36 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(2);
   PS_LAUNCH(launch_k(k_claims, prgrid, kThreads, 0, st, s));
   mark(3);
-  if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
-  PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
   // The candidates read pins and residency (final from here on) and the class
   // and stamp of unpinned blocks, which S3-S4 leave alone: under capture
   // they are counted on a side branch that runs beside the rest of S3-S4.
+  // The candidate scan writes per-step scratch only, so it forks before the
+  // grants (a step the grant then fails ignores what it wrote); the indexed
+  // queues' count applies the step's pins to persistent counts, so it waits
+  // for the grant's verdict.
   const bool fork = cap && s.policy != PS_S3FIFO;
+  const bool early = fork && !s.lg_on;
   cudaStream_t cs = st;
-  if (fork) {
-    if (cudaEventRecord(cap->fork, st) != cudaSuccess || cudaStreamWaitEvent(cap->side, cap->fork, 0) != cudaSuccess)
-      return PS_ERR_CUDA;
-    cs = cap->side;
-  }
-  const int cand_smem = (s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA ? s.G : 1) * kClasses * 5 * 4;
-  if (s.lg_on) {
-    if (launch_queue_cand(s, cs, &launches) != PS_OK) return PS_ERR_CUDA;
-  } else if (s.policy != PS_S3FIFO) {
-    // one 512-thread CTA per SM: the main branch keeps room on every SM
-    PS_LAUNCH(k_cand<<<fork ? 152 : grid_for(s.N, 1024 * 4, 152), fork ? 512 : 1024, cand_smem, cs>>>(s));
-  }
-  if (fork && cudaEventRecord(cap->join, cs) != cudaSuccess) return PS_ERR_CUDA;
+  auto launch_cand = [&]() -> int32_t {
+    if (fork) {
+      if (cudaEventRecord(cap->fork, st) != cudaSuccess || cudaStreamWaitEvent(cap->side, cap->fork, 0) != cudaSuccess)
+        return PS_ERR_CUDA;
+      cs = cap->side;
+    }
+    const int cand_smem = (s.policy == PS_PREFIXSHIELD || s.policy == PS_STATICQUOTA ? s.G : 1) * kClasses * 5 * 4;
+    if (s.lg_on) {
+      if (launch_queue_cand(s, cs, &launches) != PS_OK) return PS_ERR_CUDA;
+    } else if (s.policy != PS_S3FIFO) {
+      // one 512-thread CTA per SM: the main branch keeps room on every SM
+      PS_LAUNCH(k_cand<<<fork ? 152 : grid_for(s.N, 1024 * 4, 152), fork ? 512 : 1024, cand_smem, cs>>>(s));
+    }
+    if (fork && cudaEventRecord(cap->join, cs) != cudaSuccess) return PS_ERR_CUDA;
+    return PS_OK;
+  };
+  if (early && launch_cand() != PS_OK) return PS_ERR_CUDA;
+  if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
+  PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
+  if (!early && launch_cand() != PS_OK) return PS_ERR_CUDA;
   PS_LAUNCH(launch_k(k_instep, pgrid, kThreads, 0, st, s));
   PS_LAUNCH(launch_k(k_instep_fin, rgrid, 256, 0, st, s));
   mark(4);
@@ -2342,72 +2215,29 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
       return PS_ERR_CUDA;
     }
   }
-  // Under capture, phases that many steps skip become conditional bodies:
-  // the long-list passes of a select, and the global fallback of Alg. 2.
-  cudaGraphConditionalHandle h_fb = 0, h_long = 0;
-  bool conds = false, cond_ok = true;
-  if (cap) {
-    cudaStreamCaptureStatus cs;
-    cudaGraph_t g = nullptr;
-    // a handle that no conditional node uses can make instantiation fail:
-    // create only the ones this policy's sequence uses
-    conds = s.policy != PS_S3FIFO && !s.lg_on;
-    if (conds &&
-        !(cudaStreamGetCaptureInfo(st, &cs, nullptr, &g) == cudaSuccess && cs == cudaStreamCaptureStatusActive &&
-          cudaGraphConditionalHandleCreate(&h_long, g, 0, cudaGraphCondAssignDefault) == cudaSuccess &&
-          (s.policy != PS_PREFIXSHIELD ||
-           cudaGraphConditionalHandleCreate(&h_fb, g, 0, cudaGraphCondAssignDefault) == cudaSuccess)))
-      return PS_ERR_CUDA;
-  }
   // One exact segmented select: a digit over the candidates, the split, then
-  // the list: a long one through the multi-CTA digit passes, the tie rule
-  // and the multi-CTA marking; a short one finished by one CTA.
-  // (a body is launched only once its capture has started: a kernel launched
-  // on the auxiliary stream outside a capture would run)
-  auto select = [&](cudaStream_t q, int single, int fallback, bool cond, cudaGraphConditionalHandle hl,
-                    cudaStream_t body) {
-    PS_LAUNCH(launch_k(k_wide_pass, cgrid, 256, 0, q, s, single, fallback));
-    PS_LAUNCH(launch_k(k_wide_resolve, single ? 1 : s.G, 32, 0, q, s, single));
-    PS_LAUNCH(launch_k(k_split, cgrid, 256, 0, q, s, single, fallback, hl, cond ? 1 : 0));
-    cudaStream_t b = q;
-    if (cond) {
-      if (!cond_open(q, body, hl)) { cond_ok = false; return; }
-      b = body;
-    }
-    for (int d = 0; d < 7; ++d) PS_LAUNCH(launch_k(k_digit_pass, lgrid, 256, radix_smem, b, s, single, fallback, 1));
-    PS_LAUNCH(launch_k(k_list_finish, 1, 1024, kFinSmem, b, s, single, 1));
-    PS_LAUNCH(launch_k(k_mark_list, lgrid, 256, 0, b, s, single));
-    if (cond && !cond_close(body)) { cond_ok = false; return; }
-    PS_LAUNCH(launch_k(k_list_finish, 1, 1024, kFinSmem, q, s, single, 0));
+  // the split list finished by one CTA.  Every phase is launched on every
+  // step (a kernel of a phase with nothing to select returns at once): a
+  // conditional graph node measured about 10 us a step even when its body
+  // was skipped, more than the phase's early-returning launches.
+  auto select = [&](int single, int fallback) {
+    PS_LAUNCH(launch_k(k_wide_pass, cgrid, 256, 0, st, s, single, fallback));
+    PS_LAUNCH(launch_k(k_wide_resolve, single ? 1 : s.G, 32, 0, st, s, single));
+    PS_LAUNCH(launch_k(k_split, cgrid, 256, 0, st, s, single, fallback));
+    PS_LAUNCH(launch_k(k_list_finish, 1, 1024, kFinSmem, st, s, single));
   };
   if (s.lg_on) {
     // selected above
   } else if (s.policy == PS_PREFIXSHIELD) {
-    PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s, h_fb, conds ? 1 : 0));  // after the join: plain
-    select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
-    if (!cond_ok) return PS_ERR_CUDA;
-    cudaStream_t f = st;
-    cudaGraphConditionalHandle h_fb_long = 0;
-    if (conds) {
-      // the fallback's own long-list body nests inside the fallback's body;
-      // its handle belongs to that body graph
-      cudaGraph_t fb_body = nullptr;
-      if (!cond_open(st, cap->aux, h_fb, &fb_body) ||
-          cudaGraphConditionalHandleCreate(&h_fb_long, fb_body, 0, cudaGraphCondAssignDefault) != cudaSuccess)
-        return PS_ERR_CUDA;
-      f = cap->aux;
-    }
-    select(f, 1, 1, conds, h_fb_long, conds ? cap->aux2 : f);  // started by the debt phase's finish
-    if (!cond_ok) return PS_ERR_CUDA;
-    if (conds && !cond_close(cap->aux)) return PS_ERR_CUDA;
+    PS_LAUNCH(k_waterfill<<<1, 1024, 0, st>>>(s, 0, 0));  // after the join: plain
+    select(0, 0);
+    select(1, 1);  // the global fallback, started by the debt phase's finish
   } else if (s.policy == PS_STATICQUOTA) {
     PS_LAUNCH(k_quota_sel<<<1, 1024, 0, st>>>(s));  // after the join: plain
-    select(st, 0, 0, conds, h_long, conds ? cap->aux : st);
-    if (!cond_ok) return PS_ERR_CUDA;
+    select(0, 0);
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));  // after the join: plain
-    select(st, 1, 0, conds, h_long, conds ? cap->aux : st);
-    if (!cond_ok) return PS_ERR_CUDA;
+    select(1, 0);
   } else {
     PS_LAUNCH(launch_s3_evict(s, st));
   }
