@@ -1527,6 +1527,7 @@ __device__ __forceinline__ void wide_digit(int nrows, uint64_t mask, int* dshift
 }
 __global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int fallback) {
   s = with_args(s);
+  __shared__ uint32_t s_coarse[kRadixBins];  // one row's coarse counts (a single segment)
   __shared__ int16_t row_of[PS_MAX_GROUPS];
   __shared__ uint64_t s_pre[PS_MAX_GROUPS], s_msk[PS_MAX_GROUPS];  // the segments' prefix and mask
   __shared__ int s_nrows;
@@ -1560,31 +1561,65 @@ __global__ void __launch_bounds__(256) k_wide_pass(DevState s, int single, int f
   const int nrows = s_nrows;
   if (nrows == 0) return;
   const uint32_t stride = nrows <= kWideRows ? (uint32_t)kWideBins : (uint32_t)kRadixBins;
-  for (int64_t e0 = blockIdx.x * (int64_t)blockDim.x; e0 < s.N; e0 += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t e = e0 + threadIdx.x;
-    bool act = false, act16 = false;
-    uint32_t idx = 0;
-    if (e < s.N) {
-      const uint64_t key = s.csk[e];
-      const int seg = single ? 0 : s.blk_group[e];  // issued with the key load
-      if (key != ~0ull && !(fallback && ((s.bm_victim[e >> 5] >> (e & 31)) & 1))) {
-        const int row = row_of[seg];
+  // A 16-bit digit is also counted by its top byte (row-major, 256 a row)
+  // for the resolve.  One row takes every candidate (lru, the fallback):
+  // its 256 coarse counts would serialize global atomics, so each CTA counts
+  // them in shared memory and adds its nonzero ones once at the end.
+  const bool coarse_smem = nrows == 1 && stride == (uint32_t)kWideBins;
+  for (int k = threadIdx.x; k < kRadixBins; k += blockDim.x) s_coarse[k] = 0;
+  __syncthreads();
+  // kU candidates a thread per iteration, their loads issued together (the
+  // trip count is CTA-uniform, as the warp-aggregated increment needs)
+  constexpr int kU = 4;
+  const int64_t span = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t b0 = blockIdx.x * (int64_t)blockDim.x; b0 < s.N; b0 += span * kU) {
+    uint64_t key[kU];
+    int seg[kU];
+    uint32_t vw[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t e = b0 + u * span + threadIdx.x;
+      key[u] = ~0ull;
+      seg[u] = 0;
+      vw[u] = 0;
+      if (e < s.N) {
+        key[u] = s.csk[e];
+        if (!single) seg[u] = s.blk_group[e];
+        if (fallback) vw[u] = s.bm_victim[e >> 5];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int64_t e = b0 + u * span + threadIdx.x;
+      bool act = false, act16 = false;
+      uint32_t idx = 0;
+      if (key[u] != ~0ull && !((vw[u] >> (e & 31)) & 1)) {
+        const int row = row_of[seg[u]];
         if (row >= 0) {
-          const uint64_t msk = s_msk[seg];
-          if ((key & msk) == s_pre[seg]) {
+          const uint64_t msk = s_msk[seg[u]];
+          if ((key[u] & msk) == s_pre[seg[u]]) {
             int dsh;
             uint32_t nb;
             wide_digit(nrows, msk, &dsh, &nb);
             act = true;
             act16 = nb == (uint32_t)kWideBins;
-            idx = (uint32_t)row * stride + (uint32_t)((key >> dsh) & (nb - 1));
+            idx = (uint32_t)row * stride + (uint32_t)((key[u] >> dsh) & (nb - 1));
           }
         }
       }
+      agg_inc(s.wide_bins, idx, act);
+      const uint32_t cidx = (idx >> 16) * kRadixBins + ((idx >> 8) & 0xFF);
+      if (coarse_smem) {
+        if (act16) atomicAdd(&s_coarse[cidx], 1u);
+      } else if (stride == (uint32_t)kWideBins) {
+        agg_inc(s.wide_coarse, cidx, act16);
+      }
     }
-    agg_inc(s.wide_bins, idx, act);
-    // 16-bit digits also by their top byte (row-major, 256 a row)
-    if (stride == (uint32_t)kWideBins) agg_inc(s.wide_coarse, (idx >> 16) * kRadixBins + ((idx >> 8) & 0xFF), act16);
+  }
+  if (coarse_smem) {
+    __syncthreads();
+    for (int k = threadIdx.x; k < kRadixBins; k += blockDim.x)
+      if (s_coarse[k]) atomicAdd(s.wide_coarse + k, s_coarse[k]);
   }
 }
 
