@@ -37,7 +37,8 @@ struct ps_handle {
   cudaStream_t cap_aux = nullptr;   // conditional bodies are captured here
   cudaStream_t cap_aux2 = nullptr;  // and bodies nested in them here
   cudaStream_t cap_side = nullptr;  // a parallel branch of the step graph
-  cudaEvent_t cap_fork = nullptr, cap_join = nullptr;
+  cudaStream_t cap_side2 = nullptr; // a second one
+  cudaEvent_t cap_fork = nullptr, cap_join = nullptr, cap_fork2 = nullptr, cap_join2 = nullptr;
   cudaGraph_t graph = nullptr;
   cudaGraphExec_t exec = nullptr;
   bool exec_timing = false;
@@ -370,7 +371,8 @@ void capture_step(ps_handle* h) {
   tmpl.R = 0;
   bool ok = cudaStreamBeginCapture(h->cap_stream, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
   if (ok) {
-    const CaptureCtx ctx{h->cap_aux, h->cap_aux2, h->cap_side, h->cap_fork, h->cap_join};
+    const CaptureCtx ctx{h->cap_aux, h->cap_aux2, h->cap_side, h->cap_fork, h->cap_join,
+                         h->cap_side2, h->cap_fork2, h->cap_join2};
     const int32_t rc = launch_step(tmpl, h->cap_stream, &h->trace, &ctx);
     // a body whose capture did not close leaves an auxiliary stream capturing
     // (the side stream joined the main capture: it ends with it)
@@ -465,8 +467,11 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
                       cudaStreamCreateWithFlags(&h->cap_aux, cudaStreamNonBlocking) != cudaSuccess ||
                       cudaStreamCreateWithFlags(&h->cap_aux2, cudaStreamNonBlocking) != cudaSuccess ||
                       cudaStreamCreateWithFlags(&h->cap_side, cudaStreamNonBlocking) != cudaSuccess ||
+                      cudaStreamCreateWithFlags(&h->cap_side2, cudaStreamNonBlocking) != cudaSuccess ||
                       cudaEventCreateWithFlags(&h->cap_fork, cudaEventDisableTiming) != cudaSuccess ||
                       cudaEventCreateWithFlags(&h->cap_join, cudaEventDisableTiming) != cudaSuccess ||
+                      cudaEventCreateWithFlags(&h->cap_fork2, cudaEventDisableTiming) != cudaSuccess ||
+                      cudaEventCreateWithFlags(&h->cap_join2, cudaEventDisableTiming) != cudaSuccess ||
                       cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking) != cudaSuccess))
     rc = PS_ERR_CUDA;
   for (int k = 0; k < 2 && rc == PS_OK; ++k)
@@ -659,8 +664,11 @@ void ps_destroy(ps_handle_t* h) {
   if (h->cap_aux) cudaStreamDestroy(h->cap_aux);
   if (h->cap_aux2) cudaStreamDestroy(h->cap_aux2);
   if (h->cap_side) cudaStreamDestroy(h->cap_side);
+  if (h->cap_side2) cudaStreamDestroy(h->cap_side2);
   if (h->cap_fork) cudaEventDestroy(h->cap_fork);
   if (h->cap_join) cudaEventDestroy(h->cap_join);
+  if (h->cap_fork2) cudaEventDestroy(h->cap_fork2);
+  if (h->cap_join2) cudaEventDestroy(h->cap_join2);
   if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   for (int k = 0; k < 2; ++k)
     for (cudaEvent_t e : {h->in_ready[k], h->slot_free[k], h->done[k]})

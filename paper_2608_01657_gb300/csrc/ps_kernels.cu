@@ -129,6 +129,17 @@ __device__ uint32_t table_insert(const DevState& s, uint64_t key, uint32_t g, ui
 // first), so a delete clears only that field: an insert that takes the slot
 // at once then writes its own key and group, and no late clearing store of
 // the delete can land on them.
+// The same from the block's record as already loaded (slot with its flag,
+// key, group).
+__device__ __forceinline__ void table_delete_known(const DevState& s, uint32_t tagged, uint64_t key, uint32_t g) {
+  const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
+  const uint32_t slot = tagged & ~kDisplaced;
+  s.table[slot].blk = kNone;
+  if (!(tagged & kDisplaced)) return;  // in its home bucket: no counter passed
+  const uint32_t bucket = slot / kTableWays;
+  uint32_t x = table_home(key, g, s.tb_nbuckets_log2);
+  for (uint32_t it = 0; x != bucket && it <= mask; ++it, x = (x + 1) & mask) atomicSub(s.table_ovf + x, 1u);
+}
 __device__ void table_delete(const DevState& s, uint32_t blk) {
   const uint32_t mask = (1u << s.tb_nbuckets_log2) - 1;
   const uint32_t tagged = s.blk_slot[blk];
@@ -677,6 +688,19 @@ __device__ void undo_pin_claim(const DevState& s, const Ctl* c, int64_t t) {
   }
 }
 
+// A history entry from L2 (two 16-byte loads that skip L1: a tag may have
+// been updated by an atomic since another CTA on this SM read the line).
+__device__ __forceinline__ HistEntry ldcg_hist(const HistEntry* p) {
+  const uint4 a = __ldcg(reinterpret_cast<const uint4*>(p)), b = __ldcg(reinterpret_cast<const uint4*>(p) + 1);
+  HistEntry e;
+  e.p = (uint64_t)a.y << 32 | a.x;
+  e.g1 = a.z;
+  e.refadm = a.w;
+  e.ftag = (uint64_t)b.y << 32 | b.x;
+  e.atag = (uint64_t)b.w << 32 | b.z;
+  return e;
+}
+
 // Stage 2 (cont.): the first own claim s_i of each request, and orphans.  A
 // resident block past a request's first miss cannot be reached by lookup; it
 // is dropped (invalidated) unless some request pinned it.  Threads past the
@@ -851,24 +875,6 @@ __global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
   agg_min_u32(s.rq_fu, valid ? r.i : 0u, valid ? (uint32_t)r.m : 0u, past);
 }
 
-// hit_i = h_i + e_i per request; records the first admitting request of each
-// (group, prefix) history entry of the step.
-__global__ void k_instep_fin(DevState s) {
-  s = with_args(s);
-  const Ctl* c = s.ctl;
-  if (c->status != PS_OK) return;
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= s.R) return;
-  const int h = s.rq_h[i], si = s.rq_s[i];
-  const uint32_t fu = s.rq_fu[i];
-  const int e = (int)tmin<uint32_t>(fu, (uint32_t)si) - h;
-  s.rq_e[i] = e;
-  s.out.hit_blocks[i] = h + e;
-  const uint32_t hs = s.rq_hs[i];
-  if (s.rq_a[i] > 0 && hs != kNone)
-    atomicMax(reinterpret_cast<unsigned long long*>(&s.hist[hs].atag), (unsigned long long)step_tag(c->step, (uint32_t)i));
-}
-
 // ===========================================================================
 // Stages 3-4: metering (Eq. 1-3, OnCacheFullBlocks of Alg. 1), in request
 // order, one CTA per group.  The CTA compacts its group's requests of each
@@ -933,16 +939,27 @@ __global__ void __launch_bounds__(kMeterThreads) k_meter(DevState s0) {
       const bool mem = k < nmem;
       const int i = mem ? s_mem[k] : 0;
       int n = 0, a = 0, cid = 0, rh = 0, re = 0, rs = 0;
-      uint32_t hs = kNone;
+      uint32_t hs = kNone, fu = kNone;
       int64_t ptok = 0;
       if (mem) {
         n = s.rq_n[i]; a = s.rq_a[i]; cid = s.rq_cid[i]; hs = s.rq_hs[i];
-        rh = s.rq_h[i]; re = s.rq_e[i]; rs = s.rq_s[i];
+        rh = s.rq_h[i]; rs = s.rq_s[i]; fu = s.rq_fu[i];
         ptok = s.in_offsets[i + 1] - s.in_offsets[i];
+        // in-step hits: the leading positions of [h_i, s_i) before the first
+        // ungranted one; hit_i = h_i + e_i
+        re = (int)tmin<uint32_t>(fu, (uint32_t)rs) - rh;
+        s.rq_e[i] = re;
+        s.out.hit_blocks[i] = rh + re;
+        // the first admitting request of the (group, prefix) entry in this
+        // step: only requests of this group share its entries, and every one
+        // of them is this CTA's
+        if (a > 0 && hs != kNone)
+          atomicMax(reinterpret_cast<unsigned long long*>(&s.hist[hs].atag), (unsigned long long)step_tag(step, (uint32_t)i));
       }
       const bool pol = mem && n > 0;
+      __syncthreads();  // every member's admission tag is in place
       HistEntry he{};
-      if (pol && hs != kNone) he = s.hist[hs];
+      if (pol && hs != kNone) he = ldcg_hist(s.hist + hs);
       // charges of this group's earlier requests, per contract
       int64_t S[PS_MAX_CONTRACTS];
 #pragma unroll
@@ -2064,8 +2081,16 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
       } else {
         const ClaimEntry e = s.claims[slot];
         const uint64_t key = s.pos_key[pos];
-        if (s.blk_flags[b] & 1) {  // a victim: evict its old content
-          gold = drop_block(s, b, false);
+        // the id's old record, loaded together: a resident id is a victim,
+        // whose old content (table entry, record) leaves first
+        const uint8_t ofl = s.blk_flags[b];
+        const uint32_t oslot = s.blk_slot[b];
+        const uint64_t okey = s.blk_key[b];
+        const uint16_t ogrp = s.blk_group[b];
+        if (ofl & 1) {
+          table_delete_known(s, oslot, okey, ogrp);
+          if (s.policy == PS_S3FIFO) atomic_add_i64((ofl & 2) ? &c->s3_nM : &c->s3_nS, -1);
+          gold = ogrp;
           evicted = true;
         }
         s.blk_key[b] = key;
@@ -2167,7 +2192,6 @@ void configure_kernels(const DevState& s) {
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const CaptureCtx* cap) {
   // grids depend only on the handle's bounds (a captured graph serves any step)
   const int R = s.max_requests;
-  const int rgrid = grid_for(R, 256, 1 << 20);
   const int pgrid = grid_for(s.max_blocks, kThreads, 1 << 30);
   const int prgrid = grid_for(s.max_blocks + R, kThreads, 1 << 30);
   const int ngrid = grid_for(s.N, 256, 152 * 8);
@@ -2222,12 +2246,24 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
   if (!early && launch_cand() != PS_OK) return PS_ERR_CUDA;
   PS_LAUNCH(launch_k(k_instep, pgrid, kThreads, 0, st, s));
-  PS_LAUNCH(launch_k(k_instep_fin, rgrid, 256, 0, st, s));
   mark(4);
   PS_LAUNCH(launch_k(k_meter, s.G, 512, 0, st, s));
   mark(5);
   PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, st, s));
-  PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, st, s));
+  // The touch's second pass (promotions of resident hit blocks, gated-reuse
+  // counts) writes only the class of pinned blocks and two statistics, which
+  // nothing later in the step reads (the indexed queues' appends would: with
+  // them it stays in line): under capture it runs on a second parallel branch
+  // beside the select and the insertions, joined before the commit.
+  const bool fork2 = cap != nullptr && !s.lg_on;
+  if (fork2) {
+    if (cudaEventRecord(cap->fork2, st) != cudaSuccess || cudaStreamWaitEvent(cap->side2, cap->fork2, 0) != cudaSuccess)
+      return PS_ERR_CUDA;
+    PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, cap->side2, s));
+    if (cudaEventRecord(cap->join2, cap->side2) != cudaSuccess) return PS_ERR_CUDA;
+  } else {
+    PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, st, s));
+  }
   mark(6);
   if (fork && cudaStreamWaitEvent(st, cap->join, 0) != cudaSuccess) return PS_ERR_CUDA;
   if (s.lg_on) {
@@ -2287,7 +2323,12 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));
   if (s.lg_on && launch_queue_append(s, st, cap, &launches) != PS_OK) return PS_ERR_CUDA;
   mark(10);
-  PS_LAUNCH(launch_k(k_finalize, 1, 32, 0, st, s));
+  if (fork2) {  // the promotion branch joins the commit
+    if (cudaStreamWaitEvent(st, cap->join2, 0) != cudaSuccess) return PS_ERR_CUDA;
+    PS_LAUNCH(k_finalize<<<1, 32, 0, st>>>(s));  // after the join: plain
+  } else {
+    PS_LAUNCH(launch_k(k_finalize, 1, 32, 0, st, s));
+  }
   mark(11);
 #undef PS_LAUNCH
   if (tr) tr->launches = launches;
