@@ -357,7 +357,7 @@ struct CaptureCtx {
   cudaStream_t aux2;  // bodies of conditional nodes inside those
   cudaStream_t side;  // a parallel branch of the step graph (the candidate scan)
   cudaEvent_t fork, join;
-  cudaStream_t side2;  // a second branch (the touch's promotion pass)
+  cudaStream_t side2;  // a second branch (the touch passes)
   cudaEvent_t fork2, join2;
 };
 

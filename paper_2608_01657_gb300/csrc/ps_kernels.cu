@@ -2249,19 +2249,22 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(4);
   PS_LAUNCH(launch_k(k_meter, s.G, 512, 0, st, s));
   mark(5);
-  PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, st, s));
-  // The touch's second pass (promotions of resident hit blocks, gated-reuse
-  // counts) writes only the class of pinned blocks and two statistics, which
-  // nothing later in the step reads (the indexed queues' appends would: with
-  // them it stays in line): under capture it runs on a second parallel branch
-  // beside the select and the insertions, joined before the commit.
-  const bool fork2 = cap != nullptr && !s.lg_on;
+  // The touch passes write the stamps, counters and promotions of hit
+  // blocks (pinned: no candidate) and the in-step touches of claim entries;
+  // the select reads none of them, only the insertion does (it reads the
+  // claim entries, then clears them, which the second pass reads).  Under
+  // capture they run on a second parallel branch beside the select, joined
+  // before the insertion.  S3-FIFO and the indexed queues keep them in line
+  // (their selects read touched blocks' state).
+  const bool fork2 = cap != nullptr && !s.lg_on && s.policy != PS_S3FIFO;
   if (fork2) {
     if (cudaEventRecord(cap->fork2, st) != cudaSuccess || cudaStreamWaitEvent(cap->side2, cap->fork2, 0) != cudaSuccess)
       return PS_ERR_CUDA;
+    PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, cap->side2, s));
     PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, cap->side2, s));
     if (cudaEventRecord(cap->join2, cap->side2) != cudaSuccess) return PS_ERR_CUDA;
   } else {
+    PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, st, s));
     PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, st, s));
   }
   mark(6);
@@ -2319,16 +2322,16 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   mark(8);
   // (evictions happen in k_insert: every victim is allocated again in its step)
   mark(9);
-  PS_LAUNCH(launch_k(k_insert, pgrid, kThreads, 0, st, s));
+  if (fork2) {  // the touch branch joins the insertion
+    if (cudaStreamWaitEvent(st, cap->join2, 0) != cudaSuccess) return PS_ERR_CUDA;
+    PS_LAUNCH((k_insert<<<pgrid, kThreads, 0, st>>>(s)));  // after the join: plain
+  } else {
+    PS_LAUNCH(launch_k(k_insert, pgrid, kThreads, 0, st, s));
+  }
   if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));
   if (s.lg_on && launch_queue_append(s, st, cap, &launches) != PS_OK) return PS_ERR_CUDA;
   mark(10);
-  if (fork2) {  // the promotion branch joins the commit
-    if (cudaStreamWaitEvent(st, cap->join2, 0) != cudaSuccess) return PS_ERR_CUDA;
-    PS_LAUNCH(k_finalize<<<1, 32, 0, st>>>(s));  // after the join: plain
-  } else {
-    PS_LAUNCH(launch_k(k_finalize, 1, 32, 0, st, s));
-  }
+  PS_LAUNCH(launch_k(k_finalize, 1, 32, 0, st, s));
   mark(11);
 #undef PS_LAUNCH
   if (tr) tr->launches = launches;
