@@ -221,6 +221,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.table = cv.take<TableEntry>((size_t)kTableWays << d.tb_log2);
   t.table_ovf = cv.take<uint32_t>((size_t)1 << d.tb_log2);
   t.ledger = cv.take<int64_t>(G * d.C);
+  t.ledger_b0 = cv.take<int64_t>(G * d.C);
   t.contract_of_group = cv.take<int32_t>(G);
   t.key_words = cv.take<uint32_t>((size_t)d.bs + 2);
   t.kc_pow = cv.take<uint64_t>(2 * ((size_t)kSegBlocks + 1));

@@ -235,6 +235,7 @@ struct DevState {
   TableEntry* table;
   uint32_t* table_ovf;     // per bucket: live keys probing past it
   int64_t* ledger;         // B_{g,c}, fixed point
+  int64_t* ledger_b0;      // per step: B_{g,c} refilled to now, before the step's charges
   int32_t* contract_of_group;
   uint32_t* key_words;     // NH key schedule, bs + 2 words
   uint64_t* kc_pow;        // Kc^k mod p, k = 0..kSegBlocks, then Kc^(kSegBlocks t), t = 0..32
@@ -357,7 +358,7 @@ struct CaptureCtx {
   cudaStream_t aux2;  // bodies of conditional nodes inside those
   cudaStream_t side;  // a parallel branch of the step graph (the candidate scan)
   cudaEvent_t fork, join;
-  cudaStream_t side2;  // a second branch (the touch passes)
+  cudaStream_t side2;  // a second branch (in-step hits, metering, touch passes)
   cudaEvent_t fork2, join2;
 };
 

@@ -754,8 +754,11 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
 // Stage 3: grant new blocks against the pool.  avail = free + unpinned
 // resident = N - pinned; claims are ranked in (request, position) order; the
 // first avail ranks are materialized.  One CTA.
-__global__ void __launch_bounds__(1024) k_grant(DevState s) {
-  s = with_args(s);
+__global__ void __launch_bounds__(1024) k_grant(DevState s0) {
+  // Contract arrays are read from the parameter block: indexing the per-step
+  // copy by a run-time contract would move the whole copy to local memory.
+  const DevState s = with_args(s0);
+  extern __shared__ unsigned long long g_sum[];  // [G * C] the step's charges per (group, contract)
   Ctl* c = s.ctl;
   if (c->status != PS_OK) return;
   if (history_overflows(s, c)) {  // undone by k_claims; the error is sticky
@@ -763,7 +766,10 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
     return;
   }
   const int R = s.R;
+  const int C = s.C;
   const bool quota = s.policy == PS_STATICQUOTA;  // a_i already granted per group
+  for (int k = threadIdx.x; k < s.G * C; k += blockDim.x) g_sum[k] = 0;
+  __syncthreads();
   const int64_t avail = s.N - c->pinned;
   // Granted ranks are the first avail in (request, position) order, so the
   // grants before request i number min(avail, base_i), base_i the claims
@@ -799,6 +805,7 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
         s.rq_a[i] = a;
         s.out.admitted_blocks[i] = a;
         s.out.admitted_offsets[i] = (int32_t)lo;
+        if (a > 0) atomicAdd(&g_sum[s.in_group[i] * C + s.rq_cid[i]], (unsigned long long)a);
       }
     }
     carry += tot;
@@ -819,6 +826,38 @@ __global__ void __launch_bounds__(1024) k_grant(DevState s) {
     c->nfree = nfree;
     c->ftake = quota ? need - qv : tmin(need, nfree);
     c->mvict = need - c->ftake;
+  }
+  // The step's balances and debts (Eq. 1-3, 5) follow from each (group,
+  // contract)'s total charge, so they are settled here and the select need
+  // not wait for the per-request metering (which reads the refilled opening
+  // balances from ledger_b0).
+  __syncthreads();
+  const int64_t unit = (int64_t)1 << s.fp_shift;
+  for (int g = threadIdx.x; g < s.G; g += blockDim.x) {
+    int64_t raw = 0, norm = 0, rmax = 0;
+    for (int cc = 0; cc < C; ++cc) {
+      const int64_t b0 = refill(s.ledger[g * C + cc], s0.beta[cc], s0.rho[cc], s.now - c->t_prev);
+      s.ledger_b0[g * C + cc] = b0;
+      const int64_t b = b0 - (int64_t)g_sum[g * C + cc] * unit;  // Eq. 2 over the step's charges
+      s.ledger[g * C + cc] = b;
+      const int64_t def = tmax<int64_t>(0, -b);
+      raw += def;                                    // Eq. 3
+      norm += muldiv(def, s.rho_min, s0.rho[cc]);    // Eq. 5
+      if (b < 0) rmax = tmax(rmax, s0.rho[cc]);
+    }
+    int64_t* row = s.stats + (int64_t)g * PS_NUM_STATS;
+    row[PS_STAT_DEBT_RAW] = raw;
+    row[PS_STAT_DEBT_NORM] = norm;
+    s.out.debt_raw[g] = raw;
+    s.out.debt_norm[g] = norm;
+    s.grp_P[g] = norm;
+    s.grp_delta[g] = rmax ? muldiv(unit, s.rho_min, rmax) : 0;  // 1/W_g of Eq. 8
+    SelSeg z{};
+    z.kmin = ~0ull;
+    z.kmax = 0;
+    z.qmin = ~0ull;
+    z.qmax = 0;
+    s.sel[g] = z;
   }
 }
 
@@ -885,7 +924,8 @@ __global__ void __launch_bounds__(kThreads) k_instep(DevState s) {
 //   B_{g,c} after the request's own charge (the class of its new blocks).
 // q_r >= 1 and "(g,p) was admitted" come from the history entry as it stood at
 // the start of the step and the first request of the step that referenced /
-// admitted it.  Also writes the group's statistics, balances and debts.
+// admitted it.  Also writes the group's request statistics; the balances
+// and debts after the step are k_grant's (from the same charges).
 constexpr int kMeterThreads = 512;
 constexpr int kMeterTile = 4 * kMeterThreads;  // requests compacted per pass
 __global__ void __launch_bounds__(kMeterThreads) k_meter(DevState s0) {
@@ -901,10 +941,7 @@ __global__ void __launch_bounds__(kMeterThreads) k_meter(DevState s0) {
   __shared__ int64_t B0[PS_MAX_CONTRACTS];
   __shared__ unsigned long long s_st[7];  // the group's request statistics
   __shared__ int32_t s_mem[kMeterTile];   // this tile's members, in request order
-  if (threadIdx.x < C) {
-    const int cc = threadIdx.x;
-    B0[cc] = refill(s.ledger[g * C + cc], s0.beta[cc], s0.rho[cc], s.now - c->t_prev);
-  }
+  if (threadIdx.x < C) B0[threadIdx.x] = s.ledger_b0[g * C + threadIdx.x];  // refilled by k_grant
   if (threadIdx.x < 7) s_st[threadIdx.x] = 0;
   __syncthreads();
   int64_t carry[PS_MAX_CONTRACTS];
@@ -1016,30 +1053,6 @@ __global__ void __launch_bounds__(kMeterThreads) k_meter(DevState s0) {
     row[PS_STAT_HIT_TOKENS] += st_hit * s.bs;
     row[PS_STAT_ADMITTED_BLOCKS] += st_adm;
     row[PS_STAT_UNGRANTED_BLOCKS] += st_ungr;
-    int64_t raw = 0, norm = 0, rmax = 0;
-#pragma unroll
-    for (int cc = 0; cc < PS_MAX_CONTRACTS; ++cc) {
-      if (cc < C) {
-        const int64_t b = B0[cc] - carry[cc] * unit;  // Eq. 2 over the step's charges
-        s.ledger[g * C + cc] = b;
-        const int64_t def = tmax<int64_t>(0, -b);
-        raw += def;                                    // Eq. 3
-        norm += muldiv(def, s.rho_min, s0.rho[cc]);    // Eq. 5
-        if (b < 0) rmax = tmax(rmax, s0.rho[cc]);
-      }
-    }
-    row[PS_STAT_DEBT_RAW] = raw;
-    row[PS_STAT_DEBT_NORM] = norm;
-    s.out.debt_raw[g] = raw;
-    s.out.debt_norm[g] = norm;
-    s.grp_P[g] = norm;
-    s.grp_delta[g] = rmax ? muldiv(unit, s.rho_min, rmax) : 0;  // 1/W_g of Eq. 8
-    SelSeg z{};
-    z.kmin = ~0ull;
-    z.kmax = 0;
-    z.qmin = ~0ull;
-    z.qmax = 0;
-    s.sel[g] = z;
   }
 }
 
@@ -2187,6 +2200,7 @@ void configure_kernels(const DevState& s) {
   (void)s;
   cudaFuncSetAttribute(k_list_finish, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFinSmem);
   cudaFuncSetAttribute(k_cand, cudaFuncAttributeMaxDynamicSharedMemorySize, PS_MAX_GROUPS * kClasses * 5 * 4);
+  cudaFuncSetAttribute(k_grant, cudaFuncAttributeMaxDynamicSharedMemorySize, PS_MAX_GROUPS * PS_MAX_CONTRACTS * 8);
 }
 
 int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const CaptureCtx* cap) {
@@ -2243,30 +2257,29 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   };
   if (early && launch_cand() != PS_OK) return PS_ERR_CUDA;
   if (s.policy == PS_STATICQUOTA) PS_LAUNCH(launch_k(k_grant_quota, s.G, 1024, 0, st, s));
-  PS_LAUNCH(launch_k(k_grant, 1, 1024, 0, st, s));
+  PS_LAUNCH(launch_k(k_grant, 1, 1024, (size_t)s.G * s.C * 8, st, s));
   if (!early && launch_cand() != PS_OK) return PS_ERR_CUDA;
-  PS_LAUNCH(launch_k(k_instep, pgrid, kThreads, 0, st, s));
-  mark(4);
-  PS_LAUNCH(launch_k(k_meter, s.G, 512, 0, st, s));
-  mark(5);
-  // The touch passes write the stamps, counters and promotions of hit
-  // blocks (pinned: no candidate) and the in-step touches of claim entries;
-  // the select reads none of them, only the insertion does (it reads the
-  // claim entries, then clears them, which the second pass reads).  Under
+  // The in-step hits, the metering and the touch passes feed the insertion
+  // (the claims' in-step touches, the new blocks' class) and the statistics;
+  // the select needs only the step's debts, which k_grant settles.  Under
   // capture they run on a second parallel branch beside the select, joined
-  // before the insertion.  S3-FIFO and the indexed queues keep them in line
-  // (their selects read touched blocks' state).
+  // before the insertion (which reads, then clears, the claim entries).
+  // S3-FIFO and the indexed queues keep them in line (their selects read
+  // touched blocks' state).
   const bool fork2 = cap != nullptr && !s.lg_on && s.policy != PS_S3FIFO;
+  cudaStream_t ms = st;
   if (fork2) {
     if (cudaEventRecord(cap->fork2, st) != cudaSuccess || cudaStreamWaitEvent(cap->side2, cap->fork2, 0) != cudaSuccess)
       return PS_ERR_CUDA;
-    PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, cap->side2, s));
-    PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, cap->side2, s));
-    if (cudaEventRecord(cap->join2, cap->side2) != cudaSuccess) return PS_ERR_CUDA;
-  } else {
-    PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, st, s));
-    PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, st, s));
+    ms = cap->side2;
   }
+  PS_LAUNCH(launch_k(k_instep, pgrid, kThreads, 0, ms, s));
+  mark(4);
+  PS_LAUNCH(launch_k(k_meter, s.G, 512, 0, ms, s));
+  mark(5);
+  PS_LAUNCH(launch_k(k_touch, pgrid, kThreads, 0, ms, s));
+  PS_LAUNCH(launch_k(k_touch2, pgrid, kThreads, 0, ms, s));
+  if (fork2 && cudaEventRecord(cap->join2, cap->side2) != cudaSuccess) return PS_ERR_CUDA;
   mark(6);
   if (fork && cudaStreamWaitEvent(st, cap->join, 0) != cudaSuccess) return PS_ERR_CUDA;
   if (s.lg_on) {
