@@ -141,6 +141,7 @@ struct Dims {
   int64_t N, max_tokens, max_blocks, nwords, hist_cap, max_segments;
   int64_t s3_small_cap, s3_ghost_cap;
   uint64_t ghost_ring_cap;
+  int64_t s3_np, s3_nch, s3_nrch;
   uint32_t gh_log2;
   int32_t bs, G, C, max_requests;
   uint32_t tb_log2, cl_log2, hist_log2;
@@ -175,7 +176,16 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   d.s3_ghost_cap = N - d.s3_small_cap;
   d.gh_log2 = log2_pow2_at_least((uint64_t)((d.s3_ghost_cap + 3) / 4 > 1 ? (d.s3_ghost_cap + 3) / 4 : 1));
   if (d.gh_log2 < 1) d.gh_log2 = 1;
-  d.ghost_ring_cap = 1ull << log2_pow2_at_least((uint64_t)(2 * d.s3_ghost_cap + 64));
+  // S3-FIFO queue arrays: a region of N entries rounded up to whole chunks.
+  // Ghost FIFO ring: room for twice the ghost's capacity plus a step's pushes
+  // (at most max_blocks), so compactions are rare; at least two chunks.
+  d.s3_np = (N + kS3Chunk - 1) / kS3Chunk * kS3Chunk;
+  d.s3_nch = d.s3_np / kS3Chunk;
+  {
+    const uint64_t want = (uint64_t)(2 * (d.s3_ghost_cap + d.max_blocks));
+    d.ghost_ring_cap = 1ull << log2_pow2_at_least(want > 2 * (uint64_t)kS3Chunk ? want : 2 * (uint64_t)kS3Chunk);
+  }
+  d.s3_nrch = (int64_t)(d.ghost_ring_cap / kS3Chunk) + 1;
   // indexed queues: at most two live entries a block (its group's log and its
   // class's global log) and two a position of a step; each buffer holds eight
   // times that, so a compaction leaves at least seven eighths free
@@ -210,14 +220,12 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.blk_inval = cv.take<uint32_t>(N);
   const size_t zero_end = cv.off;  // everything above starts zeroed
   t.res_bits = cv.take<uint32_t>((size_t)d.nwords);
-  t.s3_prev = cv.take<uint32_t>(N);
-  t.s3_next = cv.take<uint32_t>(N);
-  t.s3_inval = cv.take<uint32_t>(B);
+  t.s3_arr = cv.take<uint32_t>(4 * (size_t)d.s3_np);
   t.ghost_map = cv.take<TableEntry>((size_t)kTableWays << d.gh_log2);
   t.ghost_ovf = cv.take<uint32_t>((size_t)1 << d.gh_log2);
-  t.ghost_ring_key = cv.take<uint64_t>((size_t)d.ghost_ring_cap);
-  t.ghost_ring_grp = cv.take<uint32_t>((size_t)d.ghost_ring_cap);
-  t.ghost_ring_seq = cv.take<uint64_t>((size_t)d.ghost_ring_cap);
+  t.ghost_sq = cv.take<uint64_t>((size_t)kTableWays << d.gh_log2);
+  t.ghost_ring = cv.take<uint32_t>(2 * (size_t)d.ghost_ring_cap);
+  t.ghost_bits = cv.take<uint32_t>(2 * (size_t)(d.ghost_ring_cap / 32));
   t.table = cv.take<TableEntry>((size_t)kTableWays << d.tb_log2);
   t.table_ovf = cv.take<uint32_t>((size_t)1 << d.tb_log2);
   t.ledger = cv.take<int64_t>(G * d.C);
@@ -273,6 +281,14 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.lst_blk = cv.take<uint32_t>(N);
   t.lst_seg = cv.take<uint16_t>(N);
   t.bm_chunk_cnt = cv.take<int32_t>(3 * (((size_t)d.nwords + kBmChunk - 1) / kBmChunk));  // free, evicted, invalidated
+  t.s3_attr = cv.take<uint8_t>(2 * (size_t)d.s3_np);
+  t.s3_ck = cv.take<S3Chunk>(2 * (size_t)d.s3_nch);
+  t.s3_base = cv.take<S3Base>(2 * (size_t)d.s3_nch);
+  t.s3_rck = cv.take<uint32_t>((size_t)d.s3_nrch);
+  t.s3_rbase = cv.take<uint32_t>((size_t)d.s3_nrch);
+  t.s3_plan = cv.take<S3Plan>(1);
+  t.s3_hit = cv.take<uint8_t>(B);
+  t.s3_ick = cv.take<uint32_t>(B / kS3Chunk + 1);
   if (d.lg) {
     const size_t L = (size_t)d.lg_L;
     t.lg_L = d.lg_L;
@@ -336,9 +352,6 @@ int32_t init_state(ps_handle* h, cudaStream_t st) {
     return PS_ERR_CUDA;
   if (cudaMemsetAsync(s.ghost_map, 0xFF, sizeof(TableEntry) * ((size_t)kTableWays << s.gh_nbuckets_log2), st) !=
       cudaSuccess)
-    return PS_ERR_CUDA;
-  if (cudaMemsetAsync(s.s3_prev, 0xFF, sizeof(uint32_t) * (size_t)s.N, st) != cudaSuccess ||
-      cudaMemsetAsync(s.s3_next, 0xFF, sizeof(uint32_t) * (size_t)s.N, st) != cudaSuccess)
     return PS_ERR_CUDA;
   launch_init(s, st);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
@@ -449,6 +462,7 @@ int32_t ps_create(ps_handle_t** out, int64_t capacity_blocks, int32_t block_size
   s.s3_small_pct = params->s3_small_pct; s.s3_freq_cap = params->s3_freq_cap; s.s3_move_min = params->s3_move_min_freq;
   s.s3_small_cap = d.s3_small_cap; s.s3_ghost_cap = d.s3_ghost_cap;
   s.gh_nbuckets_log2 = d.gh_log2; s.ghost_ring_cap = d.ghost_ring_cap;
+  s.s3_np = d.s3_np; s.s3_nch = d.s3_nch; s.s3_nrch = d.s3_nrch;
   s.max_requests = max_requests; s.max_tokens = max_tokens; s.max_blocks = d.max_blocks;
   s.history_capacity = params->history_capacity;
   s.tb_nbuckets_log2 = d.tb_log2; s.cl_nbuckets_log2 = d.cl_log2; s.hist_cap_log2 = d.hist_log2;
@@ -802,21 +816,22 @@ int64_t ps_export_ghost(ps_handle_t* h, void* stream, int32_t* h_group, uint64_t
   if (!h) return PS_ERR_INVALID_ARG;
   cudaStream_t st = as_stream(stream);
   const DevState& s = h->base;
-  // copy the ghost map and the ring's sequence numbers, read them here
+  // copy the ghost map and each slot's sequence number, read them here
   const size_t n = (size_t)kTableWays << s.gh_nbuckets_log2;
   std::vector<TableEntry> map(n);
-  std::vector<uint64_t> seq((size_t)s.ghost_ring_cap);
+  std::vector<uint64_t> seq(n);
   if (cudaMemcpyAsync(map.data(), s.ghost_map, n * sizeof(TableEntry), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
-      cudaMemcpyAsync(seq.data(), s.ghost_ring_seq, seq.size() * 8, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaMemcpyAsync(seq.data(), s.ghost_sq, n * 8, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
       cudaStreamSynchronize(st) != cudaSuccess)
     return PS_ERR_CUDA;
   int64_t k = 0;
-  for (const TableEntry& e : map) {
+  for (size_t i = 0; i < n; ++i) {
+    const TableEntry& e = map[i];
     if (e.blk == kNone) continue;
     if (h_group && k < cap) {
       h_group[k] = (int32_t)e.grp;
       h_key[k] = e.key;
-      h_seq[k] = seq[e.blk];
+      h_seq[k] = seq[i];
     }
     ++k;
   }

@@ -77,8 +77,10 @@ struct Ctl {
   int64_t hist_live;
   uint64_t s3_ctr, ghost_ctr;
   int64_t s3_nS, s3_nM;             // queue sizes (pinned members included)
-  uint32_t s3_head[2], s3_tail[2];  // small (0) and main (1) queues: tail = oldest
-  uint64_t ghost_head, ghost_tail;  // ghost FIFO ring positions
+  int64_t s3_len[2];                // small (0) and main (1) queue arrays: entries, oldest first
+  int32_t s3_buf;                   // which of the two array buffers holds the queues
+  int32_t ghost_rbuf;               // which of the two ghost rings holds the FIFO
+  uint64_t ghost_head, ghost_tail;  // ghost FIFO window [tail, head) (absolute positions)
   int64_t ghost_live;               // live ghost entries
   // per step
   int32_t status;          // this step's status
@@ -89,8 +91,6 @@ struct Ctl {
   int64_t n_evicted, n_alloc, n_victims_marked;
   int64_t m_fb;            // prefixshield: victims left to the global fallback
   int32_t sel_ntie, sel_k; // prefixshield tie bookkeeping
-  int64_t s3_pinned[2];    // pinned members of each S3-FIFO queue this step
-  int64_t s3_ninval;       // invalidated blocks to unlink this step
   int64_t lst_n;              // members of the select's split list
   uint32_t ticket;         // last-block-done counter for the radix passes and the split
   int32_t nlaunch;         // kernels launched by the step (conditional bodies run or not)
@@ -172,6 +172,47 @@ constexpr int kClasses = 3;
 constexpr int kWideRows = 64;
 constexpr int kWideBins = 1 << 16;
 
+// ---- S3-FIFO as sequence-ordered arrays ------------------------------------
+// Both queues are arrays of block ids in sequence order (oldest first),
+// rebuilt every step from the step's closed-form plan; chunks of kS3Chunk
+// entries are the unit of the per-step passes.
+constexpr int kS3Chunk = 2048;
+constexpr int kS3Bins = 16;      // frequencies 0..15 (a larger cap takes the sequential kernel)
+struct S3Chunk {
+  uint32_t nlive, nu, nev, pad;  // live entries, unpinned ones, unpinned with f < move threshold
+  uint32_t hist[kS3Bins];        // unpinned entries by frequency
+};
+struct S3Base {                  // exclusive prefixes of a chunk (per-region or main-then-small order)
+  uint32_t u, ev, mv, keep, ge, gt, pad0, pad1;
+};
+struct S3Plan {
+  int64_t lenS, lenM;    // queue arrays at step start
+  int64_t pcut;          // unpinned small entries before this array position are consumed
+  int64_t kS;            // small-queue evictions (ghost pushes)
+  int64_t MA;            // small -> main moves
+  int64_t UMo;           // unpinned main entries (the main phase's visit list starts with them)
+  int64_t nL;            // main phase's visit list: UMo, then the moved blocks
+  int64_t P;             // visit-list index of the final round's last visit (-1: no main phase)
+  int64_t rge_P1, rgt_P1;  // visit-list entries at or before P with f >= Rs / f > Rs
+  int64_t base_Rm1, base_R;  // reinsertions in rounds before Rs - 1 / before Rs
+  int64_t nG1, nUnvMov, nMid;
+  int64_t nKeepS, nKeepM;
+  uint64_t ctr0, ctr_end;
+  int32_t Rs;            // the final round of the main phase (0 without one)
+  int32_t fb;            // 1: the sequential kernel takes the step
+  int32_t gc;            // 1: the ghost FIFO is compacted into the other ring
+  int32_t rbuf;          // ring holding the window at step start
+  uint64_t g_head, g_tail, ra0;  // window at step start; first ring chunk's start
+  int64_t nrch;          // ring chunks over the window
+  int64_t live_old;      // live ghost entries at step start
+  int64_t X;             // oldest live entries the pushes trim (may exceed live_old)
+  int64_t born;          // pushes trimmed at once: max(0, X - live_old)
+  uint64_t pbase;        // push t (t >= born) goes to position pbase + t
+  uint64_t q;            // new window start without compaction
+  uint64_t gctr0;        // ghost counter at step start
+  int64_t n_ins, hits;   // inserted blocks; ghost hits among them
+};
+
 // Per-call arguments of a step or probe, in device memory: the step's kernels
 // read them at entry, so one captured CUDA graph serves every step.
 struct StepArgs {
@@ -224,14 +265,17 @@ struct DevState {
   uint32_t* blk_pin;       // step tag: hit in this step
   uint32_t* blk_inval;     // step tag: invalidated in this step
   uint32_t* res_bits;      // resident bitmap
-  uint32_t* s3_prev;       // S3-FIFO queue links: toward the tail (older)
-  uint32_t* s3_next;       //                      toward the head (newer)
-  uint32_t* s3_inval;      // blocks invalidated this step (to unlink)
-  TableEntry* ghost_map;   // (group, key) -> ring position (in blk)
+  // S3-FIFO queues: per buffer, the small queue's ids then the main queue's,
+  // each in a region of s3_np entries, oldest first (sequence order)
+  int64_t s3_np;           // region stride: N rounded up to a whole chunk
+  int64_t s3_nch;          // chunks a region can hold
+  int64_t s3_nrch;         // chunks a ghost ring can hold (plus one)
+  uint32_t* s3_arr;        // [2][2][s3_np]
+  TableEntry* ghost_map;   // (group, key) -> ring index (in blk)
   uint32_t* ghost_ovf;
-  uint64_t* ghost_ring_key;
-  uint32_t* ghost_ring_grp;
-  uint64_t* ghost_ring_seq;
+  uint64_t* ghost_sq;      // per map slot: the entry's ghost sequence number
+  uint32_t* ghost_ring;    // [2][ghost_ring_cap] map slot of each FIFO position
+  uint32_t* ghost_bits;    // [2][ghost_ring_cap / 32] live FIFO positions
   TableEntry* table;
   uint32_t* table_ovf;     // per bucket: live keys probing past it
   int64_t* ledger;         // B_{g,c}, fixed point
@@ -284,6 +328,15 @@ struct DevState {
   uint32_t* lst_blk;
   uint16_t* lst_seg;
   int32_t* bm_chunk_cnt;   // [3][chunks] bitmap compaction counts
+  // S3-FIFO per-step scratch
+  uint8_t* s3_attr;        // [2][s3_np] per queue entry: bit0 live, bit1 unpinned, bits 4-7 frequency
+  S3Chunk* s3_ck;          // [2][s3_nch] per-chunk counts
+  S3Base* s3_base;         // [2][s3_nch] per-chunk exclusive bases
+  uint32_t* s3_rck;        // [s3_nrch] live ghost entries per ring chunk of the window
+  uint32_t* s3_rbase;      // [s3_nrch] their exclusive prefix
+  S3Plan* s3_plan;
+  uint8_t* s3_hit;         // [max_blocks] inserted block found in the ghost
+  uint32_t* s3_ick;        // [max_blocks / kS3Chunk + 1] ghost hits per chunk of inserts
   // indexed queues (allocated only with PS_FLAG_INDEXED_QUEUES)
   int32_t lg_on;           // victims come from the queues instead of a candidate scan
   int32_t lg_L;            // logs: 3G + 3
@@ -408,8 +461,11 @@ int32_t launch_queue_select(const DevState& s, cudaStream_t st, const CaptureCtx
                             bool plain_first, int* launches);
 int32_t launch_queue_append(const DevState& s, cudaStream_t st, const CaptureCtx* cap, int* launches);
 // S3-FIFO (ps_s3fifo.cu)
-void launch_s3_evict(const DevState& s, cudaStream_t st);
-void launch_s3_insert(const DevState& s, cudaStream_t st);
+// The select: per-chunk counts, the closed-form plan, the sequential kernel
+// (used when the plan does not apply), the plan's application.
+int32_t launch_s3_select(const DevState& s, cudaStream_t st, int* launches);
+// After the insertions: ghost lookups of the new blocks, their array places.
+int32_t launch_s3_insert(const DevState& s, cudaStream_t st, int* launches);
 // A step's outputs (device) written into page-locked host buffers, the id
 // lists by their device-side counts (ps_step_host_async).
 void launch_host_out(const ps_step_out_t& dev, const ps_step_out_t& host, int32_t R, int32_t G, cudaStream_t st);

@@ -188,10 +188,8 @@ __device__ uint32_t claim_insert(const DevState& s, uint64_t key, uint32_t req) 
 __device__ uint32_t drop_block(const DevState& s, uint32_t b, bool clear_res = true) {
   table_delete(s, b);
   const uint32_t g = s.blk_group[b];
-  const uint8_t fl = s.blk_flags[b];
   s.blk_flags[b] = 0;
   if (clear_res) atomicAnd(s.res_bits + (b >> 5), ~(1u << (b & 31)));
-  if (s.policy == PS_S3FIFO) atomic_add_i64((fl & 2) ? &s.ctl->s3_nM : &s.ctl->s3_nS, -1);
   return g;
 }
 
@@ -220,8 +218,6 @@ __global__ void k_init_ctl(DevState s) {
     Ctl c{};
     c.step = 1;
     c.stamp_base = 1;
-    c.s3_head[0] = c.s3_head[1] = kNone;
-    c.s3_tail[0] = c.s3_tail[1] = kNone;
     *s.ctl = c;
   }
   for (int i = threadIdx.x; i < s.G * s.C; i += blockDim.x) s.ledger[i] = s.beta[i % s.C];
@@ -375,7 +371,6 @@ __global__ void __launch_bounds__(kValTile) k_validate(DevState s, int probe) {
     c->n_alloc = 0; c->n_victims_marked = 0; c->m_fb = 0; c->sel_ntie = 0; c->sel_k = 0; c->ticket = 0;
     c->internal_error = (vb & 2) ? 1 : 0;
     c->nlaunch = 1;  // this kernel; every later kernel of the step adds itself
-    c->s3_pinned[0] = 0; c->s3_pinned[1] = 0; c->s3_ninval = 0;
   }
 }
 
@@ -576,7 +571,6 @@ __device__ __forceinline__ bool hash_lookup_chunk(const DevState& s, Ctl* c, con
     if (in_prefix) {
       newpin = atomicExch(s.blk_pin + blk, step32) != step32;
       if (newpin && s.lg_on) pin_klass = s.blk_klass[blk];
-      if (newpin && s.policy == PS_S3FIFO) atomic_add_i64(&c->s3_pinned[(s.blk_flags[blk] >> 1) & 1], 1);
       s.pos_claim[p] = kNone;
     } else {
       s.pos_claim[p] = claim_insert(s, key, i);
@@ -729,7 +723,6 @@ __global__ void __launch_bounds__(kThreads) k_claims(DevState s) {
         ginv = drop_block(s, b);
         if (s.lg_on) kinv = s.blk_klass[b];
         atomicOr(s.bm_inval + (b >> 5), 1u << (b & 31));
-        if (s.policy == PS_S3FIFO) s.s3_inval[atomicAdd(reinterpret_cast<unsigned long long*>(&c->s3_ninval), 1ull)] = b;
         inv = true;
       }
     }
@@ -2102,7 +2095,6 @@ __global__ void __launch_bounds__(kThreads) k_insert(DevState s) {
         const uint16_t ogrp = s.blk_group[b];
         if (ofl & 1) {
           table_delete_known(s, oslot, okey, ogrp);
-          if (s.policy == PS_S3FIFO) atomic_add_i64((ofl & 2) ? &c->s3_nM : &c->s3_nS, -1);
           gold = ogrp;
           evicted = true;
         }
@@ -2147,6 +2139,17 @@ __global__ void k_finalize(DevState s) {
   c->t_prev = s.now;
   c->step += 1;
   c->stamp_base += c->nblocks;
+  if (s.policy == PS_S3FIFO) {  // the queue arrays the step wrote become current
+    const S3Plan* pl = s.s3_plan;
+    const int64_t n_ins = c->need < c->n_alloc ? c->need : c->n_alloc;
+    c->s3_len[0] = pl->nKeepS + n_ins - pl->hits;
+    c->s3_len[1] = pl->nKeepM + pl->nMid + pl->hits;
+    c->s3_buf ^= 1;
+    c->s3_ctr = pl->ctr_end + (uint64_t)n_ins;
+    c->ghost_live -= pl->hits;
+    c->s3_nS = c->s3_len[0];
+    c->s3_nM = c->s3_len[1];
+  }
 }
 
 // Read-only probe output: h_i per request, and the probe's status.
@@ -2325,8 +2328,8 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));  // after the join: plain
     select(1, 0);
-  } else {
-    PS_LAUNCH(launch_s3_evict(s, st));
+  } else if (launch_s3_select(s, st, &launches) != PS_OK) {
+    return PS_ERR_CUDA;
   }
   mark(7);
   const int nchunks = (int)((s.nwords + kBmChunk - 1) / kBmChunk);
@@ -2341,7 +2344,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   } else {
     PS_LAUNCH(launch_k(k_insert, pgrid, kThreads, 0, st, s));
   }
-  if (s.policy == PS_S3FIFO) PS_LAUNCH(launch_s3_insert(s, st));
+  if (s.policy == PS_S3FIFO && launch_s3_insert(s, st, &launches) != PS_OK) return PS_ERR_CUDA;
   if (s.lg_on && launch_queue_append(s, st, cap, &launches) != PS_OK) return PS_ERR_CUDA;
   mark(10);
   PS_LAUNCH(launch_k(k_finalize, 1, 32, 0, st, s));
