@@ -83,6 +83,16 @@ enum {
  * 1024-entry chunk, so a take that needs more finishes in the second round.
  * Same results, slower; it exercises the second round on small pools. */
 #define PS_FLAG_QUEUE_SHORT_WINDOWS 8u
+/* With s3fifo: the ghost FIFO's live entries are compacted into its second
+ * ring on every step that has any (normally only when the ring lacks room for
+ * the step's pushes).  Same results, slower; it exercises the compaction on
+ * small pools. */
+#define PS_FLAG_S3_COMPACT_GHOST 16u
+/* With s3fifo: every step's evictions run the published one-at-a-time loop on
+ * one device thread instead of the closed form computed in parallel (which
+ * falls back to that loop only where it does not apply).  Same results,
+ * slower; it checks the sequential kernel over whole traces. */
+#define PS_FLAG_S3_SEQUENTIAL 32u
 
 /* Per-group statistics, int64 each, row-major [num_groups][PS_NUM_STATS]. */
 enum {

@@ -31,6 +31,9 @@ FLAG_NO_SEGMENTATION, FLAG_NO_DEBT_GATE = 1, 2
 # the CUDA library's indexed-queue victim selection: same victims, ignored here
 FLAG_INDEXED_QUEUES = 4
 FLAG_QUEUE_SHORT_WINDOWS = 8
+# the CUDA library's S3-FIFO execution choices: same results, ignored here
+FLAG_S3_COMPACT_GHOST = 16
+FLAG_S3_SEQUENTIAL = 32
 
 
 class OrcParams(C.Structure):

@@ -28,6 +28,7 @@ STAT_NAMES = (
 POLICIES = {"lru": 0, "s3fifo": 1, "prefixshield": 2, "staticquota": 3}
 PS_OK, PS_ERR_INVALID_ARG, PS_ERR_CAPACITY, PS_ERR_CLOCK, PS_ERR_CUDA = 0, -1, -2, -3, -4
 PS_FLAG_NO_SEGMENTATION, PS_FLAG_NO_DEBT_GATE, PS_FLAG_INDEXED_QUEUES, PS_FLAG_QUEUE_SHORT_WINDOWS = 1, 2, 4, 8
+PS_FLAG_S3_COMPACT_GHOST, PS_FLAG_S3_SEQUENTIAL = 16, 32
 
 EXPORTED = ("ps_workspace_bytes", "ps_create", "ps_step", "ps_step_host", "ps_step_host_async",
             "ps_step_host_wait", "ps_stats", "ps_clear_status",

@@ -406,7 +406,7 @@ __global__ void __launch_bounds__(kPT) k_s3_plan(DevState s) {
   __syncthreads();
   const int64_t nL = UMo + MA;
   const int64_t mB = m - kS;
-  if (cap >= (uint32_t)kS3Bins || mB > nL) {  // the closed form does not apply: sequential kernel
+  if (cap >= (uint32_t)kS3Bins || mB > nL || (s.flags & PS_FLAG_S3_SEQUENTIAL)) {  // sequential kernel
     if (threadIdx.x == 0) pl->fb = 1;
     return;
   }
@@ -505,7 +505,8 @@ __global__ void __launch_bounds__(kPT) k_s3_plan(DevState s) {
   const int64_t X = live_old + kS - s.s3_ghost_cap;
   const int64_t Xo = tmin<int64_t>(tmax<int64_t>(X, 0), live_old);
   const int64_t born = tmax<int64_t>(X - live_old, 0);
-  const int gc = (int64_t)(head - tail) + kS > (int64_t)s.ghost_ring_cap ? 1 : 0;
+  const int gc = ((int64_t)(head - tail) + kS > (int64_t)s.ghost_ring_cap ||
+                  ((s.flags & PS_FLAG_S3_COMPACT_GHOST) && head > tail)) ? 1 : 0;
   const uint64_t a0 = tail & ~(uint64_t)(kS3Chunk - 1);
   const int64_t nrch = head > tail ? cdiv64((int64_t)(head - a0), kS3Chunk) : 0;
   if (threadIdx.x == 0) gq = tail;
@@ -703,7 +704,7 @@ __global__ void k_s3_fallback(DevState s) {
     ++tail;
   }
   uint64_t pbase = head;
-  if ((int64_t)(head - tail) + kS > (int64_t)rcap) {
+  if ((int64_t)(head - tail) + kS > (int64_t)rcap || ((s.flags & PS_FLAG_S3_COMPACT_GHOST) && head > tail)) {
     uint32_t* nring = ring_of(s, rb ^ 1);
     uint32_t* nbits = bits_of(s, rb ^ 1);
     uint64_t w = 0;
