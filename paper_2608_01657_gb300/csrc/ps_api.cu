@@ -76,13 +76,14 @@ KeySchedule key_schedule(uint64_t seed, int32_t bs) {
   k.kd = splitmix_next(&st) % kP61;
   if (k.kc == 0) k.kc = 1;
   if (k.kd == 0) k.kd = 1;
-  // Kc^j for j = 0..kSegBlocks, then Kc^(kSegBlocks t) for t = 0..32
+  // Kc^j for j = 0..kSegBlocks
   k.kc_pow.resize(2 * (kSegBlocks + 1));
   k.kc_pow[0] = 1;
   for (int j = 1; j <= kSegBlocks; ++j) k.kc_pow[j] = host_mul61(k.kc_pow[j - 1], k.kc);
+  // then the powers of Kc^kChunkBlocks (one chunk's multiplier), t = 0..kSegBlocks
+  const uint64_t kc_chunk = host_mul61(k.kc_pow[kSegBlocks], k.kc_pow[kSegBlocks]);
   k.kc_pow[kSegBlocks + 1] = 1;
-  for (int t = 1; t <= kSegBlocks; ++t)
-    k.kc_pow[kSegBlocks + 1 + t] = host_mul61(k.kc_pow[kSegBlocks + t], k.kc_pow[kSegBlocks]);
+  for (int t = 1; t <= kSegBlocks; ++t) k.kc_pow[kSegBlocks + 1 + t] = host_mul61(k.kc_pow[kSegBlocks + t], kc_chunk);
   return k;
 }
 
@@ -156,7 +157,7 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   d.N = N; d.bs = bs; d.G = G; d.C = P->num_contracts; d.max_requests = max_requests;
   d.max_tokens = max_tokens;
   d.max_blocks = max_tokens / bs;
-  d.max_segments = d.max_blocks / kSegBlocks + max_requests + 1;
+  d.max_segments = d.max_blocks / kChunkBlocks + max_requests + 1;
   d.nwords = (N + 31) / 32;
   // native table: 8-way buckets at load <= 1/2
   // 8-way buckets for 4N entries: at most a quarter full, so a probe rarely
@@ -252,7 +253,7 @@ size_t carve(const Dims& d, char* base, DevState* s, ps_handle* h) {
   t.pos_req = cv.take<uint32_t>(B);
   t.pos_m = cv.take<uint32_t>(B);
   t.chunks = cv.take<ChunkDesc>((size_t)d.max_segments);
-  t.val_tile = cv.take<uint64_t>(R / 256 + 1);
+  t.val_tile = cv.take<uint64_t>(R / kValTile + 1);
   t.seg_word = cv.take<uint64_t>((size_t)d.max_segments);
   t.pos_blk = cv.take<uint32_t>(B);
   t.pos_claim = cv.take<uint32_t>(B);

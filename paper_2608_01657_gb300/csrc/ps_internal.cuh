@@ -24,8 +24,10 @@ constexpr int kTableWays = 8;    // native prefix table: 8 x 16 B entries per 12
 constexpr int kClaimWays = 4;    // per-step claim map: 4 x 32 B entries per bucket
 constexpr int kRadixBits = 8;
 constexpr int kRadixBins = 1 << kRadixBits;
-constexpr int kSegBlocks = 32;   // blocks of one prompt hashed by one warp (a chunk)
+constexpr int kSegBlocks = 32;   // blocks of one chunk half (a warp's width)
+constexpr int kChunkBlocks = 2 * kSegBlocks;  // blocks of one prompt hashed by one warp (a chunk)
 constexpr int kBmChunk = 256;    // bitmap words per CTA of the id-list compaction
+constexpr int kValTile = 256;    // requests per CTA of the input validation (one published total each)
 constexpr uint64_t kP61 = (1ull << 61) - 1;  // chain modulus, a Mersenne prime
 
 // Recency stamp (native free-queue order): larger = more recently released.
@@ -109,7 +111,7 @@ struct Ctl {
   uint64_t v_sum;          // k_validate: blocks (high half) and chunks (low half) of the call
 };
 
-// One hashing chunk: up to kSegBlocks consecutive blocks of one request.
+// One hashing chunk: up to kChunkBlocks consecutive blocks of one request.
 struct __align__(16) ChunkDesc {
   int64_t o0;      // the request's first token
   uint32_t req;    // request index
@@ -282,7 +284,7 @@ struct DevState {
   int64_t* ledger_b0;      // per step: B_{g,c} refilled to now, before the step's charges
   int32_t* contract_of_group;
   uint32_t* key_words;     // NH key schedule, bs + 2 words
-  uint64_t* kc_pow;        // Kc^k mod p, k = 0..kSegBlocks, then Kc^(kSegBlocks t), t = 0..32
+  uint64_t* kc_pow;        // Kc^k mod p, k = 0..kSegBlocks, then Kc^(kChunkBlocks t), t = 0..kSegBlocks
   int64_t* stats;          // [G][PS_NUM_STATS]
   HistEntry* hist;
   // per-step scratch

@@ -233,7 +233,6 @@ __global__ void k_init_ctl(DevState s) {
 // and per-step scalars, and clears the tile words for the next call.
 // 'probe' skips the clock and step checks.  Every write is bounds-checked, so
 // inputs that turn out invalid write nothing outside the scratch arrays.
-constexpr int kValTile = 256;
 constexpr uint64_t kTileFlag = 1ull << 63;
 
 __global__ void __launch_bounds__(kValTile) k_validate(DevState s, int probe) {
@@ -263,7 +262,7 @@ __global__ void __launch_bounds__(kValTile) k_validate(DevState s, int probe) {
     if (s.in_prefix) bad |= s.in_prefix[i] == 0;
     n = bad ? 0 : (int32_t)nb;
   }
-  ns = (n + kSegBlocks - 1) / kSegBlocks;
+  ns = (n + kChunkBlocks - 1) / kChunkBlocks;
   const int tile_bad = __syncthreads_or(bad);
   // blocks in the high half, chunks in the low half of one scanned word
   uint64_t tot;
@@ -380,17 +379,21 @@ __global__ void __launch_bounds__(kValTile) k_validate(DevState s, int probe) {
 // cached prefix, the claims of every block past it, and each request's
 // history entry (OnRequest of Alg. 1).
 //
-// A chunk is up to kSegBlocks = 32 consecutive blocks of one prompt; one warp
-// takes one chunk, one lane one block.  Chunks are numbered in request order
-// (a request's chunks are consecutive) and CTAs draw their chunks in that
-// order from a ticket, so every chunk's predecessors belong to warps that
-// have already started.  Each lane reads its block's tokens with 16-byte
-// loads and forms the block digest D_m itself.  The chain
-// C_m = Kc C_{m-1} + D_m (mod 2^61 - 1) composes affine maps, so a warp scan
-// gives each block its chain value B_m relative to the chunk's start (value 0
-// entering it), and the chunk's total (B at its last block) is published
-// under a flag.  The value entering chunk k of a request is then
-//   Kc^(32k) C_seed + sum_{l<k} Kc^(32(k-1-l)) total_l,
+// A chunk is up to kChunkBlocks = 64 consecutive blocks of one prompt; one
+// warp takes one chunk, lane l its blocks l and 32 + l (two halves).  Chunks
+// are numbered in request order (a request's chunks are consecutive) and CTAs
+// draw their chunks in that order from a ticket, so every chunk's
+// predecessors belong to warps that have already started.  Each lane reads
+// its blocks' tokens with 16-byte loads and forms the block digests D_m
+// itself.  The chain C_m = Kc C_{m-1} + D_m (mod 2^61 - 1) composes affine
+// maps, so a warp scan of each half gives each block its chain value B_m
+// relative to the half's start (value 0 entering it); the chunk's total, the
+// second half's total plus Kc^(its blocks) times the first's, is published
+// under a flag.  (Two blocks a lane halve the chunks, and with them the
+// chain of dependent accesses each one pays: ticket, descriptor,
+// predecessors' totals and miss bits.)  The value entering chunk k of a
+// request is then
+//   Kc^(64k) C_seed + sum_{l<k} Kc^(64(k-1-l)) total_l,
 // and no total waits on anything, so the warp folds its k predecessors'
 // totals directly, in windows of 32 (one lane each).  With C_m the lanes form
 // their keys and probe the table.  A block is in the cached prefix iff no
@@ -496,26 +499,40 @@ __device__ __forceinline__ bool hash_lookup_chunk(const DevState& s, Ctl* c, con
   const int n = d.n;
   const int64_t sb = d.sb;
   const int k = d.k;  // chunk index within the request
-  const int m0 = k * kSegBlocks;
-  const int nb = tmin(kSegBlocks, n - m0);
+  const int m0 = k * kChunkBlocks;
+  const int nb = tmin(kChunkBlocks, n - m0);
+  const int nbA = tmin(kSegBlocks, nb), nbB = nb - nbA;  // blocks of the two halves
   const int64_t o0 = d.o0;
   const int pbase = d.pbase;
   const uint32_t g = d.group;
   const int64_t T = c->T;
-  const int m = m0 + lane;
-  // D_m, then the inclusive scan of the affine maps x -> Kc x + D
-  uint64_t bb = 0;
-  if (lane < nb) {
+  const int mA = m0 + lane, mB = m0 + kSegBlocks + lane;
+  // D_m of the lane's two blocks, then the inclusive scans of the affine maps
+  // x -> Kc x + D, one per half
+  uint64_t bA = 0, bB = 0;
+  if (lane < nbA) {
     uint64_t d1, d2;
-    block_nh<BS>(s, sk, o0 + (int64_t)m * BS, (int)(o0 & 3), s.tokens_aligned16 != 0, T, &d1, &d2);
-    bb = add61(red61(d1), mul61(s.digest_mul, red61(d2)));
+    block_nh<BS>(s, sk, o0 + (int64_t)mA * BS, (int)(o0 & 3), s.tokens_aligned16 != 0, T, &d1, &d2);
+    bA = add61(red61(d1), mul61(s.digest_mul, red61(d2)));
+  }
+  if (lane < nbB) {
+    uint64_t d1, d2;
+    block_nh<BS>(s, sk, o0 + (int64_t)mB * BS, (int)(o0 & 3), s.tokens_aligned16 != 0, T, &d1, &d2);
+    bB = add61(red61(d1), mul61(s.digest_mul, red61(d2)));
   }
 #pragma unroll
   for (int q = 0; q < 5; ++q) {
-    const uint64_t t = __shfl_up_sync(kFull, bb, 1 << q);
-    if (lane >= (1 << q)) bb = add61(bb, mul61(kc[1 << q], t));
+    const uint64_t tA = __shfl_up_sync(kFull, bA, 1 << q);
+    const uint64_t tB = __shfl_up_sync(kFull, bB, 1 << q);
+    if (lane >= (1 << q)) {
+      bA = add61(bA, mul61(kc[1 << q], tA));
+      bB = add61(bB, mul61(kc[1 << q], tB));
+    }
   }
-  const uint64_t total = __shfl_sync(kFull, bb, nb - 1);
+  const uint64_t totA = __shfl_sync(kFull, bA, nbA - 1);
+  const uint64_t totB = __shfl_sync(kFull, bB, nbB > 0 ? nbB - 1 : 0);
+  // a second half follows a full first half (Kc^32 times it)
+  const uint64_t total = nbB > 0 ? add61(mul61(kc[nbB], totA), totB) : totA;
   if (lane == 0) st_relaxed_u64(s.seg_word + j, total | kWordTotal);
   // the chain value entering the chunk
   bool ok = true;
@@ -532,16 +549,24 @@ __device__ __forceinline__ bool hash_lookup_chunk(const DevState& s, Ctl* c, con
     for (int o = 16; o > 0; o >>= 1) term = add61(term, __shfl_xor_sync(kFull, term, o));
     cin = add61(mul61(kc[(kSegBlocks + 1) + w], cin), term);
   }
-  // the lane's key and its table probe
-  uint64_t key = 0;
-  uint32_t blk = kNone;
-  if (lane < nb) {
-    const uint64_t C = add61(mul61(kc[lane + 1], cin), bb);
-    key = fix_reserved(mix64(C ^ ((uint64_t)(m + 1) * 0xD1B54A32D192ED03ull)));
-    blk = table_find(s, key, g);
+  // the lane's keys and their table probes
+  uint64_t keyA = 0, keyB = 0;
+  uint32_t blkA = kNone, blkB = kNone;
+  if (lane < nbA) {
+    const uint64_t C = add61(mul61(kc[lane + 1], cin), bA);
+    keyA = fix_reserved(mix64(C ^ ((uint64_t)(mA + 1) * 0xD1B54A32D192ED03ull)));
   }
-  const unsigned missmask = __ballot_sync(kFull, lane < nb && blk == kNone);
-  if (lane == 0) st_relaxed_u64(s.seg_word + j, total | kWordTotal | kWordMiss | (missmask ? kWordMissBit : 0));
+  if (lane < nbB) {
+    const uint64_t cinB = add61(mul61(kc[kSegBlocks], cin), totA);
+    const uint64_t C = add61(mul61(kc[lane + 1], cinB), bB);
+    keyB = fix_reserved(mix64(C ^ ((uint64_t)(mB + 1) * 0xD1B54A32D192ED03ull)));
+  }
+  if (lane < nbA) blkA = table_find(s, keyA, g);
+  if (lane < nbB) blkB = table_find(s, keyB, g);
+  const unsigned missA = __ballot_sync(kFull, lane < nbA && blkA == kNone);
+  const unsigned missB = __ballot_sync(kFull, lane < nbB && blkB == kNone);
+  const bool anymiss = (missA | missB) != 0;
+  if (lane == 0) st_relaxed_u64(s.seg_word + j, total | kWordTotal | kWordMiss | (anymiss ? kWordMissBit : 0));
   // did any earlier block of the request miss?
   bool missbefore = false;
   for (int l0 = 0; l0 < k && !missbefore; l0 += 32) {
@@ -555,36 +580,46 @@ __device__ __forceinline__ bool hash_lookup_chunk(const DevState& s, Ctl* c, con
     missbefore = __any_sync(kFull, mb);
   }
   if (!__all_sync(kFull, ok)) return false;  // a predecessor never published
-  const int first = missmask ? __ffs(missmask) - 1 : kSegBlocks;  // first miss in this chunk
-  if (!missbefore && missmask && lane == 0) s.rq_h[i] = m0 + first;  // h_i: its only writer
+  // first miss in this chunk
+  const int first = missA ? __ffs(missA) - 1 : (missB ? kSegBlocks + __ffs(missB) - 1 : kChunkBlocks);
+  if (!missbefore && anymiss && lane == 0) s.rq_h[i] = m0 + first;  // h_i: its only writer
   if (probe) return true;
-  const bool in_prefix = lane < nb && !missbefore && lane < first;
   const uint32_t step32 = (uint32_t)c->step;
-  bool newpin = false;
-  uint32_t pin_klass = 0;
-  if (lane < nb) {
-    const int64_t p = pbase + m;
+  // the cached prefix is pinned, every later block claimed
+  auto place = [&](bool act, int half, uint64_t key, uint32_t blk, uint32_t* klass) -> bool {
+    if (!act) return false;
+    const int mm = m0 + half * kSegBlocks + lane;
+    const int64_t p = pbase + mm;
     s.pos_key[p] = key;
     s.pos_req[p] = i;
-    s.pos_m[p] = (uint32_t)m;
+    s.pos_m[p] = (uint32_t)mm;
     s.pos_blk[p] = blk;
-    if (in_prefix) {
-      newpin = atomicExch(s.blk_pin + blk, step32) != step32;
-      if (newpin && s.lg_on) pin_klass = s.blk_klass[blk];
+    bool pinned = false;
+    if (!missbefore && half * kSegBlocks + lane < first) {
+      pinned = atomicExch(s.blk_pin + blk, step32) != step32;
+      if (pinned && s.lg_on) *klass = s.blk_klass[blk];
       s.pos_claim[p] = kNone;
     } else {
       s.pos_claim[p] = claim_insert(s, key, i);
     }
-  }
-  const int np = __popc(__ballot_sync(kFull, newpin));
+    return pinned;
+  };
+  uint32_t klassA = 0, klassB = 0;
+  const bool pinA = place(lane < nbA, 0, keyA, blkA, &klassA);
+  const bool pinB = place(lane < nbB, 1, keyB, blkB, &klassB);
+  const int np = __popc(__ballot_sync(kFull, pinA)) + __popc(__ballot_sync(kFull, pinB));
   if (lane == 0 && np) atomic_add_i64(&c->pinned, np);
   // hits are namespaced by group: every block the warp pins is group g's
   if (s.policy == PS_STATICQUOTA && lane == 0 && np) atomic_add_i64(s.grp_pinned + g, np);
   if (s.lg_on) {  // a pinned block is no candidate: it leaves its queues' live counts (applied in k_lg_cand)
-    const int32_t A = lg_log_a(s, g, pin_klass), B = lg_log_b(s, pin_klass);
-    agg_add_i64(s.lg_pin, (uint32_t)A, 1, newpin && A >= 0);
-    agg_add_i64(s.lg_pin, (uint32_t)B, 1, newpin && B >= 0);
+    const int32_t A1 = lg_log_a(s, g, klassA), B1 = lg_log_b(s, klassA);
+    agg_add_i64(s.lg_pin, (uint32_t)A1, 1, pinA && A1 >= 0);
+    agg_add_i64(s.lg_pin, (uint32_t)B1, 1, pinA && B1 >= 0);
+    const int32_t A2 = lg_log_a(s, g, klassB), B2 = lg_log_b(s, klassB);
+    agg_add_i64(s.lg_pin, (uint32_t)A2, 1, pinB && A2 >= 0);
+    agg_add_i64(s.lg_pin, (uint32_t)B2, 1, pinB && B2 >= 0);
   }
+  const uint64_t key = keyA;  // block 0's key, in the first chunk's lane 0
   // OnRequest of Alg. 1: the request's (group, prefix) history entry
   if (k == 0 && lane == 0) {
     const uint64_t pid = s.in_prefix ? s.in_prefix[i] : key;  // default: block 0's key
@@ -619,7 +654,7 @@ __device__ __forceinline__ bool hash_lookup_chunk(const DevState& s, Ctl* c, con
 // tickets, each held by a running warp: the waits always make progress.
 // probe = 1: the read-only probe (ps_cached_prefix): h_i only, no pins,
 // claims, history or per-position records.
-constexpr int kHashCtasPerSm = 6;
+constexpr int kHashCtasPerSm = 5;
 template <int BS>
 __global__ void __launch_bounds__(256, kHashCtasPerSm) k_hash_lookup(DevState s, int probe) {
   s = with_args(s);

@@ -23,7 +23,7 @@ using namespace ps;
 // Maximum sizes of one call: 4096 requests and 131072 full blocks.
 constexpr int64_t kNaMaxRequests = 4096;
 constexpr int64_t kNaMaxBlocks = 131072;
-constexpr int64_t kNaMaxSegments = kNaMaxBlocks / kSegBlocks + kNaMaxRequests + 1;
+constexpr int64_t kNaMaxSegments = kNaMaxBlocks / kChunkBlocks + kNaMaxRequests + 1;
 
 // Byte layout of the scratch array, every region 256-byte aligned.
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -31,7 +31,7 @@ constexpr size_t kOffCtl = 0;
 constexpr size_t kOffRq = align256(kOffCtl + sizeof(Ctl));
 constexpr size_t kRqArrays = 5;  // n, h, s, fu, pbase
 constexpr size_t kOffTile = align256(kOffRq + kRqArrays * align256(4 * kNaMaxRequests));
-constexpr size_t kOffSeg = align256(kOffTile + 8 * (kNaMaxRequests / 256 + 1));
+constexpr size_t kOffSeg = align256(kOffTile + 8 * (kNaMaxRequests / kValTile + 1));
 constexpr size_t kOffPos = align256(kOffSeg + align256(sizeof(ChunkDesc) * kNaMaxSegments) + align256(8 * kNaMaxSegments));
 constexpr size_t kScratchBytes = align256(kOffPos + align256(8 * kNaMaxBlocks) + 2 * align256(4 * kNaMaxBlocks));
 
@@ -86,7 +86,7 @@ extern "C" int32_t ps_cached_prefix_noalloc(ps_handle_t* h, void* stream, int32_
     s.max_blocks = kNaMaxBlocks;
     s.max_tokens = kNaMaxBlocks * s.bs;
   }
-  s.max_segments = s.max_blocks / kSegBlocks + s.max_requests + 1;
+  s.max_segments = s.max_blocks / kChunkBlocks + s.max_requests + 1;
   // per-call scratch, carved from the static array
   const size_t rq = align256(4 * kNaMaxRequests);
   s.ctl = reinterpret_cast<Ctl*>(base + kOffCtl);
