@@ -343,17 +343,22 @@ __global__ void __launch_bounds__(kValTile) k_validate(DevState s, int probe) {
   __threadfence();
   for (int t = threadIdx.x; t < (int)gridDim.x; t += blockDim.x) s.val_tile[t] = 0;
   if (threadIdx.x != 0) return;
+  // every value the verdict needs, loaded up front so the loads overlap
   const uint32_t vb = ldcg_u32(&c->v_bad);
   const uint64_t all = ldcg_u64(&c->v_sum);  // blocks (high half) and chunks (low half) of the step
+  const int64_t T = R > 0 ? s.in_offsets[R] : 0;
+  const int64_t first_off = R > 0 ? s.in_offsets[0] : 0;
+  const int32_t sticky = c->sticky;
+  const int64_t t_prev = c->t_prev;
+  const uint64_t step = c->step;
   c->v_bad = 0;
   c->v_ticket = 0;
   c->v_sum = 0;
-  const int64_t T = R > 0 ? s.in_offsets[R] : 0;
   int32_t st = PS_OK;
-  if (!probe && c->sticky != PS_OK) st = c->sticky;
-  else if (!probe && s.now < c->t_prev) st = PS_ERR_CLOCK;
-  else if (!probe && c->step > kMaxStep) st = PS_ERR_CAPACITY;
-  else if (vb || (R > 0 && s.in_offsets[0] != 0) || T > s.max_tokens) st = PS_ERR_INVALID_ARG;
+  if (!probe && sticky != PS_OK) st = sticky;
+  else if (!probe && s.now < t_prev) st = PS_ERR_CLOCK;
+  else if (!probe && step > kMaxStep) st = PS_ERR_CAPACITY;
+  else if (vb || first_off != 0 || T > s.max_tokens) st = PS_ERR_INVALID_ARG;
   c->status = st;
   c->T = T;
   c->hash_ticket = 0;
