@@ -129,13 +129,18 @@ __device__ void gh_erase_known(const DevState& s, uint32_t slot, uint64_t key, u
   uint32_t x = table_home(key, g, s.gh_nbuckets_log2);
   for (uint32_t it = 0; x != bucket && it <= mask; ++it, x = (x + 1) & mask) atomicSub(s.ghost_ovf + x, 1u);
 }
-// Release a slot, reading its key and group first (another thread may take
-// the slot as soon as it is released).
+// Release a slot, reading its key and group first.  Erasures and insertions
+// never run in the same kernel (a step's pushes are inserted by k_s3_push,
+// after the trimming), so no other thread rewrites the slot meanwhile.
 __device__ void gh_erase(const DevState& s, uint32_t slot) {
   const uint64_t key = __ldcg(reinterpret_cast<const unsigned long long*>(&s.ghost_map[slot].key));
   const uint32_t g = __ldcg(&s.ghost_map[slot].grp);
-  __threadfence();
   gh_erase_known(s, slot, key, g);
+}
+// The step's small-queue victims in eviction order (their ghost pushes): the
+// second half of the candidate-key scratch, which S3-FIFO does not use.
+__device__ __forceinline__ uint32_t* push_list(const DevState& s) {
+  return reinterpret_cast<uint32_t*>(s.csk) + s.N;
 }
 
 // A locate of the planner found nothing (never expected): the step goes to
@@ -599,7 +604,7 @@ __global__ void k_s3_fallback(DevState s) {
   const uint32_t step32 = (uint32_t)c->step;
   const uint32_t mm = (uint32_t)s.s3_move_min;
   uint32_t* um = reinterpret_cast<uint32_t*>(s.csk);  // the main queue's unpinned members: a ring of N
-  uint32_t* pushes = um + N;                          // the step's small-queue victims, in order
+  uint32_t* pushes = push_list(s);                    // the step's small-queue victims, in order
   auto live = [&](uint32_t b) { return (s.blk_flags[b] & 1) != 0; };
   auto unpinned = [&](uint32_t b) { return live(b) && s.blk_pin[b] != step32; };
   int64_t uh = 0, ut = 0, ucount = 0;
@@ -749,10 +754,12 @@ __global__ void k_s3_fallback(DevState s) {
 }
 
 // ===========================================================================
-// 4. The plan applied, chunk by chunk: victims, the small queue's ghost
-//    pushes, moves and main-queue visits (frequency, sequence number), the new
-//    arrays' kept and re-sequenced parts; ring chunks of the FIFO window are
-//    trimmed, or compacted into the other ring.
+// 4. The plan applied, chunk by chunk: victims (the small queue's listed in
+//    eviction order for their ghost pushes), moves and main-queue visits
+//    (frequency, sequence number), the new arrays' kept and re-sequenced
+//    parts; ring chunks of the FIFO window are trimmed, or compacted into the
+//    other ring.  The ring chunks with work come first, so that no CTA takes
+//    both a trimming chunk and a small-queue chunk before the others start.
 __global__ void __launch_bounds__(kCT) k_s3_apply(DevState s) {
   s = with_args(s);
   Ctl* c = s.ctl;
@@ -772,13 +779,18 @@ __global__ void __launch_bounds__(kCT) k_s3_apply(DevState s) {
   uint32_t* ringN = ring_of(s, gc ? rb ^ 1 : rb);
   uint32_t* bitsN = bits_of(s, gc ? rb ^ 1 : rb);
   const int64_t Xo = tmin<int64_t>(tmax<int64_t>(pl->X, 0), pl->live_old);
-  const int64_t born = pl->born;
-  const bool ring_work = gc || Xo > 0;
-  const int64_t units = chS + chM + (ring_work ? pl->nrch : 0);
+  // ring chunks with work: every chunk of the window when compacting, else
+  // those before the new start
+  int64_t nrw = 0;
+  if (gc) nrw = pl->nrch;
+  else if (Xo > 0) nrw = tmin<int64_t>(pl->nrch, cdiv64((int64_t)(pl->q - pl->ra0), kS3Chunk));
+  const int64_t units = nrw + chS + chM;
+  uint32_t* pushes = push_list(s);
   uint32_t* oS = q_region(s, buf ^ 1, 0);
   uint32_t* oM = q_region(s, buf ^ 1, 1);
-  for (int64_t u = blockIdx.x; u < units; u += gridDim.x) {
-    if (u < chS + chM) {
+  for (int64_t u0 = blockIdx.x; u0 < units; u0 += gridDim.x) {
+    if (u0 >= nrw) {
+      const int64_t u = u0 - nrw;
       const int r = u < chS ? 0 : 1;
       const int64_t ci = r ? u - chS : u;
       const int64_t len = r ? lenM : lenS;
@@ -837,19 +849,9 @@ __global__ void __launch_bounds__(kCT) k_s3_apply(DevState s) {
             q_put(s, oS, (int64_t)bb.keep + f2, b);
             continue;
           }
-          if (f < mm) {  // small-queue victim: its key enters the ghost
+          if (f < mm) {  // small-queue victim: its key enters the ghost (k_s3_push)
             mark_victim(s, b);
-            const int64_t t = (int64_t)bb.ev + f0;
-            if (t >= born) {
-              const uint64_t p = pl->pbase + (uint64_t)t;
-              const uint32_t slot = gh_insert(s, s.blk_key[b], s.blk_group[b], (uint32_t)(p & rmask), pl->gctr0 + (uint64_t)t + 1);
-              if (slot == kNone) {
-                c->internal_error = 1;
-              } else {
-                ringN[p & rmask] = slot;
-                atomicOr(bitsN + ((p & rmask) >> 5), 1u << (p & 31));
-              }
-            }
+            pushes[(int64_t)bb.ev + f0] = b;
             continue;
           }
           const int64_t mr = (int64_t)bb.mv + f1;  // moved to the main queue's head
@@ -888,7 +890,7 @@ __global__ void __launch_bounds__(kCT) k_s3_apply(DevState s) {
       }
     } else {
       // a ring chunk of the window [g_tail, g_head)
-      const int64_t k = u - chS - chM;
+      const int64_t k = u0;
       const uint64_t p0 = pl->ra0 + (uint64_t)k * kS3Chunk;
       const uint64_t tail = pl->g_tail, head = pl->g_head;
       if (!gc && p0 >= pl->q) continue;  // trimming only: nothing at or past the new start
@@ -931,8 +933,35 @@ __global__ void __launch_bounds__(kCT) k_s3_apply(DevState s) {
   }
 }
 
+// 5. The step's ghost pushes, one thread each: the key of small-queue victim t
+//    (in eviction order) enters the map with ghost sequence number gctr0 + t + 1
+//    at FIFO position pbase + t; pushes the trimming removes at once
+//    (t < born) are never written.
+__global__ void __launch_bounds__(kCT) k_s3_push(DevState s) {
+  s = with_args(s);
+  Ctl* c = s.ctl;
+  const S3Plan* pl = s.s3_plan;
+  if (c->status != PS_OK || pl->fb) return;
+  const int64_t kS = pl->kS, born = pl->born;
+  const uint64_t rmask = s.ghost_ring_cap - 1;
+  uint32_t* ring = ring_of(s, c->ghost_rbuf);  // the step's ring (the other one after a compaction)
+  uint32_t* bits = bits_of(s, c->ghost_rbuf);
+  const uint32_t* pushes = push_list(s);
+  for (int64_t t = born + blockIdx.x * (int64_t)kCT + threadIdx.x; t < kS; t += (int64_t)gridDim.x * kCT) {
+    const uint32_t b = pushes[t];
+    const uint64_t p = pl->pbase + (uint64_t)t;
+    const uint32_t slot = gh_insert(s, s.blk_key[b], s.blk_group[b], (uint32_t)(p & rmask), pl->gctr0 + (uint64_t)t + 1);
+    if (slot == kNone) {
+      c->internal_error = 1;
+    } else {
+      ring[p & rmask] = slot;
+      atomicOr(bits + ((p & rmask) >> 5), 1u << (p & 31));
+    }
+  }
+}
+
 // ===========================================================================
-// 5. After the insertions: each new block (in rank order, the order of its
+// 6. After the insertions: each new block (in rank order, the order of its
 //    sequence number) looks its key up in the ghost; a hit leaves the ghost
 //    and enters the main queue, any other block the small queue.
 __global__ void __launch_bounds__(kCT) k_s3_ins(DevState s) {
@@ -965,7 +994,7 @@ __global__ void __launch_bounds__(kCT) k_s3_ins(DevState s) {
   }
 }
 
-// 6. The new blocks' places: the small queue's after its kept members, the
+// 7. The new blocks' places: the small queue's after its kept members, the
 //    main queue's after its kept and re-sequenced members, both in rank order.
 __global__ void __launch_bounds__(kCT) k_s3_place(DevState s) {
   s = with_args(s);
@@ -1016,7 +1045,8 @@ int32_t launch_s3_select(const DevState& s, cudaStream_t st, int* launches) {
   launch_k(k_s3_plan, 1, kPT, 0, st, s);
   launch_k(k_s3_fallback, 1, 32, 0, st, s);
   launch_k(k_s3_apply, 152 * 4, kCT, 0, st, s);
-  *launches += 4;
+  launch_k(k_s3_push, 152 * 4, kCT, 0, st, s);
+  *launches += 5;
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
