@@ -465,7 +465,9 @@ int32_t launch_queue_append(const DevState& s, cudaStream_t st, const CaptureCtx
 // S3-FIFO (ps_s3fifo.cu)
 // The select: per-chunk counts, the closed-form plan, the sequential kernel
 // (used when the plan does not apply), the plan's application.
-int32_t launch_s3_select(const DevState& s, cudaStream_t st, int* launches);
+// plain_first: the first kernel follows a fork of the step graph (a plain
+// launch: a programmatic edge is kept for a kernel's only dependent).
+int32_t launch_s3_select(const DevState& s, cudaStream_t st, bool plain_first, int* launches);
 // After the insertions: ghost lookups of the new blocks, their array places.
 int32_t launch_s3_insert(const DevState& s, cudaStream_t st, int* launches);
 // A step's outputs (device) written into page-locked host buffers, the id

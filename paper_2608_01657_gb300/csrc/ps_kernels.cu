@@ -2307,9 +2307,11 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   // the select needs only the step's debts, which k_grant settles.  Under
   // capture they run on a second parallel branch beside the select, joined
   // before the insertion (which reads, then clears, the claim entries).
-  // S3-FIFO and the indexed queues keep them in line (their selects read
-  // touched blocks' state).
-  const bool fork2 = cap != nullptr && !s.lg_on && s.policy != PS_S3FIFO;
+  // The S3-FIFO select reads only unpinned blocks' frequencies, pin tags and
+  // residency, none of which these kernels write (a touch changes hit, so
+  // pinned, blocks), so it runs beside them too.  The indexed queues keep
+  // them in line (their select reads the touched blocks' new stamps).
+  const bool fork2 = cap != nullptr && !s.lg_on;
   cudaStream_t ms = st;
   if (fork2) {
     if (cudaEventRecord(cap->fork2, st) != cudaSuccess || cudaStreamWaitEvent(cap->side2, cap->fork2, 0) != cudaSuccess)
@@ -2368,7 +2370,7 @@ int32_t launch_step(const DevState& s, cudaStream_t st, StepTrace* tr, const Cap
   } else if (s.policy == PS_LRU) {
     PS_LAUNCH(k_sel_single<<<1, 32, 0, st>>>(s, 0));  // after the join: plain
     select(1, 0);
-  } else if (launch_s3_select(s, st, &launches) != PS_OK) {
+  } else if (launch_s3_select(s, st, fork2, &launches) != PS_OK) {
     return PS_ERR_CUDA;
   }
   mark(7);

@@ -1040,8 +1040,9 @@ __global__ void __launch_bounds__(kCT) k_s3_place(DevState s) {
   }
 }
 
-int32_t launch_s3_select(const DevState& s, cudaStream_t st, int* launches) {
-  launch_k(k_s3_count, 152 * 4, kCT, 0, st, s);
+int32_t launch_s3_select(const DevState& s, cudaStream_t st, bool plain_first, int* launches) {
+  if (plain_first) k_s3_count<<<152 * 4, kCT, 0, st>>>(s);
+  else launch_k(k_s3_count, 152 * 4, kCT, 0, st, s);
   launch_k(k_s3_plan, 1, kPT, 0, st, s);
   launch_k(k_s3_fallback, 1, 32, 0, st, s);
   launch_k(k_s3_apply, 152 * 4, kCT, 0, st, s);
