@@ -12,11 +12,12 @@
 //     goes to the main queue's head, the first one below it is the victim
 //     (its key enters the ghost).  Eviction t takes the small queue while the
 //     queue held at least its capacity when it started, i.e. while the
-//     members popped before it number at most D = |small| - capacity.  So the
-//     phase consumes a prefix of the small queue's unpinned members: up to
-//     its n_A-th victim, n_A = min(m, 1 + #{victims among the first D}), or
-//     all of them when it runs out of victims (that eviction then takes the
-//     main queue).
+//     members popped before it number at most D = |small| - capacity, and an
+//     unpinned member is left.  So the phase consumes a prefix of the small
+//     queue's K unpinned members: up to its n_A-th victim,
+//     n_A = min(m, 1 + #{victims among the first min(D, K - 1)}), or all of
+//     them when it runs out of victims (that eviction then takes the main
+//     queue).
 //   - Main phase.  The remaining m_B evictions visit the main queue (its
 //     unpinned members, then the moved blocks) from the tail: frequency f > 0
 //     reinserts the block at the head with f - 1, f = 0 evicts it.  So the
