@@ -77,3 +77,36 @@ def test_host_calls_refuse_bad_arguments_before_any_device_work(lib):
     assert L.ps_step_host_async(None, None, 0, 1, 0, None, None, None, None, None, None) == B.PS_ERR_INVALID_ARG
     assert L.ps_step_host(None, None, 1, 0, None, None, None, None, None, None) == B.PS_ERR_INVALID_ARG
     assert L.ps_step(None, None, 1, 0, None, None, None, None, None, None) == B.PS_ERR_INVALID_ARG
+
+
+def test_flag_and_status_constants_match_the_header():
+    """The binding's and the oracle wrapper's PS_FLAG_* values are the
+    header's (the oracle ignores the execution-choice flags, but tests pass
+    the same bits to both sides)."""
+    import oracle as O
+    from paper_2608_01657_gb300 import binding as B
+    txt = open(os.path.join(ROOT, "include", "prefixshield.h")).read()
+    flags = {m.group(1): int(m.group(2)) for m in re.finditer(r"#define\s+PS_FLAG_([A-Z0-9_]+)\s+(\d+)u", txt)}
+    assert flags, "no PS_FLAG_ definitions found"
+    for name, value in flags.items():
+        assert getattr(B, "PS_FLAG_" + name) == value, name
+        assert getattr(O, "FLAG_" + name) == value, name
+    assert len(set(flags.values())) == len(flags) and all(v & (v - 1) == 0 for v in flags.values())
+    status = dict(re.findall(r"\b(PS_OK|PS_ERR_[A-Z_]+)\s*=\s*(-?\d+)", txt))
+    for name in ("PS_OK", "PS_ERR_INVALID_ARG", "PS_ERR_CAPACITY", "PS_ERR_CLOCK", "PS_ERR_CUDA"):
+        assert getattr(B, name) == int(status[name]), name
+
+
+def test_s3fifo_layout_grows_with_the_pool_and_the_step(lib):
+    """The S3-FIFO queue arrays and ghost rings are carved for every policy:
+    the workspace grows with N (queue regions, ghost map and rings) and with
+    max_tokens / bs (a step's pushes are room in the ghost ring)."""
+    from paper_2608_01657_gb300 import binding as B
+    L = B.load()
+    p = B.Params(rho=(2.0,), beta=(6.0,)).to_c(4)
+    a = L.ps_workspace_bytes(1 << 16, 16, 4, ctypes.byref(p), 64, 1 << 16)
+    b = L.ps_workspace_bytes(1 << 17, 16, 4, ctypes.byref(p), 64, 1 << 16)
+    c = L.ps_workspace_bytes(1 << 16, 16, 4, ctypes.byref(p), 64, 1 << 22)
+    assert a > 0 and b > a and c > a
+    # two buffers of two queue regions of N u32 ids: at least 16 B a block more
+    assert b - a >= 16 * (1 << 16)
