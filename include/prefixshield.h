@@ -123,7 +123,12 @@ typedef struct {
   int32_t contract_of_group[PS_MAX_GROUPS];    /* contract used when a step passes no contract ids */
   uint64_t hash_seed;                          /* seed of the block-key function */
   int32_t s3_small_pct;                        /* S3-FIFO small queue, percent of the pool (10) */
-  int32_t s3_freq_cap;                         /* S3-FIFO counter cap (3: a two-bit counter) */
+  /* S3-FIFO counter cap (3: a two-bit counter).  A step's evictions run in
+   * parallel in closed form for caps up to 15; caps of 16 or more, and steps
+   * whose main queue would run empty (common when the small queue is near
+   * 100% of the pool), take the one-at-a-time loop on one device thread:
+   * the same results, much slower on large pools. */
+  int32_t s3_freq_cap;
   int32_t s3_move_min_freq;                    /* small->main when freq >= this (2) */
   int32_t pad0;
   int64_t history_capacity;                    /* max distinct (group, prefix id) entries */
