@@ -182,9 +182,13 @@ Dims make_dims(int64_t N, int32_t bs, int32_t G, const ps_params_t* P, int32_t m
   // (at most max_blocks), so compactions are rare; at least two chunks.
   d.s3_np = (N + kS3Chunk - 1) / kS3Chunk * kS3Chunk;
   d.s3_nch = d.s3_np / kS3Chunk;
+  // At most 2^31 positions: a FIFO index must stay below the map's empty
+  // marker (0xFFFFFFFF), and 2^31 still holds a full ghost (< 2^30 entries)
+  // plus a step's pushes (< 2^30) after a compaction.
   {
     const uint64_t want = (uint64_t)(2 * (d.s3_ghost_cap + d.max_blocks));
     d.ghost_ring_cap = 1ull << log2_pow2_at_least(want > 2 * (uint64_t)kS3Chunk ? want : 2 * (uint64_t)kS3Chunk);
+    if (d.ghost_ring_cap > (1ull << 31)) d.ghost_ring_cap = 1ull << 31;
   }
   d.s3_nrch = (int64_t)(d.ghost_ring_cap / kS3Chunk) + 1;
   // indexed queues: at most two live entries a block (its group's log and its
