@@ -282,7 +282,7 @@ int32_t ps_cached_prefix(ps_handle_t* h, void* stream, int32_t num_requests, con
  * inside a CUDA graph capture region, or code under a framework whose
  * allocator owns every device allocation.  This variant computes the same
  * counts as ps_cached_prefix() with its scratch in one fixed array compiled
- * into the library (about 2.3 MB, held on every GPU that loads the library
+ * into the library (about 2.4 MB, held on every GPU that loads the library
  * until the process exits).  It allocates nothing; the caller passes inputs
  * and outputs as for ps_cached_prefix().  Only the scratch leaves the
  * workspace: the probe reads the pool's table, which every ps_step() of the

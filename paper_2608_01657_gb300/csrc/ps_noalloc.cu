@@ -35,7 +35,7 @@ constexpr size_t kOffSeg = align256(kOffTile + 8 * (kNaMaxRequests / kValTile + 
 constexpr size_t kOffPos = align256(kOffSeg + align256(sizeof(ChunkDesc) * kNaMaxSegments) + align256(8 * kNaMaxSegments));
 constexpr size_t kScratchBytes = align256(kOffPos + align256(8 * kNaMaxBlocks) + 2 * align256(4 * kNaMaxBlocks));
 
-// The scratch itself (about 2.3 MB).  In host code 'g_probe_scratch' names a
+// The scratch itself (about 2.4 MB).  In host code 'g_probe_scratch' names a
 // host-side stand-in, not device memory: only the address returned by
 // cudaGetSymbolAddress() may be handed to a kernel.
 static __device__ __align__(256) unsigned char g_probe_scratch[kScratchBytes];
